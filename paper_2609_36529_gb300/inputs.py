@@ -1,0 +1,120 @@
+"""Seeded synthetic inputs shaped like the paper's language-modelling workloads.
+
+This module holds no arithmetic of the method itself: it only draws random
+tensors and applies the input preconditions the paper's layer applies before
+the operator (L2-normalised queries and keys, Algorithm 2; log-sigmoid forget
+gates so that log alpha <= 0; beta in (0,1) through a sigmoid).  Both the CUDA
+path's tests/benchmark and the oracle's tests draw their inputs here.
+
+Recipe (fixed tensor order q, k, q2, k2, v, beta, g, h0, dO, one
+``torch.Generator`` seeded with ``seed``):
+  q, k   ~ N(0,1) [B,T,H,dk], L2-normalised per vector in fp32
+  q2, k2 ~ N(0,1) [B,T,H,E],  L2-normalised per vector in fp32
+  v      ~ N(0,1) [B,T,H,dv]
+  beta   = sigmoid(N(0,1)) [B,T,H]              (only when requested)
+  g      = logsigmoid(N(gate_mean, 1)) [B,T,H,E] (log forget gates, <= 0)
+  h0     ~ N(0, h0_std^2) [B,H,E,dk,dv] fp32     (only when h0_std > 0)
+  dO     ~ N(0,1) [B,T,H,dv]                      (only when requested)
+q, k, q2, k2, v, dO are then cast to ``dtype``; g, beta, h0 stay fp32.
+"""
+from dataclasses import dataclass
+from typing import Optional
+
+import torch
+
+
+@dataclass(frozen=True)
+class Workload:
+    name: str
+    B: int
+    T: int
+    H: int
+    dk: int
+    dv: int
+    E: int
+    dtype: str            # "fp32" | "bf16"
+    use_delta: bool
+    with_beta: bool
+    h0_std: float = 0.0
+    backward: bool = False
+    chunk: int = 64
+
+
+# The five workloads of the paper's setting (Section 3.1, Appendix A: d=128, C=64,
+# E in {4,8,16}, 4k pretraining / 64k extension context).
+SGLA_FWD_FP32 = Workload("sgla_fwd_fp32_B1_H2_T256_d32_E4", 1, 256, 2, 32, 32, 4, "fp32",
+                         use_delta=False, with_beta=False)
+GDN_FWD_BF16 = Workload("gdn_fwd_bf16_B4_H16_T4096_d128_E8", 4, 4096, 16, 128, 128, 8, "bf16",
+                        use_delta=True, with_beta=True)
+GDN_FWDBWD_BF16 = Workload("gdn_fwdbwd_bf16_B8_H16_T8192_d128_E4", 8, 8192, 16, 128, 128, 4,
+                           "bf16", use_delta=True, with_beta=True, backward=True)
+GDN_LONG_BF16 = Workload("gdn_fwd_bf16_B1_H32_T65536_d128_E16", 1, 65536, 32, 128, 128, 16,
+                         "bf16", use_delta=True, with_beta=True, h0_std=0.1)
+WORKLOADS = {w.name: w for w in (SGLA_FWD_FP32, GDN_FWD_BF16, GDN_FWDBWD_BF16, GDN_LONG_BF16)}
+
+
+@dataclass(frozen=True)
+class DecodeWorkload:
+    name: str
+    B: int
+    H: int
+    dk: int
+    dv: int
+    E: int
+    steps: int
+    prefill: int
+
+
+DECODE = DecodeWorkload("decode_fp32_state_B256_H32_E8_d128", 256, 32, 128, 128, 8, 100, 512)
+
+
+def torch_dtype(name: str) -> torch.dtype:
+    return {"fp32": torch.float32, "bf16": torch.bfloat16}[name]
+
+
+def _unit(x: torch.Tensor) -> torch.Tensor:
+    return x / x.norm(dim=-1, keepdim=True).clamp_min(1e-12)
+
+
+def chunk_inputs(B, T, H, dk, dv, E, dtype="bf16", with_beta=True, h0_std=0.0,
+                 backward=False, device="cpu", seed=0, gate_mean=3.0,
+                 gen: Optional[torch.Generator] = None):
+    """Draw one batch of inputs for the chunkwise forward (and backward)."""
+    dev = torch.device(device)
+    if gen is None:
+        gen = torch.Generator(device=dev)
+        gen.manual_seed(seed)
+    dt = torch_dtype(dtype)
+
+    def randn(*shape):
+        return torch.randn(*shape, generator=gen, device=dev, dtype=torch.float32)
+
+    out = {}
+    out["q"] = _unit(randn(B, T, H, dk)).to(dt)
+    out["k"] = _unit(randn(B, T, H, dk)).to(dt)
+    out["q2"] = _unit(randn(B, T, H, E)).to(dt)
+    out["k2"] = _unit(randn(B, T, H, E)).to(dt)
+    out["v"] = randn(B, T, H, dv).to(dt)
+    out["beta"] = torch.sigmoid(randn(B, T, H)) if with_beta else None
+    out["g"] = torch.nn.functional.logsigmoid(randn(B, T, H, E) + gate_mean)
+    out["h0"] = randn(B, H, E, dk, dv) * h0_std if h0_std > 0 else None
+    out["dO"] = randn(B, T, H, dv).to(dt) if backward else None
+    return out
+
+
+def workload_inputs(w: Workload, device="cpu", seed=0, B=None, T=None, H=None):
+    """Inputs of a named workload, optionally with a reduced B/T/H for tests."""
+    return chunk_inputs(B or w.B, T or w.T, H or w.H, w.dk, w.dv, w.E, w.dtype, w.with_beta,
+                        w.h0_std, w.backward, device=device, seed=seed)
+
+
+def decode_inputs(B, H, dk, dv, E, dtype="fp32", with_beta=True, device="cpu",
+                  gen: Optional[torch.Generator] = None, seed=0):
+    """Inputs of one decode step: q,k [B,H,dk]; v [B,H,dv]; q2,k2,g [B,H,E]; beta [B,H]."""
+    dev = torch.device(device)
+    if gen is None:
+        gen = torch.Generator(device=dev)
+        gen.manual_seed(seed)
+    d = chunk_inputs(B, 1, H, dk, dv, E, dtype, with_beta, device=dev, gen=gen)
+    return {n: (None if t is None else t[:, 0].contiguous()) for n, t in d.items()
+            if n not in ("h0", "dO")}
