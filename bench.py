@@ -1,0 +1,530 @@
+#!/usr/bin/env python
+"""Benchmark of the triadic linear attention hot path on GB300.
+
+A step is one chunkwise forward (saving what the backward needs) plus the
+backward of triadic Gated DeltaNet on the headline workload (B=8, H=16, T=8192,
+d_k=d_v=128, E=4, chunk 64, bf16 inputs / fp32 state), synthetic seeded
+inputs.  The single-token decode step is measured in the same run on the
+decode workload (fp32 state [256,32,8,128,128], 100 steps each of sGLA and
+GDN after a 512-token chunked prefill) and reported under "decode".
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+With N > 1 (torchrun) every rank runs its own batch of independent sequences
+(heads and sequences never interact): weak scaling, no collective on the data
+path.  Rank 0 prints one JSON line.  `--impl reference` times the float64 CPU
+oracle on this machine's host cores on a bounded sample of the same workload.
+"""
+import argparse
+import ctypes
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import torch  # noqa: E402
+
+HEADLINE_METRIC = "tokens/s triadic GDN fwd+bwd (T=8K, E=4); TFLOP/s and decode GB/s vs GB300 peak"
+CHUNK = 64
+
+
+# ----------------------------------------------------------------------------- helpers
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return {"hbm_gbs": float(p["hbm_gbs"]), "bf16_tflops": float(p["bf16_tflops"]),
+                "bf16_tflops_sustained": float(p.get("bf16_tflops_sustained", p["bf16_tflops"])),
+                "source": "measured"}
+    except Exception:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+                "source": "fallback"}
+
+
+def flops_per_token_head(kernel, E, dk, dv, C=CHUNK):
+    """Algorithmic flops of one token of one head for each kernel (dense contractions).
+
+    Forward recurrence: K S_e, Q S_e, K^T diag(w_e) U  -> 6 E dk dv; T Res, A U -> 4 C dv.
+    Backward recurrence: K dS'_e, Q^T.., K^T..        -> 6 E dk dv; A^T dO, T^T dU -> 4 C dv.
+    Chunk gradients: dO S^T, dRes S^T, U dS'^T        -> 6 E dk dv; dO U^T, dU Res^T -> 4 C dv;
+                     Q K^T, K K^T, P K, P^T Q, (dKK+dKK^T) K -> 10 C dk; two C x C x C -> 4 C.
+    Chunk prep: Q K^T, K K^T -> 4 C dk; triangular solve -> C^2/3.
+    """
+    name = kernel
+    if name.startswith("fwd_recurrence") or name.startswith("bwd_recurrence"):
+        return 6 * E * dk * dv + 4 * C * dv
+    if name.startswith("bwd_chunk_grads"):
+        return 6 * E * dk * dv + 4 * C * dv + 10 * C * dk + 4 * C
+    if name.startswith("chunk_prep"):
+        return 4 * C * dk + C * C / 3
+    return 0.0
+
+
+def kernel_source_hash(kernel):
+    """Hash of the source file that defines a kernel (to invalidate stale ncu traffic)."""
+    csrc = os.path.join(ROOT, "paper_2609_36529_gb300", "csrc")
+    h = hashlib.sha256()
+    for fn in sorted(os.listdir(csrc)):
+        path = os.path.join(csrc, fn)
+        with open(path, "rb") as f:
+            data = f.read()
+        if kernel.encode() in data or fn.endswith((".cuh", ".h")):
+            h.update(fn.encode())
+            h.update(data)
+    return h.hexdigest()[:16]
+
+
+def ncu_traffic(kernel, units_per_launch):
+    """DRAM bytes per launch from the committed ncu summary, if it is still current."""
+    path = os.path.join(ROOT, "profiles", "ncu_traffic.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        rec = d[kernel]
+        if rec.get("src_hash") != kernel_source_hash(kernel):
+            return None
+        return rec["bytes_per_unit"] * units_per_launch
+    except Exception:
+        return None
+
+
+class ClockSampler:
+    """nvidia-smi samples (200 ms) of SM clock and throttle reasons while running."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device):
+        self.samples = []
+        self.proc = None
+        self.thread = None
+        sel = []
+        try:
+            uuid = str(torch.cuda.get_device_properties(device).uuid)
+            sel = ["-i", uuid if uuid.startswith("GPU-") else "GPU-" + uuid]
+        except Exception:
+            sel = []
+        self.cmd = ["nvidia-smi", "--query-gpu=" + self.FIELDS, "--format=csv,noheader,nounits",
+                    "-lms", "200"] + sel
+
+    def _reader(self):
+        for line in self.proc.stdout:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) >= 9:
+                self.samples.append(parts)
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(self.cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL,
+                                         text=True)
+            self.thread = threading.Thread(target=self._reader, daemon=True)
+            self.thread.start()
+        except Exception:
+            self.proc = None
+        return self
+
+    def stop(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+            self.thread.join(timeout=5)
+        return self.summary()
+
+    def summary(self):
+        if not self.samples:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no nvidia-smi samples"]}
+        sm, smax, power, reasons = [], [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for s in self.samples:
+            try:
+                sm.append(float(s[1]))
+                smax.append(float(s[2]))
+                power.append(float(s[3]))
+            except ValueError:
+                continue
+            for name, val in zip(names, s[5:9]):
+                if val.lower().startswith("active"):
+                    reasons.add(name)
+        loaded = [x for x in sm if x > 0.5 * max(sm)] if sm else []
+        return {"sm_mhz": statistics.median(loaded) if loaded else None,
+                "sm_max_mhz": max(smax) if smax else None,
+                "power_w_max": max(power) if power else None,
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+def bad_clocks(c):
+    if any(r in c.get("reasons", []) for r in ("hw_slowdown", "hw_thermal_slowdown",
+                                                "sw_thermal_slowdown")):
+        return True
+    if c.get("sm_mhz") and c.get("sm_max_mhz") and c["sm_mhz"] < 0.6 * c["sm_max_mhz"] \
+            and "sw_power_cap" not in c.get("reasons", []):
+        return True
+    return False
+
+
+def profile_read(lib, stream):
+    names = ctypes.create_string_buffer(64 * 32)
+    launches = (ctypes.c_int * 32)()
+    ms = (ctypes.c_float * 32)()
+    n = lib.tla_profile_end(ctypes.c_void_p(stream), names, launches, ms, 32)
+    if n < 0:
+        raise RuntimeError(f"tla_profile_end failed: {n}")
+    out = {}
+    for i in range(n):
+        nm = names.raw[64 * i:64 * (i + 1)].split(b"\0", 1)[0].decode()
+        out[nm] = {"launches": int(launches[i]), "ms": float(ms[i])}
+    return out
+
+
+# ----------------------------------------------------------------------------- our arm
+
+def run_ours(args):
+    from paper_2609_36529_gb300 import inputs, tla
+
+    ws_n, rank, local = dist_env()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if ws_n > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    lib = tla.lib()
+    lib.tla_profile_begin.restype = ctypes.c_int
+    lib.tla_profile_end.argtypes = [ctypes.c_void_p, ctypes.c_char_p,
+                                    ctypes.POINTER(ctypes.c_int), ctypes.POINTER(ctypes.c_float),
+                                    ctypes.c_int]
+    lib.tla_profile_end.restype = ctypes.c_int
+
+    def barrier():
+        if ws_n > 1:
+            torch.distributed.barrier()
+
+    def max_over_ranks(x):
+        if ws_n == 1:
+            return x
+        t = torch.tensor([x], dtype=torch.float64, device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        return float(t.item())
+
+    w = inputs.GDN_FWDBWD_BF16
+    x = inputs.workload_inputs(w, device=dev, seed=rank)
+    stream = torch.cuda.current_stream(dev)
+
+    # preallocated outputs and workspaces (allocation is outside the timed region)
+    o = torch.empty(w.B, w.T, w.H, w.dv, dtype=torch.bfloat16, device=dev)
+    p = tla.make_problem(x["q"], x["k"], x["v"], x["q2"], x["k2"], x["g"], x["beta"], None, o,
+                         None, use_delta=True)
+    fws = torch.empty(tla.fwd_workspace_bytes(p, True), dtype=torch.uint8, device=dev)
+    bws = torch.empty(tla.bwd_workspace_bytes(p), dtype=torch.uint8, device=dev)
+    grads = {"dq": torch.empty_like(x["q"]), "dk": torch.empty_like(x["k"]),
+             "dv": torch.empty_like(x["v"]), "dq2": torch.empty_like(x["q2"]),
+             "dk2": torch.empty_like(x["k2"]), "dg": torch.empty_like(x["g"]),
+             "dbeta": torch.empty_like(x["beta"])}
+
+    def step(xx):
+        tla.tla_chunk_fwd(xx["q"], xx["k"], xx["v"], xx["q2"], xx["k2"], xx["g"], xx["beta"],
+                          None, use_delta=True, save_for_bwd=True, want_ht=False, o=o,
+                          workspace=fws)
+        tla.tla_chunk_bwd(xx["q"], xx["k"], xx["v"], xx["q2"], xx["k2"], xx["g"], xx["dO"], fws,
+                          beta=xx["beta"], use_delta=True, workspace=bws, grads=grads)
+
+    for _ in range(args.warmup):
+        step(x)
+    torch.cuda.synchronize()
+    if tla.tla_last_device_status() != 0:
+        raise RuntimeError("device status not OK after warm-up")
+
+    def timed_loop():
+        barrier()
+        torch.cuda.synchronize()
+        clocks = ClockSampler(dev).start()
+        time.sleep(0.25)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        lib.tla_profile_begin()
+        e0.record(stream)
+        for _ in range(args.steps):
+            step(x)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        prof = profile_read(lib, stream.cuda_stream)
+        barrier()
+        ck = clocks.stop()
+        return e0.elapsed_time(e1), prof, ck
+
+    ms_total, prof, ck = timed_loop()
+    remeasured = False
+    if bad_clocks(ck):
+        ms_total, prof, ck = timed_loop()
+        remeasured = True
+    ms_step = max_over_ranks(ms_total / args.steps)
+    tokens_step = w.B * w.T
+    value = ws_n * tokens_step / (ms_step / 1e3)
+    if tla.tla_last_device_status() != 0:
+        raise RuntimeError("device status not OK after timed loop")
+
+    peaks = load_peaks()
+    units = w.B * w.T * w.H  # token-heads per launch
+    kernels = {}
+    for name, r in prof.items():
+        f = flops_per_token_head(name, w.E, w.dk, w.dv) * units
+        avg_ms = r["ms"] / max(r["launches"], 1)
+        kernels[name] = {"launches": r["launches"], "avg_ms": round(avg_ms, 4),
+                         "share": round(r["ms"] / max(sum(v["ms"] for v in prof.values()), 1e-9), 4),
+                         "tflops": round(f / (avg_ms / 1e3) / 1e12, 2) if f else None}
+    top = max(prof, key=lambda n: prof[n]["ms"])
+    top_flops = flops_per_token_head(top, w.E, w.dk, w.dv) * units
+    top_avg_s = prof[top]["ms"] / prof[top]["launches"] / 1e3
+    achieved = top_flops / top_avg_s / 1e12
+    peak = peaks["bf16_tflops_sustained"]
+    traffic = ncu_traffic(top, units)
+    roofline = {"kernel": top, "bound": "tensor", "achieved": round(achieved, 3),
+                "peak": peak, "unit": "TFLOP/s", "frac": round(achieved / peak, 5),
+                "traffic": traffic,
+                "peak_source": f"bf16 dense sustained, {peaks['source']} (MEASURED_PEAKS.json)"
+                if peaks["source"] == "measured" else "bf16 dense sustained, fallback"}
+    total_flops = sum(flops_per_token_head(n, w.E, w.dk, w.dv) * units * prof[n]["launches"]
+                      for n in prof) / args.steps
+    gpu_launches = sum(r["launches"] for r in prof.values())
+
+    # ---- end to end through the public API from pinned host buffers
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(args, tla, x, w, dev, stream, o, fws, bws, grads, barrier, max_over_ranks,
+                      ws_n)
+
+    # ---- decode workload
+    decode = None
+    if not args.no_decode:
+        del fws, bws
+        torch.cuda.empty_cache()
+        decode = run_decode(args, tla, inputs, dev, stream, lib, peaks, barrier, max_over_ranks,
+                            ws_n)
+
+    # ---- CPU baseline: the oracle on this host's cores (rank 0, N=1 only)
+    cpu = None
+    if rank == 0 and ws_n == 1 and not args.no_cpu_baseline:
+        cpu = oracle_baseline(x, w, seconds_target=args.cpu_seconds)
+
+    if rank == 0:
+        line = {
+            "metric": HEADLINE_METRIC, "value": round(value, 1), "unit": "tokens/s",
+            "n_gpus": ws_n, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(ms_step, 4), "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": w.name, "B": w.B, "T": w.T, "H": w.H, "dk": w.dk, "dv": w.dv,
+                       "E": w.E, "chunk": CHUNK, "variant": "triadic GDN (joint-key delta rule)",
+                       "state": "fp32", "parallelism": f"replicas x{ws_n} (independent sequences)",
+                       "l2": "inputs larger than L2 (q,k,v,dO 268 MB each per GPU)"},
+            "tflops": round(total_flops / (ms_step / 1e3) / 1e12, 3),
+            "tflops_frac": round(total_flops / (ms_step / 1e3) / 1e12 / peak, 5),
+            "roofline": roofline, "kernels": kernels, "gpu_launches": gpu_launches,
+            "clocks": ck, "clocks_remeasured": remeasured,
+            "e2e": e2e, "decode": decode, "cpu_baseline": cpu, "impl": "ours",
+        }
+        print(json.dumps(line), flush=True)
+    if ws_n > 1:
+        torch.distributed.destroy_process_group()
+
+
+def run_e2e(args, tla, x, w, dev, stream, o, fws, bws, grads, barrier, max_over_ranks, ws_n):
+    names = ["q", "k", "v", "q2", "k2", "g", "beta", "dO"]
+    host_in = {n: x[n].cpu().pin_memory() for n in names}
+    dev_in = {n: torch.empty_like(x[n]) for n in names}
+    outs = {"o": o, **grads}
+    host_out = {n: torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for n, t in outs.items()}
+    h2d = sum(t.numel() * t.element_size() for t in host_in.values())
+    d2h = sum(t.numel() * t.element_size() for t in host_out.values())
+
+    def step():
+        for n in names:
+            dev_in[n].copy_(host_in[n], non_blocking=True)
+        tla.tla_chunk_fwd(dev_in["q"], dev_in["k"], dev_in["v"], dev_in["q2"], dev_in["k2"],
+                          dev_in["g"], dev_in["beta"], None, use_delta=True, save_for_bwd=True,
+                          want_ht=False, o=o, workspace=fws)
+        tla.tla_chunk_bwd(dev_in["q"], dev_in["k"], dev_in["v"], dev_in["q2"], dev_in["k2"],
+                          dev_in["g"], dev_in["dO"], fws, beta=dev_in["beta"], use_delta=True,
+                          workspace=bws, grads=grads)
+        for n, t in outs.items():
+            host_out[n].copy_(t, non_blocking=True)
+
+    step()
+    torch.cuda.synchronize()
+    k = max(1, min(args.steps, 5))
+    barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(k):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = max_over_ranks(e0.elapsed_time(e1) / k)
+    return {"value": round(ws_n * w.B * w.T / (ms / 1e3), 1), "unit": "tokens/s",
+            "ms_per_step": round(ms, 3), "steps": k, "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "api": "paper_2609_36529_gb300.tla (ctypes -> libtla.so)"}
+
+
+def run_decode(args, tla, inputs, dev, stream, lib, peaks, barrier, max_over_ranks, ws_n):
+    dw = inputs.DECODE
+    gen = torch.Generator(dev)
+    gen.manual_seed(1000 + dist_env()[1])
+    state = torch.empty(dw.B, dw.H, dw.E, dw.dk, dw.dv, dtype=torch.float32, device=dev)
+    res = {}
+    for variant, use_delta in (("sgla", False), ("gdn", True)):
+        pre = inputs.chunk_inputs(dw.B, dw.prefill, dw.H, dw.dk, dw.dv, dw.E, dtype="bf16",
+                                  with_beta=True, device=dev, gen=gen)
+        ws = None
+        _, _, ws = tla.tla_chunk_fwd(pre["q"], pre["k"], pre["v"], pre["q2"], pre["k2"], pre["g"],
+                                     pre["beta"], None, use_delta=use_delta, save_for_bwd=False,
+                                     ht=state)
+        del pre, ws
+        steps = [inputs.decode_inputs(dw.B, dw.H, dw.dk, dw.dv, dw.E, dtype="bf16", device=dev,
+                                      gen=gen) for _ in range(dw.steps)]
+        o = torch.empty(dw.B, dw.H, dw.dv, dtype=torch.bfloat16, device=dev)
+        # warm-up launches on a one-sequence scratch state keep the measured sequence intact
+        scratch = state[:1].clone()
+        for s in steps[:3]:
+            tla.tla_decode_step(scratch, *(s[n][:1].contiguous() for n in
+                                           ("q", "k", "v", "q2", "k2", "g", "beta")),
+                                use_delta=use_delta)
+        del scratch
+        torch.cuda.synchronize()
+        barrier()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        lib.tla_profile_begin()
+        e0.record(stream)
+        for s in steps:
+            tla.tla_decode_step(state, s["q"], s["k"], s["v"], s["q2"], s["k2"], s["g"], s["beta"],
+                                use_delta=use_delta, o=o)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        prof = profile_read(lib, stream.cuda_stream)
+        ms = max_over_ranks(e0.elapsed_time(e1) / dw.steps)
+        kern_ms = prof["decode_step"]["ms"] / prof["decode_step"]["launches"]
+        bytes_step = 8.0 * dw.E * dw.dk * dw.dv * dw.B * dw.H
+        gbs = bytes_step / (kern_ms / 1e3) / 1e9
+        res[variant] = {"ms_per_step": round(ms, 4), "kernel_ms": round(kern_ms, 4),
+                        "seq_steps_per_s": round(ws_n * dw.B / (ms / 1e3), 1),
+                        "achieved_gbs": round(gbs, 1), "frac": round(gbs / peaks["hbm_gbs"], 4),
+                        "launches": prof["decode_step"]["launches"]}
+        del steps
+    return {"workload": dw.name, "unit": "GB/s", "bound": "hbm", "peak": peaks["hbm_gbs"],
+            "peak_source": f"hbm copy bandwidth, {peaks['source']}",
+            "bytes_per_step": 8 * dw.E * dw.dk * dw.dv * dw.B * dw.H,
+            "traffic": ncu_traffic("decode_step", dw.B * dw.H),
+            "state": "fp32 [256,32,8,128,128] (4.3 GB, larger than L2)", "inputs": "bf16",
+            **res}
+
+
+def oracle_baseline(x, w, seconds_target=15.0, T_sample=None):
+    """Time the float64 oracle (fwd+bwd) on a sample of whole heads on this host's cores."""
+    import oracle
+    cores = oracle.num_threads()
+    T = T_sample or w.T
+    nh = max(1, min(cores, w.B * w.H))
+    picks = [(i // w.H, i % w.H) for i in range(nh)]
+
+    def sel(t, per_token=True):
+        return torch.stack([t[b, :T, h] for b, h in picks])[:, :, None].double().cpu().numpy()
+
+    c = {n: sel(x[n]) for n in ("q", "k", "v", "q2", "k2", "g", "beta", "dO")}
+    t0 = time.perf_counter()
+    oracle.forward(c["q"], c["k"], c["v"], c["q2"], c["k2"], c["g"], c["beta"], None)
+    oracle.backward(c["q"], c["k"], c["v"], c["q2"], c["k2"], c["g"], c["dO"], c["beta"], None)
+    dt = time.perf_counter() - t0
+    tokens_equiv = nh * T / w.H   # one token = all H heads of one position
+    return {"value": round(tokens_equiv / dt, 3), "unit": "tokens/s", "cores": cores,
+            "kind": "oracle", "seconds": round(dt, 2),
+            "sample": f"{nh} whole heads (b,h) x {T} tokens of {w.name}, float64 token "
+                      f"recurrence forward + backward, OpenMP over heads; tokens/s counts "
+                      f"{nh}/{w.H} of a position's heads as {nh / w.H:.3f} tokens"}
+
+
+# ----------------------------------------------------------------------------- reference arm
+
+def run_reference(args):
+    ws_n, rank, _ = dist_env()
+    if rank != 0:
+        return
+    from paper_2609_36529_gb300 import inputs
+    import oracle
+    w = inputs.GDN_FWDBWD_BF16
+    cores = oracle.num_threads()
+    nh = max(1, min(cores, w.B * w.H))
+    T = args.ref_tokens
+    x = inputs.chunk_inputs(1, T, nh, w.dk, w.dv, w.E, dtype="bf16", with_beta=True,
+                            backward=True, device="cpu", seed=0)
+    c = {n: x[n].double().numpy() for n in ("q", "k", "v", "q2", "k2", "g", "beta", "dO")}
+
+    def step():
+        oracle.forward(c["q"], c["k"], c["v"], c["q2"], c["k2"], c["g"], c["beta"], None)
+        oracle.backward(c["q"], c["k"], c["v"], c["q2"], c["k2"], c["g"], c["dO"], c["beta"], None)
+
+    for _ in range(args.warmup):
+        step()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    dt = (time.perf_counter() - t0) / args.steps
+    tokens_equiv = nh * T / w.H
+    value = tokens_equiv / dt
+    sample = (f"{nh} heads x {T} tokens per step (shape of {w.name}: d_k=d_v={w.dk}, E={w.E}), "
+              f"float64 oracle forward + backward on {cores} host threads; tokens/s counts "
+              f"{nh}/{w.H} of a position's heads as {nh / w.H:.3f} tokens")
+    line = {"metric": HEADLINE_METRIC, "value": round(value, 3), "unit": "tokens/s",
+            "n_gpus": ws_n, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(dt * 1e3, 2), "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": w.name, "B": w.B, "T": w.T, "H": w.H, "dk": w.dk, "dv": w.dv,
+                       "E": w.E, "chunk": CHUNK, "variant": "triadic GDN (joint-key delta rule)"},
+            "impl": "reference",
+            "cpu_baseline": {"value": round(value, 3), "unit": "tokens/s", "cores": cores,
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": round(value, 3), "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-decode", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--ref-tokens", type=int, default=1024,
+                    help="tokens per head in one reference-arm step")
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl == "ours":
+        print("bench: at least 3 warm-up steps are required; using 3", file=sys.stderr)
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

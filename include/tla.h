@@ -1,0 +1,166 @@
+/*
+ * tla.h - C ABI of the GB300 (sm_103a) triadic linear attention library.
+ *
+ * Triadic linear attention (arXiv 2609.36529) keeps, per head, a third-order
+ * state S in R^{E x dk x dv} (slice e = S[:, e, :] of the paper's d x E x d
+ * tensor, stored here as [E][dk][dv]).  Each token
+ *   1. decays every slice by its own forget gate alpha_{t,e}     (Section 2.4, Eq. forget3)
+ *   2. with the joint-key delta rule, erases the value read at the joint key
+ *      k (x) k', scaled by beta_t: u = beta (v - S x1 k x2 k')   (Section 2.4, Eq. gdn3)
+ *      without it ("sGLA"): u = beta v                           (Algorithm 2)
+ *   3. writes k (x) k' (x) u                                     (Section 2.2, Eq. la3)
+ *   4. reads o = S x1 q x2 q' after the write                   (Section 2.2, Eq. la3)
+ * tla_chunk_fwd / tla_chunk_bwd compute this for whole sequences with the
+ * chunkwise-parallel form of Appendix A (Eq. joint-gram, joint-solve,
+ * joint-chunk); tla_decode_step advances the recurrence by one token.
+ *
+ * Conventions shared by every entry point
+ *  - Every pointer is a DEVICE pointer (cudaMalloc / PyTorch CUDA memory) unless
+ *    stated otherwise; the caller owns every buffer, including workspaces.
+ *    The library allocates no device memory.
+ *  - All tensors are dense, row-major, contiguous.  Token tensors use the
+ *    layout [B, T, H, D]; states use [B, H, E, dk, dv].
+ *  - `dtype` (tla_dtype) is the element type of q, k, v, q2, k2, o and of their
+ *    gradients.  Log-gates g, beta, states h0/ht/dh0, dg and dbeta are fp32.
+ *  - q, k, q2, k2 are expected to be L2-normalised by the caller (Algorithm 2
+ *    normalises them before the operator); no 1/sqrt(d) scale is applied.
+ *    g holds log alpha <= 0 (log of the per-slice forget gate).
+ *  - `stream` is a cudaStream_t passed as void*; NULL means the legacy default
+ *    stream.  Calls only enqueue work: they never synchronise the device.
+ *  - Argument errors are detected on the host before anything is launched and
+ *    return a negative status; nothing is written in that case.  Launch errors
+ *    return TLA_ERR_CUDA.  Device-side bounded waits that expire record an
+ *    error word that tla_last_device_status() reports (TLA_ERR_TIMEOUT).
+ *  - Results are deterministic: no floating-point atomics (Appendix A, Kernels).
+ */
+#ifndef TLA_H
+#define TLA_H
+
+#include <stddef.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    TLA_OK = 0,
+    TLA_ERR_INVALID_ARG = -1,  /* bad pointer, size, alignment or combination */
+    TLA_ERR_UNSUPPORTED = -2,  /* valid request outside the supported shapes   */
+    TLA_ERR_CUDA = -3,         /* a CUDA launch or runtime call failed          */
+    TLA_ERR_TIMEOUT = -4,      /* a device-side bounded wait expired            */
+    TLA_ERR_WORKSPACE = -5     /* workspace missing or smaller than required    */
+} tla_status;
+
+typedef enum { TLA_BF16 = 0, TLA_FP32 = 1 } tla_dtype;
+
+/*
+ * One chunkwise problem: B sequences of T tokens, H heads.
+ * Supported: 1 <= dk, dv <= 128 with dk, dv multiples of 16; 1 <= E <= 16;
+ * chunk == 64 (the paper's C, Appendix A); T >= 1 (a last partial chunk is
+ * allowed); B*H <= 65535.
+ */
+typedef struct {
+    int B, T, H;
+    int dk, dv, E;
+    int chunk;           /* must be 64                                         */
+    int dtype;           /* tla_dtype of q, k, v, q2, k2, o                    */
+    int use_delta;       /* 1: triadic Gated DeltaNet (Eq. gdn3); 0: sGLA      */
+    const void *q;       /* [B,T,H,dk]                                          */
+    const void *k;       /* [B,T,H,dk]                                          */
+    const void *v;       /* [B,T,H,dv]                                          */
+    const void *q2;      /* [B,T,H,E]  second query q'                          */
+    const void *k2;      /* [B,T,H,E]  second key k'                            */
+    const float *g;      /* [B,T,H,E]  log forget gates, <= 0                   */
+    const float *beta;   /* [B,T,H] write strength in (0,1); NULL => 1.
+                            Required when use_delta == 1.                       */
+    const float *h0;     /* [B,H,E,dk,dv] initial state; NULL => zero state     */
+    void *o;             /* [B,T,H,dv] output (written)                         */
+    float *ht;           /* [B,H,E,dk,dv] final state (written); may be NULL    */
+} tla_problem;
+
+/*
+ * Workspace of tla_chunk_fwd in bytes (a multiple of 256; the workspace pointer
+ * must be 256-byte aligned).  With save_for_bwd != 0 the workspace also keeps
+ * what tla_chunk_bwd needs (chunk-start states, delta-corrected values, the
+ * per-chunk UT-transform matrices); it must then stay untouched until the
+ * matching tla_chunk_bwd has run.  Returns 0 for an invalid problem.
+ */
+size_t tla_fwd_workspace_bytes(const tla_problem *p, int save_for_bwd);
+
+/*
+ * Chunkwise-parallel forward (Appendix A, Eq. joint-chunk): writes p->o and,
+ * when non-NULL, p->ht.  Steps: per-slice chunk-local cumulative log decay;
+ * per chunk R, R' (Eq. joint-gram), A = QK^T (.) R' and the UT transform
+ * T (Eq. joint-solve); then the recurrence over chunks carrying the state.
+ */
+tla_status tla_chunk_fwd(const tla_problem *p, void *workspace, size_t workspace_bytes,
+                         int save_for_bwd, void *stream);
+
+/* Workspace of tla_chunk_bwd in bytes (multiple of 256, 256-byte aligned). */
+size_t tla_bwd_workspace_bytes(const tla_problem *p);
+
+/*
+ * Backward of tla_chunk_fwd (Appendix A, Kernels: a reverse recurrence over
+ * chunks producing each chunk's state gradient, then every chunk's remaining
+ * gradients in parallel, reduced in a fixed order).
+ *   fwd_ws  workspace of a tla_chunk_fwd(p, ..., save_for_bwd=1) call on the
+ *           same problem and inputs (read only).
+ *   dO      [B,T,H,dv] dtype, gradient of o.
+ *   dht     [B,H,E,dk,dv] fp32 gradient of ht, or NULL (=> 0).
+ *   dq, dk  [B,T,H,dk] dtype;  dv [B,T,H,dv] dtype;  dq2, dk2 [B,T,H,E] dtype.
+ *   dbeta   [B,T,H] fp32; required iff p->beta != NULL, else must be NULL.
+ *   dg      [B,T,H,E] fp32 gradient of the log-gates.
+ *   dh0     [B,H,E,dk,dv] fp32; required iff p->h0 != NULL, else must be NULL.
+ */
+tla_status tla_chunk_bwd(const tla_problem *p, const void *fwd_ws, size_t fwd_ws_bytes,
+                         const void *dO, const float *dht,
+                         void *dq, void *dk, void *dv, void *dq2, void *dk2,
+                         float *dbeta, float *dg, float *dh0,
+                         void *workspace, size_t workspace_bytes, void *stream);
+
+/*
+ * One recurrent decode step for B sequences (Algorithm 2, one iteration; Eq.
+ * forget3 then Eq. gdn3 or the sGLA write, then the read of Eq. la3):
+ *   q, k [B,H,dk] dtype; v [B,H,dv] dtype; q2, k2 [B,H,E] dtype;
+ *   g [B,H,E] fp32; beta [B,H] fp32 or NULL (=> 1; required if use_delta);
+ *   state [B,H,E,dk,dv] fp32, updated in place; o [B,H,dv] dtype (written).
+ * Supported: dk, dv multiples of 16 up to 128, 1 <= E <= 16; state must be
+ * 16-byte aligned.  No workspace.
+ */
+tla_status tla_decode_step(int B, int H, int dk, int dv, int E, int use_delta, int dtype,
+                           const void *q, const void *k, const void *v,
+                           const void *q2, const void *k2, const float *g,
+                           const float *beta, float *state, void *o, void *stream);
+
+/* Human-readable name of a status code (static string). */
+const char *tla_status_string(int status);
+
+/*
+ * Synchronises `stream`, then returns TLA_ERR_TIMEOUT if a device-side bounded
+ * wait of any kernel launched since the previous call expired (and clears that
+ * record), TLA_ERR_CUDA if the stream reports an error, else TLA_OK.
+ */
+tla_status tla_last_device_status(void *stream);
+
+/*
+ * Kernel timing (tracing).  After tla_profile_begin(), every kernel the library
+ * launches is bracketed by CUDA events recorded on its launch stream (event
+ * objects are created on first use and reused; no device memory is allocated).
+ * tla_profile_end() synchronises `stream`, stops recording and reports, per
+ * kernel name in first-launch order, the number of launches and the summed
+ * device time in milliseconds.  It returns the number of distinct kernels
+ * written (at most max_kernels), or a negative status.  names_out receives
+ * max_kernels fixed-size slots of 64 bytes (NUL-terminated names).
+ */
+tla_status tla_profile_begin(void);
+int tla_profile_end(void *stream, char *names_out, int *launches_out, float *ms_out,
+                    int max_kernels);
+
+/* Library version string, e.g. "tla 0.1 sm_103a". */
+const char *tla_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* TLA_H */

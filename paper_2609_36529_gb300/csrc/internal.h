@@ -1,0 +1,67 @@
+// Host-side interfaces between the C ABI (tla_api.cu) and the kernel files.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+
+#include "../../include/tla.h"
+
+namespace tla {
+
+// Byte offsets of the private buffers inside the caller's workspaces.
+struct FwdPlan {
+    int NT;              // number of chunks, ceil(T / 64)
+    int tv;              // value columns per CTA of the SIMT recurrence
+    size_t G;            // fp32 [B,T,H,E] chunk-local inclusive log-decay
+    size_t A;            // fp32 [B,H,NT,64,64] Q K^T (.) R' (lower incl. diagonal)
+    size_t N;            // fp32 [B,H,NT,64,64] (I + L)^{-1} (delta rule only)
+    size_t S;            // fp32 [B,H,NT,E,dk,dv] chunk-start states (save_for_bwd)
+    size_t U;            // fp32 [B,T,H,dv] delta-corrected values (save_for_bwd)
+    size_t Res;          // fp32 [B,T,H,dv] residual V - W (save_for_bwd, delta rule)
+    size_t bytes;        // total
+};
+
+struct BwdPlan {
+    int tv;
+    size_t dU;           // fp32 [B,T,H,dv]
+    size_t dRes;         // fp32 [B,T,H,dv]
+    size_t dS;           // fp32 [B,H,NT,E,dk,dv] gradient of the state at each chunk's end
+    size_t bytes;
+};
+
+// Kernel timing hooks (active between tla_profile_begin / tla_profile_end).
+void prof_before(const char* name, cudaStream_t s);
+void prof_after(cudaStream_t s);
+
+// Bracket one launch: PROF_LAUNCH("name", stream, kernel<<<...>>>(...));
+#define PROF_LAUNCH(name, stream, ...)   \
+    do {                                 \
+        ::tla::prof_before(name, stream); \
+        __VA_ARGS__;                     \
+        ::tla::prof_after(stream);       \
+    } while (0)
+
+FwdPlan plan_fwd(const tla_problem& p, int save_for_bwd);
+BwdPlan plan_bwd(const tla_problem& p);
+
+// SIMT path (fp32 arithmetic on CUDA cores; any supported dtype).
+cudaError_t launch_gate_cumsum(const tla_problem& p, float* G, cudaStream_t s);
+cudaError_t launch_chunk_prep(const tla_problem& p, const float* G, float* A, float* N,
+                              cudaStream_t s);
+cudaError_t launch_fwd_recurrence(const tla_problem& p, const FwdPlan& fp, char* ws,
+                                  int save_for_bwd, cudaStream_t s);
+cudaError_t launch_bwd_recurrence(const tla_problem& p, const FwdPlan& fp, const char* fws,
+                                  const BwdPlan& bp, char* bws, const void* dO,
+                                  const float* dht, void* dv, float* dh0, cudaStream_t s);
+cudaError_t launch_bwd_chunk_grads(const tla_problem& p, const FwdPlan& fp, const char* fws,
+                                   const BwdPlan& bp, const char* bws, const void* dO,
+                                   void* dq, void* dk, void* dq2, void* dk2, float* dbeta,
+                                   float* dg, cudaStream_t s);
+
+// Decode step.
+cudaError_t launch_decode_step(int B, int H, int dk, int dv, int E, int use_delta, int dtype,
+                               const void* q, const void* k, const void* v, const void* q2,
+                               const void* k2, const float* g, const float* beta,
+                               float* state, void* o, cudaStream_t s);
+
+}  // namespace tla

@@ -1,0 +1,190 @@
+"""Thin ctypes binding of ``libtla.so`` (C ABI in include/tla.h).
+
+Argument marshalling only: every step of the path runs in the library's CUDA
+kernels.  Tensors must be contiguous CUDA tensors; outputs and workspaces are
+allocated with PyTorch (the library itself allocates nothing).  Calls are
+enqueued on the current PyTorch CUDA stream.  If the library is missing the
+first call raises: there is no fallback.
+"""
+import ctypes
+import os
+from typing import Optional
+
+import torch
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libtla.so")
+
+TLA_BF16, TLA_FP32 = 0, 1
+STATUS = {0: "TLA_OK", -1: "TLA_ERR_INVALID_ARG", -2: "TLA_ERR_UNSUPPORTED", -3: "TLA_ERR_CUDA",
+          -4: "TLA_ERR_TIMEOUT", -5: "TLA_ERR_WORKSPACE"}
+
+EXPORTED = ("tla_fwd_workspace_bytes", "tla_chunk_fwd", "tla_bwd_workspace_bytes",
+            "tla_chunk_bwd", "tla_decode_step", "tla_status_string", "tla_last_device_status",
+            "tla_version")
+
+
+class TlaError(RuntimeError):
+    def __init__(self, fn, status):
+        super().__init__(f"{fn} failed: {STATUS.get(status, status)}")
+        self.status = status
+
+
+class tla_problem(ctypes.Structure):
+    _fields_ = [("B", ctypes.c_int), ("T", ctypes.c_int), ("H", ctypes.c_int),
+                ("dk", ctypes.c_int), ("dv", ctypes.c_int), ("E", ctypes.c_int),
+                ("chunk", ctypes.c_int), ("dtype", ctypes.c_int), ("use_delta", ctypes.c_int),
+                ("q", ctypes.c_void_p), ("k", ctypes.c_void_p), ("v", ctypes.c_void_p),
+                ("q2", ctypes.c_void_p), ("k2", ctypes.c_void_p), ("g", ctypes.c_void_p),
+                ("beta", ctypes.c_void_p), ("h0", ctypes.c_void_p), ("o", ctypes.c_void_p),
+                ("ht", ctypes.c_void_p)]
+
+
+_lib = None
+
+
+def lib():
+    """Load libtla.so (raises if it has not been built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"CUDA library not built: {LIB_PATH} (run __graft_entry__.build())")
+        L = ctypes.CDLL(LIB_PATH)
+        P = ctypes.POINTER(tla_problem)
+        vp, i, sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t
+        L.tla_fwd_workspace_bytes.argtypes = [P, i]
+        L.tla_fwd_workspace_bytes.restype = sz
+        L.tla_bwd_workspace_bytes.argtypes = [P]
+        L.tla_bwd_workspace_bytes.restype = sz
+        L.tla_chunk_fwd.argtypes = [P, vp, sz, i, vp]
+        L.tla_chunk_fwd.restype = i
+        L.tla_chunk_bwd.argtypes = [P, vp, sz, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
+        L.tla_chunk_bwd.restype = i
+        L.tla_decode_step.argtypes = [i] * 7 + [vp] * 10
+        L.tla_decode_step.restype = i
+        L.tla_status_string.argtypes = [i]
+        L.tla_status_string.restype = ctypes.c_char_p
+        L.tla_last_device_status.argtypes = [vp]
+        L.tla_last_device_status.restype = i
+        L.tla_version.restype = ctypes.c_char_p
+        _lib = L
+    return _lib
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    if t is None:
+        return None
+    if not t.is_cuda or not t.is_contiguous():
+        raise ValueError("tla wants contiguous CUDA tensors")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.bfloat16:
+        return TLA_BF16
+    if t.dtype == torch.float32:
+        return TLA_FP32
+    raise ValueError(f"unsupported dtype {t.dtype}")
+
+
+def _stream():
+    return ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+
+
+def _check(fn, status):
+    if status != 0:
+        raise TlaError(fn, status)
+
+
+def make_problem(q, k, v, q2, k2, g, beta=None, h0=None, o=None, ht=None, use_delta=True,
+                 chunk=64):
+    B, T, H, dk = q.shape
+    p = tla_problem()
+    p.B, p.T, p.H, p.dk, p.dv, p.E = B, T, H, dk, v.shape[-1], q2.shape[-1]
+    p.chunk, p.dtype, p.use_delta = chunk, _dtype_code(q), int(bool(use_delta))
+    for name, t in (("q", q), ("k", k), ("v", v), ("q2", q2), ("k2", k2), ("g", g),
+                    ("beta", beta), ("h0", h0), ("o", o), ("ht", ht)):
+        setattr(p, name, _ptr(t))
+    return p
+
+
+def fwd_workspace_bytes(p: tla_problem, save_for_bwd: bool) -> int:
+    return lib().tla_fwd_workspace_bytes(ctypes.byref(p), int(save_for_bwd))
+
+
+def bwd_workspace_bytes(p: tla_problem) -> int:
+    return lib().tla_bwd_workspace_bytes(ctypes.byref(p))
+
+
+def _workspace(nbytes, device):
+    # 256-byte alignment: PyTorch's CUDA caching allocator returns 512-byte aligned blocks
+    return torch.empty(max(int(nbytes), 256), dtype=torch.uint8, device=device)
+
+
+def tla_chunk_fwd(q, k, v, q2, k2, g, beta=None, h0=None, use_delta=True, save_for_bwd=False,
+                  want_ht=True, o=None, ht=None, workspace=None):
+    """Chunkwise forward. Returns (o, ht or None, workspace)."""
+    B, T, H, _ = q.shape
+    E, dv = q2.shape[-1], v.shape[-1]
+    if o is None:
+        o = torch.empty(B, T, H, dv, dtype=q.dtype, device=q.device)
+    if ht is None and want_ht:
+        ht = torch.empty(B, H, E, q.shape[-1], dv, dtype=torch.float32, device=q.device)
+    p = make_problem(q, k, v, q2, k2, g, beta, h0, o, ht, use_delta)
+    need = fwd_workspace_bytes(p, save_for_bwd)
+    if need == 0:
+        raise TlaError("tla_fwd_workspace_bytes", -1)
+    if workspace is None or workspace.numel() < need:
+        workspace = _workspace(need, q.device)
+    _check("tla_chunk_fwd", lib().tla_chunk_fwd(ctypes.byref(p), _ptr(workspace), need,
+                                                int(save_for_bwd), _stream()))
+    return o, ht, workspace
+
+
+def tla_chunk_bwd(q, k, v, q2, k2, g, dO, fwd_workspace, beta=None, h0=None, dht=None,
+                  use_delta=True, workspace=None, grads=None):
+    """Backward of tla_chunk_fwd; fwd_workspace from a save_for_bwd=True forward.
+
+    Returns (dict of gradients dq, dk, dv, dq2, dk2, dg[, dbeta][, dh0], workspace)."""
+    p = make_problem(q, k, v, q2, k2, g, beta, h0, use_delta=use_delta)
+    # o is not read by the backward; a non-null placeholder satisfies validation
+    p.o = _ptr(dO)
+    if grads is None:
+        grads = {"dq": torch.empty_like(q), "dk": torch.empty_like(k), "dv": torch.empty_like(v),
+                 "dq2": torch.empty_like(q2), "dk2": torch.empty_like(k2),
+                 "dg": torch.empty_like(g)}
+        if beta is not None:
+            grads["dbeta"] = torch.empty_like(beta)
+        if h0 is not None:
+            grads["dh0"] = torch.empty_like(h0)
+    need = bwd_workspace_bytes(p)
+    if need == 0:
+        raise TlaError("tla_bwd_workspace_bytes", -1)
+    if workspace is None or workspace.numel() < need:
+        workspace = _workspace(need, q.device)
+    _check("tla_chunk_bwd", lib().tla_chunk_bwd(
+        ctypes.byref(p), _ptr(fwd_workspace), fwd_workspace.numel(), _ptr(dO), _ptr(dht),
+        _ptr(grads["dq"]), _ptr(grads["dk"]), _ptr(grads["dv"]), _ptr(grads["dq2"]),
+        _ptr(grads["dk2"]), _ptr(grads.get("dbeta")), _ptr(grads["dg"]), _ptr(grads.get("dh0")),
+        _ptr(workspace), need, _stream()))
+    return grads, workspace
+
+
+def tla_decode_step(state, q, k, v, q2, k2, g, beta=None, use_delta=True, o=None):
+    """One decode step; updates `state` [B,H,E,dk,dv] fp32 in place and returns o [B,H,dv]."""
+    B, H, dk = q.shape
+    dv, E = v.shape[-1], q2.shape[-1]
+    if o is None:
+        o = torch.empty(B, H, dv, dtype=q.dtype, device=q.device)
+    _check("tla_decode_step", lib().tla_decode_step(
+        B, H, dk, dv, E, int(bool(use_delta)), _dtype_code(q), _ptr(q), _ptr(k), _ptr(v),
+        _ptr(q2), _ptr(k2), _ptr(g), _ptr(beta), _ptr(state), _ptr(o), _stream()))
+    return o
+
+
+def tla_last_device_status() -> int:
+    return lib().tla_last_device_status(_stream())
+
+
+def tla_version() -> str:
+    return lib().tla_version().decode()

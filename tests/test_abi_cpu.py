@@ -1,0 +1,100 @@
+"""Host-side checks of the C-ABI library (no GPU needed, no compute calls)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def header_functions():
+    src = open(os.path.join(ROOT, "include", "tla.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(tla_[a-z0-9_]+)\s*\(", src)))
+
+
+@pytest.fixture(scope="module")
+def tla():
+    import __graft_entry__ as ge
+    ge.build_library()
+    from paper_2609_36529_gb300 import tla as t
+    return t
+
+
+def test_library_exports_every_declared_symbol(tla):
+    L = tla.lib()
+    names = header_functions()
+    assert {"tla_chunk_fwd", "tla_chunk_bwd", "tla_decode_step"} <= set(names)
+    for n in names:
+        assert hasattr(L, n), n
+    assert set(tla.EXPORTED) <= set(names)
+
+
+def test_status_strings(tla):
+    for code, name in tla.STATUS.items():
+        assert tla.lib().tla_status_string(code).decode() == name
+    assert tla.tla_version().startswith("tla")
+
+
+def _problem(tla, **kw):
+    p = tla.tla_problem()
+    p.B, p.T, p.H, p.dk, p.dv, p.E, p.chunk, p.dtype, p.use_delta = 2, 100, 3, 64, 32, 4, 64, 0, 1
+    fake = ctypes.c_void_p(0x1000)
+    for n in ("q", "k", "v", "q2", "k2", "g", "beta", "o"):
+        setattr(p, n, fake)
+    for n, v in kw.items():
+        setattr(p, n, v)
+    return p
+
+
+def test_host_validation_rejects_before_launch(tla):
+    L = tla.lib()
+    cases = [
+        (dict(chunk=32), -2), (dict(dk=20), -2), (dict(dv=256), -2), (dict(E=17), -2),
+        (dict(E=0), -1), (dict(T=0), -1), (dict(dtype=7), -1), (dict(use_delta=2), -1),
+        (dict(q=None), -1), (dict(beta=None), -1), (dict(o=None), -1),
+    ]
+    for kw, want in cases:
+        p = _problem(tla, **kw)
+        assert L.tla_chunk_fwd(ctypes.byref(p), None, 0, 0, None) == want, kw
+        assert L.tla_fwd_workspace_bytes(ctypes.byref(p), 0) == 0
+    # valid problem, missing or short workspace: rejected before any launch
+    p = _problem(tla)
+    need = L.tla_fwd_workspace_bytes(ctypes.byref(p), 1)
+    assert need > 0 and need % 256 == 0
+    assert L.tla_chunk_fwd(ctypes.byref(p), None, need, 1, None) == -5
+    assert L.tla_chunk_fwd(ctypes.byref(p), ctypes.c_void_p(0x100000), need - 1, 1, None) == -5
+    assert L.tla_chunk_fwd(ctypes.byref(p), ctypes.c_void_p(0x100010), need, 1, None) == -5
+    # sGLA may omit beta
+    p = _problem(tla, use_delta=0, beta=None)
+    assert L.tla_fwd_workspace_bytes(ctypes.byref(p), 0) > 0
+
+
+def test_host_validation_bwd_and_decode(tla):
+    L = tla.lib()
+    p = _problem(tla)
+    f = ctypes.c_void_p(0x1000)
+    # dbeta must be given iff beta is
+    assert L.tla_chunk_bwd(ctypes.byref(p), f, 1 << 40, f, None, f, f, f, f, f, None, f, None,
+                           f, 1 << 40, None) == -1
+    # h0 absent => dh0 must be NULL
+    assert L.tla_chunk_bwd(ctypes.byref(p), f, 1 << 40, f, None, f, f, f, f, f, f, f, f,
+                           f, 1 << 40, None) == -1
+    # short forward workspace
+    assert L.tla_chunk_bwd(ctypes.byref(p), None, 0, f, None, f, f, f, f, f, f, f, None,
+                           f, 1 << 40, None) == -5
+    # decode: misaligned state, unsupported dims, missing beta with the delta rule
+    assert L.tla_decode_step(2, 2, 64, 64, 4, 1, 0, f, f, f, f, f, f, f, ctypes.c_void_p(0x1004),
+                             f, None) == -1
+    assert L.tla_decode_step(2, 2, 64, 200, 4, 1, 0, f, f, f, f, f, f, f, f, f, None) == -2
+    assert L.tla_decode_step(2, 2, 64, 64, 4, 1, 0, f, f, f, f, f, f, None, f, f, None) == -1
+
+
+def test_workspace_sizes_grow_with_saving(tla):
+    L = tla.lib()
+    p = _problem(tla)
+    a = L.tla_fwd_workspace_bytes(ctypes.byref(p), 0)
+    b = L.tla_fwd_workspace_bytes(ctypes.byref(p), 1)
+    assert b > a > 0
+    assert L.tla_bwd_workspace_bytes(ctypes.byref(p)) > 0

@@ -1,0 +1,290 @@
+"""GPU parity: the CUDA path through the C ABI against the float64 oracle.
+
+Tolerances (per output tensor, oracle as reference):
+  fp32 inputs : max|err| <= 1e-4 * RMS(oracle)
+  bf16 inputs : max|err| <= 2e-2 * RMS(oracle); gradients also rel. L2 < 1%
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2609_36529_gb300 import inputs, tla
+
+pytestmark = pytest.mark.gpu
+
+TOL = {"fp32": 1e-4, "bf16": 2e-2}
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    import __graft_entry__ as ge
+    ge.build()
+    assert torch.cuda.is_available()
+
+
+def _np(t):
+    return None if t is None else t.detach().double().cpu().numpy()
+
+
+def close(name, got, ref, tol, rel_l2=None):
+    got = np.asarray(_np(got) if isinstance(got, torch.Tensor) else got, dtype=np.float64)
+    ref = np.asarray(ref, dtype=np.float64)
+    assert got.shape == ref.shape, (name, got.shape, ref.shape)
+    assert np.isfinite(got).all(), name
+    rms = float(np.sqrt(np.mean(ref ** 2)))
+    if rms == 0.0:
+        assert np.abs(got).max() <= 1e-6, name
+        return
+    err = float(np.abs(got - ref).max())
+    assert err <= tol * rms, f"{name}: max|err| {err:.3e} > {tol} x RMS {rms:.3e}"
+    if rel_l2 is not None:
+        rl = float(np.linalg.norm(got - ref) / np.linalg.norm(ref))
+        assert rl < rel_l2, f"{name}: rel L2 {rl:.3e}"
+
+
+def run_fwd(x, use_delta, save=False):
+    return tla.tla_chunk_fwd(x["q"], x["k"], x["v"], x["q2"], x["k2"], x["g"], x["beta"], x["h0"],
+                             use_delta=use_delta, save_for_bwd=save)
+
+
+def oracle_fwd(x, use_delta):
+    c = {n: _np(t) for n, t in x.items()}
+    return oracle.forward(c["q"], c["k"], c["v"], c["q2"], c["k2"], c["g"], c["beta"], c["h0"],
+                          use_delta=use_delta)
+
+
+# --- the fp32 sGLA workload exactly as specified (B1 H2 T256 d32 E4, seed 0)
+
+def test_sgla_fp32_workload_full():
+    w = inputs.SGLA_FWD_FP32
+    x = inputs.workload_inputs(w, device="cuda", seed=0)
+    o, ht, _ = run_fwd(x, w.use_delta)
+    torch.cuda.synchronize()
+    ro, rht = oracle_fwd(x, w.use_delta)
+    close("o", o, ro, TOL["fp32"])
+    close("ht", ht, rht, TOL["fp32"])
+
+
+# --- several chunks and ragged tails, both variants, both dtypes
+
+@pytest.mark.parametrize("dtype", ["fp32", "bf16"])
+@pytest.mark.parametrize("use_delta", [True, False])
+@pytest.mark.parametrize("T", [1, 63, 64, 65, 200])
+def test_fwd_small(dtype, use_delta, T):
+    x = inputs.chunk_inputs(2, T, 3, 64, 32, 3, dtype=dtype, with_beta=True, h0_std=0.2,
+                            device="cuda", seed=T)
+    o, ht, _ = run_fwd(x, use_delta)
+    torch.cuda.synchronize()
+    ro, rht = oracle_fwd(x, use_delta)
+    close("o", o, ro, TOL[dtype])
+    close("ht", ht, rht, TOL[dtype])
+
+
+@pytest.mark.parametrize("dk,dv,E", [(16, 16, 1), (32, 64, 2), (64, 48, 5), (128, 128, 4),
+                                     (48, 80, 16), (128, 128, 8), (128, 16, 16)])
+def test_fwd_shapes(dk, dv, E):
+    x = inputs.chunk_inputs(1, 150, 2, dk, dv, E, dtype="bf16", with_beta=True, h0_std=0.1,
+                            device="cuda", seed=dk + dv + E)
+    o, ht, _ = run_fwd(x, True)
+    torch.cuda.synchronize()
+    ro, rht = oracle_fwd(x, True)
+    close("o", o, ro, TOL["bf16"])
+    close("ht", ht, rht, TOL["bf16"])
+
+
+def test_fwd_sgla_no_beta_no_h0():
+    x = inputs.chunk_inputs(2, 129, 2, 32, 32, 4, dtype="fp32", with_beta=False, device="cuda",
+                            seed=5)
+    o, ht, _ = run_fwd(x, False)
+    torch.cuda.synchronize()
+    ro, rht = oracle_fwd(x, False)
+    close("o", o, ro, TOL["fp32"])
+    close("ht", ht, rht, TOL["fp32"])
+
+
+@pytest.mark.parametrize("total", [200.0, 600.0])
+def test_fwd_extreme_gates(total):
+    """Within-chunk decay of e^-200 and e^-600 in one slice (Appendix A, Numerical stability)."""
+    x = inputs.chunk_inputs(1, 128, 2, 32, 32, 3, dtype="fp32", with_beta=True, h0_std=0.3,
+                            device="cuda", seed=7)
+    x["g"][..., 0] = -total / 64.0
+    o, ht, _ = run_fwd(x, True)
+    torch.cuda.synchronize()
+    ro, rht = oracle_fwd(x, True)
+    close("o", o, ro, TOL["fp32"])
+    close("ht", ht, rht, TOL["fp32"])
+
+
+# --- backward
+
+def run_bwd(x, use_delta, dht):
+    o, ht, ws = run_fwd(x, use_delta, save=True)
+    grads, _ = tla.tla_chunk_bwd(x["q"], x["k"], x["v"], x["q2"], x["k2"], x["g"], x["dO"], ws,
+                                 beta=x["beta"], h0=x["h0"], dht=dht, use_delta=use_delta)
+    return o, ht, grads
+
+
+def oracle_bwd(x, use_delta, dht):
+    c = {n: _np(t) for n, t in x.items()}
+    return oracle.backward(c["q"], c["k"], c["v"], c["q2"], c["k2"], c["g"], c["dO"], c["beta"],
+                           c["h0"], _np(dht), use_delta=use_delta)
+
+
+@pytest.mark.parametrize("dtype", ["fp32", "bf16"])
+@pytest.mark.parametrize("use_delta", [True, False])
+@pytest.mark.parametrize("T", [1, 65, 200])
+def test_bwd_small(dtype, use_delta, T):
+    x = inputs.chunk_inputs(2, T, 2, 32, 48, 3, dtype=dtype, with_beta=True, h0_std=0.2,
+                            backward=True, device="cuda", seed=100 + T)
+    dht = torch.randn(2, 2, 3, 32, 48, device="cuda",
+                      generator=torch.Generator("cuda").manual_seed(T))
+    _, _, grads = run_bwd(x, use_delta, dht)
+    torch.cuda.synchronize()
+    ref = oracle_bwd(x, use_delta, dht)
+    assert set(ref) == set(grads)
+    for n in ref:
+        close(n, grads[n], ref[n], TOL[dtype], rel_l2=0.01 if dtype == "bf16" else None)
+
+
+def test_bwd_sgla_no_beta_no_h0():
+    x = inputs.chunk_inputs(1, 150, 2, 32, 32, 4, dtype="fp32", with_beta=False, backward=True,
+                            device="cuda", seed=11)
+    _, _, grads = run_bwd(x, False, None)
+    torch.cuda.synchronize()
+    ref = oracle_bwd(x, False, None)
+    assert set(ref) == set(grads)
+    for n in ref:
+        close(n, grads[n], ref[n], TOL["fp32"])
+
+
+@pytest.mark.parametrize("dk,dv,E", [(128, 128, 4), (64, 32, 8), (16, 128, 1)])
+def test_bwd_shapes(dk, dv, E):
+    x = inputs.chunk_inputs(1, 130, 2, dk, dv, E, dtype="bf16", with_beta=True, h0_std=0.1,
+                            backward=True, device="cuda", seed=dk * E)
+    _, _, grads = run_bwd(x, True, None)
+    torch.cuda.synchronize()
+    ref = oracle_bwd(x, True, None)
+    for n in ref:
+        close(n, grads[n], ref[n], TOL["bf16"], rel_l2=0.01)
+
+
+def test_bwd_deterministic():
+    x = inputs.chunk_inputs(2, 190, 2, 64, 64, 4, dtype="bf16", with_beta=True, h0_std=0.1,
+                            backward=True, device="cuda", seed=3)
+    _, _, g1 = run_bwd(x, True, None)
+    _, _, g2 = run_bwd(x, True, None)
+    torch.cuda.synchronize()
+    for n in g1:
+        assert torch.equal(g1[n], g2[n]), n
+
+
+# --- decode
+
+@pytest.mark.parametrize("dtype", ["fp32", "bf16"])
+@pytest.mark.parametrize("use_delta", [True, False])
+@pytest.mark.parametrize("dk,dv,E", [(128, 128, 8), (64, 48, 16), (16, 32, 1), (128, 128, 16)])
+def test_decode_steps(dtype, use_delta, dk, dv, E):
+    B, H = 3, 2
+    gen = torch.Generator("cuda").manual_seed(dk + E)
+    state = 0.1 * torch.randn(B, H, E, dk, dv, device="cuda", generator=gen)
+    ref_state = _np(state)
+    for step in range(4):
+        d = inputs.decode_inputs(B, H, dk, dv, E, dtype=dtype, device="cuda", gen=gen)
+        beta = d["beta"] if (use_delta or step % 2) else None
+        o = tla.tla_decode_step(state, d["q"], d["k"], d["v"], d["q2"], d["k2"], d["g"], beta,
+                                use_delta=use_delta)
+        torch.cuda.synchronize()
+        c = {n: _np(t) for n, t in d.items()}
+        ro, ref_state = oracle.decode_step(ref_state, c["q"], c["k"], c["v"], c["q2"], c["k2"],
+                                           c["g"], _np(beta), use_delta=use_delta)
+        close(f"o step {step}", o, ro, TOL[dtype])
+        close(f"state step {step}", state, ref_state, 1e-4)
+
+
+def test_decode_after_chunk_prefill_matches_token_recurrence():
+    """Prefill by the chunk forward, then decode: equals the oracle's recurrence over all tokens."""
+    x = inputs.chunk_inputs(2, 70, 2, 64, 64, 4, dtype="fp32", with_beta=True, device="cuda",
+                            seed=21)
+    _, ht, _ = run_fwd({n: (t[:, :64].contiguous() if t is not None and t.dim() >= 3 and t.shape[1] == 70
+                            else t) for n, t in x.items()}, True)
+    outs = []
+    for t in range(64, 70):
+        outs.append(tla.tla_decode_step(ht, *(x[n][:, t].contiguous() for n in
+                                              ("q", "k", "v", "q2", "k2", "g")),
+                                        x["beta"][:, t].contiguous()))
+    torch.cuda.synchronize()
+    ro, rht = oracle_fwd(x, True)
+    close("decode o", torch.stack(outs, 1), ro[:, 64:], TOL["fp32"])
+    close("final state", ht, rht, TOL["fp32"])
+
+
+# --- full-size workloads in the launch configuration the benchmark times, sampled heads
+
+def _sample_heads(x, bh_list, T=None):
+    """Slice inputs down to the listed (b, h) pairs (as a batch of single-head problems)."""
+    out = {}
+    for n, t in x.items():
+        if t is None:
+            out[n] = None
+        elif n == "h0":
+            out[n] = torch.stack([t[b, h] for b, h in bh_list])[:, None]
+        elif n == "beta":
+            out[n] = torch.stack([t[b, :T, h] for b, h in bh_list])[:, :, None]
+        else:
+            out[n] = torch.stack([t[b, :T, h] for b, h in bh_list])[:, :, None]
+    return out
+
+
+@pytest.mark.parametrize("name", ["gdn_fwd_bf16_B4_H16_T4096_d128_E8",
+                                  "gdn_fwd_bf16_B1_H32_T65536_d128_E16"])
+def test_full_size_forward_sampled(name):
+    w = inputs.WORKLOADS[name]
+    x = inputs.workload_inputs(w, device="cuda", seed=0)
+    o, ht, _ = run_fwd(x, w.use_delta)
+    torch.cuda.synchronize()
+    picks = [(0, 0), (w.B - 1, w.H - 1)]
+    # The forward is causal, so the first Ts outputs of the full launch must equal the
+    # oracle's outputs of the Ts-token prefix (the oracle finishes 8192 tokens in seconds).
+    Ts = min(w.T, 8192)
+    xs = _sample_heads(x, picks, Ts)
+    ro, rht = oracle_fwd(xs, w.use_delta)
+    for i, (b, h) in enumerate(picks):
+        close(f"o[:{Ts}] b{b}h{h}", o[b, :Ts, h], ro[i, :, 0], TOL[w.dtype])
+        if Ts == w.T:
+            close(f"ht b{b}h{h}", ht[b, h], rht[i, 0], TOL[w.dtype])
+
+
+def test_full_size_fwd_bwd_sampled():
+    w = inputs.GDN_FWDBWD_BF16
+    x = inputs.workload_inputs(w, device="cuda", seed=0)
+    o, ht, grads = run_bwd(x, w.use_delta, None)
+    torch.cuda.synchronize()
+    picks = [(0, 0), (w.B - 1, w.H - 1)]
+    xs = _sample_heads(x, picks)
+    ro, _ = oracle_fwd(xs, True)
+    ref = oracle_bwd(xs, True, None)
+    for i, (b, h) in enumerate(picks):
+        close(f"o b{b}h{h}", o[b, :, h], ro[i, :, 0], TOL["bf16"])
+        for n in ("dq", "dk", "dv", "dq2", "dk2", "dg"):
+            close(f"{n} b{b}h{h}", grads[n][b, :, h], ref[n][i, :, 0], TOL["bf16"], rel_l2=0.01)
+        close(f"dbeta b{b}h{h}", grads["dbeta"][b, :, h], ref["dbeta"][i, :, 0], TOL["bf16"],
+              rel_l2=0.01)
+
+
+def test_full_size_decode_sampled():
+    w = inputs.DECODE
+    gen = torch.Generator("cuda").manual_seed(0)
+    state = 0.05 * torch.randn(w.B, w.H, w.E, w.dk, w.dv, device="cuda", generator=gen)
+    picks = [(0, 0), (w.B - 1, w.H - 1), (w.B // 2, 5)]
+    ref = np.stack([_np(state[b, h]) for b, h in picks])[:, None]
+    for step in range(3):
+        d = inputs.decode_inputs(w.B, w.H, w.dk, w.dv, w.E, device="cuda", gen=gen)
+        o = tla.tla_decode_step(state, d["q"], d["k"], d["v"], d["q2"], d["k2"], d["g"], d["beta"])
+        torch.cuda.synchronize()
+        c = {n: np.stack([_np(t[b, h]) for b, h in picks])[:, None] for n, t in d.items()}
+        ro, ref = oracle.decode_step(ref, c["q"], c["k"], c["v"], c["q2"], c["k2"], c["g"],
+                                     c["beta"])
+        for i, (b, h) in enumerate(picks):
+            close(f"o step{step} b{b}h{h}", o[b, h], ro[i, 0], TOL["fp32"])
+            close(f"state step{step} b{b}h{h}", state[b, h], ref[i, 0], 1e-4)
