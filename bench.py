@@ -230,14 +230,15 @@ def run_ours(args):
     stream = torch.cuda.current_stream(dev)
 
     # preallocated outputs and workspaces (allocation is outside the timed region)
-    o = torch.empty(w.B, w.T, w.H, w.dv, dtype=torch.bfloat16, device=dev)
+    o = torch.empty(w.B, w.T, w.H, w.dv, dtype=torch.float32, device=dev)   # fp32 results
     p = tla.make_problem(x["q"], x["k"], x["v"], x["q2"], x["k2"], x["g"], x["beta"], None, o,
                          None, use_delta=True)
     fws = torch.empty(tla.fwd_workspace_bytes(p, True), dtype=torch.uint8, device=dev)
     bws = torch.empty(tla.bwd_workspace_bytes(p), dtype=torch.uint8, device=dev)
-    grads = {"dq": torch.empty_like(x["q"]), "dk": torch.empty_like(x["k"]),
-             "dv": torch.empty_like(x["v"]), "dq2": torch.empty_like(x["q2"]),
-             "dk2": torch.empty_like(x["k2"]), "dg": torch.empty_like(x["g"]),
+    f32 = dict(dtype=torch.float32, device=dev)
+    grads = {"dq": torch.empty(x["q"].shape, **f32), "dk": torch.empty(x["k"].shape, **f32),
+             "dv": torch.empty(x["v"].shape, **f32), "dq2": torch.empty(x["q2"].shape, **f32),
+             "dk2": torch.empty(x["k2"].shape, **f32), "dg": torch.empty_like(x["g"]),
              "dbeta": torch.empty_like(x["beta"])}
 
     def step(xx):
@@ -332,7 +333,7 @@ def run_ours(args):
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": {"workload": w.name, "B": w.B, "T": w.T, "H": w.H, "dk": w.dk, "dv": w.dv,
                        "E": w.E, "chunk": CHUNK, "variant": "triadic GDN (joint-key delta rule)",
-                       "state": "fp32", "parallelism": f"replicas x{ws_n} (independent sequences)",
+                       "state": "fp32", "outputs": "fp32 o and gradients", "parallelism": f"replicas x{ws_n} (independent sequences)",
                        "l2": "inputs larger than L2 (q,k,v,dO 268 MB each per GPU)"},
             "tflops": round(total_flops / (ms_step / 1e3) / 1e12, 3),
             "tflops_frac": round(total_flops / (ms_step / 1e3) / 1e12 / peak, 5),

@@ -20,8 +20,9 @@
  *    The library allocates no device memory.
  *  - All tensors are dense, row-major, contiguous.  Token tensors use the
  *    layout [B, T, H, D]; states use [B, H, E, dk, dv].
- *  - `dtype` (tla_dtype) is the element type of q, k, v, q2, k2, o and of their
- *    gradients.  Log-gates g, beta, states h0/ht/dh0, dg and dbeta are fp32.
+ *  - `dtype` (tla_dtype) is the element type of q, k, v, q2, k2; `out_dtype`
+ *    that of o and of their gradients.  Log-gates g, beta, states h0/ht/dh0,
+ *    dg and dbeta are fp32.  Arithmetic accumulates in fp32 throughout.
  *  - q, k, q2, k2 are expected to be L2-normalised by the caller (Algorithm 2
  *    normalises them before the operator); no 1/sqrt(d) scale is applied.
  *    g holds log alpha <= 0 (log of the per-slice forget gate).
@@ -63,7 +64,10 @@ typedef struct {
     int B, T, H;
     int dk, dv, E;
     int chunk;           /* must be 64                                         */
-    int dtype;           /* tla_dtype of q, k, v, q2, k2, o                    */
+    int dtype;           /* tla_dtype of q, k, v, q2, k2                       */
+    int out_dtype;       /* tla_dtype of o (forward) and of dq, dk, dv, dq2,
+                            dk2 (backward).  TLA_FP32 keeps the fp32
+                            accumulation of bf16 inputs; TLA_BF16 rounds.      */
     int use_delta;       /* 1: triadic Gated DeltaNet (Eq. gdn3); 0: sGLA      */
     const void *q;       /* [B,T,H,dk]                                          */
     const void *k;       /* [B,T,H,dk]                                          */
@@ -74,7 +78,7 @@ typedef struct {
     const float *beta;   /* [B,T,H] write strength in (0,1); NULL => 1.
                             Required when use_delta == 1.                       */
     const float *h0;     /* [B,H,E,dk,dv] initial state; NULL => zero state     */
-    void *o;             /* [B,T,H,dv] output (written)                         */
+    void *o;             /* [B,T,H,dv] out_dtype output (written)               */
     float *ht;           /* [B,H,E,dk,dv] final state (written); may be NULL    */
 } tla_problem;
 
@@ -105,9 +109,9 @@ size_t tla_bwd_workspace_bytes(const tla_problem *p);
  * gradients in parallel, reduced in a fixed order).
  *   fwd_ws  workspace of a tla_chunk_fwd(p, ..., save_for_bwd=1) call on the
  *           same problem and inputs (read only).
- *   dO      [B,T,H,dv] dtype, gradient of o.
+ *   dO      [B,T,H,dv] dtype (the input dtype), gradient of o.
  *   dht     [B,H,E,dk,dv] fp32 gradient of ht, or NULL (=> 0).
- *   dq, dk  [B,T,H,dk] dtype;  dv [B,T,H,dv] dtype;  dq2, dk2 [B,T,H,E] dtype.
+ *   dq, dk  [B,T,H,dk];  dv [B,T,H,dv];  dq2, dk2 [B,T,H,E]: all out_dtype.
  *   dbeta   [B,T,H] fp32; required iff p->beta != NULL, else must be NULL.
  *   dg      [B,T,H,E] fp32 gradient of the log-gates.
  *   dh0     [B,H,E,dk,dv] fp32; required iff p->h0 != NULL, else must be NULL.

@@ -20,6 +20,12 @@ template <> __device__ __forceinline__ __nv_bfloat16 from_f<__nv_bfloat16>(float
     return __float2bfloat16_rn(x);
 }
 
+// Store one result element in the requested output type (fp32 or bf16).
+__device__ __forceinline__ void store_out(void* base, size_t i, float v, int out_f32) {
+    if (out_f32) static_cast<float*>(base)[i] = v;
+    else static_cast<__nv_bfloat16*>(base)[i] = __float2bfloat16_rn(v);
+}
+
 // Index of element i of token (b,t,h) in a [B,T,H,D] tensor.
 __device__ __forceinline__ size_t tok_idx(int b, int t, int h, int i, int T, int H, int D) {
     return ((size_t(b) * T + t) * H + h) * D + i;

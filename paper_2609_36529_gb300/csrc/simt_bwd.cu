@@ -28,10 +28,10 @@ bwd_recurrence_kernel(const Tin* __restrict__ q, const Tin* __restrict__ k,
                       const float* __restrict__ G, const float* __restrict__ beta,
                       const float* __restrict__ Amat, const float* __restrict__ Nmat,
                       const Tin* __restrict__ dO, const float* __restrict__ dht,
-                      Tin* __restrict__ dv_out, float* __restrict__ dh0,
+                      void* __restrict__ dv_out, float* __restrict__ dh0,
                       float* __restrict__ dUbuf, float* __restrict__ dRbuf,
                       float* __restrict__ dSck, int T, int H, int dk, int dv, int E, int tv,
-                      int use_delta) {
+                      int use_delta, int out_f32) {
     const int nb = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
     const int n0 = nb * tv;
     const int tid = threadIdx.x;
@@ -135,7 +135,7 @@ bwd_recurrence_kernel(const Tin* __restrict__ q, const Tin* __restrict__ k,
                 size_t off = tok_idx(b, t0 + r, h, n0 + nn, T, H, dv);
                 dUbuf[off] = dUs[r * TVP + nn];
                 dRbuf[off] = acc;
-                dv_out[off] = from_f<Tin>(acc);
+                store_out(dv_out, off, acc, out_f32);
             }
         }
         __syncthreads();
@@ -184,15 +184,15 @@ cudaError_t launch_bwd_recurrence(const tla_problem& p, const FwdPlan& fp, const
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         kern<<<grid, 256, smem, s>>>((const Tb*)p.q, (const Tb*)p.k, (const Tb*)p.q2,
                                      (const Tb*)p.k2, G, p.beta, A, N, (const Tb*)dO, dht,
-                                     (Tb*)dv, dh0, dU, dR, dS, p.T, p.H, p.dk, p.dv, p.E, tv,
-                                     p.use_delta);
+                                     dv, dh0, dU, dR, dS, p.T, p.H, p.dk, p.dv, p.E, tv,
+                                     p.use_delta, p.out_dtype == TLA_FP32);
     } else {
         auto kern = bwd_recurrence_kernel<float>;
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         kern<<<grid, 256, smem, s>>>((const float*)p.q, (const float*)p.k, (const float*)p.q2,
                                      (const float*)p.k2, G, p.beta, A, N, (const float*)dO, dht,
-                                     (float*)dv, dh0, dU, dR, dS, p.T, p.H, p.dk, p.dv, p.E, tv,
-                                     p.use_delta);
+                                     dv, dh0, dU, dR, dS, p.T, p.H, p.dk, p.dv, p.E, tv,
+                                     p.use_delta, p.out_dtype == TLA_FP32);
     }
     prof_after(s);
     return cudaGetLastError();
@@ -222,10 +222,10 @@ bwd_chunk_grads_kernel(const Tin* __restrict__ q, const Tin* __restrict__ k,
                        const float* __restrict__ Sck, const float* __restrict__ Ubuf,
                        const float* __restrict__ Rbuf, const Tin* __restrict__ dO,
                        const float* __restrict__ dUbuf, const float* __restrict__ dRbuf,
-                       const float* __restrict__ dSck, Tin* __restrict__ dq,
-                       Tin* __restrict__ dk_out, Tin* __restrict__ dq2, Tin* __restrict__ dk2,
+                       const float* __restrict__ dSck, void* __restrict__ dq,
+                       void* __restrict__ dk_out, void* __restrict__ dq2, void* __restrict__ dk2,
                        float* __restrict__ dbeta, float* __restrict__ dg, int T, int H, int dk,
-                       int dv, int E, int use_delta) {
+                       int dv, int E, int use_delta, int out_f32) {
     const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
     const int NT = gridDim.x;
     const int tid = threadIdx.x;
@@ -535,8 +535,8 @@ bwd_chunk_grads_kernel(const Tin* __restrict__ q, const Tin* __restrict__ k,
             for (int x = r + 1; x < kChunk; ++x) ak = fmaf(B4[x * MP + r], t2[x * 33 + dd], ak);
             if (r < n && d0 + dd < dk) {
                 size_t off = tok_idx(b, t0 + r, h, d0 + dd, T, H, dk);
-                dq[off] = from_f<Tin>(aq);
-                dk_out[off] = from_f<Tin>(ak);
+                store_out(dq, off, aq, out_f32);
+                store_out(dk_out, off, ak, out_f32);
             }
         }
     }
@@ -570,8 +570,8 @@ bwd_chunk_grads_kernel(const Tin* __restrict__ q, const Tin* __restrict__ k,
     for (int i = tid; i < n * E; i += blockDim.x) {
         int r = i / E, e = i % E;
         size_t off = tok_idx(b, t0 + r, h, e, T, H, E);
-        dq2[off] = from_f<Tin>(dq2a[i]);
-        dk2[off] = from_f<Tin>(dk2a[i]);
+        store_out(dq2, off, dq2a[i], out_f32);
+        store_out(dk2, off, dk2a[i], out_f32);
     }
     if (dbeta && tid < n) dbeta[(size_t(b) * T + t0 + tid) * H + h] = dba[tid];
 }
@@ -603,16 +603,16 @@ cudaError_t launch_bwd_chunk_grads(const tla_problem& p, const FwdPlan& fp, cons
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         kern<<<grid, 256, smem, s>>>((const Tb*)p.q, (const Tb*)p.k, (const Tb*)p.v,
                                      (const Tb*)p.q2, (const Tb*)p.k2, G, p.beta, N, S, U, R,
-                                     (const Tb*)dO, dU, dR, dS, (Tb*)dq, (Tb*)dk, (Tb*)dq2,
-                                     (Tb*)dk2, dbeta, dg, p.T, p.H, p.dk, p.dv, p.E, p.use_delta);
+                                     (const Tb*)dO, dU, dR, dS, dq, dk, dq2, dk2, dbeta, dg, p.T,
+                                     p.H, p.dk, p.dv, p.E, p.use_delta, p.out_dtype == TLA_FP32);
     } else {
         auto kern = bwd_chunk_grads_kernel<float>;
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         kern<<<grid, 256, smem, s>>>((const float*)p.q, (const float*)p.k, (const float*)p.v,
                                      (const float*)p.q2, (const float*)p.k2, G, p.beta, N, S, U,
-                                     R, (const float*)dO, dU, dR, dS, (float*)dq, (float*)dk,
-                                     (float*)dq2, (float*)dk2, dbeta, dg, p.T, p.H, p.dk, p.dv,
-                                     p.E, p.use_delta);
+                                     R, (const float*)dO, dU, dR, dS, dq, dk, dq2, dk2, dbeta, dg,
+                                     p.T, p.H, p.dk, p.dv, p.E, p.use_delta,
+                                     p.out_dtype == TLA_FP32);
     }
     prof_after(s);
     return cudaGetLastError();

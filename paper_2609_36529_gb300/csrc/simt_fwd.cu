@@ -182,9 +182,9 @@ fwd_recurrence_kernel(const Tin* __restrict__ q, const Tin* __restrict__ k,
                       const Tin* __restrict__ k2, const float* __restrict__ G,
                       const float* __restrict__ beta, const float* __restrict__ h0,
                       const float* __restrict__ Amat, const float* __restrict__ Nmat,
-                      Tin* __restrict__ o, float* __restrict__ ht, float* __restrict__ Sck,
+                      void* __restrict__ o, float* __restrict__ ht, float* __restrict__ Sck,
                       float* __restrict__ Ubuf, float* __restrict__ Rbuf, int T, int H, int dk,
-                      int dv, int E, int tv, int use_delta, int save) {
+                      int dv, int E, int tv, int use_delta, int save, int out_f32) {
     const int nb = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
     const int n0 = nb * tv;
     const int tid = threadIdx.x;
@@ -303,7 +303,7 @@ fwd_recurrence_kernel(const Tin* __restrict__ q, const Tin* __restrict__ k,
             if (r >= n) continue;
             float acc = Os[r * TVP + nn];
             for (int s2 = 0; s2 <= r; ++s2) acc = fmaf(As[r * 65 + s2], Us[s2 * TVP + nn], acc);
-            o[tok_idx(b, t0 + r, h, n0 + nn, T, H, dv)] = from_f<Tin>(acc);
+            store_out(o, tok_idx(b, t0 + r, h, n0 + nn, T, H, dv), acc, out_f32);
         }
         // S_e = gamma^C_e S_e + K^T diag(w_e) U
         for (int i = tid; i < E * SE; i += blockDim.x) {
@@ -346,15 +346,15 @@ cudaError_t launch_fwd_recurrence(const tla_problem& p, const FwdPlan& fp, char*
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         kern<<<grid, 256, smem, s>>>((const Tb*)p.q, (const Tb*)p.k, (const Tb*)p.v,
                                      (const Tb*)p.q2, (const Tb*)p.k2, G, p.beta, p.h0, A, N,
-                                     (Tb*)p.o, p.ht, Sck, U, R, p.T, p.H, p.dk, p.dv, p.E, tv,
-                                     p.use_delta, save_for_bwd);
+                                     p.o, p.ht, Sck, U, R, p.T, p.H, p.dk, p.dv, p.E, tv,
+                                     p.use_delta, save_for_bwd, p.out_dtype == TLA_FP32);
     } else {
         auto kern = fwd_recurrence_kernel<float>;
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         kern<<<grid, 256, smem, s>>>((const float*)p.q, (const float*)p.k, (const float*)p.v,
                                      (const float*)p.q2, (const float*)p.k2, G, p.beta, p.h0, A,
-                                     N, (float*)p.o, p.ht, Sck, U, R, p.T, p.H, p.dk, p.dv, p.E,
-                                     tv, p.use_delta, save_for_bwd);
+                                     N, p.o, p.ht, Sck, U, R, p.T, p.H, p.dk, p.dv, p.E,
+                                     tv, p.use_delta, save_for_bwd, p.out_dtype == TLA_FP32);
     }
     prof_after(s);
     return cudaGetLastError();

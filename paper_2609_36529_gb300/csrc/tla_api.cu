@@ -21,6 +21,7 @@ static tla_status validate(const tla_problem* p) {
     if (!p) return TLA_ERR_INVALID_ARG;
     if (p->B < 1 || p->T < 1 || p->H < 1 || p->E < 1) return TLA_ERR_INVALID_ARG;
     if (p->dtype != TLA_BF16 && p->dtype != TLA_FP32) return TLA_ERR_INVALID_ARG;
+    if (p->out_dtype != TLA_BF16 && p->out_dtype != TLA_FP32) return TLA_ERR_INVALID_ARG;
     if (p->use_delta != 0 && p->use_delta != 1) return TLA_ERR_INVALID_ARG;
     if (!p->q || !p->k || !p->v || !p->q2 || !p->k2 || !p->g || !p->o) return TLA_ERR_INVALID_ARG;
     if (p->use_delta && !p->beta) return TLA_ERR_INVALID_ARG;

@@ -33,7 +33,8 @@ class TlaError(RuntimeError):
 class tla_problem(ctypes.Structure):
     _fields_ = [("B", ctypes.c_int), ("T", ctypes.c_int), ("H", ctypes.c_int),
                 ("dk", ctypes.c_int), ("dv", ctypes.c_int), ("E", ctypes.c_int),
-                ("chunk", ctypes.c_int), ("dtype", ctypes.c_int), ("use_delta", ctypes.c_int),
+                ("chunk", ctypes.c_int), ("dtype", ctypes.c_int), ("out_dtype", ctypes.c_int),
+                ("use_delta", ctypes.c_int),
                 ("q", ctypes.c_void_p), ("k", ctypes.c_void_p), ("v", ctypes.c_void_p),
                 ("q2", ctypes.c_void_p), ("k2", ctypes.c_void_p), ("g", ctypes.c_void_p),
                 ("beta", ctypes.c_void_p), ("h0", ctypes.c_void_p), ("o", ctypes.c_void_p),
@@ -97,11 +98,14 @@ def _check(fn, status):
 
 
 def make_problem(q, k, v, q2, k2, g, beta=None, h0=None, o=None, ht=None, use_delta=True,
-                 chunk=64):
+                 chunk=64, out_dtype=None):
     B, T, H, dk = q.shape
     p = tla_problem()
     p.B, p.T, p.H, p.dk, p.dv, p.E = B, T, H, dk, v.shape[-1], q2.shape[-1]
     p.chunk, p.dtype, p.use_delta = chunk, _dtype_code(q), int(bool(use_delta))
+    if out_dtype is None:
+        out_dtype = o.dtype if o is not None else torch.float32
+    p.out_dtype = _dtype_code(torch.empty(0, dtype=out_dtype))
     for name, t in (("q", q), ("k", k), ("v", v), ("q2", q2), ("k2", k2), ("g", g),
                     ("beta", beta), ("h0", h0), ("o", o), ("ht", ht)):
         setattr(p, name, _ptr(t))
@@ -122,12 +126,14 @@ def _workspace(nbytes, device):
 
 
 def tla_chunk_fwd(q, k, v, q2, k2, g, beta=None, h0=None, use_delta=True, save_for_bwd=False,
-                  want_ht=True, o=None, ht=None, workspace=None):
-    """Chunkwise forward. Returns (o, ht or None, workspace)."""
+                  want_ht=True, o=None, ht=None, workspace=None, out_dtype=torch.float32):
+    """Chunkwise forward. Returns (o, ht or None, workspace).
+
+    o is allocated in `out_dtype` (default fp32, the accumulation precision)."""
     B, T, H, _ = q.shape
     E, dv = q2.shape[-1], v.shape[-1]
     if o is None:
-        o = torch.empty(B, T, H, dv, dtype=q.dtype, device=q.device)
+        o = torch.empty(B, T, H, dv, dtype=out_dtype, device=q.device)
     if ht is None and want_ht:
         ht = torch.empty(B, H, E, q.shape[-1], dv, dtype=torch.float32, device=q.device)
     p = make_problem(q, k, v, q2, k2, g, beta, h0, o, ht, use_delta)
@@ -142,21 +148,27 @@ def tla_chunk_fwd(q, k, v, q2, k2, g, beta=None, h0=None, use_delta=True, save_f
 
 
 def tla_chunk_bwd(q, k, v, q2, k2, g, dO, fwd_workspace, beta=None, h0=None, dht=None,
-                  use_delta=True, workspace=None, grads=None):
+                  use_delta=True, workspace=None, grads=None, out_dtype=torch.float32):
     """Backward of tla_chunk_fwd; fwd_workspace from a save_for_bwd=True forward.
 
-    Returns (dict of gradients dq, dk, dv, dq2, dk2, dg[, dbeta][, dh0], workspace)."""
-    p = make_problem(q, k, v, q2, k2, g, beta, h0, use_delta=use_delta)
-    # o is not read by the backward; a non-null placeholder satisfies validation
-    p.o = _ptr(dO)
+    Returns (dict of gradients dq, dk, dv, dq2, dk2, dg[, dbeta][, dh0], workspace).
+    dq, dk, dv, dq2, dk2 are in `out_dtype` (default fp32); dg, dbeta, dh0 fp32."""
     if grads is None:
-        grads = {"dq": torch.empty_like(q), "dk": torch.empty_like(k), "dv": torch.empty_like(v),
-                 "dq2": torch.empty_like(q2), "dk2": torch.empty_like(k2),
+        od = out_dtype
+        grads = {"dq": torch.empty(q.shape, dtype=od, device=q.device),
+                 "dk": torch.empty(k.shape, dtype=od, device=q.device),
+                 "dv": torch.empty(v.shape, dtype=od, device=q.device),
+                 "dq2": torch.empty(q2.shape, dtype=od, device=q.device),
+                 "dk2": torch.empty(k2.shape, dtype=od, device=q.device),
                  "dg": torch.empty_like(g)}
         if beta is not None:
             grads["dbeta"] = torch.empty_like(beta)
         if h0 is not None:
             grads["dh0"] = torch.empty_like(h0)
+    p = make_problem(q, k, v, q2, k2, g, beta, h0, use_delta=use_delta,
+                     out_dtype=grads["dq"].dtype)
+    # o is not read by the backward; a non-null placeholder satisfies validation
+    p.o = _ptr(dO)
     need = bwd_workspace_bytes(p)
     if need == 0:
         raise TlaError("tla_bwd_workspace_bytes", -1)

@@ -40,6 +40,7 @@ def test_status_strings(tla):
 def _problem(tla, **kw):
     p = tla.tla_problem()
     p.B, p.T, p.H, p.dk, p.dv, p.E, p.chunk, p.dtype, p.use_delta = 2, 100, 3, 64, 32, 4, 64, 0, 1
+    p.out_dtype = 1
     fake = ctypes.c_void_p(0x1000)
     for n in ("q", "k", "v", "q2", "k2", "g", "beta", "o"):
         setattr(p, n, fake)
@@ -53,6 +54,7 @@ def test_host_validation_rejects_before_launch(tla):
     cases = [
         (dict(chunk=32), -2), (dict(dk=20), -2), (dict(dv=256), -2), (dict(E=17), -2),
         (dict(E=0), -1), (dict(T=0), -1), (dict(dtype=7), -1), (dict(use_delta=2), -1),
+        (dict(out_dtype=3), -1),
         (dict(q=None), -1), (dict(beta=None), -1), (dict(o=None), -1),
     ]
     for kw, want in cases:

@@ -43,6 +43,15 @@ def close(name, got, ref, tol, rel_l2=None):
         assert rl < rel_l2, f"{name}: rel L2 {rl:.3e}"
 
 
+def close_rounded(name, got, ref, tol):
+    """Results stored in bf16: allow the tolerance plus the output rounding (2^-8 |ref|)."""
+    got = _np(got)
+    ref = np.asarray(ref, dtype=np.float64)
+    rms = float(np.sqrt(np.mean(ref ** 2)))
+    excess = np.abs(got - ref) - (tol * rms + 2.0 ** -8 * np.abs(ref))
+    assert np.isfinite(got).all() and excess.max() <= 0, f"{name}: exceeds by {excess.max():.3e}"
+
+
 def run_fwd(x, use_delta, save=False):
     return tla.tla_chunk_fwd(x["q"], x["k"], x["v"], x["q2"], x["k2"], x["g"], x["beta"], x["h0"],
                              use_delta=use_delta, save_for_bwd=save)
@@ -114,6 +123,23 @@ def test_fwd_extreme_gates(total):
     ro, rht = oracle_fwd(x, True)
     close("o", o, ro, TOL["fp32"])
     close("ht", ht, rht, TOL["fp32"])
+
+
+def test_bf16_outputs_within_tolerance_plus_rounding():
+    x = inputs.chunk_inputs(2, 300, 3, 128, 128, 8, dtype="bf16", with_beta=True, h0_std=0.1,
+                            backward=True, device="cuda", seed=17)
+    o, ht, ws = tla.tla_chunk_fwd(x["q"], x["k"], x["v"], x["q2"], x["k2"], x["g"], x["beta"],
+                                  x["h0"], save_for_bwd=True, out_dtype=torch.bfloat16)
+    grads, _ = tla.tla_chunk_bwd(x["q"], x["k"], x["v"], x["q2"], x["k2"], x["g"], x["dO"], ws,
+                                 beta=x["beta"], h0=x["h0"], out_dtype=torch.bfloat16)
+    torch.cuda.synchronize()
+    assert o.dtype == torch.bfloat16 and grads["dq"].dtype == torch.bfloat16
+    ro, rht = oracle_fwd(x, True)
+    close_rounded("o", o, ro, TOL["bf16"])
+    close("ht", ht, rht, TOL["bf16"])
+    ref = oracle_bwd(x, True, None)
+    for n in ref:
+        close_rounded(n, grads[n], ref[n], TOL["bf16"])
 
 
 # --- backward
