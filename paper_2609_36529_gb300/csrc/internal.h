@@ -4,6 +4,8 @@
 #include <cuda_runtime.h>
 #include <stddef.h>
 
+#include <cuda_bf16.h>
+
 #include "../../include/tla.h"
 
 namespace tla {
@@ -18,6 +20,8 @@ struct FwdPlan {
     size_t S;            // fp32 [B,H,NT,E,dk,dv] chunk-start states (save_for_bwd)
     size_t U;            // fp32 [B,T,H,dv] delta-corrected values (save_for_bwd)
     size_t Res;          // fp32 [B,T,H,dv] residual V - W (save_for_bwd, delta rule)
+    size_t A2;           // bf16 [B,H,NT,2,128,64] [T; A T] hi and lo tiles (tensor-core path)
+    int tc_tv;           // value columns per CTA of the tensor-core recurrence (0: SIMT)
     size_t bytes;        // total
 };
 
@@ -47,7 +51,12 @@ BwdPlan plan_bwd(const tla_problem& p);
 // SIMT path (fp32 arithmetic on CUDA cores; any supported dtype).
 cudaError_t launch_gate_cumsum(const tla_problem& p, float* G, cudaStream_t s);
 cudaError_t launch_chunk_prep(const tla_problem& p, const float* G, float* A, float* N,
-                              cudaStream_t s);
+                              __nv_bfloat16* A2, cudaStream_t s);
+
+// Tensor-core path (bf16 inputs, dk = 128): value columns per CTA, or 0 if not eligible.
+int tc_fwd_tv(const tla_problem& p);
+cudaError_t launch_fwd_recurrence_tc(const tla_problem& p, const FwdPlan& fp, char* ws,
+                                     int save_for_bwd, int* err, cudaStream_t s);
 cudaError_t launch_fwd_recurrence(const tla_problem& p, const FwdPlan& fp, char* ws,
                                   int save_for_bwd, cudaStream_t s);
 cudaError_t launch_bwd_recurrence(const tla_problem& p, const FwdPlan& fp, const char* fws,

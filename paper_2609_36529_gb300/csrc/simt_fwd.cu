@@ -58,7 +58,8 @@ __global__ void __launch_bounds__(256)
 chunk_prep_kernel(const Tin* __restrict__ q, const Tin* __restrict__ k, const Tin* __restrict__ q2,
                   const Tin* __restrict__ k2, const float* __restrict__ G,
                   const float* __restrict__ beta, float* __restrict__ Aout,
-                  float* __restrict__ Nout, int T, int H, int dk, int E, int use_delta) {
+                  float* __restrict__ Nout, __nv_bfloat16* __restrict__ A2out, int T, int H,
+                  int dk, int E, int use_delta) {
     const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
     const int NT = gridDim.x;
     const int tid = threadIdx.x;
@@ -74,7 +75,8 @@ chunk_prep_kernel(const Tin* __restrict__ q, const Tin* __restrict__ k, const Ti
     float* bs = q2s + kChunk * E;
     float* Ls = bs + kChunk;
     float* Xs = Ls + kChunk * 65;
-    float* part = Xs + kChunk * 65;
+    float* As = Xs + kChunk * 65;
+    float* part = As + kChunk * 65;
 
     for (int i = tid; i < kChunk * dk; i += blockDim.x) {
         int r = i / dk, d = i % dk;
@@ -120,32 +122,59 @@ chunk_prep_kernel(const Tin* __restrict__ q, const Tin* __restrict__ k, const Ti
             if (r > s) l = bs[r] * kk * R;
         }
         Aout[mat + i] = a;
+        As[r * 65 + s] = a;
         Ls[r * 65 + s] = l;
     }
-    if (!use_delta) return;
     __syncthreads();
-    // Forward substitution, one row at a time: X[r][s] = delta_rs - sum_{j<r} L[r][j] X[j][s].
-    const int s = tid & 63, pp = tid >> 6;  // 4 partial sums per column
-    for (int r = 0; r < kChunk; ++r) {
-        float acc = 0.f;
-        for (int j = pp; j < r; j += 4) acc = fmaf(Ls[r * 65 + j], Xs[j * 65 + s], acc);
-        part[pp * 64 + s] = acc;
-        __syncthreads();
-        if (pp == 0) {
-            float x = (r == s ? 1.f : 0.f) - ((part[s] + part[64 + s]) + (part[128 + s] + part[192 + s]));
-            Xs[r * 65 + s] = x;
+    if (use_delta) {
+        // Forward substitution, one row at a time: X[r][s] = delta_rs - sum_{j<r} L[r][j] X[j][s].
+        const int s = tid & 63, pp = tid >> 6;  // 4 partial sums per column
+        for (int r = 0; r < kChunk; ++r) {
+            float acc = 0.f;
+            for (int j = pp; j < r; j += 4) acc = fmaf(Ls[r * 65 + j], Xs[j * 65 + s], acc);
+            part[pp * 64 + s] = acc;
+            __syncthreads();
+            if (pp == 0) {
+                float x = (r == s ? 1.f : 0.f) - ((part[s] + part[64 + s]) + (part[128 + s] + part[192 + s]));
+                Xs[r * 65 + s] = x;
+            }
+            __syncthreads();
         }
-        __syncthreads();
+        for (int i = tid; i < kChunk * kChunk; i += blockDim.x) Nout[mat + i] = Xs[(i >> 6) * 65 + (i & 63)];
     }
-    for (int i = tid; i < kChunk * kChunk; i += blockDim.x) Nout[mat + i] = Xs[(i >> 6) * 65 + (i & 63)];
+    if (A2out) {
+        // Operand [T; A T] (128 x 64) of the tensor-core recurrence as a bf16 pair
+        // (hi tile, then lo tile = bf16 of the remainder): T = N diag(beta)
+        // (sGLA: diag(beta)), A T = (Q K^T (.) R') T.
+        const size_t m2 = ((size_t(b) * H + h) * NT + c) * (4 * kChunk * kChunk);
+        for (int i = tid; i < kChunk * kChunk; i += blockDim.x) {
+            const int r = i >> 6, s = i & 63;
+            float t = 0.f, at = 0.f;
+            if (r >= s) {
+                const float bsv = bs[s];
+                t = (use_delta ? Xs[r * 65 + s] : (r == s ? 1.f : 0.f)) * bsv;
+                if (use_delta) {
+                    for (int j = s; j <= r; ++j) at = fmaf(As[r * 65 + j], Xs[j * 65 + s], at);
+                    at *= bsv;
+                } else {
+                    at = As[r * 65 + s] * bsv;
+                }
+            }
+            const __nv_bfloat16 th = __float2bfloat16_rn(t), ath = __float2bfloat16_rn(at);
+            A2out[m2 + i] = th;
+            A2out[m2 + kChunk * kChunk + i] = ath;
+            A2out[m2 + 2 * kChunk * kChunk + i] = __float2bfloat16_rn(t - __bfloat162float(th));
+            A2out[m2 + 3 * kChunk * kChunk + i] = __float2bfloat16_rn(at - __bfloat162float(ath));
+        }
+    }
 }
 
 static size_t prep_smem(const tla_problem& p) {
-    return sizeof(float) * (2 * kChunk * (p.dk + 1) + 3 * kChunk * p.E + kChunk + 2 * kChunk * 65 + 256);
+    return sizeof(float) * (2 * kChunk * (p.dk + 1) + 3 * kChunk * p.E + kChunk + 3 * kChunk * 65 + 256);
 }
 
 cudaError_t launch_chunk_prep(const tla_problem& p, const float* G, float* A, float* N,
-                              cudaStream_t s) {
+                              __nv_bfloat16* A2, cudaStream_t s) {
     int NT = (p.T + kChunk - 1) / kChunk;
     dim3 grid(NT, p.H, p.B);
     size_t smem = prep_smem(p);
@@ -155,13 +184,13 @@ cudaError_t launch_chunk_prep(const tla_problem& p, const float* G, float* A, fl
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         kern<<<grid, 256, smem, s>>>((const __nv_bfloat16*)p.q, (const __nv_bfloat16*)p.k,
                                      (const __nv_bfloat16*)p.q2, (const __nv_bfloat16*)p.k2, G,
-                                     p.beta, A, N, p.T, p.H, p.dk, p.E, p.use_delta);
+                                     p.beta, A, N, A2, p.T, p.H, p.dk, p.E, p.use_delta);
     } else {
         auto kern = chunk_prep_kernel<float>;
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         kern<<<grid, 256, smem, s>>>((const float*)p.q, (const float*)p.k, (const float*)p.q2,
-                                     (const float*)p.k2, G, p.beta, A, N, p.T, p.H, p.dk, p.E,
-                                     p.use_delta);
+                                     (const float*)p.k2, G, p.beta, A, N, nullptr, p.T, p.H, p.dk,
+                                     p.E, p.use_delta);
     }
     prof_after(s);
     return cudaGetLastError();

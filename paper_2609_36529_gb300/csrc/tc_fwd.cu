@@ -1,0 +1,462 @@
+// Tensor-core (tcgen05) forward recurrence over chunks, Appendix A, Eq. joint-chunk.
+//
+// One CTA of 4 warps per (b, h, block of TV value columns); value columns never
+// interact (Section 2.5, Eq. slices), so each CTA carries its own E x dk x TV
+// slab of the fp32 state in tensor memory for the whole sequence.  Per chunk of
+// C = 64 positions, with a_e = k'_e (.) gamma_e, b_e = q'_e (.) gamma_e and
+// w_e = k'_e (.) gamma^C_e / gamma_e:
+//   MMA-A  P  = [K; Q] S_all          (M=128 rows: 64 key rows, 64 query rows;
+//                                      N = E*TV columns: slice-major; K = dk)
+//   epi-A  Res = V - sum_e diag(a_e) P_K,e   (delta rule; sGLA: Res = V)
+//          Oi  = sum_e diag(b_e) P_Q,e       (kept in registers)
+//   MMA-B  [U; Oa] = [T; A T] Res      (M=128, K=64, N=TV; T and A T from the prep kernel)
+//   epi-B  O = Oi + Oa;  Ut_e = diag(w_e) U  (bf16 operand of MMA-C)
+//   MMA-C  S_all += K^T [Ut_1 .. Ut_E] (M=dk=128, K=64, N=E*TV; K^T read MN-major
+//                                      straight from the TMA-loaded key tile)
+//   epi-C  S_{[c+1]} from TMEM -> bf16 operand of the next MMA-A, checkpoint,
+//          and pre-scaled by gamma^C of the next chunk for its MMA-C.
+// Accumulation is fp32 in TMEM.  Keys and queries are bf16 inputs and enter the
+// products exactly; every other operand (the state, Res, T, A T, Ut) is carried
+// as a pair of bf16 values hi + lo (lo = bf16 of the rounding remainder), and
+// each product sums the hi*hi, hi*lo and lo*hi terms (only x*hi and x*lo when
+// the other side is an exact key or query).  This keeps the products near fp32
+// accuracy: with a single bf16 rounding of those operands the error of o and of
+// the state reaches the 2e-2 x RMS parity bound.  Key, query and value tiles
+// and the [T; A T] tiles arrive by TMA (128-byte swizzle), prefetched one chunk
+// ahead as soon as their buffers are free.  Every mbarrier wait is
+// bounded; on expiry the CTA records TLA_ERR_TIMEOUT and leaves after a
+// bounded drain of its outstanding copies and products.
+#include <algorithm>
+
+#include "common.cuh"
+#include "internal.h"
+#include "sm100.cuh"
+#include "tma_host.h"
+
+namespace tla {
+using namespace sm100;
+
+namespace {
+
+constexpr int kThreads = 128;
+constexpr int kDk = 128;
+constexpr int kBoxBytes = 64 * 64 * 2;  // one 64 x 64 bf16 TMA box
+
+struct TcFwdArgs {
+    const __nv_bfloat16* q2;
+    const __nv_bfloat16* k2;
+    const float* G;
+    const float* h0;
+    void* o;
+    float* ht;
+    float* Sck;
+    float* Ubuf;
+    float* Rbuf;
+    int* err;
+    int T, H, dv, E, NT, use_delta, save, out_f32;
+};
+
+__device__ __forceinline__ void store_row(void* base, size_t off, const float* v, int n,
+                                          int out_f32) {
+    if (out_f32) {
+        float4* d = reinterpret_cast<float4*>(static_cast<float*>(base) + off);
+        for (int i = 0; i < n / 4; ++i) d[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+    } else {
+        uint4* d = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(base) + off);
+        for (int i = 0; i < n / 8; ++i) {
+            __nv_bfloat162 p0 = __floats2bfloat162_rn(v[8 * i], v[8 * i + 1]);
+            __nv_bfloat162 p1 = __floats2bfloat162_rn(v[8 * i + 2], v[8 * i + 3]);
+            __nv_bfloat162 p2 = __floats2bfloat162_rn(v[8 * i + 4], v[8 * i + 5]);
+            __nv_bfloat162 p3 = __floats2bfloat162_rn(v[8 * i + 6], v[8 * i + 7]);
+            uint4 u;
+            u.x = *reinterpret_cast<uint32_t*>(&p0);
+            u.y = *reinterpret_cast<uint32_t*>(&p1);
+            u.z = *reinterpret_cast<uint32_t*>(&p2);
+            u.w = *reinterpret_cast<uint32_t*>(&p3);
+            d[i] = u;
+        }
+    }
+}
+
+__device__ __forceinline__ void store_f32_row(float* dst, const float* v, int n) {
+    float4* d = reinterpret_cast<float4*>(dst);
+    for (int i = 0; i < n / 4; ++i) d[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+}
+
+// Store v as a bf16 pair: hi = bf16(v) into tile_hi, lo = bf16(v - hi) into tile_lo.
+__device__ __forceinline__ void st_split(uint8_t* tile_hi, uint8_t* tile_lo, uint32_t off, float v) {
+    const __nv_bfloat16 hi = __float2bfloat16_rn(v);
+    *reinterpret_cast<__nv_bfloat16*>(tile_hi + off) = hi;
+    *reinterpret_cast<__nv_bfloat16*>(tile_lo + off) = __float2bfloat16_rn(v - __bfloat162float(hi));
+}
+
+template <int TV>
+__global__ void __launch_bounds__(kThreads, 1)
+fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
+                         const __grid_constant__ CUtensorMap map_q,
+                         const __grid_constant__ CUtensorMap map_v,
+                         const __grid_constant__ CUtensorMap map_a2, const TcFwdArgs p) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+    const int E = p.E, NE = E * TV;
+    uint8_t* sKQ = sm;                         // 2 blocks x [K rows 0-63 | Q rows 64-127] x 128 B
+    uint8_t* sA2 = sKQ + 2 * 2 * kBoxBytes;    // [T; A T] 128 x 64 bf16: hi tile, lo tile
+    uint8_t* sReg = sA2 + 4 * kBoxBytes;       // shared region, 2 * NE * 256 bytes:
+    uint8_t* sSh = sReg;                       //   S_all^T [NE][dk] hi  (MMA-A operand)
+    uint8_t* sSl = sReg + NE * 256;            //   S_all^T [NE][dk] lo
+    uint8_t* sRh = sReg;                       //   Res^T [TV][64] hi, lo (after MMA-A)
+    uint8_t* sRl = sReg + TV * 128;
+    uint8_t* sUh = sReg + TV * 256;            //   Ut^T [NE][64] hi, lo (after MMA-B)
+    uint8_t* sUl = sUh + NE * 128;
+    __nv_bfloat16* sV = reinterpret_cast<__nv_bfloat16*>(sReg + NE * 512);  // [64][TV]
+    float* ae = reinterpret_cast<float*>(sReg + NE * 512 + 64 * TV * 2);
+    float* be = ae + 64 * E;
+    float* we = be + 64 * E;
+    float* gcn = we + 64 * E;                  // gamma^C of the chunk whose coefficients are loaded
+
+    __shared__ __align__(8) uint64_t bar_kq, bar_av, bar_mma;
+    __shared__ uint32_t tmem_slot;
+
+    const int tid = threadIdx.x, warp = tid >> 5;
+    const int nb = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+    const int n0 = nb * TV;
+    const int T = p.T, H = p.H, dv = p.dv, NT = p.NT;
+    const uint32_t tcols = (2 * NE <= 256) ? 256u : 512u;
+
+    if (warp == 0) {
+        tmem_alloc(&tmem_slot, tcols);
+        tmem_relinquish();
+    }
+    if (tid == 0) {
+        mbar_init(&bar_kq, 1);
+        mbar_init(&bar_av, 1);
+        mbar_init(&bar_mma, 1);
+        fence_barrier_init();
+        tma_prefetch_desc(&map_k);
+        tma_prefetch_desc(&map_q);
+        tma_prefetch_desc(&map_v);
+        tma_prefetch_desc(&map_a2);
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tP = tmem_slot;        // columns [0, NE): P, then D2 in [0, TV)
+    const uint32_t tS = tmem_slot + NE;   // columns [NE, 2 NE): the state slab
+
+    auto issue_kq = [&](int c) {
+        mbar_arrive_expect_tx(&bar_kq, 4 * kBoxBytes);
+        for (int j = 0; j < 2; ++j) {
+            tma_load_4d(sKQ + j * 2 * kBoxBytes, &map_k, &bar_kq, 64 * j, h, c * 64, b);
+            tma_load_4d(sKQ + j * 2 * kBoxBytes + kBoxBytes, &map_q, &bar_kq, 64 * j, h, c * 64, b);
+        }
+    };
+    auto issue_av = [&](int c) {
+        mbar_arrive_expect_tx(&bar_av, 4 * kBoxBytes + 64 * TV * 2);
+        tma_load_2d(sA2, &map_a2, &bar_av, 0, ((b * H + h) * NT + c) * 256);
+        tma_load_2d(sA2 + 2 * kBoxBytes, &map_a2, &bar_av, 0, ((b * H + h) * NT + c) * 256 + 128);
+        tma_load_4d(sV, &map_v, &bar_av, n0, h, c * 64, b);
+    };
+    auto load_coefs = [&](int c) {
+        const int t0 = c * 64, n = min(64, T - t0);
+        for (int i = tid; i < 64 * E; i += kThreads) {
+            const int r = i / E, e = i - (i / E) * E;
+            const int rr = r < n ? r : n - 1;
+            const float Gr = p.G[tok_idx(b, t0 + rr, h, e, T, H, E)];
+            const float GC = p.G[tok_idx(b, t0 + n - 1, h, e, T, H, E)];
+            const float kk = r < n ? __bfloat162float(p.k2[tok_idx(b, t0 + r, h, e, T, H, E)]) : 0.f;
+            const float qq = r < n ? __bfloat162float(p.q2[tok_idx(b, t0 + r, h, e, T, H, E)]) : 0.f;
+            const float gam = expf(Gr);
+            ae[i] = kk * gam;
+            be[i] = qq * gam;
+            we[i] = kk * expf(GC - Gr);
+            if (r == 0) gcn[e] = expf(GC);
+        }
+    };
+    // State row d = tid of S_{[c]}: bf16 copy for MMA-A, checkpoint, and
+    // gamma^C_c-scaled copy in TMEM for the accumulation of chunk c.
+    auto prepare = [&](int c, bool from_h0) {
+        const int d = tid;
+        for (int e = 0; e < E; ++e) {
+            float v[TV];
+            if (from_h0) {
+                if (p.h0) {
+                    const float4* src = reinterpret_cast<const float4*>(
+                        p.h0 + ((size_t(b * H + h) * E + e) * kDk + d) * dv + n0);
+#pragma unroll
+                    for (int i = 0; i < TV / 4; ++i) {
+                        float4 x = src[i];
+                        v[4 * i] = x.x; v[4 * i + 1] = x.y; v[4 * i + 2] = x.z; v[4 * i + 3] = x.w;
+                    }
+                } else {
+#pragma unroll
+                    for (int i = 0; i < TV; ++i) v[i] = 0.f;
+                }
+            } else {
+#pragma unroll
+                for (int j = 0; j < TV; j += 16) tmem_ld16(tmem_lane_addr(tS, warp, e * TV + j), v + j);
+                tmem_wait_ld();
+            }
+#pragma unroll
+            for (int n = 0; n < TV; ++n) st_split(sSh, sSl, sw128_offset(e * TV + n, d, NE), v[n]);
+            if (p.save)
+                store_f32_row(p.Sck + ((((size_t(b) * H + h) * NT + c) * E + e) * kDk + d) * dv + n0,
+                              v, TV);
+            const float g = gcn[e];
+#pragma unroll
+            for (int n = 0; n < TV; ++n) v[n] *= g;
+#pragma unroll
+            for (int j = 0; j < TV; j += 16) tmem_st16(tmem_lane_addr(tS, warp, e * TV + j), v + j);
+        }
+        tmem_wait_st();
+    };
+
+    if (tid == 0) {
+        issue_kq(0);
+        issue_av(0);
+    }
+    load_coefs(0);
+    __syncthreads();
+    prepare(0, true);
+    fence_proxy_async_smem();
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+
+    uint32_t mma_phase = 0;
+    bool failed = false;
+    int pending_kq = 0, pending_av = 0, pending_mma = 0;  // outstanding async work (tid 0 view)
+    for (int c = 0; c < NT; ++c) {
+        const int t0 = c * 64, n = min(64, T - t0);
+        pending_kq = pending_av = 1;
+        bool ok = mbar_wait(&bar_kq, c & 1);
+        if (ok) pending_kq = 0;
+        ok = ok && mbar_wait(&bar_av, c & 1);
+        if (ok) pending_av = 0;
+        if (__syncthreads_or(!ok)) { failed = true; break; }
+        tc_fence_after();
+
+        // ---- MMA-A: P = [K; Q] S_all
+        if (tid == 0) {
+            const uint32_t idesc = idesc_bf16_f32(128, NE, 0, 0);
+#pragma unroll
+            for (int ks = 0; ks < kDk / 16; ++ks) {
+                const int blk = ks >> 2, kk = (ks & 3) * 16;
+                const uint64_t ad = smem_desc(smem_u32(sKQ) + blk * 2 * kBoxBytes + kk * 2, 16, 1024);
+                const uint32_t bo = blk * NE * 128 + kk * 2;
+                umma_bf16(tP, ad, smem_desc(smem_u32(sSh) + bo, 16, 1024), idesc, ks > 0 ? 1u : 0u);
+                umma_bf16(tP, ad, smem_desc(smem_u32(sSl) + bo, 16, 1024), idesc, 1u);
+            }
+            umma_commit(&bar_mma);
+        }
+        pending_mma = 1;
+        ok = mbar_wait(&bar_mma, mma_phase);
+        mma_phase ^= 1;
+        if (__syncthreads_or(!ok)) { failed = true; break; }
+        pending_mma = 0;
+        tc_fence_after();
+
+        // ---- epi-A
+        float oi[TV];
+        if (warp < 2) {
+            const int r = tid;
+            float w[TV];
+#pragma unroll
+            for (int i = 0; i < TV; ++i) w[i] = 0.f;
+            if (p.use_delta) {
+                for (int e = 0; e < E; ++e) {
+                    float pv[TV];
+#pragma unroll
+                    for (int j = 0; j < TV; j += 16) tmem_ld16(tmem_lane_addr(tP, warp, e * TV + j), pv + j);
+                    tmem_wait_ld();
+                    const float a = ae[r * E + e];
+#pragma unroll
+                    for (int i = 0; i < TV; ++i) w[i] = fmaf(a, pv[i], w[i]);
+                }
+            }
+            float res[TV];
+#pragma unroll
+            for (int i = 0; i < TV; ++i) {
+                res[i] = __bfloat162float(sV[r * TV + i]) - w[i];
+                st_split(sRh, sRl, sw128_offset(i, r, TV), res[i]);
+            }
+            if (p.save && p.use_delta && r < n)
+                store_f32_row(p.Rbuf + tok_idx(b, t0 + r, h, n0, T, H, dv), res, TV);
+        } else {
+            const int r = tid - 64;
+#pragma unroll
+            for (int i = 0; i < TV; ++i) oi[i] = 0.f;
+            for (int e = 0; e < E; ++e) {
+                float pv[TV];
+#pragma unroll
+                for (int j = 0; j < TV; j += 16) tmem_ld16(tmem_lane_addr(tP, warp, e * TV + j), pv + j);
+                tmem_wait_ld();
+                const float bq = be[r * E + e];
+#pragma unroll
+                for (int i = 0; i < TV; ++i) oi[i] = fmaf(bq, pv[i], oi[i]);
+            }
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        tc_fence_after();
+
+        // ---- MMA-B: [U; Oa] = [T; A T] Res  (into columns [0, TV))
+        if (tid == 0) {
+            const uint32_t idesc = idesc_bf16_f32(128, TV, 0, 0);
+#pragma unroll
+            for (int ks = 0; ks < 4; ++ks) {
+                const uint64_t ah = smem_desc(smem_u32(sA2) + ks * 32, 16, 1024);
+                const uint64_t al = smem_desc(smem_u32(sA2) + 2 * kBoxBytes + ks * 32, 16, 1024);
+                const uint64_t bh = smem_desc(smem_u32(sRh) + ks * 32, 16, 1024);
+                const uint64_t bl = smem_desc(smem_u32(sRl) + ks * 32, 16, 1024);
+                umma_bf16(tP, ah, bh, idesc, ks > 0 ? 1u : 0u);
+                umma_bf16(tP, ah, bl, idesc, 1u);
+                umma_bf16(tP, al, bh, idesc, 1u);
+            }
+            umma_commit(&bar_mma);
+        }
+        pending_mma = 1;
+        ok = mbar_wait(&bar_mma, mma_phase);
+        mma_phase ^= 1;
+        if (__syncthreads_or(!ok)) { failed = true; break; }
+        pending_mma = 0;
+        tc_fence_after();
+        if (tid == 0 && c + 1 < NT) issue_av(c + 1);   // [T; A T] and V buffers are free
+
+        // ---- epi-B
+        {
+            float d2[TV];
+#pragma unroll
+            for (int j = 0; j < TV; j += 16) tmem_ld16(tmem_lane_addr(tP, warp, j), d2 + j);
+            tmem_wait_ld();
+            if (warp < 2) {
+                const int r = tid;
+                for (int e = 0; e < E; ++e) {
+                    const float wv = we[r * E + e];
+#pragma unroll
+                    for (int i = 0; i < TV; ++i) st_split(sUh, sUl, sw128_offset(e * TV + i, r, NE), wv * d2[i]);
+                }
+                if (p.save && r < n) store_f32_row(p.Ubuf + tok_idx(b, t0 + r, h, n0, T, H, dv), d2, TV);
+            } else {
+                const int r = tid - 64;
+#pragma unroll
+                for (int i = 0; i < TV; ++i) d2[i] += oi[i];
+                if (r < n) store_row(p.o, tok_idx(b, t0 + r, h, n0, T, H, dv), d2, TV, p.out_f32);
+            }
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        tc_fence_after();
+
+        // ---- MMA-C: S_all += K^T Ut   (A = K^T, MN-major from the key rows of sKQ)
+        if (tid == 0) {
+            const uint32_t idesc = idesc_bf16_f32(128, NE, 1, 0);
+#pragma unroll
+            for (int ks = 0; ks < 4; ++ks) {
+                const uint64_t ad = smem_desc(smem_u32(sKQ) + ks * 2048, 2 * kBoxBytes, 1024);
+                umma_bf16(tS, ad, smem_desc(smem_u32(sUh) + ks * 32, 16, 1024), idesc, 1u);
+                umma_bf16(tS, ad, smem_desc(smem_u32(sUl) + ks * 32, 16, 1024), idesc, 1u);
+            }
+            umma_commit(&bar_mma);
+        }
+        pending_mma = 1;
+        if (c + 1 < NT) load_coefs(c + 1);   // overlaps MMA-C; chunk c's coefficients are done
+        ok = mbar_wait(&bar_mma, mma_phase);
+        mma_phase ^= 1;
+        if (__syncthreads_or(!ok)) { failed = true; break; }
+        pending_mma = 0;
+        tc_fence_after();
+        if (tid == 0 && c + 1 < NT) issue_kq(c + 1);   // key/query buffer is free
+
+        // ---- epi-C
+        if (c + 1 < NT) {
+            prepare(c + 1, false);
+        } else if (p.ht) {
+            const int d = tid;
+            for (int e = 0; e < E; ++e) {
+                float v[TV];
+#pragma unroll
+                for (int j = 0; j < TV; j += 16) tmem_ld16(tmem_lane_addr(tS, warp, e * TV + j), v + j);
+                tmem_wait_ld();
+                store_f32_row(p.ht + ((size_t(b * H + h) * E + e) * kDk + d) * dv + n0, v, TV);
+            }
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        tc_fence_after();
+    }
+
+    if (failed) {
+        // Bounded drain of whatever this CTA still has in flight, then leave.
+        if (tid == 0) {
+            record_device_error(p.err, TLA_ERR_TIMEOUT);
+            if (pending_mma) mbar_wait(&bar_mma, mma_phase ^ 1);
+        }
+        __syncthreads();
+        (void)pending_kq;
+        (void)pending_av;
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 0) tmem_dealloc(tmem_slot, tcols);
+}
+
+template <int TV>
+size_t tc_fwd_smem(int E) {
+    const int NE = E * TV;
+    return 1024 + 4 * kBoxBytes + 4 * kBoxBytes + NE * 512 + 64 * TV * 2 + (3 * 64 * E + E) * 4;
+}
+
+template <int TV>
+cudaError_t launch_tv(const tla_problem& p, const FwdPlan& fp, char* ws, int save, int* err,
+                      cudaStream_t s) {
+    CUtensorMap mk, mq, mv, ma;
+    const int NT = fp.NT;
+    if (!make_token_map(&mk, p.k, p.B, p.T, p.H, kDk, 64, 64, true) ||
+        !make_token_map(&mq, p.q, p.B, p.T, p.H, kDk, 64, 64, true) ||
+        !make_token_map(&mv, p.v, p.B, p.T, p.H, p.dv, TV, 64, false) ||
+        !make_matrix_map(&ma, ws + fp.A2, (long long)p.B * p.H * NT * 256, 64, 64, 128))
+        return cudaErrorInvalidValue;
+    TcFwdArgs a;
+    a.q2 = (const __nv_bfloat16*)p.q2;
+    a.k2 = (const __nv_bfloat16*)p.k2;
+    a.G = (const float*)(ws + fp.G);
+    a.h0 = p.h0;
+    a.o = p.o;
+    a.ht = p.ht;
+    a.Sck = save ? (float*)(ws + fp.S) : nullptr;
+    a.Ubuf = save ? (float*)(ws + fp.U) : nullptr;
+    a.Rbuf = (save && p.use_delta) ? (float*)(ws + fp.Res) : nullptr;
+    a.err = err;
+    a.T = p.T; a.H = p.H; a.dv = p.dv; a.E = p.E; a.NT = NT;
+    a.use_delta = p.use_delta; a.save = save; a.out_f32 = p.out_dtype == TLA_FP32;
+    const size_t smem = tc_fwd_smem<TV>(p.E);
+    auto kern = fwd_recurrence_tc_kernel<TV>;
+    cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    dim3 grid(p.dv / TV, p.H, p.B);
+    prof_before("fwd_recurrence_tc", s);
+    kern<<<grid, kThreads, smem, s>>>(mk, mq, mv, ma, a);
+    prof_after(s);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+int tc_fwd_tv(const tla_problem& p) {
+    if (p.dtype != TLA_BF16 || p.dk != kDk) return 0;
+    const int tv = p.E <= 4 ? 32 : 16;
+    if (p.dv % tv != 0 || p.E * tv > 256) return 0;
+    return tv;
+}
+
+cudaError_t launch_fwd_recurrence_tc(const tla_problem& p, const FwdPlan& fp, char* ws,
+                                     int save_for_bwd, int* err, cudaStream_t s) {
+    return fp.tc_tv == 32 ? launch_tv<32>(p, fp, ws, save_for_bwd, err, s)
+                          : launch_tv<16>(p, fp, ws, save_for_bwd, err, s);
+}
+
+}  // namespace tla

@@ -31,6 +31,20 @@ static tla_status validate(const tla_problem* p) {
     return TLA_OK;
 }
 
+static bool aligned16(const void* x) { return ((uintptr_t)x & 15) == 0; }
+
+// The tensor-core path reads q, k, v by TMA and writes rows with 16-byte stores.
+static bool tc_eligible(const tla_problem& p) {
+    return aligned16(p.q) && aligned16(p.k) && aligned16(p.v) && aligned16(p.o) &&
+           aligned16(p.h0) && aligned16(p.ht);
+}
+
+static int* device_error_word() {
+    static int* ptr = nullptr;
+    if (!ptr) cudaGetSymbolAddress((void**)&ptr, g_device_error);
+    return ptr;
+}
+
 // Value columns per CTA of the SIMT recurrences: the E x dk x tv fp32 slab
 // stays within 64 KiB of shared memory.
 static int simt_tv(const tla_problem& p) {
@@ -44,6 +58,7 @@ FwdPlan plan_fwd(const tla_problem& p, int save) {
     memset(&f, 0, sizeof(f));
     f.NT = (p.T + kChunk - 1) / kChunk;
     f.tv = simt_tv(p);
+    f.tc_tv = tc_fwd_tv(p);   // layout depends on shapes only
     const size_t tokE = (size_t)p.B * p.T * p.H * p.E * 4;
     const size_t mats = (size_t)p.B * p.H * f.NT * kChunk * kChunk * 4;
     const size_t states = (size_t)p.B * p.H * f.NT * p.E * p.dk * p.dv * 4;
@@ -52,6 +67,7 @@ FwdPlan plan_fwd(const tla_problem& p, int save) {
     f.G = off; off = align256(off + tokE);
     f.A = off; off = align256(off + mats);
     if (p.use_delta) { f.N = off; off = align256(off + mats); }
+    if (f.tc_tv) { f.A2 = off; off = align256(off + 2 * mats); }   // hi + lo 128 x 64 bf16 tiles
     if (save) {
         f.S = off; off = align256(off + states);
         f.U = off; off = align256(off + tokV);
@@ -77,6 +93,7 @@ BwdPlan plan_bwd(const tla_problem& p) {
 }
 
 static tla_status cuda_status(cudaError_t e) { return e == cudaSuccess ? TLA_OK : TLA_ERR_CUDA; }
+
 
 // ---- kernel timing: a pool of event pairs, one per launch while enabled
 struct ProfRecord {
@@ -142,8 +159,14 @@ tla_status tla_chunk_fwd(const tla_problem* p, void* workspace, size_t workspace
     cudaError_t e = launch_gate_cumsum(*p, (float*)(ws + fp.G), s);
     if (e == cudaSuccess)
         e = launch_chunk_prep(*p, (const float*)(ws + fp.G), (float*)(ws + fp.A),
-                              p->use_delta ? (float*)(ws + fp.N) : nullptr, s);
-    if (e == cudaSuccess) e = launch_fwd_recurrence(*p, fp, ws, save, s);
+                              p->use_delta ? (float*)(ws + fp.N) : nullptr,
+                              (fp.tc_tv && tc_eligible(*p)) ? (__nv_bfloat16*)(ws + fp.A2) : nullptr,
+                              s);
+    if (e == cudaSuccess) {
+        if (fp.tc_tv && tc_eligible(*p))
+            e = launch_fwd_recurrence_tc(*p, fp, ws, save, device_error_word(), s);
+        else e = launch_fwd_recurrence(*p, fp, ws, save, s);
+    }
     return cuda_status(e);
 }
 

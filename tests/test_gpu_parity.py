@@ -102,6 +102,20 @@ def test_fwd_shapes(dk, dv, E):
     close("ht", ht, rht, TOL["bf16"])
 
 
+@pytest.mark.parametrize("use_delta", [True, False])
+@pytest.mark.parametrize("T,E", [(1, 4), (63, 1), (65, 8), (200, 4), (130, 16), (257, 6)])
+def test_fwd_tensor_core_path(use_delta, T, E):
+    """bf16, dk = 128: the tcgen05 recurrence (value blocks of 32 for E <= 4, else 16)."""
+    x = inputs.chunk_inputs(2, T, 2, 128, 64, E, dtype="bf16", with_beta=True, h0_std=0.1,
+                            device="cuda", seed=T * 31 + E)
+    o, ht, _ = run_fwd(x, use_delta)
+    torch.cuda.synchronize()
+    assert tla.tla_last_device_status() == 0
+    ro, rht = oracle_fwd(x, use_delta)
+    close("o", o, ro, TOL["bf16"], rel_l2=0.01)
+    close("ht", ht, rht, TOL["bf16"], rel_l2=0.01)
+
+
 def test_fwd_sgla_no_beta_no_h0():
     x = inputs.chunk_inputs(2, 129, 2, 32, 32, 4, dtype="fp32", with_beta=False, device="cuda",
                             seed=5)
