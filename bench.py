@@ -17,6 +17,7 @@ oracle on this machine's host cores on a bounded sample of the same workload.
 """
 import argparse
 import ctypes
+import dataclasses
 import hashlib
 import json
 import os
@@ -226,6 +227,8 @@ def run_ours(args):
         return float(t.item())
 
     w = inputs.GDN_FWDBWD_BF16
+    if args.batch:   # profiling option: fewer sequences of the same shape
+        w = dataclasses.replace(w, B=args.batch, name=f"{w.name}_batch{args.batch}")
     x = inputs.workload_inputs(w, device=dev, seed=rank)
     stream = torch.cuda.current_stream(dev)
 
@@ -245,6 +248,8 @@ def run_ours(args):
         tla.tla_chunk_fwd(xx["q"], xx["k"], xx["v"], xx["q2"], xx["k2"], xx["g"], xx["beta"],
                           None, use_delta=True, save_for_bwd=True, want_ht=False, o=o,
                           workspace=fws)
+        if args.fwd_only:
+            return
         tla.tla_chunk_bwd(xx["q"], xx["k"], xx["v"], xx["q2"], xx["k2"], xx["g"], xx["dO"], fws,
                           beta=xx["beta"], use_delta=True, workspace=bws, grads=grads)
 
@@ -325,6 +330,9 @@ def run_ours(args):
     if rank == 0 and ws_n == 1 and not args.no_cpu_baseline:
         cpu = oracle_baseline(x, w, seconds_target=args.cpu_seconds)
 
+    if args.fwd_only or args.batch:
+        print("bench: profiling options given; this line is not the headline measurement",
+              file=sys.stderr)
     if rank == 0:
         line = {
             "metric": HEADLINE_METRIC, "value": round(value, 1), "unit": "tokens/s",
@@ -517,6 +525,10 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--ref-tokens", type=int, default=1024,
                     help="tokens per head in one reference-arm step")
+    ap.add_argument("--batch", type=int, default=0,
+                    help="profiling only: run B sequences instead of the workload's 8")
+    ap.add_argument("--fwd-only", action="store_true",
+                    help="profiling only: time the forward alone (not the headline metric)")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         print("bench: at least 3 warm-up steps are required; using 3", file=sys.stderr)

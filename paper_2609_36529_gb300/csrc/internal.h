@@ -21,6 +21,7 @@ struct FwdPlan {
     size_t U;            // fp32 [B,T,H,dv] delta-corrected values (save_for_bwd)
     size_t Res;          // fp32 [B,T,H,dv] residual V - W (save_for_bwd, delta rule)
     size_t A2;           // bf16 [B,H,NT,2,128,64] [T; A T] hi and lo tiles (tensor-core path)
+    size_t coef;         // fp32 [B,H,NT,3*64*E+16] per-row coefficients (tensor-core path)
     int tc_tv;           // value columns per CTA of the tensor-core recurrence (0: SIMT)
     size_t bytes;        // total
 };
@@ -51,7 +52,7 @@ BwdPlan plan_bwd(const tla_problem& p);
 // SIMT path (fp32 arithmetic on CUDA cores; any supported dtype).
 cudaError_t launch_gate_cumsum(const tla_problem& p, float* G, cudaStream_t s);
 cudaError_t launch_chunk_prep(const tla_problem& p, const float* G, float* A, float* N,
-                              __nv_bfloat16* A2, cudaStream_t s);
+                              __nv_bfloat16* A2, float* coef, cudaStream_t s);
 
 // Tensor-core path (bf16 inputs, dk = 128): value columns per CTA, or 0 if not eligible.
 int tc_fwd_tv(const tla_problem& p);

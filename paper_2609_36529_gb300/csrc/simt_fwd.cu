@@ -58,8 +58,8 @@ __global__ void __launch_bounds__(256)
 chunk_prep_kernel(const Tin* __restrict__ q, const Tin* __restrict__ k, const Tin* __restrict__ q2,
                   const Tin* __restrict__ k2, const float* __restrict__ G,
                   const float* __restrict__ beta, float* __restrict__ Aout,
-                  float* __restrict__ Nout, __nv_bfloat16* __restrict__ A2out, int T, int H,
-                  int dk, int E, int use_delta) {
+                  float* __restrict__ Nout, __nv_bfloat16* __restrict__ A2out,
+                  float* __restrict__ coef_out, int T, int H, int dk, int E, int use_delta) {
     const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
     const int NT = gridDim.x;
     const int tid = threadIdx.x;
@@ -142,6 +142,21 @@ chunk_prep_kernel(const Tin* __restrict__ q, const Tin* __restrict__ k, const Ti
         }
         for (int i = tid; i < kChunk * kChunk; i += blockDim.x) Nout[mat + i] = Xs[(i >> 6) * 65 + (i & 63)];
     }
+    if (coef_out) {
+        // Per-row coefficients of the tensor-core recurrence, one block per chunk:
+        // [k'_e gamma_e | q'_e gamma_e | k'_e gamma^C_e / gamma_e] as [64][E] each, then gamma^C_e
+        // (padded to 16).  Decays are exponentials of non-positive log differences.
+        float* cf = coef_out + ((size_t(b) * H + h) * NT + c) * (3 * kChunk * E + 16);
+        for (int i = tid; i < kChunk * E; i += blockDim.x) {
+            const int e = i % E;
+            const float Gr = Gs[i], GC = Gs[(n - 1) * E + e];
+            const float gam = expf(Gr);
+            cf[i] = k2s[i] * gam;
+            cf[kChunk * E + i] = q2s[i] * gam;
+            cf[2 * kChunk * E + i] = k2s[i] * expf(GC - Gr);
+        }
+        if (tid < 16) cf[3 * kChunk * E + tid] = tid < E ? expf(Gs[(n - 1) * E + tid]) : 0.f;
+    }
     if (A2out) {
         // Operand [T; A T] (128 x 64) of the tensor-core recurrence as a bf16 pair
         // (hi tile, then lo tile = bf16 of the remainder): T = N diag(beta)
@@ -174,7 +189,7 @@ static size_t prep_smem(const tla_problem& p) {
 }
 
 cudaError_t launch_chunk_prep(const tla_problem& p, const float* G, float* A, float* N,
-                              __nv_bfloat16* A2, cudaStream_t s) {
+                              __nv_bfloat16* A2, float* coef, cudaStream_t s) {
     int NT = (p.T + kChunk - 1) / kChunk;
     dim3 grid(NT, p.H, p.B);
     size_t smem = prep_smem(p);
@@ -184,13 +199,13 @@ cudaError_t launch_chunk_prep(const tla_problem& p, const float* G, float* A, fl
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         kern<<<grid, 256, smem, s>>>((const __nv_bfloat16*)p.q, (const __nv_bfloat16*)p.k,
                                      (const __nv_bfloat16*)p.q2, (const __nv_bfloat16*)p.k2, G,
-                                     p.beta, A, N, A2, p.T, p.H, p.dk, p.E, p.use_delta);
+                                     p.beta, A, N, A2, coef, p.T, p.H, p.dk, p.E, p.use_delta);
     } else {
         auto kern = chunk_prep_kernel<float>;
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         kern<<<grid, 256, smem, s>>>((const float*)p.q, (const float*)p.k, (const float*)p.q2,
-                                     (const float*)p.k2, G, p.beta, A, N, nullptr, p.T, p.H, p.dk,
-                                     p.E, p.use_delta);
+                                     (const float*)p.k2, G, p.beta, A, N, nullptr, nullptr, p.T,
+                                     p.H, p.dk, p.E, p.use_delta);
     }
     prof_after(s);
     return cudaGetLastError();

@@ -111,6 +111,15 @@ __device__ __forceinline__ void tma_load_4d(void* dst, const CUtensorMap* map, u
         : "memory");
 }
 
+// Plain bulk copy global -> shared (16-byte aligned addresses, size multiple of 16).
+__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+            smem_u32(dst)),
+        "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(smem_u32(bar))
+        : "memory");
+}
+
 // ---------------------------------------------------------------- TMEM
 // Allocation is a warp-wide operation; the allocated base address is written
 // to shared memory.  ncols: power of two, 32..512.
@@ -212,6 +221,23 @@ __host__ __device__ __forceinline__ uint32_t sw128_offset(int row, int k, int ro
     const int blk = k >> 6, kk = k & 63;
     return uint32_t(blk * rows * 128 + row * 128 + ((((kk >> 3) ^ (row & 7)) & 7) << 4) +
                     ((kk & 7) << 1));
+}
+
+// Store 8 consecutive values as bf16 hi/lo pairs at byte offset `off` of two tiles
+// (16-byte chunks; `off` must address the first element of a chunk).
+__device__ __forceinline__ void st8_split(uint8_t* tile_hi, uint8_t* tile_lo, uint32_t off,
+                                          const float* v) {
+    uint32_t h[4], l[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        __nv_bfloat162 hv = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
+        float2 hf = __bfloat1622float2(hv);
+        __nv_bfloat162 lv = __floats2bfloat162_rn(v[2 * i] - hf.x, v[2 * i + 1] - hf.y);
+        h[i] = *reinterpret_cast<uint32_t*>(&hv);
+        l[i] = *reinterpret_cast<uint32_t*>(&lv);
+    }
+    *reinterpret_cast<uint4*>(tile_hi + off) = make_uint4(h[0], h[1], h[2], h[3]);
+    *reinterpret_cast<uint4*>(tile_lo + off) = make_uint4(l[0], l[1], l[2], l[3]);
 }
 
 }  // namespace sm100

@@ -4,28 +4,30 @@
 // interact (Section 2.5, Eq. slices), so each CTA carries its own E x dk x TV
 // slab of the fp32 state in tensor memory for the whole sequence.  Per chunk of
 // C = 64 positions, with a_e = k'_e (.) gamma_e, b_e = q'_e (.) gamma_e and
-// w_e = k'_e (.) gamma^C_e / gamma_e:
+// w_e = k'_e (.) gamma^C_e / gamma_e (precomputed per chunk by the prep kernel):
 //   MMA-A  P  = [K; Q] S_all          (M=128 rows: 64 key rows, 64 query rows;
-//                                      N = E*TV columns: slice-major; K = dk)
+//                                      N = NE = E*TV columns, slice-major; K = dk)
 //   epi-A  Res = V - sum_e diag(a_e) P_K,e   (delta rule; sGLA: Res = V)
 //          Oi  = sum_e diag(b_e) P_Q,e       (kept in registers)
 //   MMA-B  [U; Oa] = [T; A T] Res      (M=128, K=64, N=TV; T and A T from the prep kernel)
-//   epi-B  O = Oi + Oa;  Ut_e = diag(w_e) U  (bf16 operand of MMA-C)
-//   MMA-C  S_all += K^T [Ut_1 .. Ut_E] (M=dk=128, K=64, N=E*TV; K^T read MN-major
+//   epi-B  O = Oi + Oa;  Ut_e = diag(w_e) U
+//   MMA-C  S_all += K^T [Ut_1 .. Ut_E] (M=dk=128, K=64, N=NE; K^T read MN-major
 //                                      straight from the TMA-loaded key tile)
-//   epi-C  S_{[c+1]} from TMEM -> bf16 operand of the next MMA-A, checkpoint,
-//          and pre-scaled by gamma^C of the next chunk for its MMA-C.
+//   epi-C  S_{[c+1]} from TMEM -> operand of the next MMA-A, checkpoint, and
+//          pre-scaled by gamma^C of the next chunk for its MMA-C.
 // Accumulation is fp32 in TMEM.  Keys and queries are bf16 inputs and enter the
 // products exactly; every other operand (the state, Res, T, A T, Ut) is carried
 // as a pair of bf16 values hi + lo (lo = bf16 of the rounding remainder), and
 // each product sums the hi*hi, hi*lo and lo*hi terms (only x*hi and x*lo when
 // the other side is an exact key or query).  This keeps the products near fp32
 // accuracy: with a single bf16 rounding of those operands the error of o and of
-// the state reaches the 2e-2 x RMS parity bound.  Key, query and value tiles
-// and the [T; A T] tiles arrive by TMA (128-byte swizzle), prefetched one chunk
-// ahead as soon as their buffers are free.  Every mbarrier wait is
-// bounded; on expiry the CTA records TLA_ERR_TIMEOUT and leaves after a
-// bounded drain of its outstanding copies and products.
+// the state reaches the 2e-2 x RMS parity bound.
+// The state and Ut operands are stored MN-major (one row per thread, 16-byte
+// stores), so each thread writes the TMEM row it read.  Key, query, value
+// tiles, the [T; A T] tiles and the coefficient block arrive by TMA, prefetched
+// one chunk ahead as soon as their buffers are free.  Every mbarrier wait is
+// bounded by the GPU global timer; on expiry the CTA records TLA_ERR_TIMEOUT and
+// leaves after a bounded drain of its outstanding work.
 #include <algorithm>
 
 #include "common.cuh"
@@ -43,9 +45,7 @@ constexpr int kDk = 128;
 constexpr int kBoxBytes = 64 * 64 * 2;  // one 64 x 64 bf16 TMA box
 
 struct TcFwdArgs {
-    const __nv_bfloat16* q2;
-    const __nv_bfloat16* k2;
-    const float* G;
+    const float* coef;   // [B,H,NT, 3*64*E + 16] per-chunk coefficient blocks
     const float* h0;
     void* o;
     float* ht;
@@ -64,16 +64,12 @@ __device__ __forceinline__ void store_row(void* base, size_t off, const float* v
     } else {
         uint4* d = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(base) + off);
         for (int i = 0; i < n / 8; ++i) {
-            __nv_bfloat162 p0 = __floats2bfloat162_rn(v[8 * i], v[8 * i + 1]);
-            __nv_bfloat162 p1 = __floats2bfloat162_rn(v[8 * i + 2], v[8 * i + 3]);
-            __nv_bfloat162 p2 = __floats2bfloat162_rn(v[8 * i + 4], v[8 * i + 5]);
-            __nv_bfloat162 p3 = __floats2bfloat162_rn(v[8 * i + 6], v[8 * i + 7]);
-            uint4 u;
-            u.x = *reinterpret_cast<uint32_t*>(&p0);
-            u.y = *reinterpret_cast<uint32_t*>(&p1);
-            u.z = *reinterpret_cast<uint32_t*>(&p2);
-            u.w = *reinterpret_cast<uint32_t*>(&p3);
-            d[i] = u;
+            uint32_t u[4];
+            for (int j = 0; j < 4; ++j) {
+                __nv_bfloat162 pr = __floats2bfloat162_rn(v[8 * i + 2 * j], v[8 * i + 2 * j + 1]);
+                u[j] = *reinterpret_cast<uint32_t*>(&pr);
+            }
+            d[i] = make_uint4(u[0], u[1], u[2], u[3]);
         }
     }
 }
@@ -100,20 +96,18 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
     const int E = p.E, NE = E * TV;
+    const int CB = 3 * 64 * E + 16;            // floats per coefficient block
     uint8_t* sKQ = sm;                         // 2 blocks x [K rows 0-63 | Q rows 64-127] x 128 B
-    uint8_t* sA2 = sKQ + 2 * 2 * kBoxBytes;    // [T; A T] 128 x 64 bf16: hi tile, lo tile
-    uint8_t* sReg = sA2 + 4 * kBoxBytes;       // shared region, 2 * NE * 256 bytes:
-    uint8_t* sSh = sReg;                       //   S_all^T [NE][dk] hi  (MMA-A operand)
-    uint8_t* sSl = sReg + NE * 256;            //   S_all^T [NE][dk] lo
+    uint8_t* sA2 = sKQ + 4 * kBoxBytes;        // [T; A T] 128 x 64 bf16: hi tile, lo tile
+    uint8_t* sReg = sA2 + 4 * kBoxBytes;       // shared region, NE * 512 bytes:
+    uint8_t* sSh = sReg;                       //   S_all [dk][NE] hi, MN-major (MMA-A operand)
+    uint8_t* sSl = sReg + NE * 256;            //   S_all lo
     uint8_t* sRh = sReg;                       //   Res^T [TV][64] hi, lo (after MMA-A)
     uint8_t* sRl = sReg + TV * 128;
-    uint8_t* sUh = sReg + TV * 256;            //   Ut^T [NE][64] hi, lo (after MMA-B)
+    uint8_t* sUh = sReg + TV * 256;            //   Ut [64][NE] hi, lo, MN-major (after MMA-B)
     uint8_t* sUl = sUh + NE * 128;
     __nv_bfloat16* sV = reinterpret_cast<__nv_bfloat16*>(sReg + NE * 512);  // [64][TV]
-    float* ae = reinterpret_cast<float*>(sReg + NE * 512 + 64 * TV * 2);
-    float* be = ae + 64 * E;
-    float* we = be + 64 * E;
-    float* gcn = we + 64 * E;                  // gamma^C of the chunk whose coefficients are loaded
+    float* sCoef = reinterpret_cast<float*>(sReg + NE * 512 + 64 * TV * 2);  // 2 x CB
 
     __shared__ __align__(8) uint64_t bar_kq, bar_av, bar_mma;
     __shared__ uint32_t tmem_slot;
@@ -141,7 +135,7 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    const uint32_t tP = tmem_slot;        // columns [0, NE): P, then D2 in [0, TV)
+    const uint32_t tP = tmem_slot;        // columns [0, NE): P, then [U; Oa] in [0, TV)
     const uint32_t tS = tmem_slot + NE;   // columns [NE, 2 NE): the state slab
 
     auto issue_kq = [&](int c) {
@@ -151,32 +145,20 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             tma_load_4d(sKQ + j * 2 * kBoxBytes + kBoxBytes, &map_q, &bar_kq, 64 * j, h, c * 64, b);
         }
     };
+    // [T; A T] hi/lo and V of chunk c, and its coefficient block into buffer c & 1
     auto issue_av = [&](int c) {
-        mbar_arrive_expect_tx(&bar_av, 4 * kBoxBytes + 64 * TV * 2);
-        tma_load_2d(sA2, &map_a2, &bar_av, 0, ((b * H + h) * NT + c) * 256);
-        tma_load_2d(sA2 + 2 * kBoxBytes, &map_a2, &bar_av, 0, ((b * H + h) * NT + c) * 256 + 128);
+        const size_t idx = size_t(b * H + h) * NT + c;
+        mbar_arrive_expect_tx(&bar_av, 4 * kBoxBytes + 64 * TV * 2 + CB * 4);
+        tma_load_2d(sA2, &map_a2, &bar_av, 0, int(idx * 256));
+        tma_load_2d(sA2 + 2 * kBoxBytes, &map_a2, &bar_av, 0, int(idx * 256 + 128));
         tma_load_4d(sV, &map_v, &bar_av, n0, h, c * 64, b);
+        bulk_load(sCoef + (c & 1) * CB, p.coef + idx * CB, CB * 4, &bar_av);
     };
-    auto load_coefs = [&](int c) {
-        const int t0 = c * 64, n = min(64, T - t0);
-        for (int i = tid; i < 64 * E; i += kThreads) {
-            const int r = i / E, e = i - (i / E) * E;
-            const int rr = r < n ? r : n - 1;
-            const float Gr = p.G[tok_idx(b, t0 + rr, h, e, T, H, E)];
-            const float GC = p.G[tok_idx(b, t0 + n - 1, h, e, T, H, E)];
-            const float kk = r < n ? __bfloat162float(p.k2[tok_idx(b, t0 + r, h, e, T, H, E)]) : 0.f;
-            const float qq = r < n ? __bfloat162float(p.q2[tok_idx(b, t0 + r, h, e, T, H, E)]) : 0.f;
-            const float gam = expf(Gr);
-            ae[i] = kk * gam;
-            be[i] = qq * gam;
-            we[i] = kk * expf(GC - Gr);
-            if (r == 0) gcn[e] = expf(GC);
-        }
-    };
-    // State row d = tid of S_{[c]}: bf16 copy for MMA-A, checkpoint, and
-    // gamma^C_c-scaled copy in TMEM for the accumulation of chunk c.
+    // Row d = tid of S_{[c]}: operand of MMA-A, checkpoint, and the gamma^C_c-scaled
+    // copy in TMEM for the accumulation of chunk c.
     auto prepare = [&](int c, bool from_h0) {
         const int d = tid;
+        const float* gc = sCoef + (c & 1) * CB + 3 * 64 * E;
         for (int e = 0; e < E; ++e) {
             float v[TV];
             if (from_h0) {
@@ -198,11 +180,11 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                 tmem_wait_ld();
             }
 #pragma unroll
-            for (int n = 0; n < TV; ++n) st_split(sSh, sSl, sw128_offset(e * TV + n, d, NE), v[n]);
+            for (int n = 0; n < TV; n += 8) st8_split(sSh, sSl, sw128_offset(d, e * TV + n, kDk), v + n);
             if (p.save)
                 store_f32_row(p.Sck + ((((size_t(b) * H + h) * NT + c) * E + e) * kDk + d) * dv + n0,
                               v, TV);
-            const float g = gcn[e];
+            const float g = gc[e];
 #pragma unroll
             for (int n = 0; n < TV; ++n) v[n] *= g;
 #pragma unroll
@@ -211,41 +193,43 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         tmem_wait_st();
     };
 
+    bool failed = false;
+    uint32_t mma_phase = 0;
+    int pending_mma = 0;
     if (tid == 0) {
         issue_kq(0);
         issue_av(0);
     }
-    load_coefs(0);
-    __syncthreads();
-    prepare(0, true);
-    fence_proxy_async_smem();
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
+    if (!mbar_wait(&bar_av, 0)) failed = true;
+    if (__syncthreads_or(failed)) failed = true;
+    if (!failed) {
+        prepare(0, true);
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        tc_fence_after();
+    }
 
-    uint32_t mma_phase = 0;
-    bool failed = false;
-    int pending_kq = 0, pending_av = 0, pending_mma = 0;  // outstanding async work (tid 0 view)
-    for (int c = 0; c < NT; ++c) {
+    for (int c = 0; c < NT && !failed; ++c) {
         const int t0 = c * 64, n = min(64, T - t0);
-        pending_kq = pending_av = 1;
+        const float* cf = sCoef + (c & 1) * CB;
+        const float* ae = cf;
+        const float* be = cf + 64 * E;
+        const float* we = cf + 128 * E;
         bool ok = mbar_wait(&bar_kq, c & 1);
-        if (ok) pending_kq = 0;
-        ok = ok && mbar_wait(&bar_av, c & 1);
-        if (ok) pending_av = 0;
         if (__syncthreads_or(!ok)) { failed = true; break; }
         tc_fence_after();
 
-        // ---- MMA-A: P = [K; Q] S_all
+        // ---- MMA-A: P = [K; Q] S_all    (B = S_all, MN-major, hi and lo)
         if (tid == 0) {
-            const uint32_t idesc = idesc_bf16_f32(128, NE, 0, 0);
+            const uint32_t idesc = idesc_bf16_f32(128, NE, 0, 1);
 #pragma unroll
             for (int ks = 0; ks < kDk / 16; ++ks) {
                 const int blk = ks >> 2, kk = (ks & 3) * 16;
                 const uint64_t ad = smem_desc(smem_u32(sKQ) + blk * 2 * kBoxBytes + kk * 2, 16, 1024);
-                const uint32_t bo = blk * NE * 128 + kk * 2;
-                umma_bf16(tP, ad, smem_desc(smem_u32(sSh) + bo, 16, 1024), idesc, ks > 0 ? 1u : 0u);
-                umma_bf16(tP, ad, smem_desc(smem_u32(sSl) + bo, 16, 1024), idesc, 1u);
+                umma_bf16(tP, ad, smem_desc(smem_u32(sSh) + ks * 2048, kDk * 128, 1024), idesc,
+                          ks > 0 ? 1u : 0u);
+                umma_bf16(tP, ad, smem_desc(smem_u32(sSl) + ks * 2048, kDk * 128, 1024), idesc, 1u);
             }
             umma_commit(&bar_mma);
         }
@@ -260,9 +244,21 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         float oi[TV];
         if (warp < 2) {
             const int r = tid;
-            float w[TV];
+            float res[TV];
+            {
+                const uint4* vrow = reinterpret_cast<const uint4*>(sV + r * TV);
 #pragma unroll
-            for (int i = 0; i < TV; ++i) w[i] = 0.f;
+                for (int i = 0; i < TV / 8; ++i) {
+                    uint4 u = vrow[i];
+                    const __nv_bfloat162* pr = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        float2 f = __bfloat1622float2(pr[j]);
+                        res[8 * i + 2 * j] = f.x;
+                        res[8 * i + 2 * j + 1] = f.y;
+                    }
+                }
+            }
             if (p.use_delta) {
                 for (int e = 0; e < E; ++e) {
                     float pv[TV];
@@ -271,15 +267,11 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                     tmem_wait_ld();
                     const float a = ae[r * E + e];
 #pragma unroll
-                    for (int i = 0; i < TV; ++i) w[i] = fmaf(a, pv[i], w[i]);
+                    for (int i = 0; i < TV; ++i) res[i] = fmaf(-a, pv[i], res[i]);
                 }
             }
-            float res[TV];
 #pragma unroll
-            for (int i = 0; i < TV; ++i) {
-                res[i] = __bfloat162float(sV[r * TV + i]) - w[i];
-                st_split(sRh, sRl, sw128_offset(i, r, TV), res[i]);
-            }
+            for (int i = 0; i < TV; ++i) st_split(sRh, sRl, sw128_offset(i, r, TV), res[i]);
             if (p.save && p.use_delta && r < n)
                 store_f32_row(p.Rbuf + tok_idx(b, t0 + r, h, n0, T, H, dv), res, TV);
         } else {
@@ -322,7 +314,7 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         if (__syncthreads_or(!ok)) { failed = true; break; }
         pending_mma = 0;
         tc_fence_after();
-        if (tid == 0 && c + 1 < NT) issue_av(c + 1);   // [T; A T] and V buffers are free
+        if (tid == 0 && c + 1 < NT) issue_av(c + 1);   // [T; A T], V and the other coef buffer are free
 
         // ---- epi-B
         {
@@ -334,8 +326,11 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                 const int r = tid;
                 for (int e = 0; e < E; ++e) {
                     const float wv = we[r * E + e];
+                    float u[TV];
 #pragma unroll
-                    for (int i = 0; i < TV; ++i) st_split(sUh, sUl, sw128_offset(e * TV + i, r, NE), wv * d2[i]);
+                    for (int i = 0; i < TV; ++i) u[i] = wv * d2[i];
+#pragma unroll
+                    for (int i = 0; i < TV; i += 8) st8_split(sUh, sUl, sw128_offset(r, e * TV + i, 64), u + i);
                 }
                 if (p.save && r < n) store_f32_row(p.Ubuf + tok_idx(b, t0 + r, h, n0, T, H, dv), d2, TV);
             } else {
@@ -350,21 +345,21 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         __syncthreads();
         tc_fence_after();
 
-        // ---- MMA-C: S_all += K^T Ut   (A = K^T, MN-major from the key rows of sKQ)
+        // ---- MMA-C: S_all += K^T Ut   (A = K^T MN-major from the key rows; B = Ut MN-major)
         if (tid == 0) {
-            const uint32_t idesc = idesc_bf16_f32(128, NE, 1, 0);
+            const uint32_t idesc = idesc_bf16_f32(128, NE, 1, 1);
 #pragma unroll
             for (int ks = 0; ks < 4; ++ks) {
                 const uint64_t ad = smem_desc(smem_u32(sKQ) + ks * 2048, 2 * kBoxBytes, 1024);
-                umma_bf16(tS, ad, smem_desc(smem_u32(sUh) + ks * 32, 16, 1024), idesc, 1u);
-                umma_bf16(tS, ad, smem_desc(smem_u32(sUl) + ks * 32, 16, 1024), idesc, 1u);
+                umma_bf16(tS, ad, smem_desc(smem_u32(sUh) + ks * 2048, 64 * 128, 1024), idesc, 1u);
+                umma_bf16(tS, ad, smem_desc(smem_u32(sUl) + ks * 2048, 64 * 128, 1024), idesc, 1u);
             }
             umma_commit(&bar_mma);
         }
         pending_mma = 1;
-        if (c + 1 < NT) load_coefs(c + 1);   // overlaps MMA-C; chunk c's coefficients are done
         ok = mbar_wait(&bar_mma, mma_phase);
         mma_phase ^= 1;
+        if (c + 1 < NT) ok = ok && mbar_wait(&bar_av, (c + 1) & 1);   // chunk c+1's gamma^C
         if (__syncthreads_or(!ok)) { failed = true; break; }
         pending_mma = 0;
         tc_fence_after();
@@ -390,14 +385,12 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     }
 
     if (failed) {
-        // Bounded drain of whatever this CTA still has in flight, then leave.
+        // Bounded drain of products still in flight, then leave (copies that never
+        // complete expire with the same bound in the waits above).
         if (tid == 0) {
             record_device_error(p.err, TLA_ERR_TIMEOUT);
             if (pending_mma) mbar_wait(&bar_mma, mma_phase ^ 1);
         }
-        __syncthreads();
-        (void)pending_kq;
-        (void)pending_av;
     }
     tc_fence_before();
     __syncthreads();
@@ -408,7 +401,7 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
 template <int TV>
 size_t tc_fwd_smem(int E) {
     const int NE = E * TV;
-    return 1024 + 4 * kBoxBytes + 4 * kBoxBytes + NE * 512 + 64 * TV * 2 + (3 * 64 * E + E) * 4;
+    return 1024 + 4 * kBoxBytes + 4 * kBoxBytes + NE * 512 + 64 * TV * 2 + 2 * (3 * 64 * E + 16) * 4;
 }
 
 template <int TV>
@@ -422,9 +415,7 @@ cudaError_t launch_tv(const tla_problem& p, const FwdPlan& fp, char* ws, int sav
         !make_matrix_map(&ma, ws + fp.A2, (long long)p.B * p.H * NT * 256, 64, 64, 128))
         return cudaErrorInvalidValue;
     TcFwdArgs a;
-    a.q2 = (const __nv_bfloat16*)p.q2;
-    a.k2 = (const __nv_bfloat16*)p.k2;
-    a.G = (const float*)(ws + fp.G);
+    a.coef = (const float*)(ws + fp.coef);
     a.h0 = p.h0;
     a.o = p.o;
     a.ht = p.ht;
@@ -446,17 +437,26 @@ cudaError_t launch_tv(const tla_problem& p, const FwdPlan& fp, char* ws, int sav
 
 }  // namespace
 
+// Value columns per CTA of the tensor-core recurrence (0: not eligible).  The
+// state and Ut operands are MN-major with 64-column swizzle atoms, so E * TV must
+// be a multiple of 64 (and at most 256, the widest UMMA and half of TMEM).
 int tc_fwd_tv(const tla_problem& p) {
     if (p.dtype != TLA_BF16 || p.dk != kDk) return 0;
-    const int tv = p.E <= 4 ? 32 : 16;
-    if (p.dv % tv != 0 || p.E * tv > 256) return 0;
-    return tv;
+    const int cand[3] = {32, 16, 64};
+    for (int tv : cand) {
+        const int ne = p.E * tv;
+        if (p.dv % tv == 0 && ne % 64 == 0 && ne <= 256) return tv;
+    }
+    return 0;
 }
 
 cudaError_t launch_fwd_recurrence_tc(const tla_problem& p, const FwdPlan& fp, char* ws,
                                      int save_for_bwd, int* err, cudaStream_t s) {
-    return fp.tc_tv == 32 ? launch_tv<32>(p, fp, ws, save_for_bwd, err, s)
-                          : launch_tv<16>(p, fp, ws, save_for_bwd, err, s);
+    switch (fp.tc_tv) {
+        case 16: return launch_tv<16>(p, fp, ws, save_for_bwd, err, s);
+        case 32: return launch_tv<32>(p, fp, ws, save_for_bwd, err, s);
+        default: return launch_tv<64>(p, fp, ws, save_for_bwd, err, s);
+    }
 }
 
 }  // namespace tla

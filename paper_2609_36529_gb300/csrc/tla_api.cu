@@ -67,7 +67,11 @@ FwdPlan plan_fwd(const tla_problem& p, int save) {
     f.G = off; off = align256(off + tokE);
     f.A = off; off = align256(off + mats);
     if (p.use_delta) { f.N = off; off = align256(off + mats); }
-    if (f.tc_tv) { f.A2 = off; off = align256(off + 2 * mats); }   // hi + lo 128 x 64 bf16 tiles
+    if (f.tc_tv) {
+        f.A2 = off; off = align256(off + 2 * mats);   // hi + lo 128 x 64 bf16 tiles
+        f.coef = off;
+        off = align256(off + (size_t)p.B * p.H * f.NT * (3 * kChunk * p.E + 16) * 4);
+    }
     if (save) {
         f.S = off; off = align256(off + states);
         f.U = off; off = align256(off + tokV);
@@ -161,7 +165,7 @@ tla_status tla_chunk_fwd(const tla_problem* p, void* workspace, size_t workspace
         e = launch_chunk_prep(*p, (const float*)(ws + fp.G), (float*)(ws + fp.A),
                               p->use_delta ? (float*)(ws + fp.N) : nullptr,
                               (fp.tc_tv && tc_eligible(*p)) ? (__nv_bfloat16*)(ws + fp.A2) : nullptr,
-                              s);
+                              (fp.tc_tv && tc_eligible(*p)) ? (float*)(ws + fp.coef) : nullptr, s);
     if (e == cudaSuccess) {
         if (fp.tc_tv && tc_eligible(*p))
             e = launch_fwd_recurrence_tc(*p, fp, ws, save, device_error_word(), s);
