@@ -19,7 +19,9 @@
  *    stated otherwise; the caller owns every buffer, including workspaces.
  *    The library allocates no device memory.
  *  - All tensors are dense, row-major, contiguous.  Token tensors use the
- *    layout [B, T, H, D]; states use [B, H, E, dk, dv].
+ *    layout [B, T, H, D]; states use [B, H, E, dk, dv].  Every pointer must be
+ *    16-byte aligned (PyTorch and cudaMalloc allocations are); an unaligned
+ *    pointer is rejected with TLA_ERR_INVALID_ARG.
  *  - `dtype` (tla_dtype) is the element type of q, k, v, q2, k2; `out_dtype`
  *    that of o and of their gradients.  Log-gates g, beta, states h0/ht/dh0,
  *    dg and dbeta are fp32.  Arithmetic accumulates in fp32 throughout.
@@ -128,8 +130,8 @@ tla_status tla_chunk_bwd(const tla_problem *p, const void *fwd_ws, size_t fwd_ws
  *   q, k [B,H,dk] dtype; v [B,H,dv] dtype; q2, k2 [B,H,E] dtype;
  *   g [B,H,E] fp32; beta [B,H] fp32 or NULL (=> 1; required if use_delta);
  *   state [B,H,E,dk,dv] fp32, updated in place; o [B,H,dv] dtype (written).
- * Supported: dk, dv multiples of 16 up to 128, 1 <= E <= 16; state must be
- * 16-byte aligned.  No workspace.
+ * Supported: dk, dv multiples of 16 up to 128, 1 <= E <= 16, B*H <= 65535.
+ * No workspace.
  */
 tla_status tla_decode_step(int B, int H, int dk, int dv, int E, int use_delta, int dtype,
                            const void *q, const void *k, const void *v,

@@ -22,6 +22,8 @@ struct FwdPlan {
     size_t Res;          // fp32 [B,T,H,dv] residual V - W (save_for_bwd, delta rule)
     size_t A2;           // bf16 [B,H,NT,2,128,64] [T; A T] hi and lo tiles (tensor-core path)
     size_t coef;         // fp32 [B,H,NT,3*64*E+16] per-row coefficients (tensor-core path)
+    size_t BT;           // bf16 [B,H,NT,4,64,64] A^T, T^T hi/lo (tensor-core backward)
+    int tcb;             // 1: the backward recurrence runs on tensor cores
     int tc_tv;           // value columns per CTA of the tensor-core recurrence (0: SIMT)
     size_t bytes;        // total
 };
@@ -52,7 +54,13 @@ BwdPlan plan_bwd(const tla_problem& p);
 // SIMT path (fp32 arithmetic on CUDA cores; any supported dtype).
 cudaError_t launch_gate_cumsum(const tla_problem& p, float* G, cudaStream_t s);
 cudaError_t launch_chunk_prep(const tla_problem& p, const float* G, float* A, float* N,
-                              __nv_bfloat16* A2, float* coef, cudaStream_t s);
+                              __nv_bfloat16* A2, float* coef, __nv_bfloat16* BT, cudaStream_t s);
+// Tensor-core backward recurrence (requires the tensor-core forward layout).
+int tc_bwd_ok(const tla_problem& p, int tv);
+cudaError_t launch_bwd_recurrence_tc(const tla_problem& p, const FwdPlan& fp, const char* fws,
+                                     const BwdPlan& bp, char* bws, const void* dO,
+                                     const float* dht, void* dv, float* dh0, int* err,
+                                     cudaStream_t s);
 
 // Tensor-core path (bf16 inputs, dk = 128): value columns per CTA, or 0 if not eligible.
 int tc_fwd_tv(const tla_problem& p);

@@ -59,7 +59,8 @@ chunk_prep_kernel(const Tin* __restrict__ q, const Tin* __restrict__ k, const Ti
                   const Tin* __restrict__ k2, const float* __restrict__ G,
                   const float* __restrict__ beta, float* __restrict__ Aout,
                   float* __restrict__ Nout, __nv_bfloat16* __restrict__ A2out,
-                  float* __restrict__ coef_out, int T, int H, int dk, int E, int use_delta) {
+                  float* __restrict__ coef_out, __nv_bfloat16* __restrict__ BTout, int T, int H,
+                  int dk, int E, int use_delta) {
     const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
     const int NT = gridDim.x;
     const int tid = threadIdx.x;
@@ -182,6 +183,24 @@ chunk_prep_kernel(const Tin* __restrict__ q, const Tin* __restrict__ k, const Ti
             A2out[m2 + 3 * kChunk * kChunk + i] = __float2bfloat16_rn(at - __bfloat162float(ath));
         }
     }
+    if (BTout) {
+        // Operands of the tensor-core backward recurrence as bf16 pairs, 64 x 64 each:
+        // [A^T hi | A^T lo | T^T hi | T^T lo], A^T[r][s] = A[s][r], T^T[r][s] = T[s][r].
+        const size_t m4 = ((size_t(b) * H + h) * NT + c) * (4 * kChunk * kChunk);
+        for (int i = tid; i < kChunk * kChunk; i += blockDim.x) {
+            const int r = i >> 6, s = i & 63;   // element (r, s) of the transposes
+            float at = 0.f, tt = 0.f;
+            if (s >= r) {
+                at = As[s * 65 + r];
+                tt = (use_delta ? Xs[s * 65 + r] : (s == r ? 1.f : 0.f)) * bs[r];
+            }
+            const __nv_bfloat16 ah = __float2bfloat16_rn(at), th = __float2bfloat16_rn(tt);
+            BTout[m4 + i] = ah;
+            BTout[m4 + kChunk * kChunk + i] = __float2bfloat16_rn(at - __bfloat162float(ah));
+            BTout[m4 + 2 * kChunk * kChunk + i] = th;
+            BTout[m4 + 3 * kChunk * kChunk + i] = __float2bfloat16_rn(tt - __bfloat162float(th));
+        }
+    }
 }
 
 static size_t prep_smem(const tla_problem& p) {
@@ -189,7 +208,7 @@ static size_t prep_smem(const tla_problem& p) {
 }
 
 cudaError_t launch_chunk_prep(const tla_problem& p, const float* G, float* A, float* N,
-                              __nv_bfloat16* A2, float* coef, cudaStream_t s) {
+                              __nv_bfloat16* A2, float* coef, __nv_bfloat16* BT, cudaStream_t s) {
     int NT = (p.T + kChunk - 1) / kChunk;
     dim3 grid(NT, p.H, p.B);
     size_t smem = prep_smem(p);
@@ -199,13 +218,13 @@ cudaError_t launch_chunk_prep(const tla_problem& p, const float* G, float* A, fl
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         kern<<<grid, 256, smem, s>>>((const __nv_bfloat16*)p.q, (const __nv_bfloat16*)p.k,
                                      (const __nv_bfloat16*)p.q2, (const __nv_bfloat16*)p.k2, G,
-                                     p.beta, A, N, A2, coef, p.T, p.H, p.dk, p.E, p.use_delta);
+                                     p.beta, A, N, A2, coef, BT, p.T, p.H, p.dk, p.E, p.use_delta);
     } else {
         auto kern = chunk_prep_kernel<float>;
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         kern<<<grid, 256, smem, s>>>((const float*)p.q, (const float*)p.k, (const float*)p.q2,
-                                     (const float*)p.k2, G, p.beta, A, N, nullptr, nullptr, p.T,
-                                     p.H, p.dk, p.E, p.use_delta);
+                                     (const float*)p.k2, G, p.beta, A, N, nullptr, nullptr, nullptr,
+                                     p.T, p.H, p.dk, p.E, p.use_delta);
     }
     prof_after(s);
     return cudaGetLastError();

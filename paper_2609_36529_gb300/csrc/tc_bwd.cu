@@ -1,0 +1,432 @@
+// Tensor-core (tcgen05) backward recurrence over chunks (Appendix A, Kernels: a
+// reverse pass over the chunks yields the gradient of every state slice at
+// each chunk boundary; the remaining gradients follow chunk-parallel).
+//
+// Differentiating the chunk step of Eq. joint-chunk (see tc_fwd.cu) gives, per
+// chunk c walked backwards, with dS' the gradient of the state at the chunk's end:
+//   dU   = A^T dO + sum_e diag(w_e) K dS'_e
+//   dRes = T^T dU                                   (= dV)
+//   dS_e = gamma^C_e dS'_e + Q^T diag(b_e) dO - K^T diag(a_e) dRes
+// One CTA of 4 warps per (b, h, block of TV value columns) keeps dS for its
+// value columns in TMEM.  Per chunk:
+//   MMA-A'  P' = K dS'_all              (M=64, N=NE, K=dk; dS' MN-major hi/lo)
+//   MMA-0   Y  = A^T dO                 (M=64, N=TV, K=64; A^T hi/lo, dO exact bf16)
+//   epi     dU = Y + sum_e w_e (.) P'_e  -> dU^T hi/lo operand, dU to the workspace
+//   MMA-B'  dRes = T^T dU               (M=64, N=TV, K=64; both hi/lo)
+//   epi     dRes -> workspace and dv; operand rows [-a_e (.) dRes ; b_e (.) dO]
+//   MMA-C'  dS_all += [K^T | Q^T] [-a (.) dRes ; b (.) dO]   (M=dk=128, K=128, N=NE;
+//           K^T and Q^T read MN-major from the TMA key/query tile)
+//   epi     dS_{[c]} from TMEM -> operand of the previous chunk, checkpoint, and
+//           pre-scaled by gamma^C of the previous chunk.
+// Layout of the M=64 products in TMEM: row r sits on lane 32 * (r / 16) + r % 16,
+// so lanes 0-15 of each warp own the row work and lanes 16-31 prepare dO.
+// Precision, TMA prefetch and bounded waits as in the forward kernel.
+#include "common.cuh"
+#include "internal.h"
+#include "sm100.cuh"
+#include "tc_common.cuh"
+#include "tma_host.h"
+
+namespace tla {
+using namespace sm100;
+
+namespace {
+
+constexpr int kThreads = 128;
+constexpr int kDk = 128;
+constexpr int kBoxBytes = 64 * 64 * 2;
+
+struct TcBwdArgs {
+    const float* coef;   // forward workspace coefficient blocks [B,H,NT, 3*64*E+16]
+    const float* dht;
+    void* dv_out;
+    float* dh0;
+    float* dUbuf;
+    float* dRbuf;
+    float* dSck;
+    int* err;
+    int T, H, dv, E, NT, use_delta, out_f32;
+};
+
+template <int TV>
+__global__ void __launch_bounds__(kThreads, 1)
+bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
+                         const __grid_constant__ CUtensorMap map_q,
+                         const __grid_constant__ CUtensorMap map_do,
+                         const __grid_constant__ CUtensorMap map_bt, const TcBwdArgs p) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+    const int E = p.E, NE = E * TV;
+    const int CB = 3 * 64 * E + 16;
+    uint8_t* sKQ = sm;                       // 2 blocks x [K rows | Q rows] x 128 B
+    uint8_t* sBT = sKQ + 4 * kBoxBytes;      // A^T hi, A^T lo, T^T hi, T^T lo (64 x 64 each)
+    uint8_t* sReg = sBT + 4 * kBoxBytes;     // NE * 512 bytes, reused:
+    uint8_t* sDh = sReg;                     //   dS' [dk][NE] hi / lo, MN-major (MMA-A')
+    uint8_t* sDl = sReg + NE * 256;
+    uint8_t* sUh = sReg;                     //   dU^T [TV][64] hi / lo (MMA-B')
+    uint8_t* sUl = sReg + TV * 128;
+    uint8_t* sBh = sReg;                     //   [-a dRes ; b dO] [128][NE] hi / lo (MMA-C')
+    uint8_t* sBl = sReg + NE * 256;
+    uint8_t* sOT = sReg + NE * 512;          // dO^T [TV][64] bf16 (MMA-0)
+    __nv_bfloat16* sdO = reinterpret_cast<__nv_bfloat16*>(sOT + TV * 128);   // [64][TV] (TMA)
+    float* sCoef = reinterpret_cast<float*>(sOT + TV * 128 + 64 * TV * 2);   // 2 x CB
+
+    __shared__ __align__(8) uint64_t bar_kq, bar_av, bar_mma;
+    __shared__ uint32_t tmem_slot;
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int nb = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+    const int n0 = nb * TV;
+    const int T = p.T, H = p.H, dv = p.dv, NT = p.NT;
+    const uint32_t tcols = (2 * NE + TV <= 256) ? 256u : 512u;
+    // M=64 row owned by this thread (lanes 0-15) or prepared by it (lanes 16-31)
+    const bool row_thread = lane < 16;
+    const int r64 = 16 * warp + (lane & 15);
+
+    if (warp == 0) {
+        tmem_alloc(&tmem_slot, tcols);
+        tmem_relinquish();
+    }
+    if (tid == 0) {
+        mbar_init(&bar_kq, 1);
+        mbar_init(&bar_av, 1);
+        mbar_init(&bar_mma, 1);
+        fence_barrier_init();
+        tma_prefetch_desc(&map_k);
+        tma_prefetch_desc(&map_q);
+        tma_prefetch_desc(&map_do);
+        tma_prefetch_desc(&map_bt);
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tP = tmem_slot;             // [0, NE): K dS'
+    const uint32_t tY = tmem_slot + NE;        // [NE, NE+TV): A^T dO, then dRes
+    const uint32_t tS = tmem_slot + NE + TV;   // [NE+TV, 2 NE+TV): dS
+
+    auto issue_kq = [&](int c) {
+        mbar_arrive_expect_tx(&bar_kq, 4 * kBoxBytes);
+        for (int j = 0; j < 2; ++j) {
+            tma_load_4d(sKQ + j * 2 * kBoxBytes, &map_k, &bar_kq, 64 * j, h, c * 64, b);
+            tma_load_4d(sKQ + j * 2 * kBoxBytes + kBoxBytes, &map_q, &bar_kq, 64 * j, h, c * 64, b);
+        }
+    };
+    auto issue_av = [&](int c) {
+        const size_t idx = size_t(b * H + h) * NT + c;
+        mbar_arrive_expect_tx(&bar_av, 4 * kBoxBytes + 64 * TV * 2 + CB * 4);
+        for (int j = 0; j < 4; ++j) tma_load_2d(sBT + j * kBoxBytes, &map_bt, &bar_av, 0, int(idx * 256 + 64 * j));
+        tma_load_4d(sdO, &map_do, &bar_av, n0, h, c * 64, b);
+        bulk_load(sCoef + (c & 1) * CB, p.coef + idx * CB, CB * 4, &bar_av);
+    };
+    // Row d = tid of the gradient at the end of chunk c: operand of MMA-A'(c),
+    // checkpoint for the chunk-parallel gradients, and gamma^C_c-scaled copy in TMEM.
+    auto prepare = [&](int c, bool from_dht) {
+        const int d = tid;
+        const float* gc = sCoef + (c & 1) * CB + 3 * 64 * E;
+        for (int e = 0; e < E; ++e) {
+            float v[TV];
+            if (from_dht) {
+                if (p.dht) {
+                    const float4* src = reinterpret_cast<const float4*>(
+                        p.dht + ((size_t(b * H + h) * E + e) * kDk + d) * dv + n0);
+#pragma unroll
+                    for (int i = 0; i < TV / 4; ++i) {
+                        float4 x = src[i];
+                        v[4 * i] = x.x; v[4 * i + 1] = x.y; v[4 * i + 2] = x.z; v[4 * i + 3] = x.w;
+                    }
+                } else {
+#pragma unroll
+                    for (int i = 0; i < TV; ++i) v[i] = 0.f;
+                }
+            } else {
+#pragma unroll
+                for (int j = 0; j < TV; j += 16) tmem_ld16(tmem_lane_addr(tS, warp, e * TV + j), v + j);
+                tmem_wait_ld();
+            }
+#pragma unroll
+            for (int n = 0; n < TV; n += 8) st8_split(sDh, sDl, sw128_offset(d, e * TV + n, kDk), v + n);
+            store_f32_row(p.dSck + ((((size_t(b) * H + h) * NT + c) * E + e) * kDk + d) * dv + n0, v, TV);
+            const float g = gc[e];
+#pragma unroll
+            for (int n = 0; n < TV; ++n) v[n] *= g;
+#pragma unroll
+            for (int j = 0; j < TV; j += 16) tmem_st16(tmem_lane_addr(tS, warp, e * TV + j), v + j);
+        }
+        tmem_wait_st();
+    };
+
+    bool failed = false;
+    uint32_t mma_phase = 0;
+    int pending_mma = 0;
+    if (tid == 0) {
+        issue_kq(NT - 1);
+        issue_av(NT - 1);
+    }
+    if (!mbar_wait(&bar_av, 0)) failed = true;
+    if (__syncthreads_or(failed)) failed = true;
+    if (!failed) {
+        prepare(NT - 1, true);
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        tc_fence_after();
+    }
+
+    for (int c = NT - 1; c >= 0 && !failed; --c) {
+        const int it = NT - 1 - c;                 // iteration index (barrier phases)
+        const int t0 = c * 64, n = min(64, T - t0);
+        const float* cf = sCoef + (c & 1) * CB;
+        const float* ae = cf;
+        const float* be = cf + 64 * E;
+        const float* we = cf + 128 * E;
+        bool ok = mbar_wait(&bar_kq, it & 1);
+        if (__syncthreads_or(!ok)) { failed = true; break; }
+        tc_fence_after();
+
+        // ---- step 1 (lanes 16-31): dO row -> registers and dO^T operand of MMA-0
+        float dorow[TV];
+        if (!row_thread) {
+            const uint4* src = reinterpret_cast<const uint4*>(sdO + r64 * TV);
+#pragma unroll
+            for (int i = 0; i < TV / 8; ++i) {
+                uint4 u = src[i];
+                const __nv_bfloat16* pb = reinterpret_cast<const __nv_bfloat16*>(&u);
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    *reinterpret_cast<__nv_bfloat16*>(sOT + sw128_offset(8 * i + j, r64, TV)) = pb[j];
+                    dorow[8 * i + j] = __bfloat162float(pb[j]);
+                }
+            }
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        tc_fence_after();
+
+        // ---- MMA-A' (P' = K dS') and MMA-0 (Y = A^T dO)
+        if (tid == 0) {
+            const uint32_t ida = idesc_bf16_f32(64, NE, 0, 1);
+#pragma unroll
+            for (int ks = 0; ks < kDk / 16; ++ks) {
+                const int blk = ks >> 2, kk = (ks & 3) * 16;
+                const uint64_t ad = smem_desc(smem_u32(sKQ) + blk * 2 * kBoxBytes + kk * 2, 16, 1024);
+                umma_bf16(tP, ad, smem_desc(smem_u32(sDh) + ks * 2048, kDk * 128, 1024), ida,
+                          ks > 0 ? 1u : 0u);
+                umma_bf16(tP, ad, smem_desc(smem_u32(sDl) + ks * 2048, kDk * 128, 1024), ida, 1u);
+            }
+            const uint32_t id0 = idesc_bf16_f32(64, TV, 0, 0);
+#pragma unroll
+            for (int ks = 0; ks < 4; ++ks) {
+                const uint64_t bd = smem_desc(smem_u32(sOT) + ks * 32, 16, 1024);
+                umma_bf16(tY, smem_desc(smem_u32(sBT) + ks * 32, 16, 1024), bd, id0, ks > 0 ? 1u : 0u);
+                umma_bf16(tY, smem_desc(smem_u32(sBT) + kBoxBytes + ks * 32, 16, 1024), bd, id0, 1u);
+            }
+            umma_commit(&bar_mma);
+        }
+        pending_mma = 1;
+        ok = mbar_wait(&bar_mma, mma_phase);
+        mma_phase ^= 1;
+        if (__syncthreads_or(!ok)) { failed = true; break; }
+        pending_mma = 0;
+        tc_fence_after();
+
+        // ---- dU = Y + sum_e w_e (.) P'_e   (row threads)
+        {
+            float du[TV];
+#pragma unroll
+            for (int j = 0; j < TV; j += 16) tmem_ld16(tmem_lane_addr(tY, warp, j), du + j);
+            tmem_wait_ld();
+            for (int e = 0; e < E; ++e) {
+                float pv[TV];
+#pragma unroll
+                for (int j = 0; j < TV; j += 16) tmem_ld16(tmem_lane_addr(tP, warp, e * TV + j), pv + j);
+                tmem_wait_ld();
+                const float wv = row_thread ? we[r64 * E + e] : 0.f;
+#pragma unroll
+                for (int i = 0; i < TV; ++i) du[i] = fmaf(wv, pv[i], du[i]);
+            }
+            if (row_thread) {
+#pragma unroll
+                for (int i = 0; i < TV; ++i) st_split(sUh, sUl, sw128_offset(i, r64, TV), du[i]);
+                if (r64 < n) store_f32_row(p.dUbuf + tok_idx(b, t0 + r64, h, n0, T, H, dv), du, TV);
+            }
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        tc_fence_after();
+
+        // ---- MMA-B': dRes = T^T dU   (into tY)
+        if (tid == 0) {
+            const uint32_t idb = idesc_bf16_f32(64, TV, 0, 0);
+#pragma unroll
+            for (int ks = 0; ks < 4; ++ks) {
+                const uint64_t th = smem_desc(smem_u32(sBT) + 2 * kBoxBytes + ks * 32, 16, 1024);
+                const uint64_t tl = smem_desc(smem_u32(sBT) + 3 * kBoxBytes + ks * 32, 16, 1024);
+                const uint64_t uh = smem_desc(smem_u32(sUh) + ks * 32, 16, 1024);
+                const uint64_t ul = smem_desc(smem_u32(sUl) + ks * 32, 16, 1024);
+                umma_bf16(tY, th, uh, idb, ks > 0 ? 1u : 0u);
+                umma_bf16(tY, th, ul, idb, 1u);
+                umma_bf16(tY, tl, uh, idb, 1u);
+            }
+            umma_commit(&bar_mma);
+        }
+        pending_mma = 1;
+        ok = mbar_wait(&bar_mma, mma_phase);
+        mma_phase ^= 1;
+        if (__syncthreads_or(!ok)) { failed = true; break; }
+        pending_mma = 0;
+        tc_fence_after();
+        if (tid == 0 && c > 0) issue_av(c - 1);   // A^T/T^T tiles, dO tile, other coef buffer free
+
+        // ---- operand rows of MMA-C': [-a_e (.) dRes ; b_e (.) dO]
+        {
+            float dr[TV];
+#pragma unroll
+            for (int j = 0; j < TV; j += 16) tmem_ld16(tmem_lane_addr(tY, warp, j), dr + j);
+            tmem_wait_ld();
+            if (row_thread) {
+                if (r64 < n) {
+                    const size_t off = tok_idx(b, t0 + r64, h, n0, T, H, dv);
+                    store_f32_row(p.dRbuf + off, dr, TV);
+                    store_row(p.dv_out, off, dr, TV, p.out_f32);
+                }
+                if (p.use_delta) {
+                    for (int e = 0; e < E; ++e) {
+                        const float a = -ae[r64 * E + e];
+                        float x[TV];
+#pragma unroll
+                        for (int i = 0; i < TV; ++i) x[i] = a * dr[i];
+#pragma unroll
+                        for (int i = 0; i < TV; i += 8) st8_split(sBh, sBl, sw128_offset(r64, e * TV + i, 128), x + i);
+                    }
+                }
+            } else {
+                for (int e = 0; e < E; ++e) {
+                    const float bq = be[r64 * E + e];
+                    float x[TV];
+#pragma unroll
+                    for (int i = 0; i < TV; ++i) x[i] = bq * dorow[i];
+#pragma unroll
+                    for (int i = 0; i < TV; i += 8)
+                        st8_split(sBh, sBl, sw128_offset(64 + r64, e * TV + i, 128), x + i);
+                }
+            }
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        tc_fence_after();
+
+        // ---- MMA-C': dS += [K^T | Q^T] [-a dRes ; b dO]   (sGLA: query half only)
+        if (tid == 0) {
+            const uint32_t idc = idesc_bf16_f32(128, NE, 1, 1);
+            for (int ks = p.use_delta ? 0 : 4; ks < 8; ++ks) {
+                const uint64_t ad = smem_desc(smem_u32(sKQ) + ks * 2048, 2 * kBoxBytes, 1024);
+                umma_bf16(tS, ad, smem_desc(smem_u32(sBh) + ks * 2048, 128 * 128, 1024), idc, 1u);
+                umma_bf16(tS, ad, smem_desc(smem_u32(sBl) + ks * 2048, 128 * 128, 1024), idc, 1u);
+            }
+            umma_commit(&bar_mma);
+        }
+        pending_mma = 1;
+        ok = mbar_wait(&bar_mma, mma_phase);
+        mma_phase ^= 1;
+        if (c > 0) ok = ok && mbar_wait(&bar_av, (it + 1) & 1);   // gamma^C of chunk c-1
+        if (__syncthreads_or(!ok)) { failed = true; break; }
+        pending_mma = 0;
+        tc_fence_after();
+        if (tid == 0 && c > 0) issue_kq(c - 1);
+
+        if (c > 0) {
+            prepare(c - 1, false);
+        } else if (p.dh0) {
+            const int d = tid;
+            for (int e = 0; e < E; ++e) {
+                float v[TV];
+#pragma unroll
+                for (int j = 0; j < TV; j += 16) tmem_ld16(tmem_lane_addr(tS, warp, e * TV + j), v + j);
+                tmem_wait_ld();
+                store_f32_row(p.dh0 + ((size_t(b * H + h) * E + e) * kDk + d) * dv + n0, v, TV);
+            }
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        tc_fence_after();
+    }
+
+    if (failed && tid == 0) {
+        record_device_error(p.err, TLA_ERR_TIMEOUT);
+        if (pending_mma) mbar_wait(&bar_mma, mma_phase ^ 1);
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 0) tmem_dealloc(tmem_slot, tcols);
+}
+
+template <int TV>
+size_t tc_bwd_smem(int E) {
+    const int NE = E * TV;
+    return 1024 + 8 * kBoxBytes + NE * 512 + TV * 128 + 64 * TV * 2 + 2 * (3 * 64 * E + 16) * 4;
+}
+
+template <int TV>
+cudaError_t launch_tv(const tla_problem& p, const FwdPlan& fp, const char* fws, const BwdPlan& bp,
+                      char* bws, const void* dO, const float* dht, void* dv, float* dh0, int* err,
+                      cudaStream_t s) {
+    CUtensorMap mk, mq, mo, mb;
+    const int NT = fp.NT;
+    if (!make_token_map(&mk, p.k, p.B, p.T, p.H, kDk, 64, 64, true) ||
+        !make_token_map(&mq, p.q, p.B, p.T, p.H, kDk, 64, 64, true) ||
+        !make_token_map(&mo, dO, p.B, p.T, p.H, p.dv, TV, 64, false) ||
+        !make_matrix_map(&mb, fws + fp.BT, (long long)p.B * p.H * NT * 256, 64, 64, 64))
+        return cudaErrorInvalidValue;
+    TcBwdArgs a;
+    a.coef = (const float*)(fws + fp.coef);
+    a.dht = dht;
+    a.dv_out = dv;
+    a.dh0 = dh0;
+    a.dUbuf = (float*)(bws + bp.dU);
+    a.dRbuf = (float*)(bws + bp.dRes);
+    a.dSck = (float*)(bws + bp.dS);
+    a.err = err;
+    a.T = p.T; a.H = p.H; a.dv = p.dv; a.E = p.E; a.NT = NT;
+    a.use_delta = p.use_delta; a.out_f32 = p.out_dtype == TLA_FP32;
+    const size_t smem = tc_bwd_smem<TV>(p.E);
+    auto kern = bwd_recurrence_tc_kernel<TV>;
+    cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    dim3 grid(p.dv / TV, p.H, p.B);
+    prof_before("bwd_recurrence_tc", s);
+    kern<<<grid, kThreads, smem, s>>>(mk, mq, mo, mb, a);
+    prof_after(s);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+// The backward recurrence runs on tensor cores when the forward used them and
+// the dS slab, the M=64 products and their operands fit TMEM (512 columns) and
+// shared memory.
+int tc_bwd_ok(const tla_problem& p, int tv) {
+    if (tv == 0) return 0;
+    const int ne = p.E * tv;
+    if (2 * ne + tv > 512) return 0;
+    const size_t smem = tv == 16 ? tc_bwd_smem<16>(p.E) : tv == 32 ? tc_bwd_smem<32>(p.E)
+                                                                   : tc_bwd_smem<64>(p.E);
+    return smem <= 227 * 1024 ? 1 : 0;
+}
+
+cudaError_t launch_bwd_recurrence_tc(const tla_problem& p, const FwdPlan& fp, const char* fws,
+                                     const BwdPlan& bp, char* bws, const void* dO,
+                                     const float* dht, void* dv, float* dh0, int* err,
+                                     cudaStream_t s) {
+    switch (fp.tc_tv) {
+        case 16: return launch_tv<16>(p, fp, fws, bp, bws, dO, dht, dv, dh0, err, s);
+        case 32: return launch_tv<32>(p, fp, fws, bp, bws, dO, dht, dv, dh0, err, s);
+        default: return launch_tv<64>(p, fp, fws, bp, bws, dO, dht, dv, dh0, err, s);
+    }
+}
+
+}  // namespace tla

@@ -33,6 +33,7 @@
 #include "common.cuh"
 #include "internal.h"
 #include "sm100.cuh"
+#include "tc_common.cuh"
 #include "tma_host.h"
 
 namespace tla {
@@ -55,36 +56,6 @@ struct TcFwdArgs {
     int* err;
     int T, H, dv, E, NT, use_delta, save, out_f32;
 };
-
-__device__ __forceinline__ void store_row(void* base, size_t off, const float* v, int n,
-                                          int out_f32) {
-    if (out_f32) {
-        float4* d = reinterpret_cast<float4*>(static_cast<float*>(base) + off);
-        for (int i = 0; i < n / 4; ++i) d[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
-    } else {
-        uint4* d = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(base) + off);
-        for (int i = 0; i < n / 8; ++i) {
-            uint32_t u[4];
-            for (int j = 0; j < 4; ++j) {
-                __nv_bfloat162 pr = __floats2bfloat162_rn(v[8 * i + 2 * j], v[8 * i + 2 * j + 1]);
-                u[j] = *reinterpret_cast<uint32_t*>(&pr);
-            }
-            d[i] = make_uint4(u[0], u[1], u[2], u[3]);
-        }
-    }
-}
-
-__device__ __forceinline__ void store_f32_row(float* dst, const float* v, int n) {
-    float4* d = reinterpret_cast<float4*>(dst);
-    for (int i = 0; i < n / 4; ++i) d[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
-}
-
-// Store v as a bf16 pair: hi = bf16(v) into tile_hi, lo = bf16(v - hi) into tile_lo.
-__device__ __forceinline__ void st_split(uint8_t* tile_hi, uint8_t* tile_lo, uint32_t off, float v) {
-    const __nv_bfloat16 hi = __float2bfloat16_rn(v);
-    *reinterpret_cast<__nv_bfloat16*>(tile_hi + off) = hi;
-    *reinterpret_cast<__nv_bfloat16*>(tile_lo + off) = __float2bfloat16_rn(v - __bfloat162float(hi));
-}
 
 template <int TV>
 __global__ void __launch_bounds__(kThreads, 1)

@@ -15,6 +15,8 @@ __device__ int g_device_error = 0;
 
 static size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
+static bool aligned16(const void* x) { return ((uintptr_t)x & 15) == 0; }
+
 static bool dims_ok(int d) { return d >= 16 && d <= 128 && d % 16 == 0; }
 
 static tla_status validate(const tla_problem* p) {
@@ -28,21 +30,20 @@ static tla_status validate(const tla_problem* p) {
     if (p->chunk != kChunk) return TLA_ERR_UNSUPPORTED;
     if (!dims_ok(p->dk) || !dims_ok(p->dv) || p->E > 16) return TLA_ERR_UNSUPPORTED;
     if (p->H > 65535 || p->B > 65535) return TLA_ERR_UNSUPPORTED;
+    const void* ptrs[] = {p->q, p->k, p->v, p->q2, p->k2, p->g, p->beta, p->h0, p->o, p->ht};
+    for (const void* x : ptrs)
+        if (!aligned16(x)) return TLA_ERR_INVALID_ARG;
     return TLA_OK;
 }
 
-static bool aligned16(const void* x) { return ((uintptr_t)x & 15) == 0; }
 
-// The tensor-core path reads q, k, v by TMA and writes rows with 16-byte stores.
-static bool tc_eligible(const tla_problem& p) {
-    return aligned16(p.q) && aligned16(p.k) && aligned16(p.v) && aligned16(p.o) &&
-           aligned16(p.h0) && aligned16(p.ht);
-}
-
+// Address of the error word on the current device (looked up once per device).
 static int* device_error_word() {
-    static int* ptr = nullptr;
-    if (!ptr) cudaGetSymbolAddress((void**)&ptr, g_device_error);
-    return ptr;
+    static int* ptr[64] = {nullptr};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+    if (!ptr[dev]) cudaGetSymbolAddress((void**)&ptr[dev], g_device_error);
+    return ptr[dev];
 }
 
 // Value columns per CTA of the SIMT recurrences: the E x dk x tv fp32 slab
@@ -71,6 +72,8 @@ FwdPlan plan_fwd(const tla_problem& p, int save) {
         f.A2 = off; off = align256(off + 2 * mats);   // hi + lo 128 x 64 bf16 tiles
         f.coef = off;
         off = align256(off + (size_t)p.B * p.H * f.NT * (3 * kChunk * p.E + 16) * 4);
+        f.tcb = (save && tc_bwd_ok(p, f.tc_tv)) ? 1 : 0;
+        if (f.tcb) { f.BT = off; off = align256(off + 2 * mats); }
     }
     if (save) {
         f.S = off; off = align256(off + states);
@@ -164,10 +167,12 @@ tla_status tla_chunk_fwd(const tla_problem* p, void* workspace, size_t workspace
     if (e == cudaSuccess)
         e = launch_chunk_prep(*p, (const float*)(ws + fp.G), (float*)(ws + fp.A),
                               p->use_delta ? (float*)(ws + fp.N) : nullptr,
-                              (fp.tc_tv && tc_eligible(*p)) ? (__nv_bfloat16*)(ws + fp.A2) : nullptr,
-                              (fp.tc_tv && tc_eligible(*p)) ? (float*)(ws + fp.coef) : nullptr, s);
+                              fp.tc_tv ? (__nv_bfloat16*)(ws + fp.A2) : nullptr,
+                              fp.tc_tv ? (float*)(ws + fp.coef) : nullptr,
+                              fp.tcb ? (__nv_bfloat16*)(ws + fp.BT) : nullptr,
+                              s);
     if (e == cudaSuccess) {
-        if (fp.tc_tv && tc_eligible(*p))
+        if (fp.tc_tv)
             e = launch_fwd_recurrence_tc(*p, fp, ws, save, device_error_word(), s);
         else e = launch_fwd_recurrence(*p, fp, ws, save, s);
     }
@@ -181,6 +186,11 @@ tla_status tla_chunk_bwd(const tla_problem* p, const void* fwd_ws, size_t fwd_ws
     tla_status st = validate(p);
     if (st != TLA_OK) return st;
     if (!dO || !dq || !dk || !dv || !dq2 || !dk2 || !dg) return TLA_ERR_INVALID_ARG;
+    {
+        const void* ptrs[] = {dO, dht, dq, dk, dv, dq2, dk2, dbeta, dg, dh0};
+        for (const void* x : ptrs)
+            if (!aligned16(x)) return TLA_ERR_INVALID_ARG;
+    }
     if ((p->beta != nullptr) != (dbeta != nullptr)) return TLA_ERR_INVALID_ARG;
     if ((p->h0 != nullptr) != (dh0 != nullptr)) return TLA_ERR_INVALID_ARG;
     FwdPlan fp = plan_fwd(*p, 1);
@@ -191,7 +201,9 @@ tla_status tla_chunk_bwd(const tla_problem* p, const void* fwd_ws, size_t fwd_ws
     cudaStream_t s = (cudaStream_t)stream;
     const char* fws = (const char*)fwd_ws;
     char* bws = (char*)workspace;
-    cudaError_t e = launch_bwd_recurrence(*p, fp, fws, bp, bws, dO, dht, dv, dh0, s);
+    cudaError_t e = fp.tcb ? launch_bwd_recurrence_tc(*p, fp, fws, bp, bws, dO, dht, dv, dh0,
+                                                      device_error_word(), s)
+                           : launch_bwd_recurrence(*p, fp, fws, bp, bws, dO, dht, dv, dh0, s);
     if (e == cudaSuccess)
         e = launch_bwd_chunk_grads(*p, fp, fws, bp, bws, dO, dq, dk, dq2, dk2, dbeta, dg, s);
     return cuda_status(e);
@@ -206,7 +218,11 @@ tla_status tla_decode_step(int B, int H, int dk, int dv, int E, int use_delta, i
     if (use_delta != 0 && use_delta != 1) return TLA_ERR_INVALID_ARG;
     if (!q || !k || !v || !q2 || !k2 || !g || !state || !o) return TLA_ERR_INVALID_ARG;
     if (use_delta && !beta) return TLA_ERR_INVALID_ARG;
-    if (((uintptr_t)state & 15) != 0) return TLA_ERR_INVALID_ARG;
+    {
+        const void* ptrs[] = {q, k, v, q2, k2, g, beta, state, o};
+        for (const void* x : ptrs)
+            if (!aligned16(x)) return TLA_ERR_INVALID_ARG;
+    }
     if (!dims_ok(dk) || !dims_ok(dv) || E > 16) return TLA_ERR_UNSUPPORTED;
     if ((long long)B * H > 65535) return TLA_ERR_UNSUPPORTED;  // grid.y
     return cuda_status(launch_decode_step(B, H, dk, dv, E, use_delta, dtype, q, k, v, q2, k2, g,

@@ -187,6 +187,24 @@ def test_bwd_small(dtype, use_delta, T):
         close(n, grads[n], ref[n], TOL[dtype], rel_l2=0.01 if dtype == "bf16" else None)
 
 
+@pytest.mark.parametrize("use_delta", [True, False])
+@pytest.mark.parametrize("T,E,dv", [(1, 4, 64), (64, 2, 64), (65, 4, 128), (200, 8, 64),
+                                    (130, 1, 64)])
+def test_bwd_tensor_core_path(use_delta, T, E, dv):
+    """bf16, dk = 128: tcgen05 forward and backward recurrences (+ chunk gradients)."""
+    x = inputs.chunk_inputs(2, T, 2, 128, dv, E, dtype="bf16", with_beta=True, h0_std=0.1,
+                            backward=True, device="cuda", seed=1000 + T * 7 + E)
+    dht = 0.5 * torch.randn(2, 2, E, 128, dv, device="cuda",
+                            generator=torch.Generator("cuda").manual_seed(T + E))
+    _, _, grads = run_bwd(x, use_delta, dht)
+    torch.cuda.synchronize()
+    assert tla.tla_last_device_status() == 0
+    ref = oracle_bwd(x, use_delta, dht)
+    assert set(ref) == set(grads)
+    for n in ref:
+        close(n, grads[n], ref[n], TOL["bf16"], rel_l2=0.01)
+
+
 def test_bwd_sgla_no_beta_no_h0():
     x = inputs.chunk_inputs(1, 150, 2, 32, 32, 4, dtype="fp32", with_beta=False, backward=True,
                             device="cuda", seed=11)
