@@ -55,6 +55,12 @@ BwdPlan plan_bwd(const tla_problem& p);
 cudaError_t launch_gate_cumsum(const tla_problem& p, float* G, cudaStream_t s);
 cudaError_t launch_chunk_prep(const tla_problem& p, const float* G, float* A, float* N,
                               __nv_bfloat16* A2, float* coef, __nv_bfloat16* BT, cudaStream_t s);
+// Tensor-core chunk-parallel gradients (requires the tensor-core backward recurrence).
+int tc_grads_ok(const tla_problem& p, const FwdPlan& fp);
+cudaError_t launch_bwd_chunk_grads_tc(const tla_problem& p, const FwdPlan& fp, const char* fws,
+                                      const BwdPlan& bp, const char* bws, const void* dO,
+                                      void* dq, void* dk, void* dq2, void* dk2, float* dbeta,
+                                      float* dg, int* err, cudaStream_t s);
 // Tensor-core backward recurrence (requires the tensor-core forward layout).
 int tc_bwd_ok(const tla_problem& p, int tv);
 cudaError_t launch_bwd_recurrence_tc(const tla_problem& p, const FwdPlan& fp, const char* fws,

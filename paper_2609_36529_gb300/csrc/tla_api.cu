@@ -204,8 +204,13 @@ tla_status tla_chunk_bwd(const tla_problem* p, const void* fwd_ws, size_t fwd_ws
     cudaError_t e = fp.tcb ? launch_bwd_recurrence_tc(*p, fp, fws, bp, bws, dO, dht, dv, dh0,
                                                       device_error_word(), s)
                            : launch_bwd_recurrence(*p, fp, fws, bp, bws, dO, dht, dv, dh0, s);
-    if (e == cudaSuccess)
-        e = launch_bwd_chunk_grads(*p, fp, fws, bp, bws, dO, dq, dk, dq2, dk2, dbeta, dg, s);
+    if (e == cudaSuccess) {
+        if (tc_grads_ok(*p, fp))
+            e = launch_bwd_chunk_grads_tc(*p, fp, fws, bp, bws, dO, dq, dk, dq2, dk2, dbeta, dg,
+                                          device_error_word(), s);
+        else
+            e = launch_bwd_chunk_grads(*p, fp, fws, bp, bws, dO, dq, dk, dq2, dk2, dbeta, dg, s);
+    }
     return cuda_status(e);
 }
 
