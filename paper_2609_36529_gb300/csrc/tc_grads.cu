@@ -140,9 +140,10 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     if (tid < 16) dgc[tid] = 0.f;
 
     // ---- phase 0 staging: U -> sX (hi, lo); dU, Res (sGLA: V) -> sY (hi, lo, hi, lo)
-    {
-        const int r = tid & 63, qd = tid >> 6, cw = dv / 4;
-        for (int cc = qd * cw; cc < (qd + 1) * cw; cc += 8) {
+    // (8-column chunks; consecutive threads take consecutive chunks of a row)
+    for (int ci = tid; ci < 64 * (dv / 8); ci += kThreads) {
+        const int r = ci / (dv / 8), cc = (ci % (dv / 8)) * 8;
+        {
             float u[8], du[8], rs[8];
             if (r < n) {
                 const size_t off = tok_idx(b, t0 + r, h, cc, T, H, dv);
@@ -421,16 +422,17 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     for (int e = 0; e < E && !failed; ++e) {
         const float* Se = p.Sck + (sbase + e) * kDk * dv;
         const float* dSe = p.dSck + (sbase + e) * kDk * dv;
+        const int cpr = dv / 8;   // 8-column chunks per row
         // stage S_e -> sX (hi/lo, [128 d][dv]) and A1_e = [b_e dO ; -a_e dRes] -> sY
         {
-            const int d = tid & 127, hf = tid >> 7;
-            for (int cc = hf * dv / 2; cc < (hf + 1) * dv / 2; cc += 8) {
+            for (int ci = tid; ci < 128 * cpr; ci += kThreads) {
+                const int d = ci / cpr, cc = (ci % cpr) * 8;
                 float v[8];
                 load_row8(Se + d * dv + cc, v);
                 st8_split(sX, sX + 32768, sw128_offset(d, cc, 128), v);
             }
-            const int i = d;
-            for (int cc = hf * dv / 2; cc < (hf + 1) * dv / 2; cc += 8) {
+            for (int ci = tid; ci < 128 * cpr; ci += kThreads) {
+                const int i = ci / cpr, cc = (ci % cpr) * 8;
                 float v[8];
                 if (i < 64) {
                     const float bq = q2s[i * E + e] * expf(Gs[i * E + e]);
@@ -478,9 +480,9 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         tc_fence_after();
         // stage dS'_e -> sX and A2_e = [0 ; w_e U] -> sY; Frobenius partial <dS'_e, S_e>
         {
-            const int d = tid & 127, hf = tid >> 7;
             float fro = 0.f;
-            for (int cc = hf * dv / 2; cc < (hf + 1) * dv / 2; cc += 8) {
+            for (int ci = tid; ci < 128 * cpr; ci += kThreads) {
+                const int d = ci / cpr, cc = (ci % cpr) * 8;
                 float v[8], sv[8];
                 load_row8(dSe + d * dv + cc, v);
                 load_row8(Se + d * dv + cc, sv);
@@ -488,8 +490,8 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                 st8_split(sX, sX + 32768, sw128_offset(d, cc, 128), v);
             }
             red2[tid] = fro;
-            const int i = d;
-            for (int cc = hf * dv / 2; cc < (hf + 1) * dv / 2; cc += 8) {
+            for (int ci = tid; ci < 128 * cpr; ci += kThreads) {
+                const int i = ci / cpr, cc = (ci % cpr) * 8;
                 float v[8];
                 const int r = i - 64;
                 if (i >= 64 && r < n) {

@@ -164,13 +164,14 @@ tla_status tla_chunk_fwd(const tla_problem* p, void* workspace, size_t workspace
     cudaStream_t s = (cudaStream_t)stream;
     char* ws = (char*)workspace;
     cudaError_t e = launch_gate_cumsum(*p, (float*)(ws + fp.G), s);
-    if (e == cudaSuccess)
-        e = launch_chunk_prep(*p, (const float*)(ws + fp.G), (float*)(ws + fp.A),
-                              p->use_delta ? (float*)(ws + fp.N) : nullptr,
-                              fp.tc_tv ? (__nv_bfloat16*)(ws + fp.A2) : nullptr,
-                              fp.tc_tv ? (float*)(ws + fp.coef) : nullptr,
-                              fp.tcb ? (__nv_bfloat16*)(ws + fp.BT) : nullptr,
-                              s);
+    if (e == cudaSuccess) {
+        if (fp.tc_tv)
+            e = launch_chunk_prep_tc(*p, fp, ws, device_error_word(), s);
+        else
+            e = launch_chunk_prep(*p, (const float*)(ws + fp.G), (float*)(ws + fp.A),
+                                  p->use_delta ? (float*)(ws + fp.N) : nullptr, nullptr, nullptr,
+                                  nullptr, s);
+    }
     if (e == cudaSuccess) {
         if (fp.tc_tv)
             e = launch_fwd_recurrence_tc(*p, fp, ws, save, device_error_word(), s);
