@@ -277,18 +277,18 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         for (int i = tid; i < 64 * 64; i += kThreads) B0[(i >> 6) * MP + (i & 63)] = p.Nmat[mat + i];
     float Rv[16], Rq[16];
 #pragma unroll
-    for (int j = 0; j < 16; ++j) {
-        const int r = r_base + 4 * j, s = s_own;
-        float R = 0.f, Q = 0.f;
-        if (r >= s)
-            for (int e = 0; e < E; ++e) {
-                const float gam = expf(Gs[r * E + e] - Gs[s * E + e]);
-                const float ks2 = k2s[s * E + e] * gam;
-                R = fmaf(k2s[r * E + e], ks2, R);
-                Q = fmaf(q2s[r * E + e], ks2, Q);
-            }
-        Rv[j] = R;
-        Rq[j] = Q;
+    for (int j = 0; j < 16; ++j) Rv[j] = Rq[j] = 0.f;
+    for (int e = 0; e < E; ++e) {            // 16 independent entries per slice
+        const float gs = Gs[s_own * E + e], ks = k2s[s_own * E + e];
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+            const int r = r_base + 4 * j;
+            // exp of a non-positive difference (entries above the diagonal are discarded)
+            const float gam = expf(fminf(Gs[r * E + e] - gs, 0.f));
+            const float ks2 = (r >= s_own) ? ks * gam : 0.f;
+            Rv[j] = fmaf(k2s[r * E + e], ks2, Rv[j]);
+            Rq[j] = fmaf(q2s[r * E + e], ks2, Rq[j]);
+        }
     }
     __syncthreads();
     if (p.use_delta) {
@@ -304,21 +304,32 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             for (int r = 0; r < 64; ++r) acc += B2[r * MP + tid];
             dba[tid] += acc;
         }
+        {                                               // F = dN N^T (16 independent sums)
+            float acc[16];
 #pragma unroll
-        for (int j = 0; j < 16; ++j) {                  // F = dN N^T
-            const int r = r_base + 4 * j, s = s_own;
-            float acc = 0.f;
-            for (int x = 0; x < 64; ++x) acc = fmaf(B1[r * MP + x], B0[s * MP + x], acc);
-            B3[r * MP + s] = acc;
+            for (int j = 0; j < 16; ++j) acc[j] = 0.f;
+#pragma unroll 4
+            for (int x = 0; x < 64; ++x) {
+                const float nsx = B0[s_own * MP + x];
+#pragma unroll
+                for (int j = 0; j < 16; ++j) acc[j] = fmaf(B1[(r_base + 4 * j) * MP + x], nsx, acc[j]);
+            }
+#pragma unroll
+            for (int j = 0; j < 16; ++j) B3[(r_base + 4 * j) * MP + s_own] = acc[j];
         }
         __syncthreads();
         float dL[16];
+        {                                               // dM = -N^T F, strictly lower part
 #pragma unroll
-        for (int j = 0; j < 16; ++j) {                  // dM = -N^T F, strictly lower part
-            const int r = r_base + 4 * j, s = s_own;
-            float acc = 0.f;
-            for (int x = 0; x < 64; ++x) acc = fmaf(B0[x * MP + r], B3[x * MP + s], acc);
-            dL[j] = (r > s) ? -acc : 0.f;
+            for (int j = 0; j < 16; ++j) dL[j] = 0.f;
+#pragma unroll 4
+            for (int x = 0; x < 64; ++x) {
+                const float fxs = B3[x * MP + s_own];
+#pragma unroll
+                for (int j = 0; j < 16; ++j) dL[j] = fmaf(B0[x * MP + r_base + 4 * j], fxs, dL[j]);
+            }
+#pragma unroll
+            for (int j = 0; j < 16; ++j) dL[j] = (r_base + 4 * j > s_own) ? -dL[j] : 0.f;
         }
         __syncthreads();
 #pragma unroll
@@ -425,11 +436,18 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         const int cpr = dv / 8;   // 8-column chunks per row
         // stage S_e -> sX (hi/lo, [128 d][dv]) and A1_e = [b_e dO ; -a_e dRes] -> sY
         {
-            for (int ci = tid; ci < 128 * cpr; ci += kThreads) {
-                const int d = ci / cpr, cc = (ci % cpr) * 8;
-                float v[8];
-                load_row8(Se + d * dv + cc, v);
-                st8_split(sX, sX + 32768, sw128_offset(d, cc, 128), v);
+            for (int c0 = tid; c0 < 128 * cpr; c0 += 4 * kThreads) {   // 4 chunks in flight
+                float v[4][8];
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    const int ci = c0 + k * kThreads;
+                    if (ci < 128 * cpr) load_row8(Se + (ci / cpr) * dv + (ci % cpr) * 8, v[k]);
+                }
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    const int ci = c0 + k * kThreads;
+                    if (ci < 128 * cpr) st8_split(sX, sX + 32768, sw128_offset(ci / cpr, (ci % cpr) * 8, 128), v[k]);
+                }
             }
             for (int ci = tid; ci < 128 * cpr; ci += kThreads) {
                 const int i = ci / cpr, cc = (ci % cpr) * 8;
@@ -481,13 +499,24 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         // stage dS'_e -> sX and A2_e = [0 ; w_e U] -> sY; Frobenius partial <dS'_e, S_e>
         {
             float fro = 0.f;
-            for (int ci = tid; ci < 128 * cpr; ci += kThreads) {
-                const int d = ci / cpr, cc = (ci % cpr) * 8;
-                float v[8], sv[8];
-                load_row8(dSe + d * dv + cc, v);
-                load_row8(Se + d * dv + cc, sv);
-                for (int u = 0; u < 8; ++u) fro = fmaf(v[u], sv[u], fro);
-                st8_split(sX, sX + 32768, sw128_offset(d, cc, 128), v);
+            for (int c0 = tid; c0 < 128 * cpr; c0 += 2 * kThreads) {   // 2 chunks (x2 tensors) in flight
+                float v[2][8], sv[2][8];
+#pragma unroll
+                for (int k = 0; k < 2; ++k) {
+                    const int ci = c0 + k * kThreads;
+                    if (ci < 128 * cpr) {
+                        load_row8(dSe + (ci / cpr) * dv + (ci % cpr) * 8, v[k]);
+                        load_row8(Se + (ci / cpr) * dv + (ci % cpr) * 8, sv[k]);
+                    }
+                }
+#pragma unroll
+                for (int k = 0; k < 2; ++k) {
+                    const int ci = c0 + k * kThreads;
+                    if (ci < 128 * cpr) {
+                        for (int u = 0; u < 8; ++u) fro = fmaf(v[k][u], sv[k][u], fro);
+                        st8_split(sX, sX + 32768, sw128_offset(ci / cpr, (ci % cpr) * 8, 128), v[k]);
+                    }
+                }
             }
             red2[tid] = fro;
             for (int ci = tid; ci < 128 * cpr; ci += kThreads) {
