@@ -24,6 +24,10 @@ struct FwdPlan {
     size_t coef;         // fp32 [B,H,NT,3*64*E+16] per-row coefficients (tensor-core path)
     size_t BT;           // bf16 [B,H,NT,4,64,64] A^T, T^T hi/lo (tensor-core backward)
     int tcb;             // 1: the backward recurrence runs on tensor cores
+    int ck_tiles;        // 1: state checkpoints (forward S, backward dS) are stored as bf16
+                         //    hi/lo pairs in the chunk-gradient kernel's operand layout:
+                         //    per (b,h,chunk,e) a [dk][dv] hi tile then a lo tile, 128-byte
+                         //    swizzled K-major (same 4 bytes per element as fp32)
     int tc_tv;           // value columns per CTA of the tensor-core recurrence (0: SIMT)
     size_t bytes;        // total
 };
@@ -60,6 +64,7 @@ cudaError_t launch_chunk_prep_tc(const tla_problem& p, const FwdPlan& fp, char* 
                                  cudaStream_t s);
 // Tensor-core chunk-parallel gradients (requires the tensor-core backward recurrence).
 int tc_grads_ok(const tla_problem& p, const FwdPlan& fp);
+int tc_grads_shape_ok(const tla_problem& p);
 cudaError_t launch_bwd_chunk_grads_tc(const tla_problem& p, const FwdPlan& fp, const char* fws,
                                       const BwdPlan& bp, const char* bws, const void* dO,
                                       void* dq, void* dk, void* dq2, void* dk2, float* dbeta,

@@ -45,7 +45,7 @@ struct TcBwdArgs {
     float* dRbuf;
     float* dSck;
     int* err;
-    int T, H, dv, E, NT, use_delta, out_f32;
+    int T, H, dv, E, NT, use_delta, out_f32, ck_tiles;
 };
 
 template <int TV>
@@ -146,7 +146,17 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             }
 #pragma unroll
             for (int n = 0; n < TV; n += 8) st8_split(sDh, sDl, sw128_offset(d, e * TV + n, kDk), v + n);
-            store_f32_row(p.dSck + ((((size_t(b) * H + h) * NT + c) * E + e) * kDk + d) * dv + n0, v, TV);
+            {
+                const size_t slab = (((size_t(b) * H + h) * NT + c) * E + e) * kDk * dv;
+                if (p.ck_tiles) {   // bf16 hi/lo tiles in the gradient kernel's layout
+                    uint8_t* hi = reinterpret_cast<uint8_t*>(p.dSck + slab);
+                    uint8_t* lo = hi + kDk * dv * 2;
+#pragma unroll
+                    for (int n = 0; n < TV; n += 8) st8_split(hi, lo, sw128_offset(d, n0 + n, kDk), v + n);
+                } else {
+                    store_f32_row(p.dSck + slab + size_t(d) * dv + n0, v, TV);
+                }
+            }
             const float g = gc[e];
 #pragma unroll
             for (int n = 0; n < TV; ++n) v[n] *= g;
@@ -394,6 +404,7 @@ cudaError_t launch_tv(const tla_problem& p, const FwdPlan& fp, const char* fws, 
     a.err = err;
     a.T = p.T; a.H = p.H; a.dv = p.dv; a.E = p.E; a.NT = NT;
     a.use_delta = p.use_delta; a.out_f32 = p.out_dtype == TLA_FP32;
+    a.ck_tiles = fp.ck_tiles;
     const size_t smem = tc_bwd_smem<TV>(p.E);
     auto kern = bwd_recurrence_tc_kernel<TV>;
     cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);

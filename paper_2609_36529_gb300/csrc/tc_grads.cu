@@ -106,7 +106,7 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     float* red = dgc + 16;                     // [2][128] row-dot halves
     float* red2 = red + 256;                   // [256]
 
-    __shared__ __align__(8) uint64_t bar_ld, bar_mma;
+    __shared__ __align__(8) uint64_t bar_ld, bar_mma, bar_s, bar_d;
     __shared__ uint32_t tmem_slot;
 
     if (warp == 0) {
@@ -116,6 +116,8 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     if (tid == 0) {
         mbar_init(&bar_ld, 1);
         mbar_init(&bar_mma, 1);
+        mbar_init(&bar_s, 1);
+        mbar_init(&bar_d, 1);
         fence_barrier_init();
         mbar_arrive_expect_tx(&bar_ld, 4 * kBoxBytes + (dv / 64) * kBoxBytes);
         for (int j = 0; j < 2; ++j) {
@@ -426,52 +428,45 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     }
     tc_fence_after();
 
-    // ---- phase 2: per slice
+    // ---- phase 2: per slice.  The checkpoint tiles (bf16 hi/lo, operand layout) arrive by
+    // bulk copy: S_e into sX, then dS'_e into sY once the first products have consumed A1.
     const size_t sbase = ((size_t(b) * H + h) * NT + c) * E;
+    const uint32_t slab_bytes = uint32_t(kDk) * dv * 4;   // hi tile + lo tile
+    const uint32_t LO = uint32_t(kDk) * dv * 2;           // lo tile offset of a checkpoint slab
     const int wq = warp & 3, L = wq * 32 + lane, half = warp >> 2;
+    const int cpr = dv / 8;   // 8-column chunks per row
+    uint32_t sph = 0, dph = 0;
+    if (tid == 0) {
+        mbar_arrive_expect_tx(&bar_s, slab_bytes);
+        bulk_load(sX, reinterpret_cast<const uint8_t*>(p.Sck) + sbase * kDk * dv * 4, slab_bytes, &bar_s);
+    }
     bool failed = false;
     for (int e = 0; e < E && !failed; ++e) {
-        const float* Se = p.Sck + (sbase + e) * kDk * dv;
-        const float* dSe = p.dSck + (sbase + e) * kDk * dv;
-        const int cpr = dv / 8;   // 8-column chunks per row
-        // stage S_e -> sX (hi/lo, [128 d][dv]) and A1_e = [b_e dO ; -a_e dRes] -> sY
-        {
-            for (int c0 = tid; c0 < 128 * cpr; c0 += 4 * kThreads) {   // 4 chunks in flight
-                float v[4][8];
-#pragma unroll
-                for (int k = 0; k < 4; ++k) {
-                    const int ci = c0 + k * kThreads;
-                    if (ci < 128 * cpr) load_row8(Se + (ci / cpr) * dv + (ci % cpr) * 8, v[k]);
-                }
-#pragma unroll
-                for (int k = 0; k < 4; ++k) {
-                    const int ci = c0 + k * kThreads;
-                    if (ci < 128 * cpr) st8_split(sX, sX + 32768, sw128_offset(ci / cpr, (ci % cpr) * 8, 128), v[k]);
-                }
-            }
-            for (int ci = tid; ci < 128 * cpr; ci += kThreads) {
-                const int i = ci / cpr, cc = (ci % cpr) * 8;
-                float v[8];
-                if (i < 64) {
-                    const float bq = q2s[i * E + e] * expf(Gs[i * E + e]);
-                    load_bf16x8(sDO + sw128_offset(i, cc, 64), v);
-                    for (int u = 0; u < 8; ++u) v[u] *= bq;
+        // A1_e = [b_e dO ; -a_e dRes] -> sY
+        for (int ci = tid; ci < 128 * cpr; ci += kThreads) {
+            const int i = ci / cpr, cc = (ci % cpr) * 8;
+            float v[8];
+            if (i < 64) {
+                const float bq = q2s[i * E + e] * expf(Gs[i * E + e]);
+                load_bf16x8(sDO + sw128_offset(i, cc, 64), v);
+                for (int u = 0; u < 8; ++u) v[u] *= bq;
+            } else {
+                const int r = i - 64;
+                if (p.use_delta && r < n) {
+                    const float a = -k2s[r * E + e] * expf(Gs[r * E + e]);
+                    load_row8(p.dRbuf + tok_idx(b, t0 + r, h, cc, T, H, dv), v);
+                    for (int u = 0; u < 8; ++u) v[u] *= a;
                 } else {
-                    const int r = i - 64;
-                    if (p.use_delta && r < n) {
-                        const float a = -k2s[r * E + e] * expf(Gs[r * E + e]);
-                        load_row8(p.dRbuf + tok_idx(b, t0 + r, h, cc, T, H, dv), v);
-                        for (int u = 0; u < 8; ++u) v[u] *= a;
-                    } else {
-                        for (int u = 0; u < 8; ++u) v[u] = 0.f;
-                    }
+                    for (int u = 0; u < 8; ++u) v[u] = 0.f;
                 }
-                st8_split(sY, sY + 32768, sw128_offset(i, cc, 128), v);
             }
+            st8_split(sY, sY + 32768, sw128_offset(i, cc, 128), v);
         }
+        bool ok = mbar_wait(&bar_s, sph);
+        sph ^= 1;
         fence_proxy_async_smem();
         tc_fence_before();
-        __syncthreads();
+        if (__syncthreads_or(!ok)) { failed = true; break; }
         tc_fence_after();
         if (tid == 0) {
             const uint32_t idA = idesc_bf16_f32(128, kDk, 0, 0);
@@ -480,7 +475,7 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                 const uint64_t ah = smem_desc(smem_u32(sY) + o, 16, 1024);
                 const uint64_t al = smem_desc(smem_u32(sY + 32768) + o, 16, 1024);
                 const uint64_t bh = smem_desc(smem_u32(sX) + o, 16, 1024);
-                const uint64_t bl = smem_desc(smem_u32(sX + 32768) + o, 16, 1024);
+                const uint64_t bl = smem_desc(smem_u32(sX + LO) + o, 16, 1024);
                 umma_bf16(tACC, ah, bh, idA, 1u);
                 umma_bf16(tACC, ah, bl, idA, 1u);
                 umma_bf16(tACC, al, bh, idA, 1u);
@@ -489,75 +484,19 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             for (int ks = 0; ks < kDk / 16; ++ks) {
                 const uint64_t a = smem_desc(smem_u32(sKQ) + (ks >> 2) * 2 * kBoxBytes + (ks & 3) * 32, 16, 1024);
                 umma_bf16(tP, a, smem_desc(smem_u32(sX) + ks * 2048, 16384, 1024), idP, ks > 0 ? 1u : 0u);
-                umma_bf16(tP, a, smem_desc(smem_u32(sX + 32768) + ks * 2048, 16384, 1024), idP, 1u);
+                umma_bf16(tP, a, smem_desc(smem_u32(sX + LO) + ks * 2048, 16384, 1024), idP, 1u);
             }
             umma_commit(&bar_mma);
         }
         ok = mma_wait();
         if (__syncthreads_or(!ok)) { failed = true; break; }
         tc_fence_after();
-        // stage dS'_e -> sX and A2_e = [0 ; w_e U] -> sY; Frobenius partial <dS'_e, S_e>
-        {
-            float fro = 0.f;
-            for (int c0 = tid; c0 < 128 * cpr; c0 += 2 * kThreads) {   // 2 chunks (x2 tensors) in flight
-                float v[2][8], sv[2][8];
-#pragma unroll
-                for (int k = 0; k < 2; ++k) {
-                    const int ci = c0 + k * kThreads;
-                    if (ci < 128 * cpr) {
-                        load_row8(dSe + (ci / cpr) * dv + (ci % cpr) * 8, v[k]);
-                        load_row8(Se + (ci / cpr) * dv + (ci % cpr) * 8, sv[k]);
-                    }
-                }
-#pragma unroll
-                for (int k = 0; k < 2; ++k) {
-                    const int ci = c0 + k * kThreads;
-                    if (ci < 128 * cpr) {
-                        for (int u = 0; u < 8; ++u) fro = fmaf(v[k][u], sv[k][u], fro);
-                        st8_split(sX, sX + 32768, sw128_offset(ci / cpr, (ci % cpr) * 8, 128), v[k]);
-                    }
-                }
-            }
-            red2[tid] = fro;
-            for (int ci = tid; ci < 128 * cpr; ci += kThreads) {
-                const int i = ci / cpr, cc = (ci % cpr) * 8;
-                float v[8];
-                const int r = i - 64;
-                if (i >= 64 && r < n) {
-                    const float w = k2s[r * E + e] * expf(Gs[(n - 1) * E + e] - Gs[r * E + e]);
-                    load_row8(p.Ubuf + tok_idx(b, t0 + r, h, cc, T, H, dv), v);
-                    for (int u = 0; u < 8; ++u) v[u] *= w;
-                } else {
-                    for (int u = 0; u < 8; ++u) v[u] = 0.f;
-                }
-                st8_split(sY, sY + 32768, sw128_offset(i, cc, 128), v);
-            }
+        if (tid == 0) {   // A1 consumed: dS'_e into sY
+            mbar_arrive_expect_tx(&bar_d, slab_bytes);
+            bulk_load(sY, reinterpret_cast<const uint8_t*>(p.dSck) + (sbase + e) * kDk * dv * 4,
+                      slab_bytes, &bar_d);
         }
-        fence_proxy_async_smem();
-        tc_fence_before();
-        __syncthreads();
-        tc_fence_after();
-        if (tid == 0) {
-            const uint32_t idA = idesc_bf16_f32(128, kDk, 0, 0);
-            for (int ks = 0; ks < dv / 16; ++ks) {
-                const uint32_t o = (ks >> 2) * 16384 + (ks & 3) * 32;
-                const uint64_t ah = smem_desc(smem_u32(sY) + o, 16, 1024);
-                const uint64_t al = smem_desc(smem_u32(sY + 32768) + o, 16, 1024);
-                const uint64_t bh = smem_desc(smem_u32(sX) + o, 16, 1024);
-                const uint64_t bl = smem_desc(smem_u32(sX + 32768) + o, 16, 1024);
-                umma_bf16(tACC, ah, bh, idA, 1u);
-                umma_bf16(tACC, ah, bl, idA, 1u);
-                umma_bf16(tACC, al, bh, idA, 1u);
-            }
-            const uint32_t idP = idesc_bf16_f32(128, dv, 0, 1);
-            for (int ks = 0; ks < kDk / 16; ++ks) {
-                const uint64_t a = smem_desc(smem_u32(sKQ) + (ks >> 2) * 2 * kBoxBytes + (ks & 3) * 32, 16, 1024);
-                umma_bf16(tP2, a, smem_desc(smem_u32(sX) + ks * 2048, 16384, 1024), idP, ks > 0 ? 1u : 0u);
-                umma_bf16(tP2, a, smem_desc(smem_u32(sX + 32768) + ks * 2048, 16384, 1024), idP, 1u);
-            }
-            umma_commit(&bar_mma);
-        }
-        // row dots of P_e = [K;Q] S_e (overlaps the products above)
+        // row dots of P_e = [K;Q] S_e while dS'_e is in flight
         {
             float acc = 0.f;
             const int cw = dv / 2;
@@ -581,9 +520,23 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             }
             red[half * 128 + L] = acc;
         }
-        ok = mma_wait();
+        ok = mbar_wait(&bar_d, dph);
+        dph ^= 1;
+        // <dS'_e, S_e> from the hi/lo tiles (hi + lo reproduces each value to ~2^-16)
+        {
+            float fro = 0.f;
+            for (int ci = tid; ci < 128 * cpr; ci += kThreads) {
+                const uint32_t o = sw128_offset(ci / cpr, (ci % cpr) * 8, 128);
+                float sh[8], sl[8], dh[8], dl[8];
+                load_bf16x8(sX + o, sh);
+                load_bf16x8(sX + LO + o, sl);
+                load_bf16x8(sY + o, dh);
+                load_bf16x8(sY + LO + o, dl);
+                for (int u = 0; u < 8; ++u) fro = fmaf(dh[u] + dl[u], sh[u] + sl[u], fro);
+            }
+            red2[tid] = fro;
+        }
         if (__syncthreads_or(!ok)) { failed = true; break; }
-        tc_fence_after();
         if (tid < 128) {
             const float v = red[tid] + red[128 + tid];
             if (tid < 64) dak[tid * E + e] = -v;
@@ -594,7 +547,52 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             for (int i = 0; i < kThreads; ++i) f += red2[i];
             dgc[e] = f;
         }
+        // A2_e = [0 ; w_e U] -> sX (S_e consumed)
+        for (int ci = tid; ci < 128 * cpr; ci += kThreads) {
+            const int i = ci / cpr, cc = (ci % cpr) * 8;
+            float v[8];
+            const int r = i - 64;
+            if (i >= 64 && r < n) {
+                const float w = k2s[r * E + e] * expf(Gs[(n - 1) * E + e] - Gs[r * E + e]);
+                load_row8(p.Ubuf + tok_idx(b, t0 + r, h, cc, T, H, dv), v);
+                for (int u = 0; u < 8; ++u) v[u] *= w;
+            } else {
+                for (int u = 0; u < 8; ++u) v[u] = 0.f;
+            }
+            st8_split(sX, sX + 32768, sw128_offset(i, cc, 128), v);
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
         __syncthreads();
+        tc_fence_after();
+        if (tid == 0) {
+            const uint32_t idA = idesc_bf16_f32(128, kDk, 0, 0);
+            for (int ks = 0; ks < dv / 16; ++ks) {
+                const uint32_t o = (ks >> 2) * 16384 + (ks & 3) * 32;
+                const uint64_t ah = smem_desc(smem_u32(sX) + o, 16, 1024);
+                const uint64_t al = smem_desc(smem_u32(sX + 32768) + o, 16, 1024);
+                const uint64_t bh = smem_desc(smem_u32(sY) + o, 16, 1024);
+                const uint64_t bl = smem_desc(smem_u32(sY + LO) + o, 16, 1024);
+                umma_bf16(tACC, ah, bh, idA, 1u);
+                umma_bf16(tACC, ah, bl, idA, 1u);
+                umma_bf16(tACC, al, bh, idA, 1u);
+            }
+            const uint32_t idP = idesc_bf16_f32(128, dv, 0, 1);
+            for (int ks = 0; ks < kDk / 16; ++ks) {
+                const uint64_t a = smem_desc(smem_u32(sKQ) + (ks >> 2) * 2 * kBoxBytes + (ks & 3) * 32, 16, 1024);
+                umma_bf16(tP2, a, smem_desc(smem_u32(sY) + ks * 2048, 16384, 1024), idP, ks > 0 ? 1u : 0u);
+                umma_bf16(tP2, a, smem_desc(smem_u32(sY + LO) + ks * 2048, 16384, 1024), idP, 1u);
+            }
+            umma_commit(&bar_mma);
+        }
+        ok = mma_wait();
+        if (__syncthreads_or(!ok)) { failed = true; break; }
+        tc_fence_after();
+        if (tid == 0 && e + 1 < E) {   // A2 consumed: S_{e+1} into sX
+            mbar_arrive_expect_tx(&bar_s, slab_bytes);
+            bulk_load(sX, reinterpret_cast<const uint8_t*>(p.Sck) + (sbase + e + 1) * kDk * dv * 4,
+                      slab_bytes, &bar_s);
+        }
         // row dots of P'_e = [K;Q] dS'_e (key rows)
         {
             float acc = 0.f;
@@ -681,10 +679,12 @@ size_t grads_tc_smem(int E) {
 
 }  // namespace
 
-int tc_grads_ok(const tla_problem& p, const FwdPlan& fp) {
-    return fp.tcb && p.dk == kDk && p.dv % 64 == 0 && p.dv <= 128 && p.E <= 8 &&
+int tc_grads_shape_ok(const tla_problem& p) {
+    return p.dk == kDk && p.dv % 64 == 0 && p.dv <= 128 && p.E <= 8 &&
            grads_tc_smem(p.E) <= 227 * 1024;
 }
+
+int tc_grads_ok(const tla_problem& p, const FwdPlan& fp) { return fp.ck_tiles && tc_grads_shape_ok(p); }
 
 cudaError_t launch_bwd_chunk_grads_tc(const tla_problem& p, const FwdPlan& fp, const char* fws,
                                       const BwdPlan& bp, const char* bws, const void* dO,

@@ -73,6 +73,7 @@ FwdPlan plan_fwd(const tla_problem& p, int save) {
         f.coef = off;
         off = align256(off + (size_t)p.B * p.H * f.NT * (3 * kChunk * p.E + 16) * 4);
         f.tcb = (save && tc_bwd_ok(p, f.tc_tv)) ? 1 : 0;
+        f.ck_tiles = (f.tcb && tc_grads_shape_ok(p)) ? 1 : 0;
         if (f.tcb) { f.BT = off; off = align256(off + 2 * mats); }
     }
     if (save) {
