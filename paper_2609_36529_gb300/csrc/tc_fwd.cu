@@ -422,7 +422,7 @@ cudaError_t launch_tv(const tla_problem& p, const FwdPlan& fp, char* ws, int sav
 // be a multiple of 64 (and at most 256, the widest UMMA and half of TMEM).
 int tc_fwd_tv(const tla_problem& p) {
     if (p.dtype != TLA_BF16 || p.dk != kDk) return 0;
-    const int cand[3] = {32, 16, 64};
+    const int cand[3] = {16, 32, 64};
     for (int tv : cand) {
         const int ne = p.E * tv;
         if (p.dv % tv == 0 && ne % 64 == 0 && ne <= 256) return tv;
