@@ -102,6 +102,28 @@ size_t tla_fwd_workspace_bytes(const tla_problem *p, int save_for_bwd);
 tla_status tla_chunk_fwd(const tla_problem *p, void *workspace, size_t workspace_bytes,
                          int save_for_bwd, void *stream);
 
+/*
+ * Forward without a caller-provided workspace, for callers that cannot allocate
+ * device memory (a host runtime that owns all device memory, a serving process
+ * that forbids allocation after start-up, a fixed committed memory budget).
+ * The paper has no counterpart: this is an interface convenience.  Same
+ * computation and outputs as tla_chunk_fwd(p, ws, bytes, save_for_bwd = 0, stream),
+ * with the workspace taken from a fixed device buffer built into the library
+ * (tla_noalloc_scratch_bytes() bytes, 64 MiB, held by every GPU that loads the
+ * library until the process exits).  Allocates nothing.
+ *  - Returns TLA_ERR_WORKSPACE, launching nothing, when
+ *    tla_fwd_workspace_bytes(p, 0) exceeds the buffer; other argument errors
+ *    as tla_chunk_fwd.
+ *  - All calls share the buffer: calls that overlap on the GPU (other streams,
+ *    unordered host threads) race on it.  Nothing in it needs clearing.
+ *  - The first call on each device looks up the buffer's device address; make
+ *    it before capturing the stream into a CUDA graph.
+ */
+tla_status tla_chunk_fwd_noalloc(const tla_problem *p, void *stream);
+
+/* Size in bytes of the built-in buffer used by tla_chunk_fwd_noalloc. */
+size_t tla_noalloc_scratch_bytes(void);
+
 /* Workspace of tla_chunk_bwd in bytes (multiple of 256, 256-byte aligned). */
 size_t tla_bwd_workspace_bytes(const tla_problem *p);
 

@@ -21,7 +21,7 @@ STATUS = {0: "TLA_OK", -1: "TLA_ERR_INVALID_ARG", -2: "TLA_ERR_UNSUPPORTED", -3:
 
 EXPORTED = ("tla_fwd_workspace_bytes", "tla_chunk_fwd", "tla_bwd_workspace_bytes",
             "tla_chunk_bwd", "tla_decode_step", "tla_status_string", "tla_last_device_status",
-            "tla_version")
+            "tla_version", "tla_chunk_fwd_noalloc", "tla_noalloc_scratch_bytes")
 
 
 class TlaError(RuntimeError):
@@ -68,6 +68,9 @@ def lib():
         L.tla_last_device_status.argtypes = [vp]
         L.tla_last_device_status.restype = i
         L.tla_version.restype = ctypes.c_char_p
+        L.tla_chunk_fwd_noalloc.argtypes = [P, vp]
+        L.tla_chunk_fwd_noalloc.restype = i
+        L.tla_noalloc_scratch_bytes.restype = sz
         _lib = L
     return _lib
 
@@ -145,6 +148,21 @@ def tla_chunk_fwd(q, k, v, q2, k2, g, beta=None, h0=None, use_delta=True, save_f
     _check("tla_chunk_fwd", lib().tla_chunk_fwd(ctypes.byref(p), _ptr(workspace), need,
                                                 int(save_for_bwd), _stream()))
     return o, ht, workspace
+
+
+def tla_chunk_fwd_noalloc(q, k, v, q2, k2, g, beta=None, h0=None, use_delta=True, o=None,
+                          ht=None):
+    """Forward through the entry point that allocates nothing (built-in scratch).
+
+    o and ht must be preallocated by the caller when it cannot allocate; when they
+    are None they are allocated here with PyTorch for convenience."""
+    B, T, H, _ = q.shape
+    E, dv = q2.shape[-1], v.shape[-1]
+    if o is None:
+        o = torch.empty(B, T, H, dv, dtype=torch.float32, device=q.device)
+    p = make_problem(q, k, v, q2, k2, g, beta, h0, o, ht, use_delta)
+    _check("tla_chunk_fwd_noalloc", lib().tla_chunk_fwd_noalloc(ctypes.byref(p), _stream()))
+    return o, ht
 
 
 def tla_chunk_bwd(q, k, v, q2, k2, g, dO, fwd_workspace, beta=None, h0=None, dht=None,

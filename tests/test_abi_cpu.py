@@ -100,3 +100,15 @@ def test_workspace_sizes_grow_with_saving(tla):
     b = L.tla_fwd_workspace_bytes(ctypes.byref(p), 1)
     assert b > a > 0
     assert L.tla_bwd_workspace_bytes(ctypes.byref(p)) > 0
+
+
+def test_noalloc_entry_rejects_on_host(tla):
+    """The no-allocation forward rejects bad or oversized problems before any launch."""
+    L = tla.lib()
+    cap = L.tla_noalloc_scratch_bytes()
+    assert cap == 64 << 20
+    p = _problem(tla, chunk=32)
+    assert L.tla_chunk_fwd_noalloc(ctypes.byref(p), None) == -2
+    p = _problem(tla, B=64, T=8192, H=16, dk=128, dv=128)   # workspace far above the buffer
+    assert L.tla_fwd_workspace_bytes(ctypes.byref(p), 0) > cap
+    assert L.tla_chunk_fwd_noalloc(ctypes.byref(p), None) == -5
