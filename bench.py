@@ -394,6 +394,8 @@ def run_e2e(args, tla, x, w, dev, stream, o, fws, bws, grads, barrier, max_over_
 
 def run_decode(args, tla, inputs, dev, stream, lib, peaks, barrier, max_over_ranks, ws_n):
     dw = inputs.DECODE
+    if args.decode_batch:   # profiling option: fewer sequences of the same shape
+        dw = dataclasses.replace(dw, B=args.decode_batch, name=f"{dw.name}_batch{args.decode_batch}")
     gen = torch.Generator(dev)
     gen.manual_seed(1000 + dist_env()[1])
     state = torch.empty(dw.B, dw.H, dw.E, dw.dk, dw.dv, dtype=torch.float32, device=dev)
@@ -529,6 +531,8 @@ def main():
                     help="profiling only: run B sequences instead of the workload's 8")
     ap.add_argument("--fwd-only", action="store_true",
                     help="profiling only: time the forward alone (not the headline metric)")
+    ap.add_argument("--decode-batch", type=int, default=0,
+                    help="profiling only: decode workload with this many sequences")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         print("bench: at least 3 warm-up steps are required; using 3", file=sys.stderr)

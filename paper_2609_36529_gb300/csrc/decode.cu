@@ -16,10 +16,11 @@
 namespace tla {
 
 constexpr int kDecThreads = 256;
-constexpr int kDecMaxPasses = 32;  // float4 registers per thread
 
-template <typename Tin, int TPR>  // TPR threads per slab row (TV = 4 * TPR columns)
-__global__ void __launch_bounds__(kDecThreads)
+// TPR threads per slab row (TV = 4 * TPR columns); MAXP float4 registers per thread.
+// Two or more CTAs per SM let one CTA's loads overlap another's stores.
+template <typename Tin, int TPR, int MAXP>
+__global__ void __launch_bounds__(kDecThreads, (MAXP <= 16 ? 2 : 1))
 decode_step_kernel(const Tin* __restrict__ q, const Tin* __restrict__ k,
                    const Tin* __restrict__ v, const Tin* __restrict__ q2,
                    const Tin* __restrict__ k2, const float* __restrict__ g,
@@ -55,9 +56,9 @@ decode_step_kernel(const Tin* __restrict__ q, const Tin* __restrict__ k,
     const int row_stride4 = dv / 4;
 
     // stream the slab in: all loads issued before any use
-    float4 reg[kDecMaxPasses];
+    float4 reg[MAXP];
 #pragma unroll
-    for (int p = 0; p < kDecMaxPasses; ++p) {
+    for (int p = 0; p < MAXP; ++p) {
         int row = row0 + p * RPP;
         if (p < passes && row < rows) reg[p] = __ldcs(S4 + size_t(row) * row_stride4);
         else reg[p] = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -73,7 +74,7 @@ decode_step_kernel(const Tin* __restrict__ q, const Tin* __restrict__ k,
     // decay, then partial reads at the joint key (k, k') and the joint query (q, q')
     float4 pr = make_float4(0.f, 0.f, 0.f, 0.f), pp = pr;
 #pragma unroll
-    for (int p = 0; p < kDecMaxPasses; ++p) {
+    for (int p = 0; p < MAXP; ++p) {
         int row = row0 + p * RPP;
         if (p < passes && row < rows) {
             int e = row / dk, d = row - e * dk;
@@ -124,7 +125,7 @@ decode_step_kernel(const Tin* __restrict__ q, const Tin* __restrict__ k,
     __syncthreads();
     const float4 u4 = reinterpret_cast<const float4*>(us)[quad];
 #pragma unroll
-    for (int p = 0; p < kDecMaxPasses; ++p) {
+    for (int p = 0; p < MAXP; ++p) {
         int row = row0 + p * RPP;
         if (p < passes && row < rows) {
             int e = row / dk, d = row - e * dk;
@@ -141,29 +142,29 @@ cudaError_t launch_decode_step(int B, int H, int dk, int dv, int E, int use_delt
                                const void* q, const void* k, const void* v, const void* q2,
                                const void* k2, const float* g, const float* beta,
                                float* state, void* o, cudaStream_t s) {
-    // TV = 32 columns (128-byte row segments) while the slab fits the registers, else 16.
+    // TV = 16 columns (64-byte row segments): the slab of E x dk rows takes
+    // rows / 64 float4 registers per thread (16 for E*dk <= 1024, else 32).
     const int rows = E * dk;
-    const int tpr = (rows <= kDecMaxPasses * (kDecThreads / 8) && dv % 32 == 0) ? 8 : 4;
-    const int TV = 4 * tpr;
+    const int TV = 16;
     dim3 grid(dv / TV, B * H);
     prof_before("decode_step", s);
     if (dtype == TLA_BF16) {
         using Tb = __nv_bfloat16;
-        if (tpr == 8)
-            decode_step_kernel<Tb, 8><<<grid, kDecThreads, 0, s>>>(
+        if (rows <= 16 * 64)
+            decode_step_kernel<Tb, 4, 16><<<grid, kDecThreads, 0, s>>>(
                 (const Tb*)q, (const Tb*)k, (const Tb*)v, (const Tb*)q2, (const Tb*)k2, g, beta,
                 state, (Tb*)o, dk, dv, E, use_delta);
         else
-            decode_step_kernel<Tb, 4><<<grid, kDecThreads, 0, s>>>(
+            decode_step_kernel<Tb, 4, 32><<<grid, kDecThreads, 0, s>>>(
                 (const Tb*)q, (const Tb*)k, (const Tb*)v, (const Tb*)q2, (const Tb*)k2, g, beta,
                 state, (Tb*)o, dk, dv, E, use_delta);
     } else {
-        if (tpr == 8)
-            decode_step_kernel<float, 8><<<grid, kDecThreads, 0, s>>>(
+        if (rows <= 16 * 64)
+            decode_step_kernel<float, 4, 16><<<grid, kDecThreads, 0, s>>>(
                 (const float*)q, (const float*)k, (const float*)v, (const float*)q2,
                 (const float*)k2, g, beta, state, (float*)o, dk, dv, E, use_delta);
         else
-            decode_step_kernel<float, 4><<<grid, kDecThreads, 0, s>>>(
+            decode_step_kernel<float, 4, 32><<<grid, kDecThreads, 0, s>>>(
                 (const float*)q, (const float*)k, (const float*)v, (const float*)q2,
                 (const float*)k2, g, beta, state, (float*)o, dk, dv, E, use_delta);
     }
