@@ -125,11 +125,9 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         tma_load_4d(sV, &map_v, &bar_av, n0, h, c * 64, b);
         bulk_load(sCoef + (c & 1) * CB, p.coef + idx * CB, CB * 4, &bar_av);
     };
-    // Row d = tid of S_{[c]}: operand of MMA-A, checkpoint, and the gamma^C_c-scaled
-    // copy in TMEM for the accumulation of chunk c.
-    auto prepare = [&](int c, bool from_h0) {
+    // Row d = tid of S_{[c]} (from h0 or from TMEM) as the bf16 hi/lo operand of MMA-A.
+    auto write_operand = [&](bool from_h0) {
         const int d = tid;
-        const float* gc = sCoef + (c & 1) * CB + 3 * 64 * E;
         for (int e = 0; e < E; ++e) {
             float v[TV];
             if (from_h0) {
@@ -152,6 +150,33 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             }
 #pragma unroll
             for (int n = 0; n < TV; n += 8) st8_split(sSh, sSl, sw128_offset(d, e * TV + n, kDk), v + n);
+        }
+    };
+    // Row d of S_{[c]}: checkpoint for the backward, and the gamma^C_c-scaled copy in
+    // TMEM that chunk c's state update accumulates onto.  Runs while MMA-A(c) executes.
+    auto finish_state = [&](int c, bool from_h0) {
+        const int d = tid;
+        const float* gc = sCoef + (c & 1) * CB + 3 * 64 * E;
+        for (int e = 0; e < E; ++e) {
+            float v[TV];
+            if (from_h0) {
+                if (p.h0) {
+                    const float4* src = reinterpret_cast<const float4*>(
+                        p.h0 + ((size_t(b * H + h) * E + e) * kDk + d) * dv + n0);
+#pragma unroll
+                    for (int i = 0; i < TV / 4; ++i) {
+                        float4 x = src[i];
+                        v[4 * i] = x.x; v[4 * i + 1] = x.y; v[4 * i + 2] = x.z; v[4 * i + 3] = x.w;
+                    }
+                } else {
+#pragma unroll
+                    for (int i = 0; i < TV; ++i) v[i] = 0.f;
+                }
+            } else {
+#pragma unroll
+                for (int j = 0; j < TV; j += 16) tmem_ld16(tmem_lane_addr(tS, warp, e * TV + j), v + j);
+                tmem_wait_ld();
+            }
             if (p.save) {
                 const size_t slab = (((size_t(b) * H + h) * NT + c) * E + e) * kDk * dv;
                 if (p.ck_tiles) {   // bf16 hi/lo tiles in the gradient kernel's layout
@@ -171,6 +196,19 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         }
         tmem_wait_st();
     };
+    // MMA-A: P = [K; Q] S_all    (B = S_all, MN-major, hi and lo)
+    auto issue_mma_a = [&]() {
+        const uint32_t idesc = idesc_bf16_f32(128, NE, 0, 1);
+#pragma unroll
+        for (int ks = 0; ks < kDk / 16; ++ks) {
+            const int blk = ks >> 2, kk = (ks & 3) * 16;
+            const uint64_t ad = smem_desc(smem_u32(sKQ) + blk * 2 * kBoxBytes + kk * 2, 16, 1024);
+            umma_bf16(tP, ad, smem_desc(smem_u32(sSh) + ks * 2048, kDk * 128, 1024), idesc,
+                      ks > 0 ? 1u : 0u);
+            umma_bf16(tP, ad, smem_desc(smem_u32(sSl) + ks * 2048, kDk * 128, 1024), idesc, 1u);
+        }
+        umma_commit(&bar_mma);
+    };
 
     bool failed = false;
     uint32_t mma_phase = 0;
@@ -182,11 +220,17 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     if (!mbar_wait(&bar_av, 0)) failed = true;
     if (__syncthreads_or(failed)) failed = true;
     if (!failed) {
-        prepare(0, true);
+        write_operand(true);
         fence_proxy_async_smem();
         tc_fence_before();
-        __syncthreads();
+        const bool ok = mbar_wait(&bar_kq, 0);
+        if (__syncthreads_or(!ok)) failed = true;
         tc_fence_after();
+        if (!failed) {
+            if (tid == 0) issue_mma_a();
+            pending_mma = 1;
+            finish_state(0, true);
+        }
     }
 
     for (int c = 0; c < NT && !failed; ++c) {
@@ -195,35 +239,18 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         const float* ae = cf;
         const float* be = cf + 64 * E;
         const float* we = cf + 128 * E;
-        bool ok = mbar_wait(&bar_kq, c & 1);
-        if (__syncthreads_or(!ok)) { failed = true; break; }
-        tc_fence_after();
-
-        // ---- MMA-A: P = [K; Q] S_all    (B = S_all, MN-major, hi and lo)
-        if (tid == 0) {
-            const uint32_t idesc = idesc_bf16_f32(128, NE, 0, 1);
-#pragma unroll
-            for (int ks = 0; ks < kDk / 16; ++ks) {
-                const int blk = ks >> 2, kk = (ks & 3) * 16;
-                const uint64_t ad = smem_desc(smem_u32(sKQ) + blk * 2 * kBoxBytes + kk * 2, 16, 1024);
-                umma_bf16(tP, ad, smem_desc(smem_u32(sSh) + ks * 2048, kDk * 128, 1024), idesc,
-                          ks > 0 ? 1u : 0u);
-                umma_bf16(tP, ad, smem_desc(smem_u32(sSl) + ks * 2048, kDk * 128, 1024), idesc, 1u);
-            }
-            umma_commit(&bar_mma);
-        }
-        pending_mma = 1;
-        ok = mbar_wait(&bar_mma, mma_phase);
+        // ---- wait for MMA-A(c) (issued at the end of the previous step)
+        bool ok = mbar_wait(&bar_mma, mma_phase);
         mma_phase ^= 1;
+        tc_fence_before();
         if (__syncthreads_or(!ok)) { failed = true; break; }
         pending_mma = 0;
         tc_fence_after();
 
-        // ---- epi-A
-        float oi[TV];
+        // ---- epi-A: Res (key rows) and the inter-chunk read (query rows)
+        float oi[TV], res[TV];
         if (warp < 2) {
             const int r = tid;
-            float res[TV];
             {
                 const uint4* vrow = reinterpret_cast<const uint4*>(sV + r * TV);
 #pragma unroll
@@ -251,8 +278,6 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             }
 #pragma unroll
             for (int i = 0; i < TV; ++i) st_split(sRh, sRl, sw128_offset(i, r, TV), res[i]);
-            if (p.save && p.use_delta && r < n)
-                store_f32_row(p.Rbuf + tok_idx(b, t0 + r, h, n0, T, H, dv), res, TV);
         } else {
             const int r = tid - 64;
 #pragma unroll
@@ -288,6 +313,8 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             umma_commit(&bar_mma);
         }
         pending_mma = 1;
+        if (warp < 2 && p.save && p.use_delta && tid < n)   // while MMA-B runs
+            store_f32_row(p.Rbuf + tok_idx(b, t0 + tid, h, n0, T, H, dv), res, TV);
         ok = mbar_wait(&bar_mma, mma_phase);
         mma_phase ^= 1;
         if (__syncthreads_or(!ok)) { failed = true; break; }
@@ -295,29 +322,24 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         tc_fence_after();
         if (tid == 0 && c + 1 < NT) issue_av(c + 1);   // [T; A T], V and the other coef buffer are free
 
-        // ---- epi-B
-        {
-            float d2[TV];
+        // ---- epi-B: Ut operand (key rows); O = Oi + Oa (query rows)
+        float d2[TV];
 #pragma unroll
-            for (int j = 0; j < TV; j += 16) tmem_ld16(tmem_lane_addr(tP, warp, j), d2 + j);
-            tmem_wait_ld();
-            if (warp < 2) {
-                const int r = tid;
-                for (int e = 0; e < E; ++e) {
-                    const float wv = we[r * E + e];
-                    float u[TV];
+        for (int j = 0; j < TV; j += 16) tmem_ld16(tmem_lane_addr(tP, warp, j), d2 + j);
+        tmem_wait_ld();
+        if (warp < 2) {
+            const int r = tid;
+            for (int e = 0; e < E; ++e) {
+                const float wv = we[r * E + e];
+                float u[TV];
 #pragma unroll
-                    for (int i = 0; i < TV; ++i) u[i] = wv * d2[i];
+                for (int i = 0; i < TV; ++i) u[i] = wv * d2[i];
 #pragma unroll
-                    for (int i = 0; i < TV; i += 8) st8_split(sUh, sUl, sw128_offset(r, e * TV + i, 64), u + i);
-                }
-                if (p.save && r < n) store_f32_row(p.Ubuf + tok_idx(b, t0 + r, h, n0, T, H, dv), d2, TV);
-            } else {
-                const int r = tid - 64;
-#pragma unroll
-                for (int i = 0; i < TV; ++i) d2[i] += oi[i];
-                if (r < n) store_row(p.o, tok_idx(b, t0 + r, h, n0, T, H, dv), d2, TV, p.out_f32);
+                for (int i = 0; i < TV; i += 8) st8_split(sUh, sUl, sw128_offset(r, e * TV + i, 64), u + i);
             }
+        } else {
+#pragma unroll
+            for (int i = 0; i < TV; ++i) d2[i] += oi[i];
         }
         fence_proxy_async_smem();
         tc_fence_before();
@@ -336,6 +358,16 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             umma_commit(&bar_mma);
         }
         pending_mma = 1;
+        {   // while MMA-C runs: U (key rows) and o (query rows) to global memory
+            const int r = warp < 2 ? tid : tid - 64;
+            if (r < n) {
+                if (warp < 2) {
+                    if (p.save) store_f32_row(p.Ubuf + tok_idx(b, t0 + r, h, n0, T, H, dv), d2, TV);
+                } else {
+                    store_row(p.o, tok_idx(b, t0 + r, h, n0, T, H, dv), d2, TV, p.out_f32);
+                }
+            }
+        }
         ok = mbar_wait(&bar_mma, mma_phase);
         mma_phase ^= 1;
         if (c + 1 < NT) ok = ok && mbar_wait(&bar_av, (c + 1) & 1);   // chunk c+1's gamma^C
@@ -344,9 +376,17 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         tc_fence_after();
         if (tid == 0 && c + 1 < NT) issue_kq(c + 1);   // key/query buffer is free
 
-        // ---- epi-C
+        // ---- epi-C: next chunk's operand, MMA-A(c+1), then checkpoint and scaling
         if (c + 1 < NT) {
-            prepare(c + 1, false);
+            write_operand(false);
+            fence_proxy_async_smem();
+            tc_fence_before();
+            ok = mbar_wait(&bar_kq, (c + 1) & 1);
+            if (__syncthreads_or(!ok)) { failed = true; break; }
+            tc_fence_after();
+            if (tid == 0) issue_mma_a();
+            pending_mma = 1;
+            finish_state(c + 1, false);
         } else if (p.ht) {
             const int d = tid;
             for (int e = 0; e < E; ++e) {
@@ -357,10 +397,6 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                 store_f32_row(p.ht + ((size_t(b * H + h) * E + e) * kDk + d) * dv + n0, v, TV);
             }
         }
-        fence_proxy_async_smem();
-        tc_fence_before();
-        __syncthreads();
-        tc_fence_after();
     }
 
     if (failed) {
