@@ -120,6 +120,13 @@ __device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t b
         : "memory");
 }
 
+// Hint: bring `bytes` of global memory into L2 (16-byte aligned, size multiple of 16).
+__device__ __forceinline__ void bulk_prefetch_l2(const void* src, uint32_t bytes) {
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(reinterpret_cast<uint64_t>(src)),
+                 "r"(bytes)
+                 : "memory");
+}
+
 // ---------------------------------------------------------------- TMEM
 // Allocation is a warp-wide operation; the allocated base address is written
 // to shared memory.  ncols: power of two, 32..512.

@@ -6,17 +6,22 @@
 // gradient of the state at the chunk's end, and U, Res, dU, dRes of the chunk:
 //   dQ = sum_e diag(b_e) dO S_e^T + P K,                       P = dA (.) R'
 //   dK = sum_e [diag(a_e) (-dRes) S_e^T + diag(w_e) U dS'_e^T] + (dKK + dKK^T) K + P^T Q
-//   db_e = rowdot(dO, Q S_e), da_e = -rowdot(dRes, K S_e), dw_e = rowdot(U, K dS'_e)
+//   db_e = rowdot(Q, dO S_e^T), da_e = rowdot(K, -dRes S_e^T), dw_e = rowdot(K, U dS'_e^T)
 //   dgamma^C_e = <dS'_e, S_e>_F
 //   dA = dO U^T, dT = dU Res^T (sGLA: dU V^T), and the C x C algebra of the UT
 //   transform (dN, F = dN N^T, dM = -N^T F, dL, dKK, dR, dR', dbeta).
 // Tensor-core products (fp32 accumulation in TMEM, non-exact operands as bf16 hi/lo):
 //   phase 0  [K;Q] K^T -> K K^T, Q K^T;  dO U^T -> dA;  dU Res^T -> dT   (M=64 for the last two)
-//   phase 1  (CUDA cores) C x C algebra, then ACC = [[P, 0], [Kc, P^T]] [K; Q]
-//   phase 2  per slice e:  ACC += [b_e dO ; -a_e dRes] S_e^T + [0 ; w_e U] dS'_e^T,
-//            P_e = [K;Q] S_e, P'_e = [K;Q] dS'_e (the staged S tile is read K-major for
-//            the first product and MN-major for the second)
-//   phase 3  ACC rows 0-63 -> dq, rows 64-127 -> dk; second keys/queries, log gates, beta.
+//   phase 1  (CUDA cores) C x C algebra, then ACC^T = [K; Q]^T [[P, 0], [Kc, P^T]]^T
+//   phase 2  per slice e, transposed so that TMEM lanes index the key dimension d:
+//              D1 = S_e [dO ; -dRes]^T   (128 x 128: query tokens, then key tokens)
+//              D2 = dS'_e U^T            (128 x 64)
+//            The slice's row scalings b_e, a_e, w_e are applied to D1/D2 in registers
+//            (one thread per (d, 32 tokens)), and the row dots come from the same values
+//            against the thread's column of Q or K, summed across the 128 lanes.  The
+//            unscaled operands [dO ; -dRes] and U are staged once for all slices.
+//   phase 3  dq = registers + ACC^T[:, 0:64]^T, dk = registers + ACC^T[:, 64:128]^T;
+//            second keys/queries, log gates, beta.
 #include "common.cuh"
 #include "internal.h"
 #include "sm100.cuh"
@@ -30,9 +35,11 @@ namespace {
 
 constexpr int kThreads = 256;
 constexpr int kDk = 128;
-constexpr int kBoxBytes = 64 * 64 * 2;
-constexpr int MP = 65;                     // row stride of the fp32 C x C matrices
-constexpr int kMatBytes = 64 * MP * 4;     // 16640
+constexpr int kBoxBytes = 64 * 64 * 2;     // one TMA box: 64 rows x 64 bf16
+constexpr int kNBytes = 64 * 64 * 4;       // one C x C fp32 matrix in global memory
+constexpr int MP = 68;                     // row stride (floats) of the shared C x C matrices
+constexpr int kMat = 64 * MP;              // floats per shared C x C matrix
+constexpr uint32_t kWorkBytes = 131072;    // [K;Q] tiles + phase 0/1 scratch; later two slabs
 
 struct TcGradArgs {
     const __nv_bfloat16* q2;
@@ -57,6 +64,46 @@ struct TcGradArgs {
     int T, H, dv, E, NT, use_delta, out_f32;
 };
 
+// 4 x 4 block (rows R0.., columns S0..) of a shared row-major matrix.
+__device__ __forceinline__ void ld4x4(const float* M, int R0, int S0, float (&v)[4][4]) {
+#pragma unroll
+    for (int a = 0; a < 4; ++a) {
+        const float4 x = *reinterpret_cast<const float4*>(M + (R0 + a) * MP + S0);
+        v[a][0] = x.x; v[a][1] = x.y; v[a][2] = x.z; v[a][3] = x.w;
+    }
+}
+
+// out[a][c] = sum_x A[x][R0 + a] B[x][S0 + c]  (both operands stored with x as the row).
+__device__ __forceinline__ void mm4x4(const float* A, const float* B, int R0, int S0, float (&out)[4][4]) {
+#pragma unroll
+    for (int a = 0; a < 4; ++a)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) out[a][c] = 0.f;
+#pragma unroll 4
+    for (int x = 0; x < 64; ++x) {
+        const float4 u = *reinterpret_cast<const float4*>(A + x * MP + R0);
+        const float4 w = *reinterpret_cast<const float4*>(B + x * MP + S0);
+        const float ua[4] = {u.x, u.y, u.z, u.w}, wb[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+        for (int a = 0; a < 4; ++a)
+#pragma unroll
+            for (int c = 0; c < 4; ++c) out[a][c] = fmaf(ua[a], wb[c], out[a][c]);
+    }
+}
+
+// Four consecutive values as bf16 hi/lo (8 bytes into each tile).
+__device__ __forceinline__ void st4_split(uint8_t* hi, uint8_t* lo, uint32_t off, float v0, float v1,
+                                          float v2, float v3) {
+    const __nv_bfloat162 h0 = __floats2bfloat162_rn(v0, v1), h1 = __floats2bfloat162_rn(v2, v3);
+    const float2 f0 = __bfloat1622float2(h0), f1 = __bfloat1622float2(h1);
+    const __nv_bfloat162 l0 = __floats2bfloat162_rn(v0 - f0.x, v1 - f0.y);
+    const __nv_bfloat162 l1 = __floats2bfloat162_rn(v2 - f1.x, v3 - f1.y);
+    *reinterpret_cast<uint2*>(hi + off) =
+        make_uint2(*reinterpret_cast<const uint32_t*>(&h0), *reinterpret_cast<const uint32_t*>(&h1));
+    *reinterpret_cast<uint2*>(lo + off) =
+        make_uint2(*reinterpret_cast<const uint32_t*>(&l0), *reinterpret_cast<const uint32_t*>(&l1));
+}
+
 __device__ __forceinline__ void load_row8(const float* src, float* v) {
     const float4 a = reinterpret_cast<const float4*>(src)[0];
     const float4 c = reinterpret_cast<const float4*>(src)[1];
@@ -74,6 +121,50 @@ __device__ __forceinline__ void load_bf16x8(const uint8_t* src, float* v) {
     }
 }
 
+// bf16 hi/lo split of 8 values into two tiles with different layouts.
+__device__ __forceinline__ void st8_split2(uint8_t* hi, uint32_t off_hi, uint8_t* lo,
+                                           uint32_t off_lo, const float* v) {
+    uint32_t h[4], l[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        __nv_bfloat162 hv = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
+        const float2 hf = __bfloat1622float2(hv);
+        __nv_bfloat162 lv = __floats2bfloat162_rn(v[2 * i] - hf.x, v[2 * i + 1] - hf.y);
+        h[i] = *reinterpret_cast<uint32_t*>(&hv);
+        l[i] = *reinterpret_cast<uint32_t*>(&lv);
+    }
+    *reinterpret_cast<uint4*>(hi + off_hi) = make_uint4(h[0], h[1], h[2], h[3]);
+    *reinterpret_cast<uint4*>(lo + off_lo) = make_uint4(l[0], l[1], l[2], l[3]);
+}
+
+// One halving step of a warp transpose-reduction over 2S values per lane.
+template <int S>
+__device__ __forceinline__ void xreduce_step(float* v, int lane) {
+    const bool up = (lane & S) != 0;
+#pragma unroll
+    for (int k = 0; k < S; ++k) {
+        const float send = up ? v[k] : v[k + S];
+        const float keep = up ? v[k + S] : v[k];
+        v[k] = keep + __shfl_xor_sync(0xffffffffu, send, S);
+    }
+}
+// v[0..31] per lane -> the return value of lane l is the sum over the warp's lanes of v[l].
+__device__ __forceinline__ float xreduce32(float* v, int lane) {
+    xreduce_step<16>(v, lane);
+    xreduce_step<8>(v, lane);
+    xreduce_step<4>(v, lane);
+    xreduce_step<2>(v, lane);
+    xreduce_step<1>(v, lane);
+    return v[0];
+}
+
+// Element j (0..31) of a thread's column of packed bf16 pairs, as fp32.
+__device__ __forceinline__ float unpack_bf16(const uint32_t* pk, int j) {
+    const uint32_t w = pk[j >> 1];
+    return __uint_as_float((j & 1) ? (w & 0xffff0000u) : (w << 16));
+}
+
+template <int OUT_F32>
 __global__ void __launch_bounds__(kThreads, 1)
 bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                           const __grid_constant__ CUtensorMap map_q,
@@ -85,29 +176,41 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
     const int t0 = c * 64, n = min(64, T - t0);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int T64 = 64 * dv * 2;               // bytes of a [64][dv] bf16 tile
+    const uint32_t T64 = 64u * dv * 2;         // bytes of a [64][dv] bf16 tile
+    const int nb = dv / 64;                    // 64-column blocks of a value row
 
-    uint8_t* sKQ = sm;                         // [K rows | Q rows] x 2 blocks (TMA)
-    uint8_t* sDO = sKQ + 4 * kBoxBytes;        // dO [64][dv] bf16 (TMA)
-    uint8_t* sX = sDO + 2 * kBoxBytes;         // 64 KB work tiles
-    uint8_t* sY = sX + 65536;                  // 64 KB work tiles
-    float* Gs = reinterpret_cast<float*>(sY + 65536);
-    float* k2s = Gs + 64 * E;
-    float* q2s = k2s + 64 * E;
-    float* dbq = q2s + 64 * E;
-    float* dak = dbq + 64 * E;
-    float* dwk = dak + 64 * E;
-    float* dk2a = dwk + 64 * E;
+    // persistent operands (SW128 K-major over the value dimension)
+    uint8_t* sB = sm;                          // [dO ; -dRes hi]: 128 rows, 16 KB per block
+    uint8_t* sRlo = sB + 2 * T64;              // -dRes lo: 64 rows
+    uint8_t* sUh = sRlo + T64;                 // U hi
+    uint8_t* sUl = sUh + T64;                  // U lo
+    uint8_t* W = sUl + T64;                    // 128 KB work region
+    uint8_t* sKQ = W;                          // [K rows | Q rows] per 64-column block (TMA)
+    uint8_t* scr = W + 4 * kBoxBytes;          // 96 KB: phase 0 staging, six C x C matrices, A3
+    uint8_t* bufS = W;                         // phase 2: S_e slab (hi, lo)
+    uint8_t* bufD = W + 65536;                 // phase 2: dS'_e slab (hi, lo)
+    float* Gs = reinterpret_cast<float*>(W + kWorkBytes);
+    __nv_bfloat16* k2s = reinterpret_cast<__nv_bfloat16*>(Gs + 64 * E);
+    __nv_bfloat16* q2s = k2s + 64 * E;
+    float* dk2a = reinterpret_cast<float*>(q2s + 64 * E);
     float* dq2a = dk2a + 64 * E;
     float* dGa = dq2a + 64 * E;
-    float* bs = dGa + 64 * E;                  // [64]
+    float* dwk = dGa + 64 * E;
+    float* bs = dwk + 64 * E;                  // [64]
     float* dba = bs + 64;                      // [64]
     float* dgc = dba + 64;                     // [16]
-    float* red = dgc + 16;                     // [2][128] row-dot halves
-    float* red2 = red + 256;                   // [256]
+    float* scl = dgc + 16;                     // [3][64]: b_e, a_e, w_e of the current slice
+    float* red = scl + 192;                    // [3][4][64] row-dot partials per lane quarter
+    float* frw = red + 768;                    // [8] Frobenius partials per warp
 
     __shared__ __align__(8) uint64_t bar_ld, bar_mma, bar_s, bar_d;
     __shared__ uint32_t tmem_slot;
+
+    const size_t sbase = ((size_t(b) * H + h) * NT + c) * E;   // this chunk's first slab
+    const uint32_t slab_bytes = uint32_t(kDk) * dv * 4;        // hi tile + lo tile
+    const uint32_t LO = uint32_t(kDk) * dv * 2;                // lo tile offset in a slab
+    const uint8_t* gS = reinterpret_cast<const uint8_t*>(p.Sck);
+    const uint8_t* gD = reinterpret_cast<const uint8_t*>(p.dSck);
 
     if (warp == 0) {
         tmem_alloc(&tmem_slot, 512);
@@ -119,21 +222,22 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         mbar_init(&bar_s, 1);
         mbar_init(&bar_d, 1);
         fence_barrier_init();
-        mbar_arrive_expect_tx(&bar_ld, 4 * kBoxBytes + (dv / 64) * kBoxBytes);
+        mbar_arrive_expect_tx(&bar_ld, 4 * kBoxBytes + nb * kBoxBytes);
         for (int j = 0; j < 2; ++j) {
             tma_load_4d(sKQ + j * 2 * kBoxBytes, &map_k, &bar_ld, 64 * j, h, t0, b);
             tma_load_4d(sKQ + j * 2 * kBoxBytes + kBoxBytes, &map_q, &bar_ld, 64 * j, h, t0, b);
         }
-        for (int j = 0; j < dv / 64; ++j) tma_load_4d(sDO + j * kBoxBytes, &map_do, &bar_ld, 64 * j, h, t0, b);
+        for (int j = 0; j < nb; ++j) tma_load_4d(sB + j * 2 * kBoxBytes, &map_do, &bar_ld, 64 * j, h, t0, b);
+        bulk_prefetch_l2(gS + sbase * slab_bytes, slab_bytes);
+        if (p.use_delta) bulk_prefetch_l2(p.Nmat + ((size_t(b) * H + h) * NT + c) * (64 * 64), kNBytes);
+        bulk_prefetch_l2(gD + sbase * slab_bytes, slab_bytes);
     }
-    // small per-chunk arrays
     for (int i = tid; i < 64 * E; i += kThreads) {
         const int r = i / E, e = i - (i / E) * E;
         const int rr = r < n ? r : n - 1;
         Gs[i] = p.G[tok_idx(b, t0 + rr, h, e, T, H, E)];
-        k2s[i] = r < n ? __bfloat162float(p.k2[tok_idx(b, t0 + r, h, e, T, H, E)]) : 0.f;
-        q2s[i] = r < n ? __bfloat162float(p.q2[tok_idx(b, t0 + r, h, e, T, H, E)]) : 0.f;
-        dbq[i] = dak[i] = dwk[i] = 0.f;
+        k2s[i] = r < n ? p.k2[tok_idx(b, t0 + r, h, e, T, H, E)] : __float2bfloat16_rn(0.f);
+        q2s[i] = r < n ? p.q2[tok_idx(b, t0 + r, h, e, T, H, E)] : __float2bfloat16_rn(0.f);
     }
     if (tid < 64) {
         bs[tid] = tid < n ? (p.beta ? p.beta[(size_t(b) * T + t0 + tid) * H + h] : 1.f) : 0.f;
@@ -141,50 +245,78 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     }
     if (tid < 16) dgc[tid] = 0.f;
 
-    // ---- phase 0 staging: U -> sX (hi, lo); dU, Res (sGLA: V) -> sY (hi, lo, hi, lo)
-    // (8-column chunks; consecutive threads take consecutive chunks of a row)
-    for (int ci = tid; ci < 64 * (dv / 8); ci += kThreads) {
-        const int r = ci / (dv / 8), cc = (ci % (dv / 8)) * 8;
-        {
-            float u[8], du[8], rs[8];
-            if (r < n) {
+    // ---- staging: U -> sUh/sUl; -dRes -> sB rows 64..127 (hi), sRlo (lo);
+    //      dU, Res (sGLA: V) -> scratch (hi, lo, hi, lo) for dT
+    uint8_t* sdUh = scr;
+    uint8_t* sdUl = scr + T64;
+    uint8_t* sRh = scr + 2 * T64;
+    uint8_t* sRl = scr + 3 * T64;
+    {   // every load of this thread is issued before the first split (one round of latency)
+        constexpr int kIt = 64 * 128 / 8 / kThreads;   // 8-column chunks per thread at dv = 128
+        const int cpr = dv / 8;
+        float u[kIt][8], du[kIt][8], rs[kIt][8], dr[kIt][8];
+#pragma unroll
+        for (int it = 0; it < kIt; ++it) {
+            const int ci = tid + it * kThreads, r = ci / cpr, cc = (ci % cpr) * 8;
+            if (ci < 64 * cpr && r < n) {
                 const size_t off = tok_idx(b, t0 + r, h, cc, T, H, dv);
-                load_row8(p.Ubuf + off, u);
-                load_row8(p.dUbuf + off, du);
+                load_row8(p.Ubuf + off, u[it]);
+                load_row8(p.dUbuf + off, du[it]);
                 if (p.use_delta) {
-                    load_row8(p.Rbuf + off, rs);
+                    load_row8(p.Rbuf + off, rs[it]);
+                    load_row8(p.dRbuf + off, dr[it]);
                 } else {
-                    for (int i = 0; i < 8; ++i) rs[i] = __bfloat162float(p.v[off + i]);
+                    const uint4 raw = *reinterpret_cast<const uint4*>(p.v + off);
+                    load_bf16x8(reinterpret_cast<const uint8_t*>(&raw), rs[it]);
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) dr[it][i] = 0.f;
                 }
             } else {
-                for (int i = 0; i < 8; ++i) u[i] = du[i] = rs[i] = 0.f;
+#pragma unroll
+                for (int i = 0; i < 8; ++i) u[it][i] = du[it][i] = rs[it][i] = dr[it][i] = 0.f;
             }
-            const uint32_t o = sw128_offset(r, cc, 64);
-            st8_split(sX, sX + T64, o, u);
-            st8_split(sY, sY + T64, o, du);
-            st8_split(sY + 2 * T64, sY + 3 * T64, o, rs);
+        }
+#pragma unroll
+        for (int it = 0; it < kIt; ++it) {
+            const int ci = tid + it * kThreads, r = ci / cpr, cc = (ci % cpr) * 8;
+            if (ci < 64 * cpr) {
+#pragma unroll
+                for (int i = 0; i < 8; ++i) dr[it][i] = -dr[it][i];
+                const uint32_t o = sw128_offset(r, cc, 64);
+                st8_split(sUh, sUl, o, u[it]);
+                st8_split(sdUh, sdUl, o, du[it]);
+                st8_split(sRh, sRl, o, rs[it]);
+                st8_split2(sB, sw128_offset(64 + r, cc, 128), sRlo, o, dr[it]);
+            }
         }
     }
+    fence_proxy_async_smem();
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = tmem_slot;
-    const uint32_t tACC = tmem, tP = tmem + 128, tP2 = tmem + 128 + dv;
+    const uint32_t tACC = tmem, tD1 = tmem + 128, tD2 = tmem + 256;
 
-    bool ok = mbar_wait(&bar_ld, 0);
-    fence_proxy_async_smem();
-    if (__syncthreads_or(!ok)) {
-        if (tid == 0) record_device_error(p.err, TLA_ERR_TIMEOUT);
+    uint32_t mph = 0;
+    // Failure exit: record the timeout, wait (bounded) for this CTA's copies and
+    // products still in flight, free TMEM.
+    auto bail = [&](uint64_t* pend_a, uint32_t pa, uint64_t* pend_b, uint32_t pb, bool mma) {
+        if (tid == 0) {
+            record_device_error(p.err, TLA_ERR_TIMEOUT);
+            if (pend_a) mbar_wait(pend_a, pa);
+            if (pend_b) mbar_wait(pend_b, pb);
+            if (mma) mbar_wait(&bar_mma, mph);
+        }
+        tc_fence_before();
         __syncthreads();
         if (warp == 0) tmem_dealloc(tmem, 512);
+    };
+
+    bool ok = mbar_wait(&bar_ld, 0);
+    if (__syncthreads_or(!ok)) {
+        bail(&bar_ld, 0, nullptr, 0, false);
         return;
     }
-    uint32_t mph = 0;
-    auto mma_wait = [&]() -> bool {
-        const bool w = mbar_wait(&bar_mma, mph);
-        mph ^= 1;
-        return w;
-    };
 
     // ---- phase 0 products
     if (tid == 0) {
@@ -195,42 +327,52 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         }
         const uint32_t id64 = idesc_bf16_f32(64, 64, 0, 0);
         for (int ks = 0; ks < dv / 16; ++ks) {
-            const uint32_t o = (ks >> 2) * kBoxBytes + (ks & 3) * 32;
-            const uint64_t a = smem_desc(smem_u32(sDO) + o, 16, 1024);
-            umma_bf16(tmem + 192, a, smem_desc(smem_u32(sX) + o, 16, 1024), id64, ks > 0 ? 1u : 0u);
-            umma_bf16(tmem + 192, a, smem_desc(smem_u32(sX + T64) + o, 16, 1024), id64, 1u);
-            const uint64_t uh = smem_desc(smem_u32(sY) + o, 16, 1024);
-            const uint64_t ul = smem_desc(smem_u32(sY + T64) + o, 16, 1024);
-            const uint64_t rh = smem_desc(smem_u32(sY + 2 * T64) + o, 16, 1024);
-            const uint64_t rl = smem_desc(smem_u32(sY + 3 * T64) + o, 16, 1024);
+            const uint32_t k32 = (ks & 3) * 32;
+            const uint32_t o = (ks >> 2) * kBoxBytes + k32;
+            const uint64_t a = smem_desc(smem_u32(sB) + (ks >> 2) * 2 * kBoxBytes + k32, 16, 1024);
+            umma_bf16(tmem + 192, a, smem_desc(smem_u32(sUh) + o, 16, 1024), id64, ks > 0 ? 1u : 0u);
+            umma_bf16(tmem + 192, a, smem_desc(smem_u32(sUl) + o, 16, 1024), id64, 1u);
+            const uint64_t uh = smem_desc(smem_u32(sdUh) + o, 16, 1024);
+            const uint64_t ul = smem_desc(smem_u32(sdUl) + o, 16, 1024);
+            const uint64_t rh = smem_desc(smem_u32(sRh) + o, 16, 1024);
+            const uint64_t rl = smem_desc(smem_u32(sRl) + o, 16, 1024);
             umma_bf16(tmem + 256, uh, rh, id64, ks > 0 ? 1u : 0u);
             umma_bf16(tmem + 256, uh, rl, id64, 1u);
             umma_bf16(tmem + 256, ul, rh, id64, 1u);
         }
         umma_commit(&bar_mma);
     }
-    ok = mma_wait();
+    // N (the chunk's (I + L)^-1, row-major) into registers while the products run
+    const size_t mat = ((size_t(b) * H + h) * NT + c) * (64 * 64);
+    float nv[16];
+#pragma unroll
+    for (int k = 0; k < 16; ++k) nv[k] = p.use_delta ? p.Nmat[mat + tid + k * kThreads] : 0.f;
+    ok = mbar_wait(&bar_mma, mph);
     if (__syncthreads_or(!ok)) {
-        if (tid == 0) record_device_error(p.err, TLA_ERR_TIMEOUT);
-        __syncthreads();
-        if (warp == 0) tmem_dealloc(tmem, 512);
+        bail(nullptr, 0, nullptr, 0, true);
         return;
     }
+    mph ^= 1;
     tc_fence_after();
-    // TMEM -> fp32 C x C matrices (KK, QK in sX; dA, dT in sY)
+
+    // fp32 C x C matrices in the scratch area: row-major, row stride MP (float4-aligned rows)
+    float* Mkk = reinterpret_cast<float*>(scr);
+    float* Mqk = Mkk + kMat;
+    float* MdA = Mqk + kMat;
+    float* MdT = MdA + kMat;
+    // TMEM -> KK, QK (M = 128: rows are lanes), dA, dT (M = 64: rows 16 per lane quarter)
     {
-        float* MKK = reinterpret_cast<float*>(sX);
-        float* MQK = reinterpret_cast<float*>(sX + kMatBytes);
-        float* MdA = reinterpret_cast<float*>(sY);
-        float* MdT = reinterpret_cast<float*>(sY + kMatBytes);
         const int wq = warp & 3, L = wq * 32 + lane;
         if (warp < 4) {
-            float* dst = L < 64 ? MKK + L * MP : MQK + (L - 64) * MP;
+            float* dst = (L < 64 ? Mkk : Mqk) + (L & 63) * MP;
             for (int j = 0; j < 64; j += 16) {
                 float v[16];
                 tmem_ld16(tmem_lane_addr(tmem + 128, warp, j), v);
                 tmem_wait_ld();
-                for (int i = 0; i < 16; ++i) dst[j + i] = v[i];
+#pragma unroll
+                for (int q = 0; q < 4; ++q)
+                    *reinterpret_cast<float4*>(dst + j + 4 * q) =
+                        make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
             }
         } else {
             const int r = 16 * wq + (lane & 15);
@@ -240,431 +382,460 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                 tmem_ld16(tmem_lane_addr(tmem + 256, warp, j), vt);
                 tmem_wait_ld();
                 if (lane < 16)
-                    for (int i = 0; i < 16; ++i) {
-                        MdA[r * MP + j + i] = va[i];
-                        MdT[r * MP + j + i] = vt[i];
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        *reinterpret_cast<float4*>(MdA + r * MP + j + 4 * q) =
+                            make_float4(va[4 * q], va[4 * q + 1], va[4 * q + 2], va[4 * q + 3]);
+                        *reinterpret_cast<float4*>(MdT + r * MP + j + 4 * q) =
+                            make_float4(vt[4 * q], vt[4 * q + 1], vt[4 * q + 2], vt[4 * q + 3]);
                     }
             }
         }
     }
     tc_fence_before();
     __syncthreads();
-    const int s_own = tid & 63, r_base = tid >> 6;   // entries (r_base + 4j, s_own), j < 16
-    float dA[16], dT[16], QK[16], KK[16];
-    {
-        const float* MKK = reinterpret_cast<const float*>(sX);
-        const float* MQK = reinterpret_cast<const float*>(sX + kMatBytes);
-        const float* MdA = reinterpret_cast<const float*>(sY);
-        const float* MdT = reinterpret_cast<const float*>(sY + kMatBytes);
-#pragma unroll
-        for (int j = 0; j < 16; ++j) {
-            const int r = r_base + 4 * j;
-            KK[j] = MKK[r * MP + s_own];
-            QK[j] = MQK[r * MP + s_own];
-            dA[j] = MdA[r * MP + s_own];
-            dT[j] = MdT[r * MP + s_own];
-        }
-    }
+    // ---- phase 1: C x C algebra on CUDA cores; each thread owns the 4 x 4 block of
+    // rows R0..R0+3 and columns S0..S0+3.
+    const int R0 = 4 * (tid >> 4), S0 = 4 * (tid & 15);
+    float KK[4][4], QK[4][4], dA[4][4], dT[4][4];
+    ld4x4(Mkk, R0, S0, KK);
+    ld4x4(Mqk, R0, S0, QK);
+    ld4x4(MdA, R0, S0, dA);
+    ld4x4(MdT, R0, S0, dT);
     __syncthreads();
-
-    // ---- phase 1: C x C algebra on CUDA cores
-    float* B0 = reinterpret_cast<float*>(sX);
-    float* B1 = reinterpret_cast<float*>(sX + kMatBytes);
-    float* B2 = reinterpret_cast<float*>(sX + 2 * kMatBytes);
-    float* B3 = reinterpret_cast<float*>(sY);
-    float* B4 = reinterpret_cast<float*>(sY + kMatBytes);
-    float* B5 = reinterpret_cast<float*>(sY + 2 * kMatBytes);
-    const size_t mat = ((size_t(b) * H + h) * NT + c) * (64 * 64);
+    float* Nm = reinterpret_cast<float*>(scr);   // N
+    float* NmT = Nm + kMat;                       // N^T
+    float* dNT = NmT + kMat;                       // dN^T, then dR
+    float* Fm = dNT + kMat;                       // F, then dR'
+    float* dKKm = Fm + kMat;                      // dKK
     if (p.use_delta)
-        for (int i = tid; i < 64 * 64; i += kThreads) B0[(i >> 6) * MP + (i & 63)] = p.Nmat[mat + i];
-    float Rv[16], Rq[16];
 #pragma unroll
-    for (int j = 0; j < 16; ++j) Rv[j] = Rq[j] = 0.f;
-    for (int e = 0; e < E; ++e) {            // 16 independent entries per slice
-        const float gs = Gs[s_own * E + e], ks = k2s[s_own * E + e];
+        for (int k = 0; k < 16; ++k) {
+            const int i = tid + k * kThreads, x = i >> 6, s = i & 63;
+            Nm[x * MP + s] = nv[k];
+            NmT[s * MP + x] = nv[k];
+        }
+    float Rv[4][4], Rq[4][4];   // sum_e k2_e(r) k2_e(s) exp(G_e(r) - G_e(s)), same with q2_e(r), r >= s
 #pragma unroll
-        for (int j = 0; j < 16; ++j) {
-            const int r = r_base + 4 * j;
-            // exp of a non-positive difference (entries above the diagonal are discarded)
-            const float gam = expf(fminf(Gs[r * E + e] - gs, 0.f));
-            const float ks2 = (r >= s_own) ? ks * gam : 0.f;
-            Rv[j] = fmaf(k2s[r * E + e], ks2, Rv[j]);
-            Rq[j] = fmaf(q2s[r * E + e], ks2, Rq[j]);
+    for (int a = 0; a < 4; ++a)
+#pragma unroll
+        for (int c2 = 0; c2 < 4; ++c2) Rv[a][c2] = Rq[a][c2] = 0.f;
+    for (int e = 0; e < E; ++e) {
+        float gs[4], ksv[4];
+#pragma unroll
+        for (int c2 = 0; c2 < 4; ++c2) {
+            gs[c2] = Gs[(S0 + c2) * E + e];
+            ksv[c2] = __bfloat162float(k2s[(S0 + c2) * E + e]);
+        }
+#pragma unroll
+        for (int a = 0; a < 4; ++a) {
+            const float gr = Gs[(R0 + a) * E + e];
+            const float kr = __bfloat162float(k2s[(R0 + a) * E + e]);
+            const float qr = __bfloat162float(q2s[(R0 + a) * E + e]);
+#pragma unroll
+            for (int c2 = 0; c2 < 4; ++c2) {
+                // exp of a non-positive difference (entries above the diagonal are discarded)
+                const float gam = expf(fminf(gr - gs[c2], 0.f));
+                const float ks2 = (R0 + a >= S0 + c2) ? ksv[c2] * gam : 0.f;
+                Rv[a][c2] = fmaf(kr, ks2, Rv[a][c2]);
+                Rq[a][c2] = fmaf(qr, ks2, Rq[a][c2]);
+            }
         }
     }
     __syncthreads();
+    float dKK[4][4], rp[4];
     if (p.use_delta) {
+        {   // dN = dT diag(beta) (stored transposed); column terms of dbeta: sum_r dT (.) N
+            float cp[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-        for (int j = 0; j < 16; ++j) {
-            const int r = r_base + 4 * j, s = s_own;
-            B1[r * MP + s] = dT[j] * bs[s];              // dN
-            B2[r * MP + s] = dT[j] * B0[r * MP + s];     // column terms of dbeta
+            for (int a = 0; a < 4; ++a) {
+                const float4 nr = *reinterpret_cast<const float4*>(Nm + (R0 + a) * MP + S0);
+                cp[0] = fmaf(dT[a][0], nr.x, cp[0]);
+                cp[1] = fmaf(dT[a][1], nr.y, cp[1]);
+                cp[2] = fmaf(dT[a][2], nr.z, cp[2]);
+                cp[3] = fmaf(dT[a][3], nr.w, cp[3]);
+            }
+#pragma unroll
+            for (int c2 = 0; c2 < 4; ++c2) {
+                const float bsv = bs[S0 + c2];
+                *reinterpret_cast<float4*>(dNT + (S0 + c2) * MP + R0) =
+                    make_float4(dT[0][c2] * bsv, dT[1][c2] * bsv, dT[2][c2] * bsv, dT[3][c2] * bsv);
+                cp[c2] += __shfl_xor_sync(0xffffffffu, cp[c2], 16);
+            }
+            if (lane < 16)
+#pragma unroll
+                for (int c2 = 0; c2 < 4; ++c2) red[warp * 64 + S0 + c2] = cp[c2];
         }
         __syncthreads();
         if (tid < 64) {
             float acc = 0.f;
-            for (int r = 0; r < 64; ++r) acc += B2[r * MP + tid];
+#pragma unroll
+            for (int w = 0; w < kThreads / 32; ++w) acc += red[w * 64 + tid];
             dba[tid] += acc;
         }
-        {                                               // F = dN N^T (16 independent sums)
-            float acc[16];
+        {   // F = dN N^T
+            float F[4][4];
+            mm4x4(dNT, NmT, R0, S0, F);
 #pragma unroll
-            for (int j = 0; j < 16; ++j) acc[j] = 0.f;
-#pragma unroll 4
-            for (int x = 0; x < 64; ++x) {
-                const float nsx = B0[s_own * MP + x];
-#pragma unroll
-                for (int j = 0; j < 16; ++j) acc[j] = fmaf(B1[(r_base + 4 * j) * MP + x], nsx, acc[j]);
-            }
-#pragma unroll
-            for (int j = 0; j < 16; ++j) B3[(r_base + 4 * j) * MP + s_own] = acc[j];
+            for (int a = 0; a < 4; ++a)
+                *reinterpret_cast<float4*>(Fm + (R0 + a) * MP + S0) = make_float4(F[a][0], F[a][1], F[a][2], F[a][3]);
         }
         __syncthreads();
-        float dL[16];
-        {                                               // dM = -N^T F, strictly lower part
+        float dL[4][4];   // dM = -N^T F, strictly lower part
+        mm4x4(Nm, Fm, R0, S0, dL);
 #pragma unroll
-            for (int j = 0; j < 16; ++j) dL[j] = 0.f;
-#pragma unroll 4
-            for (int x = 0; x < 64; ++x) {
-                const float fxs = B3[x * MP + s_own];
+        for (int a = 0; a < 4; ++a)
 #pragma unroll
-                for (int j = 0; j < 16; ++j) dL[j] = fmaf(B0[x * MP + r_base + 4 * j], fxs, dL[j]);
-            }
-#pragma unroll
-            for (int j = 0; j < 16; ++j) dL[j] = (r_base + 4 * j > s_own) ? -dL[j] : 0.f;
-        }
+            for (int c2 = 0; c2 < 4; ++c2) dL[a][c2] = (R0 + a > S0 + c2) ? -dL[a][c2] : 0.f;
         __syncthreads();
 #pragma unroll
-        for (int j = 0; j < 16; ++j) {
-            const int r = r_base + 4 * j, s = s_own;
-            B1[r * MP + s] = dL[j] * bs[r] * KK[j];    // dR
-            B4[r * MP + s] = dL[j] * bs[r] * Rv[j];    // dKK
-            B5[r * MP + s] = dL[j] * KK[j] * Rv[j];    // row terms of dbeta
+        for (int a = 0; a < 4; ++a) {
+            const float br = bs[R0 + a];
+            float dR[4];
+            rp[a] = 0.f;
+#pragma unroll
+            for (int c2 = 0; c2 < 4; ++c2) {
+                dR[c2] = dL[a][c2] * br * KK[a][c2];
+                dKK[a][c2] = dL[a][c2] * br * Rv[a][c2];
+                rp[a] = fmaf(dL[a][c2] * KK[a][c2], Rv[a][c2], rp[a]);   // row terms of dbeta
+            }
+            *reinterpret_cast<float4*>(dNT + (R0 + a) * MP + S0) = make_float4(dR[0], dR[1], dR[2], dR[3]);
+            *reinterpret_cast<float4*>(dKKm + (R0 + a) * MP + S0) =
+                make_float4(dKK[a][0], dKK[a][1], dKK[a][2], dKK[a][3]);
         }
     } else {
 #pragma unroll
-        for (int j = 0; j < 16; ++j) {
-            const int r = r_base + 4 * j, s = s_own;
-            B1[r * MP + s] = 0.f;
-            B4[r * MP + s] = 0.f;
-            B5[r * MP + s] = (r == s) ? dT[j] : 0.f;   // T = diag(beta)
+        for (int a = 0; a < 4; ++a) {
+            rp[a] = 0.f;
+#pragma unroll
+            for (int c2 = 0; c2 < 4; ++c2) {
+                dKK[a][c2] = 0.f;
+                if (R0 + a == S0 + c2) rp[a] = dT[a][c2];   // T = diag(beta)
+            }
+            *reinterpret_cast<float4*>(dNT + (R0 + a) * MP + S0) = make_float4(0.f, 0.f, 0.f, 0.f);
+            *reinterpret_cast<float4*>(dKKm + (R0 + a) * MP + S0) = make_float4(0.f, 0.f, 0.f, 0.f);
         }
+    }
+    // row sums of dbeta's row terms over the 16 threads of a half-warp (one half-warp per row block)
+#pragma unroll
+    for (int a = 0; a < 4; ++a) {
+#pragma unroll
+        for (int s = 1; s < 16; s <<= 1) rp[a] += __shfl_xor_sync(0xffffffffu, rp[a], s);
+    }
+    if ((tid & 15) == 0)
+#pragma unroll
+        for (int a = 0; a < 4; ++a) dba[R0 + a] += rp[a];
+    float Pv[4][4];   // P = dA (.) R'
+#pragma unroll
+    for (int a = 0; a < 4; ++a) {
+        float dRq[4];
+#pragma unroll
+        for (int c2 = 0; c2 < 4; ++c2) {
+            const bool low = R0 + a >= S0 + c2;
+            dRq[c2] = low ? dA[a][c2] * QK[a][c2] : 0.f;
+            Pv[a][c2] = low ? dA[a][c2] * Rq[a][c2] : 0.f;
+        }
+        *reinterpret_cast<float4*>(Fm + (R0 + a) * MP + S0) = make_float4(dRq[0], dRq[1], dRq[2], dRq[3]);
+    }
+    __syncthreads();
+    {   // through R (dR) and R' (dR'): one (token, slice) pair per thread
+        const float* dRm = dNT;
+        const float* dRqm = Fm;
+        for (int i = tid; i < 64 * E; i += kThreads) {
+            const int x = i / E, e = i - (i / E) * E;
+            const float gx = Gs[x * E + e];
+            const float kx = __bfloat162float(k2s[x * E + e]), qx = __bfloat162float(q2s[x * E + e]);
+            float dk2v = 0.f, dq2v = 0.f, dGv = 0.f;
+#pragma unroll 4
+            for (int s = 0; s <= x; ++s) {
+                const float gam = expf(gx - Gs[s * E + e]);
+                const float ks = __bfloat162float(k2s[s * E + e]);
+                const float dR = dRm[x * MP + s], dRq = dRqm[x * MP + s];
+                dk2v = fmaf(dR * ks, gam, dk2v);
+                dq2v = fmaf(dRq * ks, gam, dq2v);
+                dGv = fmaf((dR * kx + dRq * qx) * ks, gam, dGv);
+            }
+#pragma unroll 4
+            for (int r = x; r < 64; ++r) {
+                const float gam = expf(Gs[r * E + e] - gx);
+                const float dR = dRm[r * MP + x], dRq = dRqm[r * MP + x];
+                const float t = (dR * __bfloat162float(k2s[r * E + e]) +
+                                 dRq * __bfloat162float(q2s[r * E + e])) * gam;
+                dk2v += t;
+                dGv = fmaf(-t, kx, dGv);
+            }
+            dk2a[i] = dk2v;
+            dq2a[i] = dq2v;
+            dGa[i] = dGv;
+        }
+    }
+    __syncthreads();
+    // B operands of the last products, bf16 hi/lo (K-major, 64 rows):
+    //   Pt  = P                        (64 x 64)   -> dq rows
+    //   KPt = [dKK + dKK^T | P^T]      (64 x 128)  -> dk rows
+    uint8_t* Pth = scr;
+    uint8_t* Ptl = scr + 8192;
+    uint8_t* KPh = scr + 16384;
+    uint8_t* KPl = scr + 32768;
+#pragma unroll
+    for (int a = 0; a < 4; ++a) {
+        st4_split(Pth, Ptl, sw128_offset(R0 + a, S0, 64), Pv[a][0], Pv[a][1], Pv[a][2], Pv[a][3]);
+        float kc4[4];
+#pragma unroll
+        for (int c2 = 0; c2 < 4; ++c2) kc4[c2] = dKK[a][c2] + dKKm[(S0 + c2) * MP + R0 + a];
+        st4_split(KPh, KPl, sw128_offset(R0 + a, S0, 64), kc4[0], kc4[1], kc4[2], kc4[3]);
     }
 #pragma unroll
-    for (int j = 0; j < 16; ++j) {
-        const int r = r_base + 4 * j, s = s_own;
-        const bool low = r >= s;
-        B2[r * MP + s] = low ? dA[j] * QK[j] : 0.f;    // dR'
-        B3[r * MP + s] = low ? dA[j] * Rq[j] : 0.f;    // P = dA (.) R'
-    }
-    __syncthreads();
-    if (tid < 64) {
-        float acc = 0.f;
-        for (int s = 0; s < 64; ++s) acc += B5[tid * MP + s];
-        dba[tid] += acc;
-    }
-    for (int i = tid; i < 64 * E; i += kThreads) {      // through R (dR in B1) and R' (dR' in B2)
-        const int x = i / E, e = i - (i / E) * E;
-        const float gx = Gs[x * E + e], kx = k2s[x * E + e], qx = q2s[x * E + e];
-        float dk2v = 0.f, dq2v = 0.f, dGv = 0.f;
-        for (int s = 0; s <= x; ++s) {
-            const float gam = expf(gx - Gs[s * E + e]);
-            const float ks = k2s[s * E + e];
-            const float dR = B1[x * MP + s], dRq = B2[x * MP + s];
-            dk2v = fmaf(dR * ks, gam, dk2v);
-            dq2v = fmaf(dRq * ks, gam, dq2v);
-            dGv = fmaf((dR * kx + dRq * qx) * ks, gam, dGv);
-        }
-        for (int r = x; r < 64; ++r) {
-            const float gam = expf(Gs[r * E + e] - gx);
-            const float dR = B1[r * MP + x], dRq = B2[r * MP + x];
-            const float t = (dR * k2s[r * E + e] + dRq * q2s[r * E + e]) * gam;
-            dk2v += t;
-            dGv = fmaf(-t, kx, dGv);
-        }
-        dk2a[i] = dk2v;
-        dq2a[i] = dq2v;
-        dGa[i] = dGv;
-    }
-    __syncthreads();
-    // A3 = [[P, 0], [dKK + dKK^T, P^T]] (128 x 128) as bf16 hi/lo into sX (P in B3, dKK in B4)
-    {
-        const int i = tid >> 1, jh = tid & 1;
-        for (int j0 = jh * 64; j0 < jh * 64 + 64; j0 += 8) {
-            float v[8];
-            for (int u = 0; u < 8; ++u) {
-                const int j = j0 + u;
-                float x;
-                if (i < 64) x = (j < 64) ? B3[i * MP + j] : 0.f;
-                else {
-                    const int r = i - 64;
-                    x = (j < 64) ? B4[r * MP + j] + B4[j * MP + r] : B3[(j - 64) * MP + r];
-                }
-                v[u] = x;
-            }
-            st8_split(sX, sX + 32768, sw128_offset(i, j0, 128), v);
-        }
-    }
+    for (int c2 = 0; c2 < 4; ++c2)
+        st4_split(KPh, KPl, sw128_offset(S0 + c2, 64 + R0, 64), Pv[0][c2], Pv[1][c2], Pv[2][c2], Pv[3][c2]);
     fence_proxy_async_smem();
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
+    // ACC^T (lanes = key dimension d, columns = output rows): [K]^T Pt^T, then [K;Q]^T KPt^T
     if (tid == 0) {
-        const uint32_t id = idesc_bf16_f32(128, kDk, 0, 1);
+        const uint32_t id = idesc_bf16_f32(128, 64, 1, 0);
+        for (int ks = 0; ks < 4; ++ks) {
+            const uint64_t a = smem_desc(smem_u32(sKQ) + ks * 2048, 2 * kBoxBytes, 1024);
+            umma_bf16(tACC, a, smem_desc(smem_u32(Pth) + ks * 32, 16, 1024), id, ks > 0 ? 1u : 0u);
+            umma_bf16(tACC, a, smem_desc(smem_u32(Ptl) + ks * 32, 16, 1024), id, 1u);
+        }
         for (int ks = 0; ks < 8; ++ks) {
-            const uint32_t o = (ks >> 2) * 16384 + (ks & 3) * 32;
-            const uint64_t bq = smem_desc(smem_u32(sKQ) + ks * 2048, 2 * kBoxBytes, 1024);
-            umma_bf16(tACC, smem_desc(smem_u32(sX) + o, 16, 1024), bq, id, ks > 0 ? 1u : 0u);
-            umma_bf16(tACC, smem_desc(smem_u32(sX + 32768) + o, 16, 1024), bq, id, 1u);
+            const uint64_t a = smem_desc(smem_u32(sKQ) + ks * 2048, 2 * kBoxBytes, 1024);
+            const uint32_t o = (ks >> 2) * 8192 + (ks & 3) * 32;
+            umma_bf16(tACC + 64, a, smem_desc(smem_u32(KPh) + o, 16, 1024), id, ks > 0 ? 1u : 0u);
+            umma_bf16(tACC + 64, a, smem_desc(smem_u32(KPl) + o, 16, 1024), id, 1u);
         }
         umma_commit(&bar_mma);
     }
-    ok = mma_wait();
+    // this thread's key dimension d and token block, and its columns of K and Q (bf16 pairs)
+    const int wq = warp & 3, tb = 32 * (warp >> 2), d = wq * 32 + lane;
+    uint32_t kc[16], qc[16];
+    {
+        const uint8_t* kb = sKQ + (d >> 6) * 2 * kBoxBytes;
+#pragma unroll
+        for (int m = 0; m < 16; ++m) {
+            const int t = tb + 2 * m;
+            const uint32_t o0 = sw128_offset(t, d & 63, 64), o1 = sw128_offset(t + 1, d & 63, 64);
+            kc[m] = uint32_t(*reinterpret_cast<const uint16_t*>(kb + o0)) |
+                    (uint32_t(*reinterpret_cast<const uint16_t*>(kb + o1)) << 16);
+            qc[m] = uint32_t(*reinterpret_cast<const uint16_t*>(kb + kBoxBytes + o0)) |
+                    (uint32_t(*reinterpret_cast<const uint16_t*>(kb + kBoxBytes + o1)) << 16);
+        }
+    }
+    ok = mbar_wait(&bar_mma, mph);
     if (__syncthreads_or(!ok)) {
-        if (tid == 0) record_device_error(p.err, TLA_ERR_TIMEOUT);
-        __syncthreads();
-        if (warp == 0) tmem_dealloc(tmem, 512);
+        bail(nullptr, 0, nullptr, 0, true);
         return;
     }
+    mph ^= 1;
     tc_fence_after();
 
-    // ---- phase 2: per slice.  The checkpoint tiles (bf16 hi/lo, operand layout) arrive by
-    // bulk copy: S_e into sX, then dS'_e into sY once the first products have consumed A1.
-    const size_t sbase = ((size_t(b) * H + h) * NT + c) * E;
-    const uint32_t slab_bytes = uint32_t(kDk) * dv * 4;   // hi tile + lo tile
-    const uint32_t LO = uint32_t(kDk) * dv * 2;           // lo tile offset of a checkpoint slab
-    const int wq = warp & 3, L = wq * 32 + lane, half = warp >> 2;
-    const int cpr = dv / 8;   // 8-column chunks per row
+    // ---- phase 2: per slice.  S_e and dS'_e slabs (bf16 hi/lo, operand layout) arrive by
+    // bulk copy over the work region; the next pair is requested once the products and the
+    // Frobenius sum have consumed the current one.
     uint32_t sph = 0, dph = 0;
-    if (tid == 0) {
+    auto issue_slabs = [&](int e) {
         mbar_arrive_expect_tx(&bar_s, slab_bytes);
-        bulk_load(sX, reinterpret_cast<const uint8_t*>(p.Sck) + sbase * kDk * dv * 4, slab_bytes, &bar_s);
-    }
-    bool failed = false;
-    for (int e = 0; e < E && !failed; ++e) {
-        // A1_e = [b_e dO ; -a_e dRes] -> sY
-        for (int ci = tid; ci < 128 * cpr; ci += kThreads) {
-            const int i = ci / cpr, cc = (ci % cpr) * 8;
-            float v[8];
-            if (i < 64) {
-                const float bq = q2s[i * E + e] * expf(Gs[i * E + e]);
-                load_bf16x8(sDO + sw128_offset(i, cc, 64), v);
-                for (int u = 0; u < 8; ++u) v[u] *= bq;
-            } else {
-                const int r = i - 64;
-                if (p.use_delta && r < n) {
-                    const float a = -k2s[r * E + e] * expf(Gs[r * E + e]);
-                    load_row8(p.dRbuf + tok_idx(b, t0 + r, h, cc, T, H, dv), v);
-                    for (int u = 0; u < 8; ++u) v[u] *= a;
-                } else {
-                    for (int u = 0; u < 8; ++u) v[u] = 0.f;
-                }
-            }
-            st8_split(sY, sY + 32768, sw128_offset(i, cc, 128), v);
+        bulk_load(bufS, gS + (sbase + e) * slab_bytes, slab_bytes, &bar_s);
+        mbar_arrive_expect_tx(&bar_d, slab_bytes);
+        bulk_load(bufD, gD + (sbase + e) * slab_bytes, slab_bytes, &bar_d);
+        if (e + 1 < E) {
+            bulk_prefetch_l2(gS + (sbase + e + 1) * slab_bytes, slab_bytes);
+            bulk_prefetch_l2(gD + (sbase + e + 1) * slab_bytes, slab_bytes);
         }
-        bool ok = mbar_wait(&bar_s, sph);
-        sph ^= 1;
-        fence_proxy_async_smem();
+    };
+    if (tid == 0) issue_slabs(0);
+    float acq[32], ack[32];
+#pragma unroll
+    for (int j = 0; j < 32; ++j) acq[j] = ack[j] = 0.f;
+    for (int e = 0; e < E; ++e) {
+        if (tid < 192) {   // b_e, a_e, w_e of the 64 tokens
+            const int r = tid & 63, i = r * E + e;
+            float s;
+            if (tid < 64) s = __bfloat162float(q2s[i]) * expf(Gs[i]);
+            else if (tid < 128) s = __bfloat162float(k2s[i]) * expf(Gs[i]);
+            else s = __bfloat162float(k2s[i]) * expf(Gs[(n - 1) * E + e] - Gs[i]);
+            scl[tid] = s;
+        }
+        const bool ok_s = mbar_wait(&bar_s, sph);
+        const bool ok_d = mbar_wait(&bar_d, dph);
         tc_fence_before();
-        if (__syncthreads_or(!ok)) { failed = true; break; }
+        if (__syncthreads_or(!(ok_s && ok_d))) {
+            bail(&bar_s, sph, &bar_d, dph, false);
+            return;
+        }
+        sph ^= 1;
+        dph ^= 1;
         tc_fence_after();
         if (tid == 0) {
-            const uint32_t idA = idesc_bf16_f32(128, kDk, 0, 0);
+            const uint32_t id128 = idesc_bf16_f32(128, 128, 0, 0);
+            const uint32_t id64 = idesc_bf16_f32(128, 64, 0, 0);
             for (int ks = 0; ks < dv / 16; ++ks) {
-                const uint32_t o = (ks >> 2) * 16384 + (ks & 3) * 32;
-                const uint64_t ah = smem_desc(smem_u32(sY) + o, 16, 1024);
-                const uint64_t al = smem_desc(smem_u32(sY + 32768) + o, 16, 1024);
-                const uint64_t bh = smem_desc(smem_u32(sX) + o, 16, 1024);
-                const uint64_t bl = smem_desc(smem_u32(sX + LO) + o, 16, 1024);
-                umma_bf16(tACC, ah, bh, idA, 1u);
-                umma_bf16(tACC, ah, bl, idA, 1u);
-                umma_bf16(tACC, al, bh, idA, 1u);
-            }
-            const uint32_t idP = idesc_bf16_f32(128, dv, 0, 1);
-            for (int ks = 0; ks < kDk / 16; ++ks) {
-                const uint64_t a = smem_desc(smem_u32(sKQ) + (ks >> 2) * 2 * kBoxBytes + (ks & 3) * 32, 16, 1024);
-                umma_bf16(tP, a, smem_desc(smem_u32(sX) + ks * 2048, 16384, 1024), idP, ks > 0 ? 1u : 0u);
-                umma_bf16(tP, a, smem_desc(smem_u32(sX + LO) + ks * 2048, 16384, 1024), idP, 1u);
+                const uint32_t k32 = (ks & 3) * 32;
+                const uint32_t o128 = (ks >> 2) * 16384 + k32, o64 = (ks >> 2) * 8192 + k32;
+                const uint64_t sh = smem_desc(smem_u32(bufS) + o128, 16, 1024);
+                const uint64_t sl = smem_desc(smem_u32(bufS + LO) + o128, 16, 1024);
+                const uint64_t bh = smem_desc(smem_u32(sB) + o128, 16, 1024);
+                const uint64_t rl = smem_desc(smem_u32(sRlo) + o64, 16, 1024);
+                umma_bf16(tD1, sh, bh, id128, ks > 0 ? 1u : 0u);
+                umma_bf16(tD1, sl, bh, id128, 1u);
+                if (p.use_delta) umma_bf16(tD1 + 64, sh, rl, id64, 1u);
+                const uint64_t dh = smem_desc(smem_u32(bufD) + o128, 16, 1024);
+                const uint64_t dl = smem_desc(smem_u32(bufD + LO) + o128, 16, 1024);
+                const uint64_t uh = smem_desc(smem_u32(sUh) + o64, 16, 1024);
+                const uint64_t ul = smem_desc(smem_u32(sUl) + o64, 16, 1024);
+                umma_bf16(tD2, dh, uh, id64, ks > 0 ? 1u : 0u);
+                umma_bf16(tD2, dl, uh, id64, 1u);
+                umma_bf16(tD2, dh, ul, id64, 1u);
             }
             umma_commit(&bar_mma);
         }
-        ok = mma_wait();
-        if (__syncthreads_or(!ok)) { failed = true; break; }
-        tc_fence_after();
-        if (tid == 0) {   // A1 consumed: dS'_e into sY
-            mbar_arrive_expect_tx(&bar_d, slab_bytes);
-            bulk_load(sY, reinterpret_cast<const uint8_t*>(p.dSck) + (sbase + e) * kDk * dv * 4,
-                      slab_bytes, &bar_d);
-        }
-        // row dots of P_e = [K;Q] S_e while dS'_e is in flight
-        {
-            float acc = 0.f;
-            const int cw = dv / 2;
-            for (int j = half * cw; j < half * cw + cw; j += 16) {
-                float pv[16];
-                tmem_ld16(tmem_lane_addr(tP, warp, j), pv);
-                tmem_wait_ld();
-                float x[16];
-                if (L < 64) {
-                    if (L < n && p.use_delta) {
-                        load_row8(p.dRbuf + tok_idx(b, t0 + L, h, j, T, H, dv), x);
-                        load_row8(p.dRbuf + tok_idx(b, t0 + L, h, j + 8, T, H, dv), x + 8);
-                    } else {
-                        for (int u = 0; u < 16; ++u) x[u] = 0.f;
-                    }
-                } else {
-                    load_bf16x8(sDO + sw128_offset(L - 64, j, 64), x);
-                    load_bf16x8(sDO + sw128_offset(L - 64, j + 8, 64), x + 8);
-                }
-                for (int u = 0; u < 16; ++u) acc = fmaf(x[u], pv[u], acc);
-            }
-            red[half * 128 + L] = acc;
-        }
-        ok = mbar_wait(&bar_d, dph);
-        dph ^= 1;
-        // <dS'_e, S_e> from the hi/lo tiles (hi + lo reproduces each value to ~2^-16)
-        {
+        {   // <dS'_e, S_e> from the hi/lo tiles (hi + lo reproduces each value to ~2^-16)
             float fro = 0.f;
-            for (int ci = tid; ci < 128 * cpr; ci += kThreads) {
-                const uint32_t o = sw128_offset(ci / cpr, (ci % cpr) * 8, 128);
+            for (uint32_t o = tid * 16; o < LO; o += kThreads * 16) {
                 float sh[8], sl[8], dh[8], dl[8];
-                load_bf16x8(sX + o, sh);
-                load_bf16x8(sX + LO + o, sl);
-                load_bf16x8(sY + o, dh);
-                load_bf16x8(sY + LO + o, dl);
+                load_bf16x8(bufS + o, sh);
+                load_bf16x8(bufS + LO + o, sl);
+                load_bf16x8(bufD + o, dh);
+                load_bf16x8(bufD + LO + o, dl);
+#pragma unroll
                 for (int u = 0; u < 8; ++u) fro = fmaf(dh[u] + dl[u], sh[u] + sl[u], fro);
             }
-            red2[tid] = fro;
+#pragma unroll
+            for (int s = 16; s >= 1; s >>= 1) fro += __shfl_xor_sync(0xffffffffu, fro, s);
+            if (lane == 0) frw[warp] = fro;
         }
-        if (__syncthreads_or(!ok)) { failed = true; break; }
-        if (tid < 128) {
-            const float v = red[tid] + red[128 + tid];
-            if (tid < 64) dak[tid * E + e] = -v;
-            else dbq[(tid - 64) * E + e] = v;
+        ok = mbar_wait(&bar_mma, mph);
+        if (__syncthreads_or(!ok)) {
+            bail(nullptr, 0, nullptr, 0, true);
+            return;
         }
-        if (tid == 0) {
+        mph ^= 1;
+        tc_fence_after();
+        if (tid == 0 && e + 1 < E) issue_slabs(e + 1);
+        {
+            float z[32];
+            // D1 query columns: dq += b_e (dO S_e^T); db_e = rowdot(Q, dO S_e^T)
+            tmem_ld16(tmem_lane_addr(tD1, warp, tb), z);
+            tmem_ld16(tmem_lane_addr(tD1, warp, tb + 16), z + 16);
+            tmem_wait_ld();
+#pragma unroll
+            for (int j = 0; j < 32; ++j) {
+                acq[j] = fmaf(scl[tb + j], z[j], acq[j]);
+                z[j] *= unpack_bf16(qc, j);
+            }
+            red[(0 * 4 + wq) * 64 + tb + lane] = xreduce32(z, lane);
+            // D1 key columns: dk += a_e (-dRes S_e^T); da_e = rowdot(K, -dRes S_e^T)
+            tmem_ld16(tmem_lane_addr(tD1, warp, 64 + tb), z);
+            tmem_ld16(tmem_lane_addr(tD1, warp, 64 + tb + 16), z + 16);
+            tmem_wait_ld();
+#pragma unroll
+            for (int j = 0; j < 32; ++j) {
+                ack[j] = fmaf(scl[64 + tb + j], z[j], ack[j]);
+                z[j] *= unpack_bf16(kc, j);
+            }
+            red[(1 * 4 + wq) * 64 + tb + lane] = xreduce32(z, lane);
+            // D2: dk += w_e (U dS'_e^T); dw_e = rowdot(K, U dS'_e^T)
+            tmem_ld16(tmem_lane_addr(tD2, warp, tb), z);
+            tmem_ld16(tmem_lane_addr(tD2, warp, tb + 16), z + 16);
+            tmem_wait_ld();
+#pragma unroll
+            for (int j = 0; j < 32; ++j) {
+                ack[j] = fmaf(scl[128 + tb + j], z[j], ack[j]);
+                z[j] *= unpack_bf16(kc, j);
+            }
+            red[(2 * 4 + wq) * 64 + tb + lane] = xreduce32(z, lane);
+        }
+        tc_fence_before();
+        __syncthreads();
+        if (tid < 64) {   // this slice's row dots -> dq2, dk2, dG (a_e = k2 gamma, b_e = q2 gamma, w_e)
+            const int i = tid * E + e;
+            float db = 0.f, da = 0.f, dw = 0.f;
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                db += red[(0 * 4 + q) * 64 + tid];
+                da += red[(1 * 4 + q) * 64 + tid];
+                dw += red[(2 * 4 + q) * 64 + tid];
+            }
+            const float gam = expf(Gs[i]);
+            const float wdec = expf(Gs[(n - 1) * E + e] - Gs[i]);
+            const float k2v = __bfloat162float(k2s[i]), q2v = __bfloat162float(q2s[i]);
+            dk2a[i] += da * gam + dw * wdec;
+            dq2a[i] += db * gam;
+            dGa[i] += da * (k2v * gam) + db * (q2v * gam) - dw * (k2v * wdec);
+            dwk[i] = dw;
+        } else if (tid == 64) {
             float f = 0.f;
-            for (int i = 0; i < kThreads; ++i) f += red2[i];
+            for (int w = 0; w < kThreads / 32; ++w) f += frw[w];
             dgc[e] = f;
         }
-        // A2_e = [0 ; w_e U] -> sX (S_e consumed)
-        for (int ci = tid; ci < 128 * cpr; ci += kThreads) {
-            const int i = ci / cpr, cc = (ci % cpr) * 8;
-            float v[8];
-            const int r = i - 64;
-            if (i >= 64 && r < n) {
-                const float w = k2s[r * E + e] * expf(Gs[(n - 1) * E + e] - Gs[r * E + e]);
-                load_row8(p.Ubuf + tok_idx(b, t0 + r, h, cc, T, H, dv), v);
-                for (int u = 0; u < 8; ++u) v[u] *= w;
-            } else {
-                for (int u = 0; u < 8; ++u) v[u] = 0.f;
-            }
-            st8_split(sX, sX + 32768, sw128_offset(i, cc, 128), v);
-        }
-        fence_proxy_async_smem();
-        tc_fence_before();
-        __syncthreads();
-        tc_fence_after();
-        if (tid == 0) {
-            const uint32_t idA = idesc_bf16_f32(128, kDk, 0, 0);
-            for (int ks = 0; ks < dv / 16; ++ks) {
-                const uint32_t o = (ks >> 2) * 16384 + (ks & 3) * 32;
-                const uint64_t ah = smem_desc(smem_u32(sX) + o, 16, 1024);
-                const uint64_t al = smem_desc(smem_u32(sX + 32768) + o, 16, 1024);
-                const uint64_t bh = smem_desc(smem_u32(sY) + o, 16, 1024);
-                const uint64_t bl = smem_desc(smem_u32(sY + LO) + o, 16, 1024);
-                umma_bf16(tACC, ah, bh, idA, 1u);
-                umma_bf16(tACC, ah, bl, idA, 1u);
-                umma_bf16(tACC, al, bh, idA, 1u);
-            }
-            const uint32_t idP = idesc_bf16_f32(128, dv, 0, 1);
-            for (int ks = 0; ks < kDk / 16; ++ks) {
-                const uint64_t a = smem_desc(smem_u32(sKQ) + (ks >> 2) * 2 * kBoxBytes + (ks & 3) * 32, 16, 1024);
-                umma_bf16(tP2, a, smem_desc(smem_u32(sY) + ks * 2048, 16384, 1024), idP, ks > 0 ? 1u : 0u);
-                umma_bf16(tP2, a, smem_desc(smem_u32(sY + LO) + ks * 2048, 16384, 1024), idP, 1u);
-            }
-            umma_commit(&bar_mma);
-        }
-        ok = mma_wait();
-        if (__syncthreads_or(!ok)) { failed = true; break; }
-        tc_fence_after();
-        if (tid == 0 && e + 1 < E) {   // A2 consumed: S_{e+1} into sX
-            mbar_arrive_expect_tx(&bar_s, slab_bytes);
-            bulk_load(sX, reinterpret_cast<const uint8_t*>(p.Sck) + (sbase + e + 1) * kDk * dv * 4,
-                      slab_bytes, &bar_s);
-        }
-        // row dots of P'_e = [K;Q] dS'_e (key rows)
-        {
-            float acc = 0.f;
-            const int cw = dv / 2;
-            for (int j = half * cw; j < half * cw + cw; j += 16) {
-                float pv[16];
-                tmem_ld16(tmem_lane_addr(tP2, warp, j), pv);
-                tmem_wait_ld();
-                if (L < n) {
-                    float x[16];
-                    load_row8(p.Ubuf + tok_idx(b, t0 + L, h, j, T, H, dv), x);
-                    load_row8(p.Ubuf + tok_idx(b, t0 + L, h, j + 8, T, H, dv), x + 8);
-                    for (int u = 0; u < 16; ++u) acc = fmaf(x[u], pv[u], acc);
-                }
-            }
-            red[half * 128 + L] = acc;
-        }
-        __syncthreads();
-        if (tid < 64) dwk[tid * E + e] = red[tid] + red[128 + tid];
-        tc_fence_before();
-        __syncthreads();
-        tc_fence_after();
-    }
-    if (failed) {
-        if (tid == 0) record_device_error(p.err, TLA_ERR_TIMEOUT);
-        tc_fence_before();
-        __syncthreads();
-        if (warp == 0) tmem_dealloc(tmem, 512);
-        return;
     }
 
-    // ---- phase 3: dq (ACC rows 0-63), dk (rows 64-127)
+    // ---- phase 3: dq, dk = register sums + ACC^T, staged as [64 tokens][128] fp32 tiles in the
+    // (now idle) work region and written as whole rows
     {
-        const int row = L < 64 ? L : L - 64;
-        void* dst = L < 64 ? p.dq : p.dk;
-        for (int j = half * 64; j < half * 64 + 64; j += 16) {
-            float v[16];
-            tmem_ld16(tmem_lane_addr(tACC, warp, j), v);
-            tmem_wait_ld();
-            if (row < n) store_row(dst, tok_idx(b, t0 + row, h, j, T, H, kDk), v, 16, p.out_f32);
+        float* dqs = reinterpret_cast<float*>(W);
+        float* dks = dqs + 64 * kDk;
+        float v[32];
+        tmem_ld16(tmem_lane_addr(tACC, warp, tb), v);
+        tmem_ld16(tmem_lane_addr(tACC, warp, tb + 16), v + 16);
+        tmem_wait_ld();
+#pragma unroll
+        for (int j = 0; j < 32; ++j) dqs[(tb + j) * kDk + d] = acq[j] + v[j];
+        tmem_ld16(tmem_lane_addr(tACC, warp, 64 + tb), v);
+        tmem_ld16(tmem_lane_addr(tACC, warp, 64 + tb + 16), v + 16);
+        tmem_wait_ld();
+#pragma unroll
+        for (int j = 0; j < 32; ++j) dks[(tb + j) * kDk + d] = ack[j] + v[j];
+        __syncthreads();
+        for (int i = tid; i < 2 * 64 * (kDk / 4); i += kThreads) {
+            const int m = i >= 64 * (kDk / 4), j = i - m * 64 * (kDk / 4);
+            const int t = j / (kDk / 4), c4 = (j % (kDk / 4)) * 4;
+            if (t >= n) continue;
+            const float4 x = *reinterpret_cast<const float4*>((m ? dks : dqs) + t * kDk + c4);
+            const size_t off = tok_idx(b, t0 + t, h, c4, T, H, kDk);
+            void* dst = m ? p.dk : p.dq;
+            if (OUT_F32) {
+                *reinterpret_cast<float4*>(static_cast<float*>(dst) + off) = x;
+            } else {
+                const __nv_bfloat162 lo = __floats2bfloat162_rn(x.x, x.y), hi = __floats2bfloat162_rn(x.z, x.w);
+                *reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(dst) + off) =
+                    make_uint2(*reinterpret_cast<const uint32_t*>(&lo), *reinterpret_cast<const uint32_t*>(&hi));
+            }
         }
-    }
-    for (int i = tid; i < 64 * E; i += kThreads) {
-        const int e = i - (i / E) * E;
-        const float gam = expf(Gs[i]);
-        const float wdec = expf(Gs[(n - 1) * E + e] - Gs[i]);
-        const float a = k2s[i] * gam, bq = q2s[i] * gam, w = k2s[i] * wdec;
-        dk2a[i] += dak[i] * gam + dwk[i] * wdec;
-        dq2a[i] += dbq[i] * gam;
-        dGa[i] += dak[i] * a + dbq[i] * bq - dwk[i] * w;
     }
     __syncthreads();
-    if (tid < E) {
-        const int e = tid;
+    if (warp < E) {   // one warp per slice: dgamma^C, then the reverse cumulative sum of dG
+        const int e = warp;
+        const float gl = Gs[(n - 1) * E + e];
         float dGC = 0.f;
-        for (int r = 0; r < n; ++r) {
-            const float w = k2s[r * E + e] * expf(Gs[(n - 1) * E + e] - Gs[r * E + e]);
-            dGC = fmaf(dwk[r * E + e], w, dGC);
+        for (int r = lane; r < n; r += 32)
+            dGC = fmaf(dwk[r * E + e], __bfloat162float(k2s[r * E + e]) * expf(gl - Gs[r * E + e]), dGC);
+#pragma unroll
+        for (int s = 16; s >= 1; s >>= 1) dGC += __shfl_xor_sync(0xffffffffu, dGC, s);
+        dGC = fmaf(dgc[e], expf(gl), dGC);
+        const int r0 = 2 * lane, r1 = r0 + 1;
+        const float a0 = r0 < n ? dGa[r0 * E + e] + (r0 == n - 1 ? dGC : 0.f) : 0.f;
+        const float a1 = r1 < n ? dGa[r1 * E + e] + (r1 == n - 1 ? dGC : 0.f) : 0.f;
+        const float pair = a0 + a1;
+        float suf = pair;   // inclusive suffix sum over lanes
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+            const float v = __shfl_down_sync(0xffffffffu, suf, off);
+            if (lane + off < 32) suf += v;
         }
-        dGC = fmaf(dgc[e], expf(Gs[(n - 1) * E + e]), dGC);
-        dGa[(n - 1) * E + e] += dGC;
-        float acc = 0.f;
-        for (int r = n - 1; r >= 0; --r) {
-            acc += dGa[r * E + e];
-            p.dg[tok_idx(b, t0 + r, h, e, T, H, E)] = acc;
-        }
+        float above = __shfl_down_sync(0xffffffffu, suf, 1);   // sum over the lanes above
+        if (lane == 31) above = 0.f;
+        const float s1 = a1 + above;
+        if (r0 < n) p.dg[tok_idx(b, t0 + r0, h, e, T, H, E)] = a0 + s1;
+        if (r1 < n) p.dg[tok_idx(b, t0 + r1, h, e, T, H, E)] = s1;
     }
     for (int i = tid; i < n * E; i += kThreads) {
         const int r = i / E, e = i - (i / E) * E;
         const size_t off = tok_idx(b, t0 + r, h, e, T, H, E);
-        store_out(p.dq2, off, dq2a[i], p.out_f32);
-        store_out(p.dk2, off, dk2a[i], p.out_f32);
+        store_out(p.dq2, off, dq2a[i], OUT_F32);
+        store_out(p.dk2, off, dk2a[i], OUT_F32);
     }
     if (p.dbeta && tid < n) p.dbeta[(size_t(b) * T + t0 + tid) * H + h] = dba[tid];
     tc_fence_before();
@@ -673,15 +844,17 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     if (warp == 0) tmem_dealloc(tmem, 512);
 }
 
-size_t grads_tc_smem(int E) {
-    return 1024 + 6 * kBoxBytes + 2 * 65536 + (9 * 64 * E + 64 + 64 + 16 + 256 + 256) * 4;
+size_t grads_tc_smem(int E, int dv) {
+    const size_t T64 = size_t(64) * dv * 2;
+    const size_t small = size_t(64) * E * (4 + 2 + 2 + 4 * 4) + (64 + 64 + 16 + 192 + 768 + 8) * 4;
+    return 1024 + 5 * T64 + kWorkBytes + small;
 }
 
 }  // namespace
 
 int tc_grads_shape_ok(const tla_problem& p) {
     return p.dk == kDk && p.dv % 64 == 0 && p.dv <= 128 && p.E <= 8 &&
-           grads_tc_smem(p.E) <= 227 * 1024;
+           grads_tc_smem(p.E, p.dv) <= 227 * 1024;
 }
 
 int tc_grads_ok(const tla_problem& p, const FwdPlan& fp) { return fp.ck_tiles && tc_grads_shape_ok(p); }
@@ -712,12 +885,12 @@ cudaError_t launch_bwd_chunk_grads_tc(const tla_problem& p, const FwdPlan& fp, c
     a.err = err;
     a.T = p.T; a.H = p.H; a.dv = p.dv; a.E = p.E; a.NT = fp.NT;
     a.use_delta = p.use_delta; a.out_f32 = p.out_dtype == TLA_FP32;
-    const size_t smem = grads_tc_smem(p.E);
-    cudaFuncSetAttribute(bwd_chunk_grads_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                         (int)smem);
+    const size_t smem = grads_tc_smem(p.E, p.dv);
+    auto kern = a.out_f32 ? bwd_chunk_grads_tc_kernel<1> : bwd_chunk_grads_tc_kernel<0>;
+    cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     dim3 grid(fp.NT, p.H, p.B);
     prof_before("bwd_chunk_grads_tc", s);
-    bwd_chunk_grads_tc_kernel<<<grid, kThreads, smem, s>>>(mk, mq, mo, a);
+    kern<<<grid, kThreads, smem, s>>>(mk, mq, mo, a);
     prof_after(s);
     return cudaGetLastError();
 }
