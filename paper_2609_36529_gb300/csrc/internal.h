@@ -18,8 +18,9 @@ struct FwdPlan {
     size_t A;            // fp32 [B,H,NT,64,64] Q K^T (.) R' (lower incl. diagonal)
     size_t N;            // fp32 [B,H,NT,64,64] (I + L)^{-1} (delta rule only)
     size_t S;            // fp32 [B,H,NT,E,dk,dv] chunk-start states (save_for_bwd)
-    size_t U;            // fp32 [B,T,H,dv] delta-corrected values (save_for_bwd)
-    size_t Res;          // fp32 [B,T,H,dv] residual V - W (save_for_bwd, delta rule)
+    size_t U;            // delta-corrected values (save_for_bwd): fp32 [B,T,H,dv], or token tiles
+    size_t Res;          // residual V - W (save_for_bwd; delta rule, or any rule with token
+                         // tiles, where sGLA stores V): fp32 [B,T,H,dv], or token tiles
     size_t A2;           // bf16 [B,H,NT,2,128,64] [T; A T] hi and lo tiles (tensor-core path)
     size_t coef;         // fp32 [B,H,NT,3*64*E+16] per-row coefficients (tensor-core path)
     size_t BT;           // bf16 [B,H,NT,4,64,64] A^T, T^T hi/lo (tensor-core backward)
@@ -27,15 +28,18 @@ struct FwdPlan {
     int ck_tiles;        // 1: state checkpoints (forward S, backward dS) are stored as bf16
                          //    hi/lo pairs in the chunk-gradient kernel's operand layout:
                          //    per (b,h,chunk,e) a [dk][dv] hi tile then a lo tile, 128-byte
-                         //    swizzled K-major (same 4 bytes per element as fp32)
+                         //    swizzled K-major (same 4 bytes per element as fp32); U, Res
+                         //    and the backward's dU, -dRes are then token tiles: per
+                         //    (b,h,chunk) 64 rows x dv bf16 hi then lo, SW128 K-major 64-row
+                         //    blocks, rows past T zero
     int tc_tv;           // value columns per CTA of the tensor-core recurrence (0: SIMT)
     size_t bytes;        // total
 };
 
 struct BwdPlan {
     int tv;
-    size_t dU;           // fp32 [B,T,H,dv]
-    size_t dRes;         // fp32 [B,T,H,dv]
+    size_t dU;           // fp32 [B,T,H,dv], or token tiles (FwdPlan::ck_tiles)
+    size_t dRes;         // fp32 [B,T,H,dv] dRes, or token tiles of -dRes (delta rule)
     size_t dS;           // fp32 [B,H,NT,E,dk,dv] gradient of the state at each chunk's end
     size_t bytes;
 };

@@ -259,7 +259,8 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             if (row_thread) {
 #pragma unroll
                 for (int i = 0; i < TV; ++i) st_split(sUh, sUl, sw128_offset(i, r64, TV), du[i]);
-                if (r64 < n) store_f32_row(p.dUbuf + tok_idx(b, t0 + r64, h, n0, T, H, dv), du, TV);
+                if (p.ck_tiles) store_tok_tile(p.dUbuf, (size_t(b) * H + h) * NT + c, dv, r64, n0, du, TV, r64 < n);
+                else if (r64 < n) store_f32_row(p.dUbuf + tok_idx(b, t0 + r64, h, n0, T, H, dv), du, TV);
             }
         }
         fence_proxy_async_smem();
@@ -299,8 +300,14 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             if (row_thread) {
                 if (r64 < n) {
                     const size_t off = tok_idx(b, t0 + r64, h, n0, T, H, dv);
-                    store_f32_row(p.dRbuf + off, dr, TV);
+                    if (!p.ck_tiles) store_f32_row(p.dRbuf + off, dr, TV);
                     store_row(p.dv_out, off, dr, TV, p.out_f32);
+                }
+                if (p.ck_tiles && p.use_delta) {   // -dRes, the operand sign the gradient kernel uses
+                    float ndr[TV];
+#pragma unroll
+                    for (int i = 0; i < TV; ++i) ndr[i] = -dr[i];
+                    store_tok_tile(p.dRbuf, (size_t(b) * H + h) * NT + c, dv, r64, n0, ndr, TV, r64 < n);
                 }
                 if (p.use_delta) {
                     for (int e = 0; e < E; ++e) {

@@ -4,6 +4,8 @@
 #include <cuda_bf16.h>
 #include <stdint.h>
 
+#include "sm100.cuh"
+
 namespace tla {
 
 __device__ __forceinline__ void store_row(void* base, size_t off, const float* v, int n,
@@ -36,5 +38,21 @@ __device__ __forceinline__ void st_split(uint8_t* tile_hi, uint8_t* tile_lo, uin
     *reinterpret_cast<__nv_bfloat16*>(tile_lo + off) = __float2bfloat16_rn(v - __bfloat162float(hi));
 }
 
+
+// Token tile of one chunk: 64 rows x dv as bf16 hi (64*dv*2 bytes) then bf16 lo, each in
+// SW128 K-major 64-row blocks of 64 columns -- the operand layout of the chunk-gradient
+// kernel, which copies a tile into shared memory as is.  Writes columns n0..n0+cnt of row r
+// (zeros when !valid, so that padded rows of the last chunk read as zero).
+__device__ __forceinline__ void store_tok_tile(float* base, size_t chunk, int dv, int r, int n0,
+                                               const float* v, int cnt, bool valid) {
+    uint8_t* hi = reinterpret_cast<uint8_t*>(base) + chunk * (size_t(64) * dv * 4);
+    uint8_t* lo = hi + size_t(64) * dv * 2;
+    for (int i = 0; i < cnt; i += 8) {
+        float z[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) z[k] = valid ? v[i + k] : 0.f;
+        sm100::st8_split(hi, lo, sm100::sw128_offset(r, n0 + i, 64), z);
+    }
+}
 
 }  // namespace tla

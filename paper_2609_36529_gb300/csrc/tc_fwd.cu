@@ -313,8 +313,10 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             umma_commit(&bar_mma);
         }
         pending_mma = 1;
-        if (warp < 2 && p.save && p.use_delta && tid < n)   // while MMA-B runs
-            store_f32_row(p.Rbuf + tok_idx(b, t0 + tid, h, n0, T, H, dv), res, TV);
+        if (warp < 2 && p.Rbuf) {   // while MMA-B runs
+            if (p.ck_tiles) store_tok_tile(p.Rbuf, (size_t(b) * H + h) * NT + c, dv, tid, n0, res, TV, tid < n);
+            else if (tid < n) store_f32_row(p.Rbuf + tok_idx(b, t0 + tid, h, n0, T, H, dv), res, TV);
+        }
         ok = mbar_wait(&bar_mma, mma_phase);
         mma_phase ^= 1;
         if (__syncthreads_or(!ok)) { failed = true; break; }
@@ -360,12 +362,13 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         pending_mma = 1;
         {   // while MMA-C runs: U (key rows) and o (query rows) to global memory
             const int r = warp < 2 ? tid : tid - 64;
-            if (r < n) {
-                if (warp < 2) {
-                    if (p.save) store_f32_row(p.Ubuf + tok_idx(b, t0 + r, h, n0, T, H, dv), d2, TV);
-                } else {
-                    store_row(p.o, tok_idx(b, t0 + r, h, n0, T, H, dv), d2, TV, p.out_f32);
+            if (warp < 2) {
+                if (p.save) {
+                    if (p.ck_tiles) store_tok_tile(p.Ubuf, (size_t(b) * H + h) * NT + c, dv, r, n0, d2, TV, r < n);
+                    else if (r < n) store_f32_row(p.Ubuf + tok_idx(b, t0 + r, h, n0, T, H, dv), d2, TV);
                 }
+            } else if (r < n) {
+                store_row(p.o, tok_idx(b, t0 + r, h, n0, T, H, dv), d2, TV, p.out_f32);
             }
         }
         ok = mbar_wait(&bar_mma, mma_phase);
@@ -436,7 +439,7 @@ cudaError_t launch_tv(const tla_problem& p, const FwdPlan& fp, char* ws, int sav
     a.ht = p.ht;
     a.Sck = save ? (float*)(ws + fp.S) : nullptr;
     a.Ubuf = save ? (float*)(ws + fp.U) : nullptr;
-    a.Rbuf = (save && p.use_delta) ? (float*)(ws + fp.Res) : nullptr;
+    a.Rbuf = (save && (p.use_delta || fp.ck_tiles)) ? (float*)(ws + fp.Res) : nullptr;
     a.err = err;
     a.T = p.T; a.H = p.H; a.dv = p.dv; a.E = p.E; a.NT = NT;
     a.use_delta = p.use_delta; a.save = save; a.out_f32 = p.out_dtype == TLA_FP32;

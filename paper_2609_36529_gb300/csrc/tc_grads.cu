@@ -44,7 +44,6 @@ constexpr uint32_t kWorkBytes = 131072;    // [K;Q] tiles + phase 0/1 scratch; l
 struct TcGradArgs {
     const __nv_bfloat16* q2;
     const __nv_bfloat16* k2;
-    const __nv_bfloat16* v;
     const float* G;
     const float* beta;
     const float* Nmat;
@@ -104,12 +103,6 @@ __device__ __forceinline__ void st4_split(uint8_t* hi, uint8_t* lo, uint32_t off
         make_uint2(*reinterpret_cast<const uint32_t*>(&l0), *reinterpret_cast<const uint32_t*>(&l1));
 }
 
-__device__ __forceinline__ void load_row8(const float* src, float* v) {
-    const float4 a = reinterpret_cast<const float4*>(src)[0];
-    const float4 c = reinterpret_cast<const float4*>(src)[1];
-    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = c.x; v[5] = c.y; v[6] = c.z; v[7] = c.w;
-}
-
 __device__ __forceinline__ void load_bf16x8(const uint8_t* src, float* v) {
     const uint4 u = *reinterpret_cast<const uint4*>(src);
     const __nv_bfloat162* p = reinterpret_cast<const __nv_bfloat162*>(&u);
@@ -119,22 +112,6 @@ __device__ __forceinline__ void load_bf16x8(const uint8_t* src, float* v) {
         v[2 * i] = f.x;
         v[2 * i + 1] = f.y;
     }
-}
-
-// bf16 hi/lo split of 8 values into two tiles with different layouts.
-__device__ __forceinline__ void st8_split2(uint8_t* hi, uint32_t off_hi, uint8_t* lo,
-                                           uint32_t off_lo, const float* v) {
-    uint32_t h[4], l[4];
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        __nv_bfloat162 hv = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
-        const float2 hf = __bfloat1622float2(hv);
-        __nv_bfloat162 lv = __floats2bfloat162_rn(v[2 * i] - hf.x, v[2 * i + 1] - hf.y);
-        h[i] = *reinterpret_cast<uint32_t*>(&hv);
-        l[i] = *reinterpret_cast<uint32_t*>(&lv);
-    }
-    *reinterpret_cast<uint4*>(hi + off_hi) = make_uint4(h[0], h[1], h[2], h[3]);
-    *reinterpret_cast<uint4*>(lo + off_lo) = make_uint4(l[0], l[1], l[2], l[3]);
 }
 
 // One halving step of a warp transpose-reduction over 2S values per lane.
@@ -222,12 +199,24 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         mbar_init(&bar_s, 1);
         mbar_init(&bar_d, 1);
         fence_barrier_init();
-        mbar_arrive_expect_tx(&bar_ld, 4 * kBoxBytes + nb * kBoxBytes);
+        const size_t ci = (size_t(b) * H + h) * NT + c;
+        const uint32_t tt = 2 * T64;   // one token tile: hi then lo
+        // one arrival per phase (the barrier counts a single arrival): every byte of the
+        // tensor loads and the token-tile copies is announced here, before any copy starts
+        mbar_arrive_expect_tx(&bar_ld, 4 * kBoxBytes + nb * kBoxBytes + 3 * tt + (p.use_delta ? tt : 0));
         for (int j = 0; j < 2; ++j) {
             tma_load_4d(sKQ + j * 2 * kBoxBytes, &map_k, &bar_ld, 64 * j, h, t0, b);
             tma_load_4d(sKQ + j * 2 * kBoxBytes + kBoxBytes, &map_q, &bar_ld, 64 * j, h, t0, b);
         }
         for (int j = 0; j < nb; ++j) tma_load_4d(sB + j * 2 * kBoxBytes, &map_do, &bar_ld, 64 * j, h, t0, b);
+        bulk_load(sUh, reinterpret_cast<const uint8_t*>(p.Ubuf) + ci * tt, tt, &bar_ld);
+        bulk_load(scr, reinterpret_cast<const uint8_t*>(p.dUbuf) + ci * tt, tt, &bar_ld);
+        bulk_load(scr + tt, reinterpret_cast<const uint8_t*>(p.Rbuf) + ci * tt, tt, &bar_ld);
+        if (p.use_delta) {
+            const uint8_t* g = reinterpret_cast<const uint8_t*>(p.dRbuf) + ci * tt;
+            for (int j = 0; j < nb; ++j) bulk_load(sB + j * 16384 + 8192, g + j * 8192, 8192, &bar_ld);
+            bulk_load(sRlo, g + T64, T64, &bar_ld);
+        }
         bulk_prefetch_l2(gS + sbase * slab_bytes, slab_bytes);
         if (p.use_delta) bulk_prefetch_l2(p.Nmat + ((size_t(b) * H + h) * NT + c) * (64 * 64), kNBytes);
         bulk_prefetch_l2(gD + sbase * slab_bytes, slab_bytes);
@@ -245,51 +234,15 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     }
     if (tid < 16) dgc[tid] = 0.f;
 
-    // ---- staging: U -> sUh/sUl; -dRes -> sB rows 64..127 (hi), sRlo (lo);
-    //      dU, Res (sGLA: V) -> scratch (hi, lo, hi, lo) for dT
+    // ---- staging: the token tiles arrive by bulk copy (U -> sUh/sUl; dU, Res -> scratch for
+    //      dT; -dRes -> sB rows 64..127 (hi) and sRlo (lo)); sGLA has no -dRes operand
     uint8_t* sdUh = scr;
     uint8_t* sdUl = scr + T64;
     uint8_t* sRh = scr + 2 * T64;
     uint8_t* sRl = scr + 3 * T64;
-    {   // every load of this thread is issued before the first split (one round of latency)
-        constexpr int kIt = 64 * 128 / 8 / kThreads;   // 8-column chunks per thread at dv = 128
-        const int cpr = dv / 8;
-        float u[kIt][8], du[kIt][8], rs[kIt][8], dr[kIt][8];
-#pragma unroll
-        for (int it = 0; it < kIt; ++it) {
-            const int ci = tid + it * kThreads, r = ci / cpr, cc = (ci % cpr) * 8;
-            if (ci < 64 * cpr && r < n) {
-                const size_t off = tok_idx(b, t0 + r, h, cc, T, H, dv);
-                load_row8(p.Ubuf + off, u[it]);
-                load_row8(p.dUbuf + off, du[it]);
-                if (p.use_delta) {
-                    load_row8(p.Rbuf + off, rs[it]);
-                    load_row8(p.dRbuf + off, dr[it]);
-                } else {
-                    const uint4 raw = *reinterpret_cast<const uint4*>(p.v + off);
-                    load_bf16x8(reinterpret_cast<const uint8_t*>(&raw), rs[it]);
-#pragma unroll
-                    for (int i = 0; i < 8; ++i) dr[it][i] = 0.f;
-                }
-            } else {
-#pragma unroll
-                for (int i = 0; i < 8; ++i) u[it][i] = du[it][i] = rs[it][i] = dr[it][i] = 0.f;
-            }
-        }
-#pragma unroll
-        for (int it = 0; it < kIt; ++it) {
-            const int ci = tid + it * kThreads, r = ci / cpr, cc = (ci % cpr) * 8;
-            if (ci < 64 * cpr) {
-#pragma unroll
-                for (int i = 0; i < 8; ++i) dr[it][i] = -dr[it][i];
-                const uint32_t o = sw128_offset(r, cc, 64);
-                st8_split(sUh, sUl, o, u[it]);
-                st8_split(sdUh, sdUl, o, du[it]);
-                st8_split(sRh, sRl, o, rs[it]);
-                st8_split2(sB, sw128_offset(64 + r, cc, 128), sRlo, o, dr[it]);
-            }
-        }
-    }
+    if (!p.use_delta)
+        for (int i = tid; i < nb * 512; i += kThreads)
+            *reinterpret_cast<uint4*>(sB + (i >> 9) * 16384 + 8192 + (i & 511) * 16) = make_uint4(0, 0, 0, 0);
     fence_proxy_async_smem();
     tc_fence_before();
     __syncthreads();
@@ -871,13 +824,12 @@ cudaError_t launch_bwd_chunk_grads_tc(const tla_problem& p, const FwdPlan& fp, c
     TcGradArgs a;
     a.q2 = (const __nv_bfloat16*)p.q2;
     a.k2 = (const __nv_bfloat16*)p.k2;
-    a.v = (const __nv_bfloat16*)p.v;
     a.G = (const float*)(fws + fp.G);
     a.beta = p.beta;
     a.Nmat = p.use_delta ? (const float*)(fws + fp.N) : nullptr;
     a.Sck = (const float*)(fws + fp.S);
     a.Ubuf = (const float*)(fws + fp.U);
-    a.Rbuf = p.use_delta ? (const float*)(fws + fp.Res) : nullptr;
+    a.Rbuf = (const float*)(fws + fp.Res);
     a.dUbuf = (const float*)(bws + bp.dU);
     a.dRbuf = (const float*)(bws + bp.dRes);
     a.dSck = (const float*)(bws + bp.dS);

@@ -63,7 +63,7 @@ FwdPlan plan_fwd(const tla_problem& p, int save) {
     const size_t tokE = (size_t)p.B * p.T * p.H * p.E * 4;
     const size_t mats = (size_t)p.B * p.H * f.NT * kChunk * kChunk * 4;
     const size_t states = (size_t)p.B * p.H * f.NT * p.E * p.dk * p.dv * 4;
-    const size_t tokV = (size_t)p.B * p.T * p.H * p.dv * 4;
+    const size_t tokV = (size_t)p.B * f.NT * kChunk * p.H * p.dv * 4;   // whole chunks (token tiles)
     size_t off = 0;
     f.G = off; off = align256(off + tokE);
     f.A = off; off = align256(off + mats);
@@ -79,7 +79,7 @@ FwdPlan plan_fwd(const tla_problem& p, int save) {
     if (save) {
         f.S = off; off = align256(off + states);
         f.U = off; off = align256(off + tokV);
-        if (p.use_delta) { f.Res = off; off = align256(off + tokV); }
+        if (p.use_delta || f.ck_tiles) { f.Res = off; off = align256(off + tokV); }
     }
     f.bytes = off;
     return f;
@@ -90,7 +90,7 @@ BwdPlan plan_bwd(const tla_problem& p) {
     memset(&b, 0, sizeof(b));
     const int NT = (p.T + kChunk - 1) / kChunk;
     b.tv = simt_tv(p);
-    const size_t tokV = (size_t)p.B * p.T * p.H * p.dv * 4;
+    const size_t tokV = (size_t)p.B * NT * kChunk * p.H * p.dv * 4;   // whole chunks (token tiles)
     const size_t states = (size_t)p.B * p.H * NT * p.E * p.dk * p.dv * 4;
     size_t off = 0;
     b.dU = off; off = align256(off + tokV);
