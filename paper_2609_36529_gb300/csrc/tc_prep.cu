@@ -23,7 +23,9 @@ namespace {
 constexpr int kThreads = 256;
 constexpr int kDk = 128;
 constexpr int kBoxBytes = 64 * 64 * 2;
-constexpr int MP = 65;
+constexpr int MP = 68;                        // row stride (floats) of the C x C matrices
+constexpr int kSlot = 64 * MP;                // floats per matrix slot (17408 bytes)
+constexpr int XS = 20;                        // row stride of the transposed 16 x 16 diagonal blocks
 
 struct TcPrepArgs {
     const __nv_bfloat16* q2;
@@ -39,10 +41,24 @@ struct TcPrepArgs {
     int T, H, E, NT, use_delta;
 };
 
-__device__ __forceinline__ void put_pair(__nv_bfloat16* hi, __nv_bfloat16* lo, float x) {
-    const __nv_bfloat16 h = __float2bfloat16_rn(x);
-    *hi = h;
-    *lo = __float2bfloat16_rn(x - __bfloat162float(h));
+__device__ __forceinline__ void ld4(const float* src, float* v) {
+    const float4 x = *reinterpret_cast<const float4*>(src);
+    v[0] = x.x; v[1] = x.y; v[2] = x.z; v[3] = x.w;
+}
+__device__ __forceinline__ void st4(float* dst, float v0, float v1, float v2, float v3) {
+    *reinterpret_cast<float4*>(dst) = make_float4(v0, v1, v2, v3);
+}
+// Four consecutive values as bf16 hi/lo pairs (8 bytes into each of two global arrays).
+__device__ __forceinline__ void put4(__nv_bfloat16* hi, __nv_bfloat16* lo, float v0, float v1,
+                                     float v2, float v3) {
+    const __nv_bfloat162 h0 = __floats2bfloat162_rn(v0, v1), h1 = __floats2bfloat162_rn(v2, v3);
+    const float2 f0 = __bfloat1622float2(h0), f1 = __bfloat1622float2(h1);
+    const __nv_bfloat162 l0 = __floats2bfloat162_rn(v0 - f0.x, v1 - f0.y);
+    const __nv_bfloat162 l1 = __floats2bfloat162_rn(v2 - f1.x, v3 - f1.y);
+    *reinterpret_cast<uint2*>(hi) =
+        make_uint2(*reinterpret_cast<const uint32_t*>(&h0), *reinterpret_cast<const uint32_t*>(&h1));
+    *reinterpret_cast<uint2*>(lo) =
+        make_uint2(*reinterpret_cast<const uint32_t*>(&l0), *reinterpret_cast<const uint32_t*>(&l1));
 }
 
 __global__ void __launch_bounds__(kThreads, 2)
@@ -55,12 +71,15 @@ chunk_prep_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
     const int t0 = c * 64, n = min(64, T - t0);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    uint8_t* sKQ = sm;
-    float* ML = reinterpret_cast<float*>(sm + 4 * kBoxBytes);   // K K^T -> L
-    float* MA = ML + 64 * MP;                                   // Q K^T -> A
-    float* MX = MA + 64 * MP;                                   // N = (I + L)^{-1}
-    float* MW = MX + 64 * MP;                                   // block products
-    float* Gs = MW + 64 * MP;
+    // five matrix slots; the TMA key/query tile overlays slots 3-4 until the products are read
+    float* slot = reinterpret_cast<float*>(sm);
+    float* LT = slot;                 // L^T (K K^T first)
+    float* MX = slot + kSlot;         // N = (I + L)^{-1} (Q K^T first)
+    float* MAT = slot + 2 * kSlot;    // A^T
+    float* MW = slot + 3 * kSlot;     // off-diagonal block products, then T
+    float* XT = slot + 4 * kSlot;     // transposed 16 x 16 diagonal blocks of N, 4 x [16][XS]
+    uint8_t* sKQ = sm + 3 * kSlot * 4;   // 1024-aligned (3 x 17408 = 51 x 1024)
+    float* Gs = slot + 5 * kSlot;
     float* k2s = Gs + 64 * E;
     float* q2s = k2s + 64 * E;
     float* bs = q2s + 64 * E;
@@ -95,7 +114,10 @@ chunk_prep_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     const uint32_t tmem = tmem_slot;
     bool ok = mbar_wait(&bar_ld, 0);
     if (__syncthreads_or(!ok)) {
-        if (tid == 0) record_device_error(p.err, TLA_ERR_TIMEOUT);
+        if (tid == 0) {
+            record_device_error(p.err, TLA_ERR_TIMEOUT);
+            mbar_wait(&bar_ld, 0);   // bounded: the copies still in flight
+        }
         __syncthreads();
         if (warp == 0) tmem_dealloc(tmem, 64);
         return;
@@ -110,20 +132,24 @@ chunk_prep_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     }
     ok = mbar_wait(&bar_mma, 0);
     if (__syncthreads_or(!ok)) {
-        if (tid == 0) record_device_error(p.err, TLA_ERR_TIMEOUT);
+        if (tid == 0) {
+            record_device_error(p.err, TLA_ERR_TIMEOUT);
+            mbar_wait(&bar_mma, 0);
+        }
         __syncthreads();
         if (warp == 0) tmem_dealloc(tmem, 64);
         return;
     }
     tc_fence_after();
-    if (warp < 4) {   // rows 0-63: K K^T, rows 64-127: Q K^T
+    if (warp < 4) {   // rows 0-63: K K^T -> slot 0, rows 64-127: Q K^T -> slot 1
         const int L = warp * 32 + lane;
-        float* dst = L < 64 ? ML + L * MP : MA + (L - 64) * MP;
+        float* dst = (L < 64 ? LT : MX) + (L & 63) * MP;
         for (int j = 0; j < 64; j += 16) {
             float v[16];
             tmem_ld16(tmem_lane_addr(tmem, warp, j), v);
             tmem_wait_ld();
-            for (int i = 0; i < 16; ++i) dst[j + i] = v[i];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) st4(dst + j + 4 * q, v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
         }
     }
     tc_fence_before();
@@ -131,92 +157,191 @@ chunk_prep_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     tc_fence_after();
     if (warp == 0) tmem_dealloc(tmem, 64);
 
-    // A and L in place
-    const size_t mat = ((size_t(b) * H + h) * NT + c) * (64 * 64);
-    for (int i = tid; i < 64 * 64; i += kThreads) {
-        const int r = i >> 6, s = i & 63;
-        float a = 0.f, l = 0.f;
-        if (r >= s) {
-            float R = 0.f, Rq = 0.f;
-            for (int e = 0; e < E; ++e) {
-                const float gam = expf(Gs[r * E + e] - Gs[s * E + e]);
-                const float ks2 = k2s[s * E + e] * gam;
-                R = fmaf(k2s[r * E + e], ks2, R);
-                Rq = fmaf(q2s[r * E + e], ks2, Rq);
+    // ---- A and L on 4 x 4 blocks: thread owns rows R0..R0+3, columns S0..S0+3
+    const int R0 = 4 * (tid >> 4), S0 = 4 * (tid & 15);
+    const bool live = R0 + 3 >= S0;   // blocks entirely above the diagonal are zero
+    float KK[4][4], Av[4][4], Lv[4][4];
+#pragma unroll
+    for (int a = 0; a < 4; ++a) {
+        ld4(LT + (R0 + a) * MP + S0, KK[a]);
+        ld4(MX + (R0 + a) * MP + S0, Av[a]);   // Q K^T for now
+    }
+    __syncthreads();
+    if (live) {
+        float R[4][4], Rq[4][4];
+#pragma unroll
+        for (int a = 0; a < 4; ++a)
+#pragma unroll
+            for (int c2 = 0; c2 < 4; ++c2) R[a][c2] = Rq[a][c2] = 0.f;
+        for (int e = 0; e < E; ++e) {
+            float gs[4], ks[4];
+#pragma unroll
+            for (int c2 = 0; c2 < 4; ++c2) {
+                gs[c2] = Gs[(S0 + c2) * E + e];
+                ks[c2] = k2s[(S0 + c2) * E + e];
             }
-            a = MA[r * MP + s] * Rq;
-            if (r > s) l = bs[r] * ML[r * MP + s] * R;
+#pragma unroll
+            for (int a = 0; a < 4; ++a) {
+                const float gr = Gs[(R0 + a) * E + e], kr = k2s[(R0 + a) * E + e], qr = q2s[(R0 + a) * E + e];
+#pragma unroll
+                for (int c2 = 0; c2 < 4; ++c2) {
+                    // exp of a non-positive log-decay difference (Eq. joint-gram); the
+                    // clamp only matters above the diagonal, where the entry is discarded
+                    const float ks2 = ks[c2] * expf(fminf(gr - gs[c2], 0.f));
+                    R[a][c2] = fmaf(kr, ks2, R[a][c2]);
+                    Rq[a][c2] = fmaf(qr, ks2, Rq[a][c2]);
+                }
+            }
         }
-        MA[r * MP + s] = a;
-        ML[r * MP + s] = l;
-        p.Aout[mat + i] = a;
+#pragma unroll
+        for (int a = 0; a < 4; ++a)
+#pragma unroll
+            for (int c2 = 0; c2 < 4; ++c2) {
+                const int r = R0 + a, s2 = S0 + c2;
+                Av[a][c2] = (r >= s2) ? Av[a][c2] * Rq[a][c2] : 0.f;
+                Lv[a][c2] = (r > s2) ? bs[r] * KK[a][c2] * R[a][c2] : 0.f;
+            }
+    } else {
+#pragma unroll
+        for (int a = 0; a < 4; ++a)
+#pragma unroll
+            for (int c2 = 0; c2 < 4; ++c2) Av[a][c2] = Lv[a][c2] = 0.f;
+    }
+    const size_t mat = ((size_t(b) * H + h) * NT + c) * (64 * 64);
+#pragma unroll
+    for (int a = 0; a < 4; ++a) {
+        *reinterpret_cast<float4*>(p.Aout + mat + (R0 + a) * 64 + S0) = make_float4(Av[a][0], Av[a][1], Av[a][2], Av[a][3]);
+    }
+#pragma unroll
+    for (int c2 = 0; c2 < 4; ++c2) {
+        st4(MAT + (S0 + c2) * MP + R0, Av[0][c2], Av[1][c2], Av[2][c2], Av[3][c2]);
+        st4(LT + (S0 + c2) * MP + R0, Lv[0][c2], Lv[1][c2], Lv[2][c2], Lv[3][c2]);
     }
     __syncthreads();
 
-    // N = (I + L)^{-1}: diagonal 16 x 16 blocks (warps 0-3, lane = column), then the rest
+    // ---- N = (I + L)^{-1} (Eq. joint-solve): the four 16 x 16 diagonal blocks by forward
+    // substitution (warps 0-3, lane = column), then the off-diagonal blocks by distance
     if (p.use_delta) {
         if (warp < 4 && lane < 16) {
-            const int o = 16 * warp, s = lane;
+            const int o = 16 * warp, s2 = lane;
             float x[16];
 #pragma unroll
             for (int r = 0; r < 16; ++r) {
-                float acc = (r == s) ? 1.f : 0.f;
+                float acc = (r == s2) ? 1.f : 0.f;
 #pragma unroll
-                for (int j = 0; j < r; ++j) acc = fmaf(-ML[(o + r) * MP + o + j], x[j], acc);
+                for (int j = 0; j < r; ++j) acc = fmaf(-LT[(o + j) * MP + o + r], x[j], acc);
                 x[r] = acc;
             }
 #pragma unroll
-            for (int r = 0; r < 16; ++r) MX[(o + r) * MP + o + s] = x[r];
+            for (int r = 0; r < 16; ++r) {
+                MX[(o + r) * MP + o + s2] = x[r];
+                XT[warp * 16 * XS + s2 * XS + r] = x[r];
+            }
         }
-        // zero the strictly upper blocks
-        for (int i = tid; i < 64 * 64; i += kThreads) {
-            const int r = i >> 6, s = i & 63;
-            if ((s >> 4) > (r >> 4)) MX[r * MP + s] = 0.f;
+        for (int i = tid; i < 64 * 64; i += kThreads) {   // zero the strictly upper blocks
+            const int r = i >> 6, s2 = i & 63;
+            if ((s2 >> 4) > (r >> 4)) MX[r * MP + s2] = 0.f;
         }
         __syncthreads();
         for (int dist = 1; dist < 4; ++dist) {
-            const int nblk = 4 - dist;   // blocks (i, i - dist), i = dist..3
-            // W_ij = sum_{k=j}^{i-1} L_ik X_kj
-            for (int idx = tid; idx < nblk * 256; idx += kThreads) {
-                const int bi = dist + idx / 256, bj = bi - dist, e2 = idx & 255;
-                const int r = 16 * bi + (e2 >> 4), s = 16 * bj + (e2 & 15);
-                float acc = 0.f;
-                for (int x = 16 * bj; x < 16 * bi; ++x) acc = fmaf(ML[r * MP + x], MX[x * MP + s], acc);
-                MW[r * MP + s] = acc;
+            const int tasks = (4 - dist) * 16;   // 4 x 4 blocks of the blocks (i, i - dist)
+            const int bi = dist + (tid >> 4), bj = bi - dist;
+            const int r0 = 16 * bi + 4 * ((tid >> 2) & 3), s0 = 16 * bj + 4 * (tid & 3);
+            if (tid < tasks) {   // W_ij = sum_{k=j}^{i-1} L_ik X_kj
+                float w[4][4];
+#pragma unroll
+                for (int a = 0; a < 4; ++a)
+#pragma unroll
+                    for (int c2 = 0; c2 < 4; ++c2) w[a][c2] = 0.f;
+#pragma unroll 4
+                for (int x = 16 * bj; x < 16 * bi; ++x) {
+                    float l[4], xv[4];
+                    ld4(LT + x * MP + r0, l);
+                    ld4(MX + x * MP + s0, xv);
+#pragma unroll
+                    for (int a = 0; a < 4; ++a)
+#pragma unroll
+                        for (int c2 = 0; c2 < 4; ++c2) w[a][c2] = fmaf(l[a], xv[c2], w[a][c2]);
+                }
+#pragma unroll
+                for (int a = 0; a < 4; ++a) st4(MW + (r0 + a) * MP + s0, w[a][0], w[a][1], w[a][2], w[a][3]);
             }
             __syncthreads();
-            // X_ij = -X_ii W_ij
-            for (int idx = tid; idx < nblk * 256; idx += kThreads) {
-                const int bi = dist + idx / 256, bj = bi - dist, e2 = idx & 255;
-                const int r = 16 * bi + (e2 >> 4), s = 16 * bj + (e2 & 15);
-                float acc = 0.f;
-                for (int x = 16 * bi; x <= r; ++x) acc = fmaf(MX[r * MP + x], MW[x * MP + s], acc);
-                MX[r * MP + s] = -acc;
+            if (tid < tasks) {   // X_ij = -X_ii W_ij
+                float xo[4][4];
+#pragma unroll
+                for (int a = 0; a < 4; ++a)
+#pragma unroll
+                    for (int c2 = 0; c2 < 4; ++c2) xo[a][c2] = 0.f;
+                const float* xt = XT + bi * 16 * XS;
+#pragma unroll 4
+                for (int x = 0; x < 16; ++x) {
+                    float xi[4], wv[4];
+                    ld4(xt + x * XS + (r0 - 16 * bi), xi);
+                    ld4(MW + (16 * bi + x) * MP + s0, wv);
+#pragma unroll
+                    for (int a = 0; a < 4; ++a)
+#pragma unroll
+                        for (int c2 = 0; c2 < 4; ++c2) xo[a][c2] = fmaf(xi[a], wv[c2], xo[a][c2]);
+                }
+#pragma unroll
+                for (int a = 0; a < 4; ++a) st4(MX + (r0 + a) * MP + s0, -xo[a][0], -xo[a][1], -xo[a][2], -xo[a][3]);
             }
             __syncthreads();
         }
-        for (int i = tid; i < 64 * 64; i += kThreads) p.Nout[mat + i] = MX[(i >> 6) * MP + (i & 63)];
-    } else {
-        for (int i = tid; i < 64 * 64; i += kThreads) MX[(i >> 6) * MP + (i & 63)] = ((i >> 6) == (i & 63)) ? 1.f : 0.f;
-        __syncthreads();
+        for (int i = tid; i < 64 * 16; i += kThreads) {
+            const int r = i >> 4, c4 = (i & 15) * 4;
+            *reinterpret_cast<float4*>(p.Nout + mat + r * 64 + c4) = *reinterpret_cast<const float4*>(MX + r * MP + c4);
+        }
     }
-    // T = N diag(beta) into MW; then A T, and the bf16 pairs
-    for (int i = tid; i < 64 * 64; i += kThreads) {
-        const int r = i >> 6, s = i & 63;
-        MW[r * MP + s] = (r >= s) ? MX[r * MP + s] * bs[s] : 0.f;
+    // ---- T = N diag(beta) (sGLA: diag(beta)), then A T; bf16 hi/lo tiles
+    float Tv[4][4];
+#pragma unroll
+    for (int a = 0; a < 4; ++a) {
+        float nr[4];
+        if (p.use_delta) ld4(MX + (R0 + a) * MP + S0, nr);
+#pragma unroll
+        for (int c2 = 0; c2 < 4; ++c2) {
+            const int r = R0 + a, s2 = S0 + c2;
+            const float nv = p.use_delta ? nr[c2] : (r == s2 ? 1.f : 0.f);
+            Tv[a][c2] = (r >= s2) ? nv * bs[s2] : 0.f;
+        }
     }
+#pragma unroll
+    for (int a = 0; a < 4; ++a) st4(MW + (R0 + a) * MP + S0, Tv[a][0], Tv[a][1], Tv[a][2], Tv[a][3]);
     __syncthreads();
+    float ATv[4][4];   // (A T)[r][s] = sum_{j=s}^{r} A[r][j] T[j][s]
+#pragma unroll
+    for (int a = 0; a < 4; ++a)
+#pragma unroll
+        for (int c2 = 0; c2 < 4; ++c2) ATv[a][c2] = 0.f;
+    if (live) {
+#pragma unroll 4
+        for (int j = S0; j < R0 + 4; ++j) {
+            float av[4], tv[4];
+            ld4(MAT + j * MP + R0, av);
+            ld4(MW + j * MP + S0, tv);
+#pragma unroll
+            for (int a = 0; a < 4; ++a)
+#pragma unroll
+                for (int c2 = 0; c2 < 4; ++c2) ATv[a][c2] = fmaf(av[a], tv[c2], ATv[a][c2]);
+        }
+    }
     const size_t m2 = ((size_t(b) * H + h) * NT + c) * (4 * 64 * 64);
-    for (int i = tid; i < 64 * 64; i += kThreads) {
-        const int r = i >> 6, s = i & 63;
-        float at = 0.f;
-        for (int j = s; j <= r; ++j) at = fmaf(MA[r * MP + j], MW[j * MP + s], at);
-        const float t = MW[r * MP + s];
-        put_pair(p.A2out + m2 + i, p.A2out + m2 + 2 * 4096 + i, t);
-        put_pair(p.A2out + m2 + 4096 + i, p.A2out + m2 + 3 * 4096 + i, at);
-        if (p.BTout) {   // element (r, s) of A^T and T^T
-            put_pair(p.BTout + m2 + i, p.BTout + m2 + 4096 + i, MA[s * MP + r]);
-            put_pair(p.BTout + m2 + 2 * 4096 + i, p.BTout + m2 + 3 * 4096 + i, MW[s * MP + r]);
+    __nv_bfloat16* A2 = p.A2out + m2;   // [T ; A T] hi (128 x 64), then lo
+#pragma unroll
+    for (int a = 0; a < 4; ++a) {
+        const int o = (R0 + a) * 64 + S0;
+        put4(A2 + o, A2 + 8192 + o, Tv[a][0], Tv[a][1], Tv[a][2], Tv[a][3]);
+        put4(A2 + 4096 + o, A2 + 12288 + o, ATv[a][0], ATv[a][1], ATv[a][2], ATv[a][3]);
+    }
+    if (p.BTout) {   // [A^T hi, A^T lo, T^T hi, T^T lo], 64 x 64 each
+        __nv_bfloat16* BT = p.BTout + m2;
+#pragma unroll
+        for (int c2 = 0; c2 < 4; ++c2) {
+            const int o = (S0 + c2) * 64 + R0;
+            put4(BT + o, BT + 4096 + o, Av[0][c2], Av[1][c2], Av[2][c2], Av[3][c2]);
+            put4(BT + 8192 + o, BT + 12288 + o, Tv[0][c2], Tv[1][c2], Tv[2][c2], Tv[3][c2]);
         }
     }
     // coefficient block
@@ -232,7 +357,7 @@ chunk_prep_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     if (tid < 16) cf[192 * E + tid] = tid < E ? expf(Gs[(n - 1) * E + tid]) : 0.f;
 }
 
-size_t prep_tc_smem(int E) { return 1024 + 4 * kBoxBytes + 4 * 64 * MP * 4 + (3 * 64 * E + 64) * 4; }
+size_t prep_tc_smem(int E) { return 1024 + size_t(5) * kSlot * 4 + (3 * 64 * E + 64) * 4; }
 
 }  // namespace
 
