@@ -164,8 +164,6 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     uint8_t* W = sUl + T64;                    // 128 KB work region
     uint8_t* sKQ = W;                          // [K rows | Q rows] per 64-column block (TMA)
     uint8_t* scr = W + 4 * kBoxBytes;          // 96 KB: phase 0 staging, six C x C matrices, A3
-    uint8_t* bufS = W;                         // phase 2: S_e slab (hi, lo)
-    uint8_t* bufD = W + 65536;                 // phase 2: dS'_e slab (hi, lo)
     float* Gs = reinterpret_cast<float*>(W + kWorkBytes);
     __nv_bfloat16* k2s = reinterpret_cast<__nv_bfloat16*>(Gs + 64 * E);
     __nv_bfloat16* q2s = k2s + 64 * E;
@@ -176,11 +174,11 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     float* bs = dwk + 64 * E;                  // [64]
     float* dba = bs + 64;                      // [64]
     float* dgc = dba + 64;                     // [16]
-    float* scl = dgc + 16;                     // [3][64]: b_e, a_e, w_e of the current slice
-    float* red = scl + 192;                    // [3][4][64] row-dot partials per lane quarter
-    float* frw = red + 768;                    // [8] Frobenius partials per warp
+    float* scl = dgc + 16;                     // [2][3][64]: b_e, a_e, w_e (slice parity)
+    float* red = scl + 384;                    // [3][4][64] row-dot partials per lane quarter
+    float* frw = red + 768;                    // [2][8] Frobenius partials per warp (slice parity)
 
-    __shared__ __align__(8) uint64_t bar_ld, bar_mma, bar_s, bar_d;
+    __shared__ __align__(8) uint64_t bar_ld, bar_mma, bar_fro, bar_q[4];
     __shared__ uint32_t tmem_slot;
 
     const size_t sbase = ((size_t(b) * H + h) * NT + c) * E;   // this chunk's first slab
@@ -196,8 +194,8 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     if (tid == 0) {
         mbar_init(&bar_ld, 1);
         mbar_init(&bar_mma, 1);
-        mbar_init(&bar_s, 1);
-        mbar_init(&bar_d, 1);
+        for (int q = 0; q < 4; ++q) mbar_init(&bar_q[q], 1);
+        mbar_init(&bar_fro, kThreads / 32 - 1);   // one arrival per warp 1..7
         fence_barrier_init();
         const size_t ci = (size_t(b) * H + h) * NT + c;
         const uint32_t tt = 2 * T64;   // one token tile: hi then lo
@@ -248,7 +246,7 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = tmem_slot;
-    const uint32_t tACC = tmem, tD1 = tmem + 128, tD2 = tmem + 256;
+    const uint32_t tACC = tmem;   // phase 2: D1/D2 at columns 128/256 (even slices), 320/448 (odd)
 
     uint32_t mph = 0;
     // Failure exit: record the timeout, wait (bounded) for this CTA's copies and
@@ -584,144 +582,191 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     mph ^= 1;
     tc_fence_after();
 
-    // ---- phase 2: per slice.  S_e and dS'_e slabs (bf16 hi/lo, operand layout) arrive by
-    // bulk copy over the work region; the next pair is requested once the products and the
-    // Frobenius sum have consumed the current one.
-    uint32_t sph = 0, dph = 0;
-    auto issue_slabs = [&](int e) {
-        mbar_arrive_expect_tx(&bar_s, slab_bytes);
-        bulk_load(bufS, gS + (sbase + e) * slab_bytes, slab_bytes, &bar_s);
-        mbar_arrive_expect_tx(&bar_d, slab_bytes);
-        bulk_load(bufD, gD + (sbase + e) * slab_bytes, slab_bytes, &bar_d);
+    // ---- phase 2: per slice.  S_e and dS'_e (bf16 hi/lo, operand layout) arrive by bulk copy,
+    // one 64-column half per quarter of the work region with its own barrier.  Thread 0 issues
+    // the slice's products (it is held for about their execution time) and, once they and the
+    // Frobenius sum of warps 1-7 are done, the next slice's copies; slice e-1's epilogue runs
+    // on all warps meanwhile (D1/D2 double-buffered in TMEM).
+    uint32_t qph = 0, pend = 0, fph = 0;   // quarter phases, loads in flight (thread 0), bar_fro phase
+    auto quarter = [&](int which, int j) { return W + (2 * j + which) * 32768; };   // 0: S, 1: dS'
+    auto issue_slice = [&](int e) {
+        for (int j = 0; j < nb; ++j)
+            for (int which = 0; which < 2; ++which) {
+                uint8_t* dst = quarter(which, j);
+                const uint8_t* src = (which ? gD : gS) + (sbase + e) * slab_bytes + j * 16384;
+                uint64_t* bar = &bar_q[2 * j + which];
+                mbar_arrive_expect_tx(bar, 32768);
+                bulk_load(dst, src, 16384, bar);
+                bulk_load(dst + 16384, src + LO, 16384, bar);
+                pend |= 1u << (2 * j + which);
+            }
         if (e + 1 < E) {
             bulk_prefetch_l2(gS + (sbase + e + 1) * slab_bytes, slab_bytes);
             bulk_prefetch_l2(gD + (sbase + e + 1) * slab_bytes, slab_bytes);
         }
     };
-    if (tid == 0) issue_slabs(0);
+    auto fail = [&](bool mma) {   // timeout: record it, drain this CTA's copies and products
+        if (tid == 0) {
+            record_device_error(p.err, TLA_ERR_TIMEOUT);
+            for (int q = 0; q < 4; ++q)
+                if ((pend >> q) & 1) mbar_wait(&bar_q[q], (qph >> q) & 1);
+            if (mma) mbar_wait(&bar_mma, mph);
+        }
+        tc_fence_before();
+        __syncthreads();
+        if (warp == 0) tmem_dealloc(tmem, 512);
+    };
+    if (tid == 0) issue_slice(0);
     float acq[32], ack[32];
 #pragma unroll
     for (int j = 0; j < 32; ++j) acq[j] = ack[j] = 0.f;
-    for (int e = 0; e < E; ++e) {
-        if (tid < 192) {   // b_e, a_e, w_e of the 64 tokens
-            const int r = tid & 63, i = r * E + e;
-            float s;
-            if (tid < 64) s = __bfloat162float(q2s[i]) * expf(Gs[i]);
-            else if (tid < 128) s = __bfloat162float(k2s[i]) * expf(Gs[i]);
-            else s = __bfloat162float(k2s[i]) * expf(Gs[(n - 1) * E + e] - Gs[i]);
-            scl[tid] = s;
-        }
-        const bool ok_s = mbar_wait(&bar_s, sph);
-        const bool ok_d = mbar_wait(&bar_d, dph);
-        tc_fence_before();
-        if (__syncthreads_or(!(ok_s && ok_d))) {
-            bail(&bar_s, sph, &bar_d, dph, false);
-            return;
-        }
-        sph ^= 1;
-        dph ^= 1;
-        tc_fence_after();
-        if (tid == 0) {
-            const uint32_t id128 = idesc_bf16_f32(128, 128, 0, 0);
-            const uint32_t id64 = idesc_bf16_f32(128, 64, 0, 0);
-            for (int ks = 0; ks < dv / 16; ++ks) {
-                const uint32_t k32 = (ks & 3) * 32;
-                const uint32_t o128 = (ks >> 2) * 16384 + k32, o64 = (ks >> 2) * 8192 + k32;
-                const uint64_t sh = smem_desc(smem_u32(bufS) + o128, 16, 1024);
-                const uint64_t sl = smem_desc(smem_u32(bufS + LO) + o128, 16, 1024);
-                const uint64_t bh = smem_desc(smem_u32(sB) + o128, 16, 1024);
-                const uint64_t rl = smem_desc(smem_u32(sRlo) + o64, 16, 1024);
-                umma_bf16(tD1, sh, bh, id128, ks > 0 ? 1u : 0u);
-                umma_bf16(tD1, sl, bh, id128, 1u);
-                if (p.use_delta) umma_bf16(tD1 + 64, sh, rl, id64, 1u);
-                const uint64_t dh = smem_desc(smem_u32(bufD) + o128, 16, 1024);
-                const uint64_t dl = smem_desc(smem_u32(bufD + LO) + o128, 16, 1024);
-                const uint64_t uh = smem_desc(smem_u32(sUh) + o64, 16, 1024);
-                const uint64_t ul = smem_desc(smem_u32(sUl) + o64, 16, 1024);
-                umma_bf16(tD2, dh, uh, id64, ks > 0 ? 1u : 0u);
-                umma_bf16(tD2, dl, uh, id64, 1u);
-                umma_bf16(tD2, dh, ul, id64, 1u);
+    const uint32_t qmask = nb == 2 ? 15u : 3u;
+    for (int e = 0; e <= E; ++e) {   // e == E only finishes slice E-1
+        const bool act = e < E;
+        const int pb = e & 1;
+        bool ok = true;
+        if (act) {
+            if (tid < 192) {   // b_e, a_e, w_e of the 64 tokens
+                const int r = tid & 63, i = r * E + e;
+                float sv;
+                if (tid < 64) sv = __bfloat162float(q2s[i]) * expf(Gs[i]);
+                else if (tid < 128) sv = __bfloat162float(k2s[i]) * expf(Gs[i]);
+                else sv = __bfloat162float(k2s[i]) * expf(Gs[(n - 1) * E + e] - Gs[i]);
+                scl[pb * 192 + tid] = sv;
             }
-            umma_commit(&bar_mma);
-        }
-        {   // <dS'_e, S_e> from the hi/lo tiles (hi + lo reproduces each value to ~2^-16)
-            float fro = 0.f;
-            for (uint32_t o = tid * 16; o < LO; o += kThreads * 16) {
-                float sh[8], sl[8], dh[8], dl[8];
-                load_bf16x8(bufS + o, sh);
-                load_bf16x8(bufS + LO + o, sl);
-                load_bf16x8(bufD + o, dh);
-                load_bf16x8(bufD + LO + o, dl);
-#pragma unroll
-                for (int u = 0; u < 8; ++u) fro = fmaf(dh[u] + dl[u], sh[u] + sl[u], fro);
+            for (int q = 0; q < 4; ++q)
+                if ((qmask >> q) & 1) ok = mbar_wait(&bar_q[q], (qph >> q) & 1) && ok;
+            tc_fence_before();
+            if (__syncthreads_or(!ok)) {
+                fail(false);
+                return;
             }
+            qph ^= qmask;
+            pend &= ~qmask;
+            tc_fence_after();
+            if (warp == 0) {
+                if (lane == 0) {   // D1 = S_e [dO; -dRes]^T, D2 = dS'_e U^T
+                    const uint32_t d1 = pb ? tmem + 320 : tmem + 128, d2 = pb ? tmem + 448 : tmem + 256;
+                    const uint32_t id128 = idesc_bf16_f32(128, 128, 0, 0);
+                    const uint32_t id64 = idesc_bf16_f32(128, 64, 0, 0);
+                    for (int j = 0; j < nb; ++j) {
+                        const uint32_t qs = smem_u32(quarter(0, j)), qd = smem_u32(quarter(1, j));
+                        for (int kk = 0; kk < 4; ++kk) {
+                            const uint32_t k32 = kk * 32, acc = (j > 0 || kk > 0) ? 1u : 0u;
+                            const uint64_t sh = smem_desc(qs + k32, 16, 1024);
+                            const uint64_t sl = smem_desc(qs + 16384 + k32, 16, 1024);
+                            const uint64_t bh = smem_desc(smem_u32(sB) + j * 16384 + k32, 16, 1024);
+                            umma_bf16(d1, sh, bh, id128, acc);
+                            umma_bf16(d1, sl, bh, id128, 1u);
+                            if (p.use_delta)
+                                umma_bf16(d1 + 64, sh, smem_desc(smem_u32(sRlo) + j * 8192 + k32, 16, 1024), id64, 1u);
+                            const uint64_t dh = smem_desc(qd + k32, 16, 1024);
+                            const uint64_t dl = smem_desc(qd + 16384 + k32, 16, 1024);
+                            const uint64_t uh = smem_desc(smem_u32(sUh) + j * 8192 + k32, 16, 1024);
+                            const uint64_t ul = smem_desc(smem_u32(sUl) + j * 8192 + k32, 16, 1024);
+                            umma_bf16(d2, dh, uh, id64, acc);
+                            umma_bf16(d2, dl, uh, id64, 1u);
+                            umma_bf16(d2, dh, ul, id64, 1u);
+                        }
+                    }
+                    umma_commit(&bar_mma);
+                    // the slabs are free once the products and the Frobenius sum have read them
+                    ok = mbar_wait(&bar_mma, mph) && mbar_wait(&bar_fro, fph);
+                    if (ok && e + 1 < E) issue_slice(e + 1);
+                }
+                __syncwarp();
+            } else {   // <dS'_e, S_e> (hi + lo reproduces each value to ~2^-16), warps 1..7
+                float fro = 0.f;
+                for (int j = 0; j < nb; ++j) {
+                    const uint8_t* qsb = quarter(0, j);
+                    const uint8_t* qdb = quarter(1, j);
+                    for (uint32_t o = (tid - 32) * 16; o < 16384; o += (kThreads - 32) * 16) {
+                        float sh[8], sl[8], dh[8], dl[8];
+                        load_bf16x8(qsb + o, sh);
+                        load_bf16x8(qsb + 16384 + o, sl);
+                        load_bf16x8(qdb + o, dh);
+                        load_bf16x8(qdb + 16384 + o, dl);
 #pragma unroll
-            for (int s = 16; s >= 1; s >>= 1) fro += __shfl_xor_sync(0xffffffffu, fro, s);
-            if (lane == 0) frw[warp] = fro;
+                        for (int u = 0; u < 8; ++u) fro = fmaf(dh[u] + dl[u], sh[u] + sl[u], fro);
+                    }
+                }
+#pragma unroll
+                for (int sft = 16; sft >= 1; sft >>= 1) fro += __shfl_xor_sync(0xffffffffu, fro, sft);
+                if (lane == 0) {
+                    frw[pb * 8 + warp] = fro;
+                    mbar_arrive(&bar_fro);
+                }
+            }
         }
-        ok = mbar_wait(&bar_mma, mph);
-        if (__syncthreads_or(!ok)) {
-            bail(nullptr, 0, nullptr, 0, true);
-            return;
-        }
-        mph ^= 1;
-        tc_fence_after();
-        if (tid == 0 && e + 1 < E) issue_slabs(e + 1);
-        {
+        if (e > 0) {   // epilogue of slice e-1 (its D1/D2 and scales)
+            const int ep = (e - 1) & 1;
+            const uint32_t d1 = ep ? tmem + 320 : tmem + 128, d2 = ep ? tmem + 448 : tmem + 256;
+            const float* sc = scl + ep * 192;
             float z[32];
             // D1 query columns: dq += b_e (dO S_e^T); db_e = rowdot(Q, dO S_e^T)
-            tmem_ld16(tmem_lane_addr(tD1, warp, tb), z);
-            tmem_ld16(tmem_lane_addr(tD1, warp, tb + 16), z + 16);
+            tmem_ld16(tmem_lane_addr(d1, warp, tb), z);
+            tmem_ld16(tmem_lane_addr(d1, warp, tb + 16), z + 16);
             tmem_wait_ld();
 #pragma unroll
-            for (int j = 0; j < 32; ++j) {
-                acq[j] = fmaf(scl[tb + j], z[j], acq[j]);
-                z[j] *= unpack_bf16(qc, j);
+            for (int jj = 0; jj < 32; ++jj) {
+                acq[jj] = fmaf(sc[tb + jj], z[jj], acq[jj]);
+                z[jj] *= unpack_bf16(qc, jj);
             }
             red[(0 * 4 + wq) * 64 + tb + lane] = xreduce32(z, lane);
             // D1 key columns: dk += a_e (-dRes S_e^T); da_e = rowdot(K, -dRes S_e^T)
-            tmem_ld16(tmem_lane_addr(tD1, warp, 64 + tb), z);
-            tmem_ld16(tmem_lane_addr(tD1, warp, 64 + tb + 16), z + 16);
+            tmem_ld16(tmem_lane_addr(d1, warp, 64 + tb), z);
+            tmem_ld16(tmem_lane_addr(d1, warp, 64 + tb + 16), z + 16);
             tmem_wait_ld();
 #pragma unroll
-            for (int j = 0; j < 32; ++j) {
-                ack[j] = fmaf(scl[64 + tb + j], z[j], ack[j]);
-                z[j] *= unpack_bf16(kc, j);
+            for (int jj = 0; jj < 32; ++jj) {
+                ack[jj] = fmaf(sc[64 + tb + jj], z[jj], ack[jj]);
+                z[jj] *= unpack_bf16(kc, jj);
             }
             red[(1 * 4 + wq) * 64 + tb + lane] = xreduce32(z, lane);
             // D2: dk += w_e (U dS'_e^T); dw_e = rowdot(K, U dS'_e^T)
-            tmem_ld16(tmem_lane_addr(tD2, warp, tb), z);
-            tmem_ld16(tmem_lane_addr(tD2, warp, tb + 16), z + 16);
+            tmem_ld16(tmem_lane_addr(d2, warp, tb), z);
+            tmem_ld16(tmem_lane_addr(d2, warp, tb + 16), z + 16);
             tmem_wait_ld();
 #pragma unroll
-            for (int j = 0; j < 32; ++j) {
-                ack[j] = fmaf(scl[128 + tb + j], z[j], ack[j]);
-                z[j] *= unpack_bf16(kc, j);
+            for (int jj = 0; jj < 32; ++jj) {
+                ack[jj] = fmaf(sc[128 + tb + jj], z[jj], ack[jj]);
+                z[jj] *= unpack_bf16(kc, jj);
             }
             red[(2 * 4 + wq) * 64 + tb + lane] = xreduce32(z, lane);
         }
         tc_fence_before();
-        __syncthreads();
-        if (tid < 64) {   // this slice's row dots -> dq2, dk2, dG (a_e = k2 gamma, b_e = q2 gamma, w_e)
-            const int i = tid * E + e;
-            float db = 0.f, da = 0.f, dw = 0.f;
+        if (__syncthreads_or(!ok)) {
+            fail(act);
+            return;
+        }
+        tc_fence_after();
+        if (act) {
+            mph ^= 1;
+            fph ^= 1;
+        }
+        if (e > 0) {   // slice e-1's row dots -> dq2, dk2, dG (a_e = k2 gamma, b_e = q2 gamma, w_e)
+            const int es = e - 1;
+            if (tid < 64) {
+                const int i = tid * E + es;
+                float db = 0.f, da = 0.f, dw = 0.f;
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                db += red[(0 * 4 + q) * 64 + tid];
-                da += red[(1 * 4 + q) * 64 + tid];
-                dw += red[(2 * 4 + q) * 64 + tid];
+                for (int q = 0; q < 4; ++q) {
+                    db += red[(0 * 4 + q) * 64 + tid];
+                    da += red[(1 * 4 + q) * 64 + tid];
+                    dw += red[(2 * 4 + q) * 64 + tid];
+                }
+                const float gam = expf(Gs[i]);
+                const float wdec = expf(Gs[(n - 1) * E + es] - Gs[i]);
+                const float k2v = __bfloat162float(k2s[i]), q2v = __bfloat162float(q2s[i]);
+                dk2a[i] += da * gam + dw * wdec;
+                dq2a[i] += db * gam;
+                dGa[i] += da * (k2v * gam) + db * (q2v * gam) - dw * (k2v * wdec);
+                dwk[i] = dw;
+            } else if (tid == 64) {
+                float f = 0.f;
+                for (int w = 1; w < kThreads / 32; ++w) f += frw[(es & 1) * 8 + w];
+                dgc[es] = f;
             }
-            const float gam = expf(Gs[i]);
-            const float wdec = expf(Gs[(n - 1) * E + e] - Gs[i]);
-            const float k2v = __bfloat162float(k2s[i]), q2v = __bfloat162float(q2s[i]);
-            dk2a[i] += da * gam + dw * wdec;
-            dq2a[i] += db * gam;
-            dGa[i] += da * (k2v * gam) + db * (q2v * gam) - dw * (k2v * wdec);
-            dwk[i] = dw;
-        } else if (tid == 64) {
-            float f = 0.f;
-            for (int w = 0; w < kThreads / 32; ++w) f += frw[w];
-            dgc[e] = f;
         }
     }
 
@@ -799,8 +844,8 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
 
 size_t grads_tc_smem(int E, int dv) {
     const size_t T64 = size_t(64) * dv * 2;
-    const size_t small = size_t(64) * E * (4 + 2 + 2 + 4 * 4) + (64 + 64 + 16 + 192 + 768 + 8) * 4;
-    return 1024 + 5 * T64 + kWorkBytes + small;
+    const size_t small = size_t(64) * E * (4 + 2 + 2 + 4 * 4) + (64 + 64 + 16 + 384 + 768 + 16) * 4;
+    return 1024 + 5 * T64 + kWorkBytes + small;   // small: Gs, k2s, q2s, dk2a, dq2a, dGa, dwk, bs, dba, dgc, scl, red, frw
 }
 
 }  // namespace
