@@ -82,6 +82,21 @@ typedef struct {
     const float *h0;     /* [B,H,E,dk,dv] initial state; NULL => zero state     */
     void *o;             /* [B,T,H,dv] out_dtype output (written)               */
     float *ht;           /* [B,H,E,dk,dv] final state (written); may be NULL    */
+    /* Packed documents (Appendix A, Kernels: variable-length sequences packed
+     * into one batch, each evolved from its own initial state).  NULL: B
+     * independent sequences of T tokens.  Otherwise a HOST array of n_docs + 1
+     * token offsets, cu_seqlens[0] = 0 <= cu_seqlens[i] <= cu_seqlens[i+1],
+     * cu_seqlens[n_docs] = T, with B = 1: document i is tokens
+     * [cu_seqlens[i], cu_seqlens[i+1]) of the single sequence, its chunks start
+     * at its first token (the last one may be partial; empty documents are
+     * allowed), and h0, ht, dht and dh0 are [n_docs,H,E,dk,dv].  The library
+     * copies a chunk table built from it into the forward workspace (a
+     * cudaMemcpyAsync from pageable host memory on the call's stream), so the
+     * backward reads it from there.  Packed documents run on the tensor-core
+     * path only (bf16 inputs, dk = 128, dv a multiple of 64, E <= 8, save or
+     * not); other shapes return TLA_ERR_UNSUPPORTED.                        */
+    const int *cu_seqlens;
+    int n_docs;
 } tla_problem;
 
 /*

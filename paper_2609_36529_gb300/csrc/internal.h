@@ -12,7 +12,10 @@ namespace tla {
 
 // Byte offsets of the private buffers inside the caller's workspaces.
 struct FwdPlan {
-    int NT;              // number of chunks, ceil(T / 64)
+    int NT;              // chunks per sequence, ceil(T / 64); packed documents: all chunks
+    int nseq;            // independent states: B, or the number of packed documents
+    size_t ctab;         // packed documents: int2 [NT] (first token, rows) of every chunk
+    size_t dtab;         // packed documents: int4 [n_docs] (first token, chunks, first chunk, tokens)
     int tv;              // value columns per CTA of the SIMT recurrence
     size_t G;            // fp32 [B,T,H,E] chunk-local inclusive log-decay
     size_t A;            // fp32 [B,H,NT,64,64] Q K^T (.) R' (lower incl. diagonal)
@@ -57,10 +60,13 @@ void prof_after(cudaStream_t s);
     } while (0)
 
 FwdPlan plan_fwd(const tla_problem& p, int save_for_bwd);
+// Chunks of a problem: ceil(T / 64) per sequence, or the sum over packed documents.
+int chunk_count(const tla_problem& p);
 BwdPlan plan_bwd(const tla_problem& p);
 
 // SIMT path (fp32 arithmetic on CUDA cores; any supported dtype).
-cudaError_t launch_gate_cumsum(const tla_problem& p, float* G, cudaStream_t s);
+cudaError_t launch_gate_cumsum(const tla_problem& p, const FwdPlan& fp, const char* ws, float* G,
+                               cudaStream_t s);
 cudaError_t launch_chunk_prep(const tla_problem& p, const float* G, float* A, float* N,
                               __nv_bfloat16* A2, float* coef, __nv_bfloat16* BT, cudaStream_t s);
 // Per-chunk preparation of the tensor-core path (A, N, [T; A T], [A^T; T^T], coefficients).

@@ -19,8 +19,9 @@
 namespace tla {
 
 // ---------------------------------------------------------------------------
-__global__ void gate_cumsum_kernel(const float* __restrict__ g, float* __restrict__ G, int B,
-                                   int T, int H, int E, int NT) {
+__global__ void gate_cumsum_kernel(const float* __restrict__ g, float* __restrict__ G,
+                                   const int2* __restrict__ ctab, int B, int T, int H, int E,
+                                   int NT) {
     long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x;
     long long total = (long long)B * NT * H * E;
     if (idx >= total) return;
@@ -32,6 +33,11 @@ __global__ void gate_cumsum_kernel(const float* __restrict__ g, float* __restric
     int b = int(x / NT);
     int t0 = c * kChunk;
     int n = min(kChunk, T - t0);
+    if (ctab) {   // packed documents: the chunk's first token and rows
+        const int2 cr = ctab[c];
+        t0 = cr.x;
+        n = cr.y;
+    }
     float acc = 0.f;
     for (int r = 0; r < n; ++r) {
         size_t off = tok_idx(b, t0 + r, h, e, T, H, E);
@@ -40,13 +46,16 @@ __global__ void gate_cumsum_kernel(const float* __restrict__ g, float* __restric
     }
 }
 
-cudaError_t launch_gate_cumsum(const tla_problem& p, float* G, cudaStream_t s) {
-    int NT = (p.T + kChunk - 1) / kChunk;
+cudaError_t launch_gate_cumsum(const tla_problem& p, const FwdPlan& fp, const char* ws, float* G,
+                               cudaStream_t s) {
+    const int NT = fp.NT;
     long long total = (long long)p.B * NT * p.H * p.E;
+    if (total == 0) return cudaSuccess;
     int threads = 256;
     long long blocks = (total + threads - 1) / threads;
+    const int2* ctab = p.cu_seqlens ? (const int2*)(ws + fp.ctab) : nullptr;
     prof_before("gate_cumsum", s);
-    gate_cumsum_kernel<<<(unsigned)blocks, threads, 0, s>>>(p.g, G, p.B, p.T, p.H, p.E, NT);
+    gate_cumsum_kernel<<<(unsigned)blocks, threads, 0, s>>>(p.g, G, ctab, p.B, p.T, p.H, p.E, NT);
     prof_after(s);
     return cudaGetLastError();
 }

@@ -45,6 +45,7 @@ struct TcBwdArgs {
     float* dRbuf;
     float* dSck;
     int* err;
+    const int4* dtab;    // packed documents: (first token, chunks, first chunk, tokens); else NULL
     int T, H, dv, E, NT, use_delta, out_f32, ck_tiles;
 };
 
@@ -76,10 +77,25 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     __shared__ uint32_t tmem_slot;
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int nb = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+    const int nb = blockIdx.x, h = blockIdx.y, sb = blockIdx.z;   // sb: sequence or document
     const int n0 = nb * TV;
     const int T = p.T, H = p.H, dv = p.dv, NT = p.NT;
     const uint32_t tcols = (2 * NE + TV <= 256) ? 256u : 512u;
+    // token batch, first token, tokens, chunks and first chunk (in the workspaces) of this state
+    int b = sb, tbeg = 0, tlen = T, nct = NT, cb = 0;
+    if (p.dtab) {
+        const int4 dd = p.dtab[sb];
+        b = 0; tbeg = dd.x; nct = dd.y; cb = dd.z; tlen = dd.w;
+    }
+    if (nct == 0) {   // empty document: the gradient of the initial state is that of the final one
+        if (p.dh0)
+            for (int e = 0; e < E; ++e)
+                for (int n = 0; n < TV; ++n) {
+                    const size_t o = ((size_t(sb * H + h) * E + e) * kDk + tid) * dv + n0 + n;
+                    p.dh0[o] = p.dht ? p.dht[o] : 0.f;
+                }
+        return;
+    }
     // M=64 row owned by this thread (lanes 0-15) or prepared by it (lanes 16-31)
     const bool row_thread = lane < 16;
     const int r64 = 16 * warp + (lane & 15);
@@ -108,15 +124,15 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     auto issue_kq = [&](int c) {
         mbar_arrive_expect_tx(&bar_kq, 4 * kBoxBytes);
         for (int j = 0; j < 2; ++j) {
-            tma_load_4d(sKQ + j * 2 * kBoxBytes, &map_k, &bar_kq, 64 * j, h, c * 64, b);
-            tma_load_4d(sKQ + j * 2 * kBoxBytes + kBoxBytes, &map_q, &bar_kq, 64 * j, h, c * 64, b);
+            tma_load_4d(sKQ + j * 2 * kBoxBytes, &map_k, &bar_kq, 64 * j, h, tbeg + c * 64, b);
+            tma_load_4d(sKQ + j * 2 * kBoxBytes + kBoxBytes, &map_q, &bar_kq, 64 * j, h, tbeg + c * 64, b);
         }
     };
     auto issue_av = [&](int c) {
-        const size_t idx = size_t(b * H + h) * NT + c;
+        const size_t idx = size_t(b * H + h) * NT + cb + c;
         mbar_arrive_expect_tx(&bar_av, 4 * kBoxBytes + 64 * TV * 2 + CB * 4);
         for (int j = 0; j < 4; ++j) tma_load_2d(sBT + j * kBoxBytes, &map_bt, &bar_av, 0, int(idx * 256 + 64 * j));
-        tma_load_4d(sdO, &map_do, &bar_av, n0, h, c * 64, b);
+        tma_load_4d(sdO, &map_do, &bar_av, n0, h, tbeg + c * 64, b);
         bulk_load(sCoef + (c & 1) * CB, p.coef + idx * CB, CB * 4, &bar_av);
     };
     // Row d = tid of the gradient at the end of chunk c: operand of MMA-A'(c),
@@ -129,7 +145,7 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             if (from_dht) {
                 if (p.dht) {
                     const float4* src = reinterpret_cast<const float4*>(
-                        p.dht + ((size_t(b * H + h) * E + e) * kDk + d) * dv + n0);
+                        p.dht + ((size_t(sb * H + h) * E + e) * kDk + d) * dv + n0);
 #pragma unroll
                     for (int i = 0; i < TV / 4; ++i) {
                         float4 x = src[i];
@@ -147,7 +163,7 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
 #pragma unroll
             for (int n = 0; n < TV; n += 8) st8_split(sDh, sDl, sw128_offset(d, e * TV + n, kDk), v + n);
             {
-                const size_t slab = (((size_t(b) * H + h) * NT + c) * E + e) * kDk * dv;
+                const size_t slab = (((size_t(b) * H + h) * NT + cb + c) * E + e) * kDk * dv;
                 if (p.ck_tiles) {   // bf16 hi/lo tiles in the gradient kernel's layout
                     uint8_t* hi = reinterpret_cast<uint8_t*>(p.dSck + slab);
                     uint8_t* lo = hi + kDk * dv * 2;
@@ -170,22 +186,22 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     uint32_t mma_phase = 0;
     int pending_mma = 0;
     if (tid == 0) {
-        issue_kq(NT - 1);
-        issue_av(NT - 1);
+        issue_kq(nct - 1);
+        issue_av(nct - 1);
     }
     if (!mbar_wait(&bar_av, 0)) failed = true;
     if (__syncthreads_or(failed)) failed = true;
     if (!failed) {
-        prepare(NT - 1, true);
+        prepare(nct - 1, true);
         fence_proxy_async_smem();
         tc_fence_before();
         __syncthreads();
         tc_fence_after();
     }
 
-    for (int c = NT - 1; c >= 0 && !failed; --c) {
-        const int it = NT - 1 - c;                 // iteration index (barrier phases)
-        const int t0 = c * 64, n = min(64, T - t0);
+    for (int c = nct - 1; c >= 0 && !failed; --c) {
+        const int it = nct - 1 - c;                // iteration index (barrier phases)
+        const int t0 = tbeg + c * 64, n = min(64, tlen - c * 64);
         const float* cf = sCoef + (c & 1) * CB;
         const float* ae = cf;
         const float* be = cf + 64 * E;
@@ -259,7 +275,7 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             if (row_thread) {
 #pragma unroll
                 for (int i = 0; i < TV; ++i) st_split(sUh, sUl, sw128_offset(i, r64, TV), du[i]);
-                if (p.ck_tiles) store_tok_tile(p.dUbuf, (size_t(b) * H + h) * NT + c, dv, r64, n0, du, TV, r64 < n);
+                if (p.ck_tiles) store_tok_tile(p.dUbuf, (size_t(b) * H + h) * NT + cb + c, dv, r64, n0, du, TV, r64 < n);
                 else if (r64 < n) store_f32_row(p.dUbuf + tok_idx(b, t0 + r64, h, n0, T, H, dv), du, TV);
             }
         }
@@ -307,7 +323,7 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                     float ndr[TV];
 #pragma unroll
                     for (int i = 0; i < TV; ++i) ndr[i] = -dr[i];
-                    store_tok_tile(p.dRbuf, (size_t(b) * H + h) * NT + c, dv, r64, n0, ndr, TV, r64 < n);
+                    store_tok_tile(p.dRbuf, (size_t(b) * H + h) * NT + cb + c, dv, r64, n0, ndr, TV, r64 < n);
                 }
                 if (p.use_delta) {
                     for (int e = 0; e < E; ++e) {
@@ -364,7 +380,7 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
 #pragma unroll
                 for (int j = 0; j < TV; j += 16) tmem_ld16(tmem_lane_addr(tS, warp, e * TV + j), v + j);
                 tmem_wait_ld();
-                store_f32_row(p.dh0 + ((size_t(b * H + h) * E + e) * kDk + d) * dv + n0, v, TV);
+                store_f32_row(p.dh0 + ((size_t(sb * H + h) * E + e) * kDk + d) * dv + n0, v, TV);
             }
         }
         fence_proxy_async_smem();
@@ -412,10 +428,11 @@ cudaError_t launch_tv(const tla_problem& p, const FwdPlan& fp, const char* fws, 
     a.T = p.T; a.H = p.H; a.dv = p.dv; a.E = p.E; a.NT = NT;
     a.use_delta = p.use_delta; a.out_f32 = p.out_dtype == TLA_FP32;
     a.ck_tiles = fp.ck_tiles;
+    a.dtab = p.cu_seqlens ? (const int4*)(fws + fp.dtab) : nullptr;
     const size_t smem = tc_bwd_smem<TV>(p.E);
     auto kern = bwd_recurrence_tc_kernel<TV>;
     cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    dim3 grid(p.dv / TV, p.H, p.B);
+    dim3 grid(p.dv / TV, p.H, fp.nseq);
     prof_before("bwd_recurrence_tc", s);
     kern<<<grid, kThreads, smem, s>>>(mk, mq, mo, mb, a);
     prof_after(s);

@@ -54,6 +54,7 @@ struct TcFwdArgs {
     float* Ubuf;
     float* Rbuf;
     int* err;
+    const int4* dtab;    // packed documents: (first token, chunks, first chunk, tokens); else NULL
     int T, H, dv, E, NT, use_delta, save, out_f32, ck_tiles;
 };
 
@@ -84,10 +85,25 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     __shared__ uint32_t tmem_slot;
 
     const int tid = threadIdx.x, warp = tid >> 5;
-    const int nb = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+    const int nb = blockIdx.x, h = blockIdx.y, sb = blockIdx.z;   // sb: sequence or document
     const int n0 = nb * TV;
     const int T = p.T, H = p.H, dv = p.dv, NT = p.NT;
     const uint32_t tcols = (2 * NE <= 256) ? 256u : 512u;
+    // token batch, first token, tokens, chunks and first chunk (in the workspace) of this state
+    int b = sb, tbeg = 0, tlen = T, nct = NT, cb = 0;
+    if (p.dtab) {
+        const int4 dd = p.dtab[sb];
+        b = 0; tbeg = dd.x; nct = dd.y; cb = dd.z; tlen = dd.w;
+    }
+    if (nct == 0) {   // empty document: the final state is the initial one
+        if (p.ht)
+            for (int e = 0; e < E; ++e)
+                for (int n = 0; n < TV; ++n) {
+                    const size_t o = ((size_t(sb * H + h) * E + e) * kDk + tid) * dv + n0 + n;
+                    p.ht[o] = p.h0 ? p.h0[o] : 0.f;
+                }
+        return;
+    }
 
     if (warp == 0) {
         tmem_alloc(&tmem_slot, tcols);
@@ -112,17 +128,17 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     auto issue_kq = [&](int c) {
         mbar_arrive_expect_tx(&bar_kq, 4 * kBoxBytes);
         for (int j = 0; j < 2; ++j) {
-            tma_load_4d(sKQ + j * 2 * kBoxBytes, &map_k, &bar_kq, 64 * j, h, c * 64, b);
-            tma_load_4d(sKQ + j * 2 * kBoxBytes + kBoxBytes, &map_q, &bar_kq, 64 * j, h, c * 64, b);
+            tma_load_4d(sKQ + j * 2 * kBoxBytes, &map_k, &bar_kq, 64 * j, h, tbeg + c * 64, b);
+            tma_load_4d(sKQ + j * 2 * kBoxBytes + kBoxBytes, &map_q, &bar_kq, 64 * j, h, tbeg + c * 64, b);
         }
     };
     // [T; A T] hi/lo and V of chunk c, and its coefficient block into buffer c & 1
     auto issue_av = [&](int c) {
-        const size_t idx = size_t(b * H + h) * NT + c;
+        const size_t idx = size_t(b * H + h) * NT + cb + c;
         mbar_arrive_expect_tx(&bar_av, 4 * kBoxBytes + 64 * TV * 2 + CB * 4);
         tma_load_2d(sA2, &map_a2, &bar_av, 0, int(idx * 256));
         tma_load_2d(sA2 + 2 * kBoxBytes, &map_a2, &bar_av, 0, int(idx * 256 + 128));
-        tma_load_4d(sV, &map_v, &bar_av, n0, h, c * 64, b);
+        tma_load_4d(sV, &map_v, &bar_av, n0, h, tbeg + c * 64, b);
         bulk_load(sCoef + (c & 1) * CB, p.coef + idx * CB, CB * 4, &bar_av);
     };
     // Row d = tid of S_{[c]} (from h0 or from TMEM) as the bf16 hi/lo operand of MMA-A.
@@ -133,7 +149,7 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             if (from_h0) {
                 if (p.h0) {
                     const float4* src = reinterpret_cast<const float4*>(
-                        p.h0 + ((size_t(b * H + h) * E + e) * kDk + d) * dv + n0);
+                        p.h0 + ((size_t(sb * H + h) * E + e) * kDk + d) * dv + n0);
 #pragma unroll
                     for (int i = 0; i < TV / 4; ++i) {
                         float4 x = src[i];
@@ -162,7 +178,7 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             if (from_h0) {
                 if (p.h0) {
                     const float4* src = reinterpret_cast<const float4*>(
-                        p.h0 + ((size_t(b * H + h) * E + e) * kDk + d) * dv + n0);
+                        p.h0 + ((size_t(sb * H + h) * E + e) * kDk + d) * dv + n0);
 #pragma unroll
                     for (int i = 0; i < TV / 4; ++i) {
                         float4 x = src[i];
@@ -178,7 +194,7 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                 tmem_wait_ld();
             }
             if (p.save) {
-                const size_t slab = (((size_t(b) * H + h) * NT + c) * E + e) * kDk * dv;
+                const size_t slab = (((size_t(b) * H + h) * NT + cb + c) * E + e) * kDk * dv;
                 if (p.ck_tiles) {   // bf16 hi/lo tiles in the gradient kernel's layout
                     uint8_t* hi = reinterpret_cast<uint8_t*>(p.Sck + slab);
                     uint8_t* lo = hi + kDk * dv * 2;
@@ -233,8 +249,8 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         }
     }
 
-    for (int c = 0; c < NT && !failed; ++c) {
-        const int t0 = c * 64, n = min(64, T - t0);
+    for (int c = 0; c < nct && !failed; ++c) {
+        const int t0 = tbeg + c * 64, n = min(64, tlen - c * 64);
         const float* cf = sCoef + (c & 1) * CB;
         const float* ae = cf;
         const float* be = cf + 64 * E;
@@ -314,7 +330,7 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         }
         pending_mma = 1;
         if (warp < 2 && p.Rbuf) {   // while MMA-B runs
-            if (p.ck_tiles) store_tok_tile(p.Rbuf, (size_t(b) * H + h) * NT + c, dv, tid, n0, res, TV, tid < n);
+            if (p.ck_tiles) store_tok_tile(p.Rbuf, (size_t(b) * H + h) * NT + cb + c, dv, tid, n0, res, TV, tid < n);
             else if (tid < n) store_f32_row(p.Rbuf + tok_idx(b, t0 + tid, h, n0, T, H, dv), res, TV);
         }
         ok = mbar_wait(&bar_mma, mma_phase);
@@ -322,7 +338,7 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         if (__syncthreads_or(!ok)) { failed = true; break; }
         pending_mma = 0;
         tc_fence_after();
-        if (tid == 0 && c + 1 < NT) issue_av(c + 1);   // [T; A T], V and the other coef buffer are free
+        if (tid == 0 && c + 1 < nct) issue_av(c + 1);   // [T; A T], V and the other coef buffer are free
 
         // ---- epi-B: Ut operand (key rows); O = Oi + Oa (query rows)
         float d2[TV];
@@ -364,7 +380,7 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             const int r = warp < 2 ? tid : tid - 64;
             if (warp < 2) {
                 if (p.save) {
-                    if (p.ck_tiles) store_tok_tile(p.Ubuf, (size_t(b) * H + h) * NT + c, dv, r, n0, d2, TV, r < n);
+                    if (p.ck_tiles) store_tok_tile(p.Ubuf, (size_t(b) * H + h) * NT + cb + c, dv, r, n0, d2, TV, r < n);
                     else if (r < n) store_f32_row(p.Ubuf + tok_idx(b, t0 + r, h, n0, T, H, dv), d2, TV);
                 }
             } else if (r < n) {
@@ -373,14 +389,14 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         }
         ok = mbar_wait(&bar_mma, mma_phase);
         mma_phase ^= 1;
-        if (c + 1 < NT) ok = ok && mbar_wait(&bar_av, (c + 1) & 1);   // chunk c+1's gamma^C
+        if (c + 1 < nct) ok = ok && mbar_wait(&bar_av, (c + 1) & 1);   // chunk c+1's gamma^C
         if (__syncthreads_or(!ok)) { failed = true; break; }
         pending_mma = 0;
         tc_fence_after();
-        if (tid == 0 && c + 1 < NT) issue_kq(c + 1);   // key/query buffer is free
+        if (tid == 0 && c + 1 < nct) issue_kq(c + 1);   // key/query buffer is free
 
         // ---- epi-C: next chunk's operand, MMA-A(c+1), then checkpoint and scaling
-        if (c + 1 < NT) {
+        if (c + 1 < nct) {
             write_operand(false);
             fence_proxy_async_smem();
             tc_fence_before();
@@ -397,7 +413,7 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
 #pragma unroll
                 for (int j = 0; j < TV; j += 16) tmem_ld16(tmem_lane_addr(tS, warp, e * TV + j), v + j);
                 tmem_wait_ld();
-                store_f32_row(p.ht + ((size_t(b * H + h) * E + e) * kDk + d) * dv + n0, v, TV);
+                store_f32_row(p.ht + ((size_t(sb * H + h) * E + e) * kDk + d) * dv + n0, v, TV);
             }
         }
     }
@@ -444,10 +460,11 @@ cudaError_t launch_tv(const tla_problem& p, const FwdPlan& fp, char* ws, int sav
     a.T = p.T; a.H = p.H; a.dv = p.dv; a.E = p.E; a.NT = NT;
     a.use_delta = p.use_delta; a.save = save; a.out_f32 = p.out_dtype == TLA_FP32;
     a.ck_tiles = fp.ck_tiles;
+    a.dtab = p.cu_seqlens ? (const int4*)(ws + fp.dtab) : nullptr;
     const size_t smem = tc_fwd_smem<TV>(p.E);
     auto kern = fwd_recurrence_tc_kernel<TV>;
     cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    dim3 grid(p.dv / TV, p.H, p.B);
+    dim3 grid(p.dv / TV, p.H, fp.nseq);
     prof_before("fwd_recurrence_tc", s);
     kern<<<grid, kThreads, smem, s>>>(mk, mq, mv, ma, a);
     prof_after(s);

@@ -60,6 +60,7 @@ struct TcGradArgs {
     float* dbeta;
     float* dg;
     int* err;
+    const int2* ctab;    // packed documents: (first token, rows) of each chunk; else NULL
     int T, H, dv, E, NT, use_delta, out_f32;
 };
 
@@ -141,7 +142,7 @@ __device__ __forceinline__ float unpack_bf16(const uint32_t* pk, int j) {
     return __uint_as_float((j & 1) ? (w & 0xffff0000u) : (w << 16));
 }
 
-template <int OUT_F32>
+template <int OUT_F32, bool PACKED>
 __global__ void __launch_bounds__(kThreads, 1)
 bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                           const __grid_constant__ CUtensorMap map_q,
@@ -151,7 +152,14 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                                              ~uintptr_t(1023));
     const int E = p.E, dv = p.dv, T = p.T, H = p.H, NT = p.NT;
     const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
-    const int t0 = c * 64, n = min(64, T - t0);
+    // first token and rows of this chunk (packed documents: from the chunk table; a separate
+    // instance, so that the regular one keeps t0 a compile-time multiple of 64)
+    int t0 = c * 64, n = min(64, T - t0);
+    if (PACKED) {
+        const int2 cr = p.ctab[c];
+        t0 = cr.x;
+        n = cr.y;
+    }
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const uint32_t T64 = 64u * dv * 2;         // bytes of a [64][dv] bf16 tile
     const int nb = dv / 64;                    // 64-column blocks of a value row
@@ -880,10 +888,12 @@ cudaError_t launch_bwd_chunk_grads_tc(const tla_problem& p, const FwdPlan& fp, c
     a.dSck = (const float*)(bws + bp.dS);
     a.dq = dq; a.dk = dk; a.dq2 = dq2; a.dk2 = dk2; a.dbeta = dbeta; a.dg = dg;
     a.err = err;
+    a.ctab = p.cu_seqlens ? (const int2*)(fws + fp.ctab) : nullptr;
     a.T = p.T; a.H = p.H; a.dv = p.dv; a.E = p.E; a.NT = fp.NT;
     a.use_delta = p.use_delta; a.out_f32 = p.out_dtype == TLA_FP32;
     const size_t smem = grads_tc_smem(p.E, p.dv);
-    auto kern = a.out_f32 ? bwd_chunk_grads_tc_kernel<1> : bwd_chunk_grads_tc_kernel<0>;
+    auto kern = a.ctab ? (a.out_f32 ? bwd_chunk_grads_tc_kernel<1, true> : bwd_chunk_grads_tc_kernel<0, true>)
+                       : (a.out_f32 ? bwd_chunk_grads_tc_kernel<1, false> : bwd_chunk_grads_tc_kernel<0, false>);
     cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     dim3 grid(fp.NT, p.H, p.B);
     prof_before("bwd_chunk_grads_tc", s);

@@ -38,6 +38,7 @@ struct TcPrepArgs {
     __nv_bfloat16* BTout;
     float* coef;
     int* err;
+    const int2* ctab;    // packed documents: (first token, rows) of each chunk; else NULL
     int T, H, E, NT, use_delta;
 };
 
@@ -69,7 +70,12 @@ chunk_prep_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                                              ~uintptr_t(1023));
     const int E = p.E, T = p.T, H = p.H, NT = p.NT;
     const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
-    const int t0 = c * 64, n = min(64, T - t0);
+    int t0 = c * 64, n = min(64, T - t0);
+    if (p.ctab) {
+        const int2 cr = p.ctab[c];
+        t0 = cr.x;
+        n = cr.y;
+    }
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     // five matrix slots; the TMA key/query tile overlays slots 3-4 until the products are read
     float* slot = reinterpret_cast<float*>(sm);
@@ -378,6 +384,7 @@ cudaError_t launch_chunk_prep_tc(const tla_problem& p, const FwdPlan& fp, char* 
     a.BTout = fp.tcb ? (__nv_bfloat16*)(ws + fp.BT) : nullptr;
     a.coef = (float*)(ws + fp.coef);
     a.err = err;
+    a.ctab = p.cu_seqlens ? (const int2*)(ws + fp.ctab) : nullptr;
     a.T = p.T; a.H = p.H; a.E = p.E; a.NT = fp.NT; a.use_delta = p.use_delta;
     const size_t smem = prep_tc_smem(p.E);
     cudaFuncSetAttribute(chunk_prep_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);

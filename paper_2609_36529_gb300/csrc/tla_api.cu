@@ -2,6 +2,7 @@
 // Declarations and the contract of every entry point: include/tla.h.
 #include <string.h>
 
+#include <algorithm>
 #include <mutex>
 #include <vector>
 
@@ -33,6 +34,13 @@ static tla_status validate(const tla_problem* p) {
     const void* ptrs[] = {p->q, p->k, p->v, p->q2, p->k2, p->g, p->beta, p->h0, p->o, p->ht};
     for (const void* x : ptrs)
         if (!aligned16(x)) return TLA_ERR_INVALID_ARG;
+    if (p->cu_seqlens) {   // packed documents: B = 1, offsets 0 = cu[0] <= ... <= cu[n_docs] = T
+        if (p->B != 1 || p->n_docs < 1) return TLA_ERR_INVALID_ARG;
+        if (p->n_docs > 65535) return TLA_ERR_UNSUPPORTED;
+        if (p->cu_seqlens[0] != 0 || p->cu_seqlens[p->n_docs] != p->T) return TLA_ERR_INVALID_ARG;
+        for (int d = 0; d < p->n_docs; ++d)
+            if (p->cu_seqlens[d + 1] < p->cu_seqlens[d]) return TLA_ERR_INVALID_ARG;
+    }
     return TLA_OK;
 }
 
@@ -54,10 +62,19 @@ static int simt_tv(const tla_problem& p) {
     return 8;
 }
 
+int chunk_count(const tla_problem& p) {
+    if (!p.cu_seqlens) return (p.T + kChunk - 1) / kChunk;
+    long long nc = 0;
+    for (int d = 0; d < p.n_docs; ++d)
+        nc += (p.cu_seqlens[d + 1] - p.cu_seqlens[d] + kChunk - 1) / kChunk;
+    return (int)nc;
+}
+
 FwdPlan plan_fwd(const tla_problem& p, int save) {
     FwdPlan f;
     memset(&f, 0, sizeof(f));
-    f.NT = (p.T + kChunk - 1) / kChunk;
+    f.NT = chunk_count(p);
+    f.nseq = p.cu_seqlens ? p.n_docs : p.B;
     f.tv = simt_tv(p);
     f.tc_tv = tc_fwd_tv(p);   // layout depends on shapes only
     const size_t tokE = (size_t)p.B * p.T * p.H * p.E * 4;
@@ -81,6 +98,10 @@ FwdPlan plan_fwd(const tla_problem& p, int save) {
         f.U = off; off = align256(off + tokV);
         if (p.use_delta || f.ck_tiles) { f.Res = off; off = align256(off + tokV); }
     }
+    if (p.cu_seqlens) {
+        f.ctab = off; off = align256(off + (size_t)f.NT * sizeof(int2));
+        f.dtab = off; off = align256(off + (size_t)p.n_docs * sizeof(int4));
+    }
     f.bytes = off;
     return f;
 }
@@ -88,7 +109,7 @@ FwdPlan plan_fwd(const tla_problem& p, int save) {
 BwdPlan plan_bwd(const tla_problem& p) {
     BwdPlan b;
     memset(&b, 0, sizeof(b));
-    const int NT = (p.T + kChunk - 1) / kChunk;
+    const int NT = chunk_count(p);
     b.tv = simt_tv(p);
     const size_t tokV = (size_t)p.B * NT * kChunk * p.H * p.dv * 4;   // whole chunks (token tiles)
     const size_t states = (size_t)p.B * p.H * NT * p.E * p.dk * p.dv * 4;
@@ -164,7 +185,25 @@ tla_status tla_chunk_fwd(const tla_problem* p, void* workspace, size_t workspace
         return TLA_ERR_WORKSPACE;
     cudaStream_t s = (cudaStream_t)stream;
     char* ws = (char*)workspace;
-    cudaError_t e = launch_gate_cumsum(*p, (float*)(ws + fp.G), s);
+    if (p->cu_seqlens) {   // packed documents: tensor-core path only; chunk and document tables
+        if (!fp.tc_tv) return TLA_ERR_UNSUPPORTED;
+        std::vector<int2> ct(fp.NT);
+        std::vector<int4> dt(p->n_docs);
+        int g = 0;
+        for (int d = 0; d < p->n_docs; ++d) {
+            const int t0 = p->cu_seqlens[d], len = p->cu_seqlens[d + 1] - t0;
+            const int nc = (len + kChunk - 1) / kChunk;
+            dt[d] = make_int4(t0, nc, g, len);
+            for (int c = 0; c < nc; ++c) ct[g++] = make_int2(t0 + c * kChunk, std::min(kChunk, len - c * kChunk));
+        }
+        cudaError_t ce = cudaMemcpyAsync(ws + fp.ctab, ct.data(), ct.size() * sizeof(int2),
+                                         cudaMemcpyHostToDevice, s);
+        if (ce == cudaSuccess)
+            ce = cudaMemcpyAsync(ws + fp.dtab, dt.data(), dt.size() * sizeof(int4),
+                                 cudaMemcpyHostToDevice, s);
+        if (ce != cudaSuccess) return TLA_ERR_CUDA;
+    }
+    cudaError_t e = launch_gate_cumsum(*p, fp, ws, (float*)(ws + fp.G), s);
     if (e == cudaSuccess) {
         if (fp.tc_tv)
             e = launch_chunk_prep_tc(*p, fp, ws, device_error_word(), s);
@@ -197,6 +236,7 @@ tla_status tla_chunk_bwd(const tla_problem* p, const void* fwd_ws, size_t fwd_ws
     if ((p->h0 != nullptr) != (dh0 != nullptr)) return TLA_ERR_INVALID_ARG;
     FwdPlan fp = plan_fwd(*p, 1);
     BwdPlan bp = plan_bwd(*p);
+    if (p->cu_seqlens && !(fp.tcb && tc_grads_ok(*p, fp))) return TLA_ERR_UNSUPPORTED;
     if (!fwd_ws || fwd_ws_bytes < fp.bytes || ((uintptr_t)fwd_ws & 255)) return TLA_ERR_WORKSPACE;
     if (!workspace || workspace_bytes < bp.bytes || ((uintptr_t)workspace & 255))
         return TLA_ERR_WORKSPACE;

@@ -16,10 +16,14 @@ Recipe (fixed tensor order q, k, q2, k2, v, beta, g, h0, dO, one
   h0     ~ N(0, h0_std^2) [B,H,E,dk,dv] fp32     (only when h0_std > 0)
   dO     ~ N(0,1) [B,T,H,dv]                      (only when requested)
 q, k, q2, k2, v, dO are then cast to ``dtype``; g, beta, h0 stay fp32.
+Packed documents: the same draws for one sequence of sum(lengths) tokens, initial
+states per document from a generator seeded with ``seed + 1``, and document lengths
+log-normal around a mean (sigma 1) with the last one cut to the total.
 """
 from dataclasses import dataclass
 from typing import Optional
 
+import numpy as np
 import torch
 
 
@@ -100,6 +104,40 @@ def chunk_inputs(B, T, H, dk, dv, E, dtype="bf16", with_beta=True, h0_std=0.0,
     out["h0"] = randn(B, H, E, dk, dv) * h0_std if h0_std > 0 else None
     out["dO"] = randn(B, T, H, dv).to(dt) if backward else None
     return out
+
+
+def packed_inputs(lens, H, dk, dv, E, dtype="bf16", with_beta=True, h0_std=0.0,
+                  backward=False, device="cpu", seed=0):
+    """Inputs of packed documents of the given lengths: one sequence of sum(lens) tokens
+    (B = 1) drawn like chunk_inputs, initial states per document ([n_docs,H,E,dk,dv]) and
+    the host token offsets cu_seqlens (n_docs + 1 values, starting at 0)."""
+    T = int(sum(int(n) for n in lens))
+    x = chunk_inputs(1, T, H, dk, dv, E, dtype, with_beta, 0.0, backward, device=device,
+                     seed=seed)
+    if h0_std > 0:
+        gen = torch.Generator(device=torch.device(device))
+        gen.manual_seed(seed + 1)
+        x["h0"] = torch.randn(len(lens), H, E, dk, dv, generator=gen, device=torch.device(device),
+                              dtype=torch.float32) * h0_std
+    cu = [0]
+    for n in lens:
+        cu.append(cu[-1] + int(n))
+    return x, cu
+
+
+def packed_lengths(total, mean_len, seed=0, min_len=1):
+    """Document lengths summing to `total`: log-normal around `mean_len` (sigma 1), the
+    last one cut to fit -- a stand-in for the length mix of a packed pretraining batch."""
+    rng = np.random.default_rng(seed)
+    mu = np.log(mean_len) - 0.5
+    lens = []
+    left = int(total)
+    while left > 0:
+        n = max(min_len, int(rng.lognormal(mu, 1.0)))
+        n = min(n, left)
+        lens.append(n)
+        left -= n
+    return lens
 
 
 def workload_inputs(w: Workload, device="cpu", seed=0, B=None, T=None, H=None):

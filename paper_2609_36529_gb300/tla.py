@@ -38,7 +38,8 @@ class tla_problem(ctypes.Structure):
                 ("q", ctypes.c_void_p), ("k", ctypes.c_void_p), ("v", ctypes.c_void_p),
                 ("q2", ctypes.c_void_p), ("k2", ctypes.c_void_p), ("g", ctypes.c_void_p),
                 ("beta", ctypes.c_void_p), ("h0", ctypes.c_void_p), ("o", ctypes.c_void_p),
-                ("ht", ctypes.c_void_p)]
+                ("ht", ctypes.c_void_p), ("cu_seqlens", ctypes.POINTER(ctypes.c_int)),
+                ("n_docs", ctypes.c_int)]
 
 
 _lib = None
@@ -100,8 +101,13 @@ def _check(fn, status):
         raise TlaError(fn, status)
 
 
+def _n_states(q, cu_seqlens):
+    return q.shape[0] if cu_seqlens is None else len(cu_seqlens) - 1
+
+
 def make_problem(q, k, v, q2, k2, g, beta=None, h0=None, o=None, ht=None, use_delta=True,
-                 chunk=64, out_dtype=None):
+                 chunk=64, out_dtype=None, cu_seqlens=None):
+    """cu_seqlens: None, or the host token offsets of packed documents (B = 1)."""
     B, T, H, dk = q.shape
     p = tla_problem()
     p.B, p.T, p.H, p.dk, p.dv, p.E = B, T, H, dk, v.shape[-1], q2.shape[-1]
@@ -112,6 +118,12 @@ def make_problem(q, k, v, q2, k2, g, beta=None, h0=None, o=None, ht=None, use_de
     for name, t in (("q", q), ("k", k), ("v", v), ("q2", q2), ("k2", k2), ("g", g),
                     ("beta", beta), ("h0", h0), ("o", o), ("ht", ht)):
         setattr(p, name, _ptr(t))
+    if cu_seqlens is not None:
+        cu = [int(x) for x in cu_seqlens]
+        arr = (ctypes.c_int * len(cu))(*cu)
+        p._cu_keepalive = arr   # the library reads it during the call
+        p.cu_seqlens = ctypes.cast(arr, ctypes.POINTER(ctypes.c_int))
+        p.n_docs = len(cu) - 1
     return p
 
 
@@ -129,17 +141,20 @@ def _workspace(nbytes, device):
 
 
 def tla_chunk_fwd(q, k, v, q2, k2, g, beta=None, h0=None, use_delta=True, save_for_bwd=False,
-                  want_ht=True, o=None, ht=None, workspace=None, out_dtype=torch.float32):
+                  want_ht=True, o=None, ht=None, workspace=None, out_dtype=torch.float32,
+                  cu_seqlens=None):
     """Chunkwise forward. Returns (o, ht or None, workspace).
 
-    o is allocated in `out_dtype` (default fp32, the accumulation precision)."""
+    o is allocated in `out_dtype` (default fp32, the accumulation precision).  With
+    cu_seqlens (host offsets of packed documents, B = 1) h0 and ht are per document."""
     B, T, H, _ = q.shape
     E, dv = q2.shape[-1], v.shape[-1]
     if o is None:
         o = torch.empty(B, T, H, dv, dtype=out_dtype, device=q.device)
     if ht is None and want_ht:
-        ht = torch.empty(B, H, E, q.shape[-1], dv, dtype=torch.float32, device=q.device)
-    p = make_problem(q, k, v, q2, k2, g, beta, h0, o, ht, use_delta)
+        ht = torch.empty(_n_states(q, cu_seqlens), H, E, q.shape[-1], dv, dtype=torch.float32,
+                         device=q.device)
+    p = make_problem(q, k, v, q2, k2, g, beta, h0, o, ht, use_delta, cu_seqlens=cu_seqlens)
     need = fwd_workspace_bytes(p, save_for_bwd)
     if need == 0:
         raise TlaError("tla_fwd_workspace_bytes", -1)
@@ -151,7 +166,7 @@ def tla_chunk_fwd(q, k, v, q2, k2, g, beta=None, h0=None, use_delta=True, save_f
 
 
 def tla_chunk_fwd_noalloc(q, k, v, q2, k2, g, beta=None, h0=None, use_delta=True, o=None,
-                          ht=None):
+                          ht=None, cu_seqlens=None):
     """Forward through the entry point that allocates nothing (built-in scratch).
 
     o and ht must be preallocated by the caller when it cannot allocate; when they
@@ -160,13 +175,14 @@ def tla_chunk_fwd_noalloc(q, k, v, q2, k2, g, beta=None, h0=None, use_delta=True
     E, dv = q2.shape[-1], v.shape[-1]
     if o is None:
         o = torch.empty(B, T, H, dv, dtype=torch.float32, device=q.device)
-    p = make_problem(q, k, v, q2, k2, g, beta, h0, o, ht, use_delta)
+    p = make_problem(q, k, v, q2, k2, g, beta, h0, o, ht, use_delta, cu_seqlens=cu_seqlens)
     _check("tla_chunk_fwd_noalloc", lib().tla_chunk_fwd_noalloc(ctypes.byref(p), _stream()))
     return o, ht
 
 
 def tla_chunk_bwd(q, k, v, q2, k2, g, dO, fwd_workspace, beta=None, h0=None, dht=None,
-                  use_delta=True, workspace=None, grads=None, out_dtype=torch.float32):
+                  use_delta=True, workspace=None, grads=None, out_dtype=torch.float32,
+                  cu_seqlens=None):
     """Backward of tla_chunk_fwd; fwd_workspace from a save_for_bwd=True forward.
 
     Returns (dict of gradients dq, dk, dv, dq2, dk2, dg[, dbeta][, dh0], workspace).
@@ -184,7 +200,7 @@ def tla_chunk_bwd(q, k, v, q2, k2, g, dO, fwd_workspace, beta=None, h0=None, dht
         if h0 is not None:
             grads["dh0"] = torch.empty_like(h0)
     p = make_problem(q, k, v, q2, k2, g, beta, h0, use_delta=use_delta,
-                     out_dtype=grads["dq"].dtype)
+                     out_dtype=grads["dq"].dtype, cu_seqlens=cu_seqlens)
     # o is not read by the backward; a non-null placeholder satisfies validation
     p.o = _ptr(dO)
     need = bwd_workspace_bytes(p)

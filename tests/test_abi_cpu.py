@@ -112,3 +112,35 @@ def test_noalloc_entry_rejects_on_host(tla):
     p = _problem(tla, B=64, T=8192, H=16, dk=128, dv=128)   # workspace far above the buffer
     assert L.tla_fwd_workspace_bytes(ctypes.byref(p), 0) > cap
     assert L.tla_chunk_fwd_noalloc(ctypes.byref(p), None) == -5
+
+
+def test_packed_documents_validation(tla):
+    """cu_seqlens (Appendix A, Kernels: packed documents) is checked on the host."""
+    L = tla.lib()
+
+    def packed(cu, **kw):
+        args = dict(B=1, T=cu[-1])
+        args.update(kw)
+        p = _problem(tla, **args)
+        arr = (ctypes.c_int * len(cu))(*cu)
+        p._keep = arr
+        p.cu_seqlens = ctypes.cast(arr, ctypes.POINTER(ctypes.c_int))
+        p.n_docs = len(cu) - 1
+        return p
+
+    ok = packed([0, 10, 10, 100])   # an empty document is allowed
+    need = L.tla_fwd_workspace_bytes(ctypes.byref(ok), 1)
+    assert need > 0 and need % 256 == 0
+    # each document starts its own chunks: 1 + 0 + 2 chunks instead of 2 for 100 tokens
+    plain = _problem(tla, B=1, T=100)
+    assert need > L.tla_fwd_workspace_bytes(ctypes.byref(plain), 1)
+    bad = [packed([1, 10, 100]), packed([0, 50, 40, 100]), packed([0, 10, 99], T=100),
+           packed([0, 100], B=2)]
+    for p in bad:
+        assert L.tla_fwd_workspace_bytes(ctypes.byref(p), 1) == 0
+        assert L.tla_chunk_fwd(ctypes.byref(p), None, 0, 0, None) == -1
+    p = packed([0, 100])
+    p.n_docs = 0
+    assert L.tla_chunk_fwd(ctypes.byref(p), None, 0, 0, None) == -1
+    # packed documents run on the tensor-core path only (here d_k = 64): refused before a launch
+    assert L.tla_chunk_fwd(ctypes.byref(ok), ctypes.c_void_p(0x100000), need, 1, None) == -2
