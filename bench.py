@@ -6,7 +6,9 @@ backward of triadic Gated DeltaNet on the headline workload (B=8, H=16, T=8192,
 d_k=d_v=128, E=4, chunk 64, bf16 inputs / fp32 state), synthetic seeded
 inputs.  The single-token decode step is measured in the same run on the
 decode workload (fp32 state [256,32,8,128,128], 100 steps each of sGLA and
-GDN after a 512-token chunked prefill) and reported under "decode".
+GDN after a 512-token chunked prefill) and reported under "decode", and the
+same step with the headline's tokens packed into documents of log-normal length
+around 1000 tokens (cu_seqlens, each document from its own state) under "packed".
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
@@ -318,6 +320,10 @@ def run_ours(args):
                       ws_n)
 
     # ---- decode workload
+    packed = None
+    if not args.no_packed:
+        packed = run_packed(args, tla, inputs, w, dev, stream, barrier, max_over_ranks, ws_n, rank)
+        packed["vs_uniform_batch"] = round(packed["value"] / value, 4)
     decode = None
     if not args.no_decode:
         del fws, bws
@@ -347,7 +353,7 @@ def run_ours(args):
             "tflops_frac": round(total_flops / (ms_step / 1e3) / 1e12 / peak, 5),
             "roofline": roofline, "kernels": kernels, "gpu_launches": gpu_launches,
             "clocks": ck, "clocks_remeasured": remeasured,
-            "e2e": e2e, "decode": decode, "cpu_baseline": cpu, "impl": "ours",
+            "e2e": e2e, "packed": packed, "decode": decode, "cpu_baseline": cpu, "impl": "ours",
         }
         print(json.dumps(line), flush=True)
     if ws_n > 1:
@@ -419,6 +425,57 @@ def run_e2e(args, tla, x, w, dev, stream, o, fws, bws, grads, barrier, max_over_
             "pipeline": "3 streams (host->device, compute, device->host), 2 device copies of "
                         "inputs and outputs; every step uploads all inputs and downloads o "
                         "and every gradient"}
+
+
+def run_packed(args, tla, inputs, w, dev, stream, barrier, max_over_ranks, ws_n, rank):
+    """The headline step's tokens as packed documents (Appendix A, Kernels): one sequence of
+    B*T tokens split into documents of log-normal length around 1000 tokens, each from its
+    own zero state; forward + backward per step through the public API (cu_seqlens)."""
+    total = w.B * w.T
+    lens = inputs.packed_lengths(total, 1000, seed=rank)
+    x, cu = inputs.packed_inputs(lens, w.H, w.dk, w.dv, w.E, dtype=w.dtype, backward=True,
+                                 device=dev, seed=100 + rank)
+    o = torch.empty(1, total, w.H, w.dv, dtype=torch.float32, device=dev)
+    p = tla.make_problem(x["q"], x["k"], x["v"], x["q2"], x["k2"], x["g"], x["beta"], None, o,
+                         None, use_delta=True, cu_seqlens=cu)
+    fws = torch.empty(tla.fwd_workspace_bytes(p, True), dtype=torch.uint8, device=dev)
+    bws = torch.empty(tla.bwd_workspace_bytes(p), dtype=torch.uint8, device=dev)
+    f32 = dict(dtype=torch.float32, device=dev)
+    grads = {"dq": torch.empty(x["q"].shape, **f32), "dk": torch.empty(x["k"].shape, **f32),
+             "dv": torch.empty(x["v"].shape, **f32), "dq2": torch.empty(x["q2"].shape, **f32),
+             "dk2": torch.empty(x["k2"].shape, **f32), "dg": torch.empty_like(x["g"]),
+             "dbeta": torch.empty_like(x["beta"])}
+
+    def step():
+        tla.tla_chunk_fwd(x["q"], x["k"], x["v"], x["q2"], x["k2"], x["g"], x["beta"], None,
+                          use_delta=True, save_for_bwd=True, want_ht=False, o=o, workspace=fws,
+                          cu_seqlens=cu)
+        tla.tla_chunk_bwd(x["q"], x["k"], x["v"], x["q2"], x["k2"], x["g"], x["dO"], fws,
+                          beta=x["beta"], use_delta=True, workspace=bws, grads=grads,
+                          cu_seqlens=cu)
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    torch.cuda.synchronize()
+    k = max(3, min(args.steps, 5))
+    barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(k):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    if tla.tla_last_device_status() != 0:
+        raise RuntimeError("device status not OK after the packed-document loop")
+    ms = max_over_ranks(e0.elapsed_time(e1) / k)
+    nc = sum((n + 63) // 64 for n in lens)
+    return {"workload": f"gdn_fwdbwd_bf16_packed_T{total}_H{w.H}_d{w.dk}_E{w.E}",
+            "value": round(ws_n * total / (ms / 1e3), 1), "unit": "tokens/s",
+            "ms_per_step": round(ms, 4), "steps": k, "docs": len(lens),
+            "doc_len": {"mean": round(total / len(lens), 1), "min": min(lens), "max": max(lens)},
+            "chunks": nc, "chunks_uniform_batch": total // 64,
+            "data": "synthetic; lengths log-normal around 1000 tokens (sigma 1), seeded"}
 
 
 def run_decode(args, tla, inputs, dev, stream, lib, peaks, barrier, max_over_ranks, ws_n):
@@ -552,6 +609,7 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-decode", action="store_true")
+    ap.add_argument("--no-packed", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--ref-tokens", type=int, default=1024,
