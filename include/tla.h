@@ -58,7 +58,8 @@ typedef enum { TLA_BF16 = 0, TLA_FP32 = 1 } tla_dtype;
 
 /*
  * One chunkwise problem: B sequences of T tokens, H heads.
- * Supported: 1 <= dk, dv <= 128 with dk, dv multiples of 16; 1 <= E <= 16;
+ * Supported: 1 <= dk, dv <= 128 with dk, dv multiples of 16; 1 <= E <= 32, with
+ * dk <= 64 when E > 16 (the paper's E = 16/32 variants use d_k = 32/64);
  * chunk == 64 (the paper's C, Appendix A); T >= 1 (a last partial chunk is
  * allowed); B*H <= 65535.
  */
@@ -97,6 +98,10 @@ typedef struct {
      * not); other shapes return TLA_ERR_UNSUPPORTED.                        */
     const int *cu_seqlens;
     int n_docs;
+    /* 1: one scalar log forget gate per head and token, shared by all E slices
+     * (the per-head gate variant): g is [B,T,H] and the backward's dg is
+     * [B,T,H].  0: g and dg are [B,T,H,E].                                   */
+    int gate_per_head;
 } tla_problem;
 
 /*
@@ -152,7 +157,7 @@ size_t tla_bwd_workspace_bytes(const tla_problem *p);
  *   dht     [B,H,E,dk,dv] fp32 gradient of ht, or NULL (=> 0).
  *   dq, dk  [B,T,H,dk];  dv [B,T,H,dv];  dq2, dk2 [B,T,H,E]: all out_dtype.
  *   dbeta   [B,T,H] fp32; required iff p->beta != NULL, else must be NULL.
- *   dg      [B,T,H,E] fp32 gradient of the log-gates.
+ *   dg      [B,T,H,E] fp32 gradient of the log-gates ([B,T,H] with gate_per_head).
  *   dh0     [B,H,E,dk,dv] fp32; required iff p->h0 != NULL, else must be NULL.
  */
 tla_status tla_chunk_bwd(const tla_problem *p, const void *fwd_ws, size_t fwd_ws_bytes,
@@ -167,7 +172,8 @@ tla_status tla_chunk_bwd(const tla_problem *p, const void *fwd_ws, size_t fwd_ws
  *   q, k [B,H,dk] dtype; v [B,H,dv] dtype; q2, k2 [B,H,E] dtype;
  *   g [B,H,E] fp32; beta [B,H] fp32 or NULL (=> 1; required if use_delta);
  *   state [B,H,E,dk,dv] fp32, updated in place; o [B,H,dv] dtype (written).
- * Supported: dk, dv multiples of 16 up to 128, 1 <= E <= 16, B*H <= 65535.
+ * Supported: dk, dv multiples of 16 up to 128, 1 <= E <= 32 with E*dk <= 2048,
+ * B*H <= 65535.  A per-head gate is passed as E equal values of g.
  * No workspace.
  */
 tla_status tla_decode_step(int B, int H, int dk, int dv, int E, int use_delta, int dtype,

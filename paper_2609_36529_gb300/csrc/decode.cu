@@ -38,7 +38,7 @@ decode_step_kernel(const Tin* __restrict__ q, const Tin* __restrict__ k,
     const int rows = E * dk;
     const int passes = (rows + RPP - 1) / RPP;
 
-    __shared__ float qs[128], ks[128], q2s[16], k2s[16], al[16];
+    __shared__ float qs[128], ks[128], q2s[32], k2s[32], al[32];
     __shared__ float4 red_r[NW][TPR], red_p[NW][TPR];
     __shared__ __align__(16) float us[TV];
     __shared__ float qk_s, q2k2_s;

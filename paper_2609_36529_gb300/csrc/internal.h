@@ -44,6 +44,7 @@ struct BwdPlan {
     size_t dU;           // fp32 [B,T,H,dv], or token tiles (FwdPlan::ck_tiles)
     size_t dRes;         // fp32 [B,T,H,dv] dRes, or token tiles of -dRes (delta rule)
     size_t dS;           // fp32 [B,H,NT,E,dk,dv] gradient of the state at each chunk's end
+    size_t dgE;          // per-head gate: fp32 [B,T,H,E] per-slice gate gradient before the sum
     size_t bytes;
 };
 
@@ -99,6 +100,9 @@ cudaError_t launch_bwd_chunk_grads(const tla_problem& p, const FwdPlan& fp, cons
                                    const BwdPlan& bp, const char* bws, const void* dO,
                                    void* dq, void* dk, void* dq2, void* dk2, float* dbeta,
                                    float* dg, cudaStream_t s);
+
+// dst[i] = sum_e src[i * E + e] (gradient of a per-head gate).
+cudaError_t launch_sum_slices(const float* src, float* dst, long long n, int E, cudaStream_t s);
 
 // Decode step.
 cudaError_t launch_decode_step(int B, int H, int dk, int dv, int E, int use_delta, int dtype,

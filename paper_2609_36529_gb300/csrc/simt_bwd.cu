@@ -257,7 +257,7 @@ bwd_chunk_grads_kernel(const Tin* __restrict__ q, const Tin* __restrict__ k,
     float* bs = dGa + kChunk * E;        // [64]
     float* dba = bs + kChunk;            // dbeta accumulator [64]
     float* dgc = dba + kChunk;           // [E] d gamma^C (Frobenius products)
-    float* red = dgc + 16;               // [256]
+    float* red = dgc + 32;               // [256]
 
     for (int i = tid; i < kChunk * E; i += blockDim.x) {
         int r = i / E, e = i % E;
@@ -271,7 +271,7 @@ bwd_chunk_grads_kernel(const Tin* __restrict__ q, const Tin* __restrict__ k,
         bs[r] = r < n ? (beta ? beta[(size_t(b) * T + t0 + r) * H + h] : 1.f) : 0.f;
         dba[r] = 0.f;
     }
-    if (tid < 16) dgc[tid] = 0.f;
+    if (tid < 32) dgc[tid] = 0.f;
     const size_t mat = ((size_t(b) * H + h) * NT + c) * (kChunk * kChunk);
     if (use_delta)
         for (int i = tid; i < kChunk * kChunk; i += blockDim.x) B0[(i >> 6) * MP + (i & 63)] = Nmat[mat + i];
@@ -576,9 +576,28 @@ bwd_chunk_grads_kernel(const Tin* __restrict__ q, const Tin* __restrict__ k,
     if (dbeta && tid < n) dbeta[(size_t(b) * T + t0 + tid) * H + h] = dba[tid];
 }
 
+// Gradient of a per-head gate: the sum over the slices of the per-slice gradient (fixed order).
+__global__ void sum_slices_kernel(const float* __restrict__ src, float* __restrict__ dst,
+                                  long long n, int E) {
+    const long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x;
+    if (i >= n) return;
+    float acc = 0.f;
+    for (int e = 0; e < E; ++e) acc += src[i * E + e];
+    dst[i] = acc;
+}
+
+cudaError_t launch_sum_slices(const float* src, float* dst, long long n, int E, cudaStream_t s) {
+    if (n == 0) return cudaSuccess;
+    const int threads = 256;
+    prof_before("sum_slices", s);
+    sum_slices_kernel<<<unsigned((n + threads - 1) / threads), threads, 0, s>>>(src, dst, n, E);
+    prof_after(s);
+    return cudaGetLastError();
+}
+
 static size_t grads_smem(const tla_problem& p) {
     return sizeof(float) * (6 * kChunk * 65 + 4 * kChunk * 33 + 2 * 32 * 33 + 9 * kChunk * p.E +
-                            2 * kChunk + 16 + 256);
+                            2 * kChunk + 32 + 256);
 }
 
 cudaError_t launch_bwd_chunk_grads(const tla_problem& p, const FwdPlan& fp, const char* fws,

@@ -21,7 +21,7 @@ namespace tla {
 // ---------------------------------------------------------------------------
 __global__ void gate_cumsum_kernel(const float* __restrict__ g, float* __restrict__ G,
                                    const int2* __restrict__ ctab, int B, int T, int H, int E,
-                                   int NT) {
+                                   int NT, int per_head) {
     long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x;
     long long total = (long long)B * NT * H * E;
     if (idx >= total) return;
@@ -41,7 +41,7 @@ __global__ void gate_cumsum_kernel(const float* __restrict__ g, float* __restric
     float acc = 0.f;
     for (int r = 0; r < n; ++r) {
         size_t off = tok_idx(b, t0 + r, h, e, T, H, E);
-        acc += g[off];
+        acc += per_head ? g[(size_t(b) * T + t0 + r) * H + h] : g[off];   // per-head gate: every slice
         G[off] = acc;
     }
 }
@@ -55,7 +55,8 @@ cudaError_t launch_gate_cumsum(const tla_problem& p, const FwdPlan& fp, const ch
     long long blocks = (total + threads - 1) / threads;
     const int2* ctab = p.cu_seqlens ? (const int2*)(ws + fp.ctab) : nullptr;
     prof_before("gate_cumsum", s);
-    gate_cumsum_kernel<<<(unsigned)blocks, threads, 0, s>>>(p.g, G, ctab, p.B, p.T, p.H, p.E, NT);
+    gate_cumsum_kernel<<<(unsigned)blocks, threads, 0, s>>>(p.g, G, ctab, p.B, p.T, p.H, p.E, NT,
+                                                            p.gate_per_head);
     prof_after(s);
     return cudaGetLastError();
 }

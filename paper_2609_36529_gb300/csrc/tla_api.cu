@@ -29,7 +29,9 @@ static tla_status validate(const tla_problem* p) {
     if (!p->q || !p->k || !p->v || !p->q2 || !p->k2 || !p->g || !p->o) return TLA_ERR_INVALID_ARG;
     if (p->use_delta && !p->beta) return TLA_ERR_INVALID_ARG;
     if (p->chunk != kChunk) return TLA_ERR_UNSUPPORTED;
-    if (!dims_ok(p->dk) || !dims_ok(p->dv) || p->E > 16) return TLA_ERR_UNSUPPORTED;
+    if (!dims_ok(p->dk) || !dims_ok(p->dv) || p->E > 32) return TLA_ERR_UNSUPPORTED;
+    if (p->E > 16 && p->dk > 64) return TLA_ERR_UNSUPPORTED;   // shared-memory state slab
+    if (p->gate_per_head != 0 && p->gate_per_head != 1) return TLA_ERR_INVALID_ARG;
     if (p->H > 65535 || p->B > 65535) return TLA_ERR_UNSUPPORTED;
     const void* ptrs[] = {p->q, p->k, p->v, p->q2, p->k2, p->g, p->beta, p->h0, p->o, p->ht};
     for (const void* x : ptrs)
@@ -117,6 +119,7 @@ BwdPlan plan_bwd(const tla_problem& p) {
     b.dU = off; off = align256(off + tokV);
     b.dRes = off; off = align256(off + tokV);
     b.dS = off; off = align256(off + states);
+    if (p.gate_per_head) { b.dgE = off; off = align256(off + (size_t)p.B * p.T * p.H * p.E * 4); }
     b.bytes = off;
     return b;
 }
@@ -243,16 +246,19 @@ tla_status tla_chunk_bwd(const tla_problem* p, const void* fwd_ws, size_t fwd_ws
     cudaStream_t s = (cudaStream_t)stream;
     const char* fws = (const char*)fwd_ws;
     char* bws = (char*)workspace;
+    float* dgs = p->gate_per_head ? (float*)(bws + bp.dgE) : dg;   // per-slice gate gradient
     cudaError_t e = fp.tcb ? launch_bwd_recurrence_tc(*p, fp, fws, bp, bws, dO, dht, dv, dh0,
                                                       device_error_word(), s)
                            : launch_bwd_recurrence(*p, fp, fws, bp, bws, dO, dht, dv, dh0, s);
     if (e == cudaSuccess) {
         if (tc_grads_ok(*p, fp))
-            e = launch_bwd_chunk_grads_tc(*p, fp, fws, bp, bws, dO, dq, dk, dq2, dk2, dbeta, dg,
+            e = launch_bwd_chunk_grads_tc(*p, fp, fws, bp, bws, dO, dq, dk, dq2, dk2, dbeta, dgs,
                                           device_error_word(), s);
         else
-            e = launch_bwd_chunk_grads(*p, fp, fws, bp, bws, dO, dq, dk, dq2, dk2, dbeta, dg, s);
+            e = launch_bwd_chunk_grads(*p, fp, fws, bp, bws, dO, dq, dk, dq2, dk2, dbeta, dgs, s);
     }
+    if (e == cudaSuccess && p->gate_per_head)
+        e = launch_sum_slices(dgs, dg, (long long)p->B * p->T * p->H, p->E, s);
     return cuda_status(e);
 }
 
@@ -270,7 +276,7 @@ tla_status tla_decode_step(int B, int H, int dk, int dv, int E, int use_delta, i
         for (const void* x : ptrs)
             if (!aligned16(x)) return TLA_ERR_INVALID_ARG;
     }
-    if (!dims_ok(dk) || !dims_ok(dv) || E > 16) return TLA_ERR_UNSUPPORTED;
+    if (!dims_ok(dk) || !dims_ok(dv) || E > 32 || E * dk > 2048) return TLA_ERR_UNSUPPORTED;
     if ((long long)B * H > 65535) return TLA_ERR_UNSUPPORTED;  // grid.y
     return cuda_status(launch_decode_step(B, H, dk, dv, E, use_delta, dtype, q, k, v, q2, k2, g,
                                           beta, state, o, (cudaStream_t)stream));

@@ -39,7 +39,7 @@ class tla_problem(ctypes.Structure):
                 ("q2", ctypes.c_void_p), ("k2", ctypes.c_void_p), ("g", ctypes.c_void_p),
                 ("beta", ctypes.c_void_p), ("h0", ctypes.c_void_p), ("o", ctypes.c_void_p),
                 ("ht", ctypes.c_void_p), ("cu_seqlens", ctypes.POINTER(ctypes.c_int)),
-                ("n_docs", ctypes.c_int)]
+                ("n_docs", ctypes.c_int), ("gate_per_head", ctypes.c_int)]
 
 
 _lib = None
@@ -107,11 +107,13 @@ def _n_states(q, cu_seqlens):
 
 def make_problem(q, k, v, q2, k2, g, beta=None, h0=None, o=None, ht=None, use_delta=True,
                  chunk=64, out_dtype=None, cu_seqlens=None):
-    """cu_seqlens: None, or the host token offsets of packed documents (B = 1)."""
+    """cu_seqlens: None, or the host token offsets of packed documents (B = 1).
+    A 3-d g ([B,T,H]) is one gate per head shared by all slices (gate_per_head)."""
     B, T, H, dk = q.shape
     p = tla_problem()
     p.B, p.T, p.H, p.dk, p.dv, p.E = B, T, H, dk, v.shape[-1], q2.shape[-1]
     p.chunk, p.dtype, p.use_delta = chunk, _dtype_code(q), int(bool(use_delta))
+    p.gate_per_head = int(g.dim() == 3)
     if out_dtype is None:
         out_dtype = o.dtype if o is not None else torch.float32
     p.out_dtype = _dtype_code(torch.empty(0, dtype=out_dtype))

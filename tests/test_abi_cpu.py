@@ -52,7 +52,8 @@ def _problem(tla, **kw):
 def test_host_validation_rejects_before_launch(tla):
     L = tla.lib()
     cases = [
-        (dict(chunk=32), -2), (dict(dk=20), -2), (dict(dv=256), -2), (dict(E=17), -2),
+        (dict(chunk=32), -2), (dict(dk=20), -2), (dict(dv=256), -2), (dict(E=33), -2),
+        (dict(E=17, dk=128), -2), (dict(gate_per_head=2), -1),
         (dict(E=0), -1), (dict(T=0), -1), (dict(dtype=7), -1), (dict(use_delta=2), -1),
         (dict(out_dtype=3), -1),
         (dict(q=None), -1), (dict(beta=None), -1), (dict(o=None), -1),
@@ -90,6 +91,8 @@ def test_host_validation_bwd_and_decode(tla):
     assert L.tla_decode_step(2, 2, 64, 64, 4, 1, 0, f, f, f, f, f, f, f, ctypes.c_void_p(0x1004),
                              f, None) == -1
     assert L.tla_decode_step(2, 2, 64, 200, 4, 1, 0, f, f, f, f, f, f, f, f, f, None) == -2
+    assert L.tla_decode_step(2, 2, 64, 64, 33, 1, 0, f, f, f, f, f, f, f, f, f, None) == -2
+    assert L.tla_decode_step(2, 2, 128, 64, 32, 1, 0, f, f, f, f, f, f, f, f, f, None) == -2
     assert L.tla_decode_step(2, 2, 64, 64, 4, 1, 0, f, f, f, f, f, f, None, f, f, None) == -1
 
 
