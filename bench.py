@@ -8,7 +8,8 @@ inputs.  The single-token decode step is measured in the same run on the
 decode workload (fp32 state [256,32,8,128,128], 100 steps each of sGLA and
 GDN after a 512-token chunked prefill) and reported under "decode", and the
 same step with the headline's tokens packed into documents of log-normal length
-around 1000 tokens (cu_seqlens, each document from its own state) under "packed".
+around 1000 tokens (cu_seqlens, each document from its own state) under "packed";
+the per-head-gate and E = 32 / d_k = 64 variants under "variants".
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
@@ -324,6 +325,10 @@ def run_ours(args):
     if not args.no_packed:
         packed = run_packed(args, tla, inputs, w, dev, stream, barrier, max_over_ranks, ws_n, rank)
         packed["vs_uniform_batch"] = round(packed["value"] / value, 4)
+    variants = None
+    if not args.no_variants:
+        variants = run_variants(args, tla, inputs, w, dev, stream, barrier, max_over_ranks, ws_n,
+                                rank, value)
     decode = None
     if not args.no_decode:
         del fws, bws
@@ -353,7 +358,7 @@ def run_ours(args):
             "tflops_frac": round(total_flops / (ms_step / 1e3) / 1e12 / peak, 5),
             "roofline": roofline, "kernels": kernels, "gpu_launches": gpu_launches,
             "clocks": ck, "clocks_remeasured": remeasured,
-            "e2e": e2e, "packed": packed, "decode": decode, "cpu_baseline": cpu, "impl": "ours",
+            "e2e": e2e, "packed": packed, "variants": variants, "decode": decode, "cpu_baseline": cpu, "impl": "ours",
         }
         print(json.dumps(line), flush=True)
     if ws_n > 1:
@@ -476,6 +481,65 @@ def run_packed(args, tla, inputs, w, dev, stream, barrier, max_over_ranks, ws_n,
             "doc_len": {"mean": round(total / len(lens), 1), "min": min(lens), "max": max(lens)},
             "chunks": nc, "chunks_uniform_batch": total // 64,
             "data": "synthetic; lengths log-normal around 1000 tokens (sigma 1), seeded"}
+
+
+def _time_steps(step, k, warm, stream, barrier, max_over_ranks):
+    for _ in range(warm):
+        step()
+    torch.cuda.synchronize()
+    barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(k):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    return max_over_ranks(e0.elapsed_time(e1) / k)
+
+
+def run_variants(args, tla, inputs, w, dev, stream, barrier, max_over_ranks, ws_n, rank,
+                 headline):
+    """Forward + backward tokens/s of the shape/gate variants: one log gate per head on the
+    headline workload (tensor-core path), and E = 32 slices with d_k = 64 (Table 4's
+    iso-state variant; CUDA-core path) on one 8192-token sequence."""
+    out = {}
+    cases = [("gate_per_head", w.B, w.T, w.H, w.dk, w.dv, w.E, True),
+             ("E32_dk64", 1, w.T, w.H, 64, w.dv, 32, False)]
+    for name, B, T, H, dk, dv, E, per_head in cases:
+        x = inputs.chunk_inputs(B, T, H, dk, dv, E, dtype=w.dtype, with_beta=True,
+                                backward=True, device=dev, seed=200 + rank)
+        if per_head:
+            x["g"] = x["g"][..., 0].contiguous()
+        o = torch.empty(B, T, H, dv, dtype=torch.float32, device=dev)
+        p = tla.make_problem(x["q"], x["k"], x["v"], x["q2"], x["k2"], x["g"], x["beta"], None,
+                             o, None, use_delta=True)
+        fws = torch.empty(tla.fwd_workspace_bytes(p, True), dtype=torch.uint8, device=dev)
+        bws = torch.empty(tla.bwd_workspace_bytes(p), dtype=torch.uint8, device=dev)
+        f32 = dict(dtype=torch.float32, device=dev)
+        grads = {n: torch.empty(x[k].shape, **f32) for n, k in
+                 (("dq", "q"), ("dk", "k"), ("dv", "v"), ("dq2", "q2"), ("dk2", "k2"),
+                  ("dg", "g"), ("dbeta", "beta"))}
+
+        def step():
+            tla.tla_chunk_fwd(x["q"], x["k"], x["v"], x["q2"], x["k2"], x["g"], x["beta"], None,
+                              use_delta=True, save_for_bwd=True, want_ht=False, o=o,
+                              workspace=fws)
+            tla.tla_chunk_bwd(x["q"], x["k"], x["v"], x["q2"], x["k2"], x["g"], x["dO"], fws,
+                              beta=x["beta"], use_delta=True, workspace=bws, grads=grads)
+
+        ms = _time_steps(step, 3, 3, stream, barrier, max_over_ranks)
+        val = ws_n * B * T / (ms / 1e3)
+        out[name] = {"config": {"B": B, "T": T, "H": H, "dk": dk, "dv": dv, "E": E,
+                                "gate": "per head [B,T,H]" if per_head else "per slice"},
+                     "value": round(val, 1), "unit": "tokens/s", "ms_per_step": round(ms, 4),
+                     "path": "tensor cores" if dk == 128 else "CUDA cores (fp32 SIMT)"}
+        if per_head:
+            out[name]["vs_headline"] = round(val / headline, 4)
+        del x, fws, bws, grads, o
+    if tla.tla_last_device_status() != 0:
+        raise RuntimeError("device status not OK after the variant loops")
+    return out
 
 
 def run_decode(args, tla, inputs, dev, stream, lib, peaks, barrier, max_over_ranks, ws_n):
@@ -610,6 +674,7 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-decode", action="store_true")
     ap.add_argument("--no-packed", action="store_true")
+    ap.add_argument("--no-variants", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--ref-tokens", type=int, default=1024,
