@@ -34,6 +34,11 @@ def _load():
         lib.tla_oracle_chunk_forward.argtypes = [i] * 8 + [_dp] * 10
         lib.tla_oracle_backward.argtypes = [i] * 7 + [_dp] * 18
         lib.tla_oracle_decode_step.argtypes = [i] * 6 + [_dp] * 9
+        d = ctypes.c_double
+        lib.tla_oracle_prologue.argtypes = [i] * 7 + [d] + [_dp] * 13
+        lib.tla_oracle_prologue_backward.argtypes = [i] * 7 + [d] + [_dp] * 19
+        lib.tla_oracle_gate_norm.argtypes = [i] * 4 + [d] + [_dp] * 4
+        lib.tla_oracle_gate_norm_backward.argtypes = [i] * 4 + [d] + [_dp] * 7
         lib.tla_oracle_num_threads.restype = ctypes.c_int
         lib.tla_oracle_set_threads.argtypes = [i]
         _lib = lib
@@ -119,3 +124,64 @@ def decode_step(state, q, k, v, q2, k2, g, beta=None, use_delta=True):
     _load().tla_oracle_decode_step(B, H, dk, dv, E, int(bool(use_delta)), _p(q), _p(k), _p(v),
                                    _p(q2), _p(k2), _p(g), _p(beta), _p(st), _p(o))
     return o, st
+
+
+def prologue(P, conv_w, gate_in, gate_bias, A_log, beta_in, dk, dv, E, eps=1e-6):
+    """Layer input path of Algorithm 4: causal depthwise convolution of the projection
+    output P [B,T,H,2dk+dv+2E] (per head [q|k|v|q'|k']) with conv_w [H,C,K], SiLU on
+    q,k,v, softplus on q',k', L2 normalisation of q,k,q',k'; log gates
+    -exp(A_log) softplus(gate_in + gate_bias) and beta = sigmoid(beta_in).
+    Returns dict q, k, v, q2, k2, g, beta (beta None without beta_in)."""
+    P, conv_w, gate_in, gate_bias, A_log, beta_in = map(
+        _f64, (P, conv_w, gate_in, gate_bias, A_log, beta_in))
+    B, T, H, C = P.shape
+    K = conv_w.shape[-1]
+    out = {"q": np.zeros((B, T, H, dk)), "k": np.zeros((B, T, H, dk)),
+           "v": np.zeros((B, T, H, dv)), "q2": np.zeros((B, T, H, E)),
+           "k2": np.zeros((B, T, H, E)), "g": np.zeros((B, T, H, E)),
+           "beta": np.zeros((B, T, H)) if beta_in is not None else None}
+    _load().tla_oracle_prologue(B, T, H, dk, dv, E, K, float(eps), _p(P), _p(conv_w),
+                                _p(gate_in), _p(gate_bias), _p(A_log), _p(beta_in),
+                                _p(out["q"]), _p(out["k"]), _p(out["v"]), _p(out["q2"]),
+                                _p(out["k2"]), _p(out["g"]), _p(out["beta"]))
+    return out
+
+
+def prologue_backward(P, conv_w, gate_in, gate_bias, A_log, beta_in, grads, dk, dv, E,
+                      eps=1e-6):
+    """Gradients of prologue(): grads holds dq, dk, dv, dq2, dk2, dg (and dbeta).
+    Returns dict dP, dconv_w, dgate_in, dgate_bias, dA_log (and dbeta_in)."""
+    P, conv_w, gate_in, gate_bias, A_log, beta_in = map(
+        _f64, (P, conv_w, gate_in, gate_bias, A_log, beta_in))
+    gr = {n: _f64(grads.get(n)) for n in ("dq", "dk", "dv", "dq2", "dk2", "dg", "dbeta")}
+    B, T, H, C = P.shape
+    K = conv_w.shape[-1]
+    out = {"dP": np.zeros_like(P), "dconv_w": np.zeros_like(conv_w),
+           "dgate_in": np.zeros_like(gate_in), "dgate_bias": np.zeros_like(gate_bias),
+           "dA_log": np.zeros_like(A_log),
+           "dbeta_in": np.zeros_like(beta_in) if beta_in is not None else None}
+    _load().tla_oracle_prologue_backward(
+        B, T, H, dk, dv, E, K, float(eps), _p(P), _p(conv_w), _p(gate_in), _p(gate_bias),
+        _p(A_log), _p(beta_in), _p(gr["dq"]), _p(gr["dk"]), _p(gr["dv"]), _p(gr["dq2"]),
+        _p(gr["dk2"]), _p(gr["dg"]), _p(gr["dbeta"]), _p(out["dP"]), _p(out["dconv_w"]),
+        _p(out["dgate_in"]), _p(out["dgate_bias"]), _p(out["dA_log"]), _p(out["dbeta_in"]))
+    return {n: a for n, a in out.items() if a is not None}
+
+
+def gate_norm(o, z, w_norm, eps=1e-6):
+    """Output gate of Algorithm 4: RMSNorm(o) (weight w_norm [dv]) times sigmoid(z)."""
+    o, z, w_norm = map(_f64, (o, z, w_norm))
+    B, T, H, dv = o.shape
+    y = np.zeros_like(o)
+    _load().tla_oracle_gate_norm(B, T, H, dv, float(eps), _p(o), _p(z), _p(w_norm), _p(y))
+    return y
+
+
+def gate_norm_backward(o, z, w_norm, dy, eps=1e-6):
+    """Gradients of gate_norm(): returns dict do, dz, dw_norm."""
+    o, z, w_norm, dy = map(_f64, (o, z, w_norm, dy))
+    B, T, H, dv = o.shape
+    out = {"do": np.zeros_like(o), "dz": np.zeros_like(o), "dw_norm": np.zeros_like(w_norm)}
+    _load().tla_oracle_gate_norm_backward(B, T, H, dv, float(eps), _p(o), _p(z), _p(w_norm),
+                                          _p(dy), _p(out["do"]), _p(out["dz"]), _p(out["dw_norm"]))
+    return out

@@ -25,6 +25,8 @@
  *   chunk forward      pinned (agrees with the token recurrence, including
  *                      extreme within-chunk decay)
  *   decode step        pinned (one token of the pinned token recurrence)
+ *   layer prologue     pinned (torch F.conv1d / F.silu / F.softplus restatement,
+ *   and output gate     its autograd for the backward, causality, unit norms)
  */
 #include <math.h>
 #include <stdint.h>
@@ -498,4 +500,228 @@ void tla_oracle_chunk_forward(int B, int T, int H, int dk, int dv, int E, int us
         if (ht) memcpy(ht + (size_t)bh * ssz, S, ssz * sizeof(double));
         free(S); free(G); free(R); free(Rq); free(L); free(Tm); free(Res); free(U); free(bt);
     }
+}
+
+/* ------------------------------------------------------------------------
+ * Layer input path and output gate of Algorithm 4 (and the input-projection
+ * paragraph of Appendix A): what surrounds the operator in a triadic layer.
+ *
+ * Input prologue, per (b, t, h), with C = 2 dk + dv + 2 E channels per head in
+ * the order [q | k | v | q' | k'] of the projection output P [B,T,H,C]:
+ *   a_c(t) = sum_{j<K} w[h,c,j] P_c(t - K + 1 + j)      causal depthwise conv
+ *            (P before the first token is zero)
+ *   q = n(silu(a_q)), k = n(silu(a_k)), v = silu(a_v),
+ *   q' = n(softplus(a_q')), k' = n(softplus(a_k')),
+ *   n(x) = x / sqrt(sum x^2 + eps)                       (L2 normalisation)
+ *   g_e = log alpha_e = -exp(A_log[h,e]) softplus(gate_in_e + gate_bias[h,e])
+ *   beta = sigmoid(beta_in)
+ * Output gate, per (b, t, h) over the dv channels:
+ *   y = o / sqrt(mean(o^2) + eps) * w_norm * sigmoid(z)
+ * The backward functions are the hand-derived chains of these definitions.
+ * ---------------------------------------------------------------------- */
+static double o_sigmoid(double x) { return 1.0 / (1.0 + exp(-x)); }
+static double o_softplus(double x) { return x > 30.0 ? x : log1p(exp(x)); }
+
+/* Pre-activation a[C] of one token of one head (causal depthwise convolution). */
+static void conv_token(const double *P, const double *w, int T, int H, int C, int K,
+                       int b, int t, int h, double *a) {
+    for (int c = 0; c < C; ++c) {
+        double acc = 0.0;
+        for (int j = 0; j < K; ++j) {
+            const int ts = t - K + 1 + j;
+            if (ts >= 0) acc += w[((size_t)h * C + c) * K + j] * P[IDX_TOK(b, ts, h, c, T, H, C)];
+        }
+        a[c] = acc;
+    }
+}
+
+void tla_oracle_prologue(int B, int T, int H, int dk, int dv, int E, int K, double eps,
+                         const double *P, const double *w, const double *gate_in,
+                         const double *gate_bias, const double *A_log, const double *beta_in,
+                         double *q, double *k, double *v, double *q2, double *k2, double *g,
+                         double *beta) {
+    const int C = 2 * dk + dv + 2 * E;
+#pragma omp parallel for collapse(2) schedule(static)
+    for (int b = 0; b < B; ++b)
+        for (int t = 0; t < T; ++t) {
+            double *a = (double *)malloc(sizeof(double) * C);
+            for (int h = 0; h < H; ++h) {
+                conv_token(P, w, T, H, C, K, b, t, h, a);
+                /* groups: offset, width, activation (0 silu, 1 softplus), normalised, output */
+                const int off[5] = {0, dk, 2 * dk, 2 * dk + dv, 2 * dk + dv + E};
+                const int wid[5] = {dk, dk, dv, E, E};
+                const int act[5] = {0, 0, 0, 1, 1};
+                const int nrm[5] = {1, 1, 0, 1, 1};
+                double *dst[5] = {q, k, v, q2, k2};
+                for (int gi = 0; gi < 5; ++gi) {
+                    double ss = 0.0;
+                    for (int i = 0; i < wid[gi]; ++i) {
+                        const double x = a[off[gi] + i];
+                        const double y = act[gi] ? o_softplus(x) : x * o_sigmoid(x);
+                        a[off[gi] + i] = y;
+                        ss += y * y;
+                    }
+                    const double scale = nrm[gi] ? 1.0 / sqrt(ss + eps) : 1.0;
+                    for (int i = 0; i < wid[gi]; ++i)
+                        dst[gi][IDX_TOK(b, t, h, i, T, H, wid[gi])] = a[off[gi] + i] * scale;
+                }
+                for (int e = 0; e < E; ++e) {
+                    const size_t i = IDX_TOK(b, t, h, e, T, H, E);
+                    g[i] = -exp(A_log[h * E + e]) * o_softplus(gate_in[i] + gate_bias[h * E + e]);
+                }
+                if (beta_in) {
+                    const size_t i = ((size_t)b * T + t) * H + h;
+                    beta[i] = o_sigmoid(beta_in[i]);
+                }
+            }
+            free(a);
+        }
+}
+
+void tla_oracle_prologue_backward(int B, int T, int H, int dk, int dv, int E, int K, double eps,
+                                  const double *P, const double *w, const double *gate_in,
+                                  const double *gate_bias, const double *A_log,
+                                  const double *beta_in, const double *dq, const double *dk_,
+                                  const double *dv_, const double *dq2, const double *dk2,
+                                  const double *dg, const double *dbeta, double *dP, double *dw,
+                                  double *dgate_in, double *dgate_bias, double *dA_log,
+                                  double *dbeta_in) {
+    const int C = 2 * dk + dv + 2 * E;
+    double *da = (double *)calloc((size_t)B * T * H * C, sizeof(double));
+#pragma omp parallel for collapse(2) schedule(static)
+    for (int b = 0; b < B; ++b)
+        for (int t = 0; t < T; ++t) {
+            double *a = (double *)malloc(sizeof(double) * C);
+            double *y = (double *)malloc(sizeof(double) * C);
+            for (int h = 0; h < H; ++h) {
+                conv_token(P, w, T, H, C, K, b, t, h, a);
+                const int off[5] = {0, dk, 2 * dk, 2 * dk + dv, 2 * dk + dv + E};
+                const int wid[5] = {dk, dk, dv, E, E};
+                const int act[5] = {0, 0, 0, 1, 1};
+                const int nrm[5] = {1, 1, 0, 1, 1};
+                const double *gy[5] = {dq, dk_, dv_, dq2, dk2};
+                for (int gi = 0; gi < 5; ++gi) {
+                    double ss = 0.0;
+                    for (int i = 0; i < wid[gi]; ++i) {
+                        const double x = a[off[gi] + i];
+                        y[off[gi] + i] = act[gi] ? o_softplus(x) : x * o_sigmoid(x);
+                        ss += y[off[gi] + i] * y[off[gi] + i];
+                    }
+                    const double n = nrm[gi] ? sqrt(ss + eps) : 1.0;
+                    /* d(x/n)/dx: (dy - u (u.dy)) / n with u = x/n; identity without the norm */
+                    double udy = 0.0;
+                    for (int i = 0; i < wid[gi]; ++i)
+                        udy += (y[off[gi] + i] / n) * gy[gi][IDX_TOK(b, t, h, i, T, H, wid[gi])];
+                    for (int i = 0; i < wid[gi]; ++i) {
+                        const double u = y[off[gi] + i] / n;
+                        const double dyi = gy[gi][IDX_TOK(b, t, h, i, T, H, wid[gi])];
+                        const double dx = nrm[gi] ? (dyi - u * udy) / n : dyi;
+                        const double x = a[off[gi] + i], s = o_sigmoid(x);
+                        const double dact = act[gi] ? s : s * (1.0 + x * (1.0 - s));
+                        da[IDX_TOK(b, t, h, off[gi] + i, T, H, C)] = dx * dact;
+                    }
+                }
+                for (int e = 0; e < E; ++e) {
+                    const size_t i = IDX_TOK(b, t, h, e, T, H, E);
+                    const double z = gate_in[i] + gate_bias[h * E + e];
+                    dgate_in[i] = dg[i] * (-exp(A_log[h * E + e])) * o_sigmoid(z);
+                }
+                if (beta_in) {
+                    const size_t i = ((size_t)b * T + t) * H + h;
+                    const double s = o_sigmoid(beta_in[i]);
+                    dbeta_in[i] = dbeta[i] * s * (1.0 - s);
+                }
+            }
+            free(a);
+            free(y);
+        }
+    /* transposed convolution and the weight correlation */
+#pragma omp parallel for collapse(2) schedule(static)
+    for (int b = 0; b < B; ++b)
+        for (int t = 0; t < T; ++t)
+            for (int h = 0; h < H; ++h)
+                for (int c = 0; c < C; ++c) {
+                    double acc = 0.0;
+                    for (int j = 0; j < K; ++j) {
+                        const int td = t + K - 1 - j;
+                        if (td < T) acc += w[((size_t)h * C + c) * K + j] * da[IDX_TOK(b, td, h, c, T, H, C)];
+                    }
+                    dP[IDX_TOK(b, t, h, c, T, H, C)] = acc;
+                }
+#pragma omp parallel for collapse(2) schedule(static)
+    for (int h = 0; h < H; ++h)
+        for (int c = 0; c < C; ++c)
+            for (int j = 0; j < K; ++j) {
+                double acc = 0.0;
+                for (int b = 0; b < B; ++b)
+                    for (int t = 0; t < T; ++t) {
+                        const int ts = t - K + 1 + j;
+                        if (ts >= 0) acc += da[IDX_TOK(b, t, h, c, T, H, C)] * P[IDX_TOK(b, ts, h, c, T, H, C)];
+                    }
+                dw[((size_t)h * C + c) * K + j] = acc;
+            }
+    for (int h = 0; h < H; ++h)
+        for (int e = 0; e < E; ++e) {
+            double sb = 0.0, sa = 0.0;
+            for (int b = 0; b < B; ++b)
+                for (int t = 0; t < T; ++t) {
+                    const size_t i = IDX_TOK(b, t, h, e, T, H, E);
+                    const double z = gate_in[i] + gate_bias[h * E + e];
+                    sb += dgate_in[i];
+                    sa += dg[i] * (-exp(A_log[h * E + e]) * o_softplus(z));   /* dg * g */
+                }
+            dgate_bias[h * E + e] = sb;
+            dA_log[h * E + e] = sa;
+        }
+    free(da);
+}
+
+void tla_oracle_gate_norm(int B, int T, int H, int dv, double eps, const double *o,
+                          const double *z, const double *wn, double *y) {
+#pragma omp parallel for collapse(2) schedule(static)
+    for (int b = 0; b < B; ++b)
+        for (int t = 0; t < T; ++t)
+            for (int h = 0; h < H; ++h) {
+                double ss = 0.0;
+                for (int i = 0; i < dv; ++i) {
+                    const double x = o[IDX_TOK(b, t, h, i, T, H, dv)];
+                    ss += x * x;
+                }
+                const double r = 1.0 / sqrt(ss / dv + eps);
+                for (int i = 0; i < dv; ++i) {
+                    const size_t j = IDX_TOK(b, t, h, i, T, H, dv);
+                    y[j] = o[j] * r * wn[i] * o_sigmoid(z[j]);
+                }
+            }
+}
+
+void tla_oracle_gate_norm_backward(int B, int T, int H, int dv, double eps, const double *o,
+                                   const double *z, const double *wn, const double *dy,
+                                   double *d_o, double *dz, double *dwn) {
+    memset(dwn, 0, sizeof(double) * dv);
+    for (int b = 0; b < B; ++b)
+        for (int t = 0; t < T; ++t)
+            for (int h = 0; h < H; ++h) {
+                double ss = 0.0;
+                for (int i = 0; i < dv; ++i) {
+                    const double x = o[IDX_TOK(b, t, h, i, T, H, dv)];
+                    ss += x * x;
+                }
+                const double r = 1.0 / sqrt(ss / dv + eps);
+                double dot = 0.0;   /* sum_i dnh_i nh_i */
+                for (int i = 0; i < dv; ++i) {
+                    const size_t j = IDX_TOK(b, t, h, i, T, H, dv);
+                    const double nh = o[j] * r, s = o_sigmoid(z[j]);
+                    const double dnh = dy[j] * wn[i] * s;
+                    dz[j] = dy[j] * nh * wn[i] * s * (1.0 - s);
+                    dwn[i] += dy[j] * nh * s;
+                    dot += dnh * nh;
+                }
+                for (int i = 0; i < dv; ++i) {
+                    const size_t j = IDX_TOK(b, t, h, i, T, H, dv);
+                    const double nh = o[j] * r, s = o_sigmoid(z[j]);
+                    const double dnh = dy[j] * wn[i] * s;
+                    d_o[j] = r * (dnh - nh * dot / dv);
+                }
+            }
 }

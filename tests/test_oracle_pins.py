@@ -305,3 +305,89 @@ def test_backward_vs_autograd_flat(delta):
     for x, gname in names.items():
         np.testing.assert_allclose(gr[gname], t[x].grad.numpy(), rtol=1e-10, atol=1e-10,
                                    err_msg=x)
+
+
+# --- layer input path and output gate (Algorithm 4; Appendix A, Input projections)
+
+def _layer_inputs(seed, B=2, T=37, H=2, dk=8, dv=16, E=3, K=4):
+    rng = np.random.default_rng(seed)
+    C = 2 * dk + dv + 2 * E
+    return dict(P=rng.standard_normal((B, T, H, C)), conv_w=0.5 * rng.standard_normal((H, C, K)),
+                gate_in=rng.standard_normal((B, T, H, E)), gate_bias=rng.standard_normal((H, E)),
+                A_log=0.3 * rng.standard_normal((H, E)), beta_in=rng.standard_normal((B, T, H))), \
+        (dk, dv, E)
+
+
+def _torch_prologue(x, dk, dv, E, eps=1e-6):
+    """The same layer written with library routines: a grouped F.conv1d over a left-padded
+    sequence (causal depthwise convolution), F.silu / F.softplus, torch reductions."""
+    import torch.nn.functional as F
+    P, w = x["P"], x["conv_w"]
+    B, T, H, C = P.shape
+    K = w.shape[-1]
+    seq = P.permute(0, 2, 3, 1).reshape(B, H * C, T)
+    a = F.conv1d(F.pad(seq, (K - 1, 0)), w.reshape(H * C, 1, K), groups=H * C)
+    a = a.reshape(B, H, C, T).permute(0, 3, 1, 2)
+    parts = torch.split(a, [dk, dk, dv, E, E], dim=-1)
+
+    def unit(y):
+        return y / torch.sqrt((y * y).sum(-1, keepdim=True) + eps)
+
+    out = {"q": unit(F.silu(parts[0])), "k": unit(F.silu(parts[1])), "v": F.silu(parts[2]),
+           "q2": unit(F.softplus(parts[3])), "k2": unit(F.softplus(parts[4])),
+           "g": -torch.exp(x["A_log"]) * F.softplus(x["gate_in"] + x["gate_bias"]),
+           "beta": torch.sigmoid(x["beta_in"])}
+    return out
+
+
+def test_layer_prologue_matches_library_form():
+    x, (dk, dv, E) = _layer_inputs(1)
+    ref = _torch_prologue({n: torch.tensor(a) for n, a in x.items()}, dk, dv, E)
+    got = oracle.prologue(**x, dk=dk, dv=dv, E=E)
+    for n in ref:
+        np.testing.assert_allclose(got[n], ref[n].numpy(), rtol=0, atol=1e-12, err_msg=n)
+    for n in ("q", "k", "q2", "k2"):   # unit vectors up to eps
+        np.testing.assert_allclose(np.linalg.norm(got[n], axis=-1), 1.0, atol=1e-4)
+
+
+def test_layer_prologue_is_causal():
+    x, (dk, dv, E) = _layer_inputs(2)
+    base = oracle.prologue(**x, dk=dk, dv=dv, E=E)
+    y = dict(x)
+    y["P"] = x["P"].copy()
+    y["P"][:, 20:] += 3.0    # change every projection from token 20 on
+    moved = oracle.prologue(**y, dk=dk, dv=dv, E=E)
+    for n in ("q", "k", "v", "q2", "k2"):
+        np.testing.assert_array_equal(moved[n][:, :20], base[n][:, :20])
+        assert np.abs(moved[n][:, 20:] - base[n][:, 20:]).max() > 1e-3
+
+
+def test_layer_prologue_backward_matches_autograd():
+    x, (dk, dv, E) = _layer_inputs(3)
+    tx = {n: torch.tensor(a, requires_grad=True) for n, a in x.items()}
+    out = _torch_prologue(tx, dk, dv, E)
+    rng = np.random.default_rng(4)
+    cot = {n: rng.standard_normal(tuple(t.shape)) for n, t in out.items()}
+    sum((out[n] * torch.tensor(cot[n])).sum() for n in out).backward()
+    grads = {"d" + n: cot[n] for n in ("q", "k", "v", "q2", "k2", "g")}
+    grads["dbeta"] = cot["beta"]
+    got = oracle.prologue_backward(**x, grads=grads, dk=dk, dv=dv, E=E)
+    pairs = {"dP": "P", "dconv_w": "conv_w", "dgate_in": "gate_in", "dgate_bias": "gate_bias",
+             "dA_log": "A_log", "dbeta_in": "beta_in"}
+    for gname, xname in pairs.items():
+        np.testing.assert_allclose(got[gname], tx[xname].grad.numpy(), rtol=1e-9, atol=1e-10,
+                                   err_msg=gname)
+
+
+def test_output_gate_matches_library_form_and_autograd():
+    rng = np.random.default_rng(5)
+    o, z = rng.standard_normal((2, 9, 3, 32)), rng.standard_normal((2, 9, 3, 32))
+    w = 1.0 + 0.1 * rng.standard_normal(32)
+    to, tz, tw = (torch.tensor(a, requires_grad=True) for a in (o, z, w))
+    ref = torch.nn.functional.rms_norm(to, (32,), tw, eps=1e-6) * torch.sigmoid(tz)
+    np.testing.assert_allclose(oracle.gate_norm(o, z, w), ref.detach().numpy(), atol=1e-12)
+    dy = rng.standard_normal(o.shape)
+    (ref * torch.tensor(dy)).sum().backward()
+    got = oracle.gate_norm_backward(o, z, w, dy)
+    for gname, t in (("do", to), ("dz", tz), ("dw_norm", tw)):
+        np.testing.assert_allclose(got[gname], t.grad.numpy(), rtol=1e-9, atol=1e-10, err_msg=gname)
