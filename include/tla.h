@@ -185,6 +185,83 @@ tla_status tla_decode_step(int B, int H, int dk, int dv, int E, int use_delta, i
 const char *tla_status_string(int status);
 
 /*
+ * Layer input path of Algorithm 4 (Appendix A, Input projections): from the
+ * output P of the one projection GEMM to the operator's inputs.  The GEMMs
+ * themselves (W u for P, W_alpha u, W_beta u) are plain GEMMs of the caller.
+ * Per (b, t, h), with C = 2 dk + dv + 2 E channels per head ordered
+ * [q | k | v | q' | k']:
+ *   a_c(t) = sum_{j<K} conv_w[h,c,j] P_c(t - K + 1 + j)   (causal depthwise
+ *            convolution of width K; P before token 0 is zero)
+ *   q = n(silu(a_q)), k = n(silu(a_k)), v = silu(a_v),
+ *   q' = n(softplus(a_q')), k' = n(softplus(a_k')), n(x) = x / sqrt(|x|^2 + eps)
+ *   g = log alpha = -exp(A_log) softplus(gate_in + gate_bias),  beta = sigmoid(beta_in)
+ * All pointers 16-byte aligned; sizes as stated; outputs are written.
+ */
+typedef struct {
+    int B, T, H, dk, dv, E;
+    int K;               /* convolution width, 1..4                              */
+    int dtype;           /* tla_dtype of P and of q, k, v, q2, k2                */
+    float eps;           /* L2-normalisation epsilon                             */
+    const void *P;       /* [B,T,H,C] projection output                          */
+    const float *conv_w; /* [H,C,K]                                              */
+    const float *gate_in;   /* [B,T,H,E]  W_alpha u                              */
+    const float *gate_bias; /* [H,E]                                             */
+    const float *A_log;     /* [H,E]                                             */
+    const float *beta_in;   /* [B,T,H]  W_beta u, or NULL (then beta is NULL)    */
+    void *q, *k, *v, *q2, *k2;   /* [B,T,H,dk|dk|dv|E|E] dtype                  */
+    float *g;            /* [B,T,H,E]                                            */
+    float *beta;         /* [B,T,H], NULL iff beta_in is NULL                    */
+} tla_prologue_args;
+
+/* Forward of the input path.  Supported: dk, dv multiples of 16 up to 128,
+ * 1 <= E <= 32, 1 <= K <= 4, B*H <= 65535. */
+tla_status tla_layer_prologue(const tla_prologue_args *a, void *stream);
+
+/* Workspace of tla_layer_prologue_bwd in bytes (per-segment partial sums). */
+size_t tla_layer_prologue_bwd_workspace_bytes(const tla_prologue_args *a);
+
+/*
+ * Backward of the input path.  grad_dtype is the tla_dtype of dq, dk, dv, dq2,
+ * dk2 (what tla_chunk_bwd produced); dg [B,T,H,E] and dbeta [B,T,H] are fp32
+ * (dbeta NULL iff beta_in NULL).  Writes dP [B,T,H,C] (dtype), dconv_w [H,C,K],
+ * dgate_in [B,T,H,E], dgate_bias [H,E], dA_log [H,E] and dbeta_in [B,T,H] (fp32).
+ * The sums over tokens are taken in a fixed order (deterministic).
+ */
+tla_status tla_layer_prologue_bwd(const tla_prologue_args *a, int grad_dtype, const void *dq,
+                                  const void *dk, const void *dv, const void *dq2,
+                                  const void *dk2, const float *dg, const float *dbeta,
+                                  void *dP, float *dconv_w, float *dgate_in, float *dgate_bias,
+                                  float *dA_log, float *dbeta_in, void *workspace,
+                                  size_t workspace_bytes, void *stream);
+
+/*
+ * Output gate of Algorithm 4: per (b, t, h) over dv channels
+ *   y = o / sqrt(mean(o^2) + eps) * w_norm * sigmoid(z).
+ */
+typedef struct {
+    int B, T, H, dv;
+    int o_dtype;         /* tla_dtype of o (the operator's output)               */
+    int dtype;           /* tla_dtype of z and y                                 */
+    float eps;
+    const void *o;       /* [B,T,H,dv]                                           */
+    const void *z;       /* [B,T,H,dv]  gate pre-activation (W_g2 W_g1 u + b_g)   */
+    const float *w_norm; /* [dv]                                                 */
+    void *y;             /* [B,T,H,dv] (written)                                 */
+} tla_gate_args;
+
+/* Forward of the output gate (dv a multiple of 16 up to 128). */
+tla_status tla_output_gate(const tla_gate_args *a, void *stream);
+
+/* Workspace of tla_output_gate_bwd in bytes. */
+size_t tla_output_gate_bwd_workspace_bytes(const tla_gate_args *a);
+
+/* Backward: dy [B,T,H,dv] (dtype) -> d_o (o_dtype), dz (dtype), dw_norm [dv]
+ * fp32 (fixed-order sums). */
+tla_status tla_output_gate_bwd(const tla_gate_args *a, const void *dy, void *d_o, void *dz,
+                               float *dw_norm, void *workspace, size_t workspace_bytes,
+                               void *stream);
+
+/*
  * Synchronises `stream`, then returns TLA_ERR_TIMEOUT if a device-side bounded
  * wait of any kernel launched since the previous call expired (and clears that
  * record), TLA_ERR_CUDA if the stream reports an error, else TLA_OK.

@@ -140,6 +140,28 @@ def packed_lengths(total, mean_len, seed=0, min_len=1):
     return lens
 
 
+def layer_inputs(B, T, H, dk, dv, E, K=4, dtype="bf16", device="cpu", seed=0):
+    """Inputs of the layer input path and output gate (Algorithm 4), one generator:
+    P ~ N(0,1) [B,T,H,2dk+dv+2E] (dtype), conv_w ~ N(0,1/K) [H,C,K], gate_in ~ N(0,1)
+    [B,T,H,E], gate_bias ~ N(1,1) [H,E], A_log ~ N(-1,0.5^2) [H,E], beta_in ~ N(0,1) [B,T,H],
+    o ~ N(0,1) [B,T,H,dv] fp32, z ~ N(0,1) [B,T,H,dv] (dtype), w_norm ~ 1 + 0.1 N(0,1) [dv];
+    all but P and z fp32."""
+    dev = torch.device(device)
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(seed)
+    dt = torch_dtype(dtype)
+    C = 2 * dk + dv + 2 * E
+
+    def randn(*shape):
+        return torch.randn(*shape, generator=gen, device=dev, dtype=torch.float32)
+
+    return {"P": randn(B, T, H, C).to(dt), "conv_w": randn(H, C, K) / K ** 0.5,
+            "gate_in": randn(B, T, H, E), "gate_bias": randn(H, E) + 1.0,
+            "A_log": 0.5 * randn(H, E) - 1.0, "beta_in": randn(B, T, H),
+            "o": randn(B, T, H, dv), "z": randn(B, T, H, dv).to(dt),
+            "w_norm": 1.0 + 0.1 * randn(dv)}
+
+
 def workload_inputs(w: Workload, device="cpu", seed=0, B=None, T=None, H=None):
     """Inputs of a named workload, optionally with a reduced B/T/H for tests."""
     return chunk_inputs(B or w.B, T or w.T, H or w.H, w.dk, w.dv, w.E, w.dtype, w.with_beta,

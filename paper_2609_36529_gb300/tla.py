@@ -21,7 +21,10 @@ STATUS = {0: "TLA_OK", -1: "TLA_ERR_INVALID_ARG", -2: "TLA_ERR_UNSUPPORTED", -3:
 
 EXPORTED = ("tla_fwd_workspace_bytes", "tla_chunk_fwd", "tla_bwd_workspace_bytes",
             "tla_chunk_bwd", "tla_decode_step", "tla_status_string", "tla_last_device_status",
-            "tla_version", "tla_chunk_fwd_noalloc", "tla_noalloc_scratch_bytes")
+            "tla_version", "tla_chunk_fwd_noalloc", "tla_noalloc_scratch_bytes",
+            "tla_layer_prologue", "tla_layer_prologue_bwd_workspace_bytes",
+            "tla_layer_prologue_bwd", "tla_output_gate", "tla_output_gate_bwd_workspace_bytes",
+            "tla_output_gate_bwd")
 
 
 class TlaError(RuntimeError):
@@ -40,6 +43,24 @@ class tla_problem(ctypes.Structure):
                 ("beta", ctypes.c_void_p), ("h0", ctypes.c_void_p), ("o", ctypes.c_void_p),
                 ("ht", ctypes.c_void_p), ("cu_seqlens", ctypes.POINTER(ctypes.c_int)),
                 ("n_docs", ctypes.c_int), ("gate_per_head", ctypes.c_int)]
+
+
+class tla_prologue_args(ctypes.Structure):
+    _fields_ = [("B", ctypes.c_int), ("T", ctypes.c_int), ("H", ctypes.c_int),
+                ("dk", ctypes.c_int), ("dv", ctypes.c_int), ("E", ctypes.c_int),
+                ("K", ctypes.c_int), ("dtype", ctypes.c_int), ("eps", ctypes.c_float),
+                ("P", ctypes.c_void_p), ("conv_w", ctypes.c_void_p), ("gate_in", ctypes.c_void_p),
+                ("gate_bias", ctypes.c_void_p), ("A_log", ctypes.c_void_p),
+                ("beta_in", ctypes.c_void_p), ("q", ctypes.c_void_p), ("k", ctypes.c_void_p),
+                ("v", ctypes.c_void_p), ("q2", ctypes.c_void_p), ("k2", ctypes.c_void_p),
+                ("g", ctypes.c_void_p), ("beta", ctypes.c_void_p)]
+
+
+class tla_gate_args(ctypes.Structure):
+    _fields_ = [("B", ctypes.c_int), ("T", ctypes.c_int), ("H", ctypes.c_int),
+                ("dv", ctypes.c_int), ("o_dtype", ctypes.c_int), ("dtype", ctypes.c_int),
+                ("eps", ctypes.c_float), ("o", ctypes.c_void_p), ("z", ctypes.c_void_p),
+                ("w_norm", ctypes.c_void_p), ("y", ctypes.c_void_p)]
 
 
 _lib = None
@@ -72,6 +93,19 @@ def lib():
         L.tla_chunk_fwd_noalloc.argtypes = [P, vp]
         L.tla_chunk_fwd_noalloc.restype = i
         L.tla_noalloc_scratch_bytes.restype = sz
+        PA, GA = ctypes.POINTER(tla_prologue_args), ctypes.POINTER(tla_gate_args)
+        L.tla_layer_prologue.argtypes = [PA, vp]
+        L.tla_layer_prologue.restype = i
+        L.tla_layer_prologue_bwd_workspace_bytes.argtypes = [PA]
+        L.tla_layer_prologue_bwd_workspace_bytes.restype = sz
+        L.tla_layer_prologue_bwd.argtypes = [PA, i] + [vp] * 14 + [sz, vp]
+        L.tla_layer_prologue_bwd.restype = i
+        L.tla_output_gate.argtypes = [GA, vp]
+        L.tla_output_gate.restype = i
+        L.tla_output_gate_bwd_workspace_bytes.argtypes = [GA]
+        L.tla_output_gate_bwd_workspace_bytes.restype = sz
+        L.tla_output_gate_bwd.argtypes = [GA, vp, vp, vp, vp, vp, sz, vp]
+        L.tla_output_gate_bwd.restype = i
         _lib = L
     return _lib
 
@@ -236,3 +270,95 @@ def tla_last_device_status() -> int:
 
 def tla_version() -> str:
     return lib().tla_version().decode()
+
+
+# --- layer input path and output gate (Algorithm 4)
+
+def _prologue_args(P, conv_w, gate_in, gate_bias, A_log, beta_in, dk, dv, E, eps, out):
+    B, T, H, C = P.shape
+    assert C == 2 * dk + dv + 2 * E, "P channels must be 2 dk + dv + 2 E per head"
+    a = tla_prologue_args()
+    a.B, a.T, a.H, a.dk, a.dv, a.E, a.K = B, T, H, dk, dv, E, conv_w.shape[-1]
+    a.dtype, a.eps = _dtype_code(P), float(eps)
+    for name, t in (("P", P), ("conv_w", conv_w), ("gate_in", gate_in), ("gate_bias", gate_bias),
+                    ("A_log", A_log), ("beta_in", beta_in)):
+        setattr(a, name, _ptr(t))
+    for name in ("q", "k", "v", "q2", "k2", "g", "beta"):
+        setattr(a, name, _ptr(out.get(name)))
+    return a
+
+
+def layer_prologue(P, conv_w, gate_in, gate_bias, A_log, beta_in, dk, dv, E, eps=1e-6):
+    """Input path of Algorithm 4 from the projection output P [B,T,H,2dk+dv+2E] (per head
+    [q|k|v|q'|k']): returns q, k, v, q2, k2 (P's dtype), g and beta (fp32)."""
+    B, T, H, _ = P.shape
+    dev, dt = P.device, P.dtype
+    out = {"q": torch.empty(B, T, H, dk, dtype=dt, device=dev),
+           "k": torch.empty(B, T, H, dk, dtype=dt, device=dev),
+           "v": torch.empty(B, T, H, dv, dtype=dt, device=dev),
+           "q2": torch.empty(B, T, H, E, dtype=dt, device=dev),
+           "k2": torch.empty(B, T, H, E, dtype=dt, device=dev),
+           "g": torch.empty(B, T, H, E, dtype=torch.float32, device=dev),
+           "beta": torch.empty(B, T, H, dtype=torch.float32, device=dev)
+           if beta_in is not None else None}
+    a = _prologue_args(P, conv_w, gate_in, gate_bias, A_log, beta_in, dk, dv, E, eps, out)
+    _check("tla_layer_prologue", lib().tla_layer_prologue(ctypes.byref(a), _stream()))
+    return out
+
+
+def layer_prologue_bwd(P, conv_w, gate_in, gate_bias, A_log, beta_in, dk, dv, E, grads,
+                       eps=1e-6):
+    """Backward of layer_prologue.  grads: dq, dk, dv, dq2, dk2 (one dtype), dg, dbeta.
+    Returns dP (P's dtype), dconv_w, dgate_in, dgate_bias, dA_log, dbeta_in (fp32)."""
+    a = _prologue_args(P, conv_w, gate_in, gate_bias, A_log, beta_in, dk, dv, E, eps, {})
+    # output slots are not read by the backward; any non-null aligned pointer passes validation
+    for name in ("q", "k", "v", "q2", "k2", "g"):
+        setattr(a, name, _ptr(P))
+    a.beta = _ptr(beta_in) if beta_in is not None else None
+    f32 = dict(dtype=torch.float32, device=P.device)
+    out = {"dP": torch.empty_like(P), "dconv_w": torch.empty_like(conv_w),
+           "dgate_in": torch.empty_like(gate_in), "dgate_bias": torch.empty_like(gate_bias),
+           "dA_log": torch.empty_like(A_log),
+           "dbeta_in": torch.empty(beta_in.shape, **f32) if beta_in is not None else None}
+    need = lib().tla_layer_prologue_bwd_workspace_bytes(ctypes.byref(a))
+    if need == 0:
+        raise TlaError("tla_layer_prologue_bwd_workspace_bytes", -1)
+    ws = _workspace(need, P.device)
+    _check("tla_layer_prologue_bwd", lib().tla_layer_prologue_bwd(
+        ctypes.byref(a), _dtype_code(grads["dq"]), _ptr(grads["dq"]), _ptr(grads["dk"]),
+        _ptr(grads["dv"]), _ptr(grads["dq2"]), _ptr(grads["dk2"]), _ptr(grads["dg"]),
+        _ptr(grads.get("dbeta")), _ptr(out["dP"]), _ptr(out["dconv_w"]), _ptr(out["dgate_in"]),
+        _ptr(out["dgate_bias"]), _ptr(out["dA_log"]), _ptr(out["dbeta_in"]), _ptr(ws), need,
+        _stream()))
+    return {n: t for n, t in out.items() if t is not None}
+
+
+def _gate_args(o, z, w_norm, eps, y):
+    B, T, H, dv = o.shape
+    a = tla_gate_args()
+    a.B, a.T, a.H, a.dv = B, T, H, dv
+    a.o_dtype, a.dtype, a.eps = _dtype_code(o), _dtype_code(z), float(eps)
+    a.o, a.z, a.w_norm, a.y = _ptr(o), _ptr(z), _ptr(w_norm), _ptr(y)
+    return a
+
+
+def output_gate(o, z, w_norm, eps=1e-6):
+    """Output gate of Algorithm 4: RMSNorm(o) * w_norm * sigmoid(z), in z's dtype."""
+    y = torch.empty(o.shape, dtype=z.dtype, device=o.device)
+    a = _gate_args(o, z, w_norm, eps, y)
+    _check("tla_output_gate", lib().tla_output_gate(ctypes.byref(a), _stream()))
+    return y
+
+
+def output_gate_bwd(o, z, w_norm, dy, eps=1e-6):
+    """Backward of output_gate: returns do (o's dtype), dz (z's dtype), dw_norm (fp32)."""
+    out = {"do": torch.empty_like(o), "dz": torch.empty_like(z), "dw_norm": torch.empty_like(w_norm)}
+    a = _gate_args(o, z, w_norm, eps, dy)
+    need = lib().tla_output_gate_bwd_workspace_bytes(ctypes.byref(a))
+    if need == 0:
+        raise TlaError("tla_output_gate_bwd_workspace_bytes", -1)
+    ws = _workspace(need, o.device)
+    _check("tla_output_gate_bwd", lib().tla_output_gate_bwd(
+        ctypes.byref(a), _ptr(dy), _ptr(out["do"]), _ptr(out["dz"]), _ptr(out["dw_norm"]),
+        _ptr(ws), need, _stream()))
+    return out

@@ -147,3 +147,47 @@ def test_packed_documents_validation(tla):
     assert L.tla_chunk_fwd(ctypes.byref(p), None, 0, 0, None) == -1
     # packed documents run on the tensor-core path only (here d_k = 64): refused before a launch
     assert L.tla_chunk_fwd(ctypes.byref(ok), ctypes.c_void_p(0x100000), need, 1, None) == -2
+
+
+def test_layer_io_validation(tla):
+    """Input prologue and output gate (Algorithm 4): argument checks before any launch."""
+    L = tla.lib()
+    f = ctypes.c_void_p(0x1000)
+
+    def prologue(**kw):
+        a = tla.tla_prologue_args()
+        a.B, a.T, a.H, a.dk, a.dv, a.E, a.K, a.dtype, a.eps = 2, 100, 3, 64, 64, 4, 4, 0, 1e-6
+        for n in ("P", "conv_w", "gate_in", "gate_bias", "A_log", "beta_in", "q", "k", "v",
+                  "q2", "k2", "g", "beta"):
+            setattr(a, n, f)
+        for n, v in kw.items():
+            setattr(a, n, v)
+        return a
+
+    for kw, want in [(dict(K=5), -2), (dict(K=0), -1), (dict(E=33), -2), (dict(dk=20), -2),
+                     (dict(beta=None), -1), (dict(P=None), -1), (dict(eps=0.0), -1),
+                     (dict(dtype=5), -1), (dict(q=ctypes.c_void_p(0x1004)), -1)]:
+        assert L.tla_layer_prologue(ctypes.byref(prologue(**kw)), None) == want, kw
+    ok = prologue()
+    need = L.tla_layer_prologue_bwd_workspace_bytes(ctypes.byref(ok))
+    assert need > 0 and need % 256 == 0
+    args = [f] * 14
+    assert L.tla_layer_prologue_bwd(ctypes.byref(ok), 1, *args[:13], None, need, None) == -5
+    assert L.tla_layer_prologue_bwd(ctypes.byref(ok), 3, *args, need, None) == -1
+
+    def gate(**kw):
+        a = tla.tla_gate_args()
+        a.B, a.T, a.H, a.dv, a.o_dtype, a.dtype, a.eps = 2, 10, 3, 64, 1, 0, 1e-6
+        for n in ("o", "z", "w_norm", "y"):
+            setattr(a, n, f)
+        for n, v in kw.items():
+            setattr(a, n, v)
+        return a
+
+    for kw, want in [(dict(dv=20), -2), (dict(o=None), -1), (dict(o_dtype=9), -1),
+                     (dict(eps=-1.0), -1)]:
+        assert L.tla_output_gate(ctypes.byref(gate(**kw)), None) == want, kw
+    g = gate()
+    need = L.tla_output_gate_bwd_workspace_bytes(ctypes.byref(g))
+    assert need > 0
+    assert L.tla_output_gate_bwd(ctypes.byref(g), f, f, f, f, None, need, None) == -5
