@@ -9,7 +9,8 @@ decode workload (fp32 state [256,32,8,128,128], 100 steps each of sGLA and
 GDN after a 512-token chunked prefill) and reported under "decode", and the
 same step with the headline's tokens packed into documents of log-normal length
 around 1000 tokens (cu_seqlens, each document from its own state) under "packed";
-the per-head-gate and E = 32 / d_k = 64 variants under "variants".
+the per-head-gate and E = 32 / d_k = 64 variants under "variants"; the layer's
+fused input path and output gate (GB/s) under "layer_io".
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
@@ -329,6 +330,10 @@ def run_ours(args):
     if not args.no_variants:
         variants = run_variants(args, tla, inputs, w, dev, stream, barrier, max_over_ranks, ws_n,
                                 rank, value)
+    layer = None
+    if not args.no_layer:
+        layer = run_layer_io(args, tla, inputs, w, dev, stream, barrier, max_over_ranks, rank,
+                             load_peaks())
     decode = None
     if not args.no_decode:
         del fws, bws
@@ -358,7 +363,7 @@ def run_ours(args):
             "tflops_frac": round(total_flops / (ms_step / 1e3) / 1e12 / peak, 5),
             "roofline": roofline, "kernels": kernels, "gpu_launches": gpu_launches,
             "clocks": ck, "clocks_remeasured": remeasured,
-            "e2e": e2e, "packed": packed, "variants": variants, "decode": decode, "cpu_baseline": cpu, "impl": "ours",
+            "e2e": e2e, "packed": packed, "variants": variants, "layer_io": layer, "decode": decode, "cpu_baseline": cpu, "impl": "ours",
         }
         print(json.dumps(line), flush=True)
     if ws_n > 1:
@@ -542,6 +547,41 @@ def run_variants(args, tla, inputs, w, dev, stream, barrier, max_over_ranks, ws_
     return out
 
 
+def run_layer_io(args, tla, inputs, w, dev, stream, barrier, max_over_ranks, rank, peaks):
+    """The layer's input path and output gate (Algorithm 4) on the headline's token-heads
+    (bf16 projection output, K = 4 convolution, fp32 operator output and gradients): device
+    time per call and algorithmic bytes (each tensor read or written once) per second."""
+    B, T, H, dk, dv, E, K = w.B, w.T, w.H, w.dk, w.dv, w.E, 4
+    x = inputs.layer_inputs(B, T, H, dk, dv, E, K, dtype=w.dtype, device=dev, seed=300 + rank)
+    args_p = [x[n] for n in ("P", "conv_w", "gate_in", "gate_bias", "A_log", "beta_in")]
+    gen = torch.Generator(dev).manual_seed(301 + rank)
+    grads = {n: torch.randn(B, T, H, c, device=dev, generator=gen)
+             for n, c in (("dq", dk), ("dk", dk), ("dv", dv), ("dq2", E), ("dk2", E), ("dg", E))}
+    grads["dbeta"] = torch.randn(B, T, H, device=dev, generator=gen)
+    dy = torch.randn(B, T, H, dv, device=dev, generator=gen).to(x["z"].dtype)
+    units = B * T * H
+    C = 2 * dk + dv + 2 * E
+    eb = 2 if w.dtype == "bf16" else 4
+    bytes_per = {   # per token-head, every tensor touched once
+        "prologue_fwd": C * eb + E * 4 + 4 + C * eb + E * 4 + 4,
+        "prologue_bwd": C * eb + (2 * dk + dv + 2 * E) * 4 + E * 4 + 4 + E * 4 + 4 + C * eb + E * 4 + 4,
+        "gate_fwd": dv * 4 + dv * eb + dv * eb,
+        "gate_bwd": dv * 4 + 2 * dv * eb + dv * 4 + dv * eb}
+    calls = {"prologue_fwd": lambda: tla.layer_prologue(*args_p, dk, dv, E),
+             "prologue_bwd": lambda: tla.layer_prologue_bwd(*args_p, dk, dv, E, grads),
+             "gate_fwd": lambda: tla.output_gate(x["o"], x["z"], x["w_norm"]),
+             "gate_bwd": lambda: tla.output_gate_bwd(x["o"], x["z"], x["w_norm"], dy)}
+    peak = peaks["hbm_gbs"]
+    out = {"workload": f"layer_io_B{B}_H{H}_T{T}_d{dk}_E{E}_K{K}", "unit": "GB/s", "peak": peak,
+           "peak_source": "hbm copy bandwidth, " + peaks["source"]}
+    for name, fn in calls.items():
+        ms = _time_steps(fn, 3, 3, stream, barrier, max_over_ranks)
+        gbs = bytes_per[name] * units / (ms / 1e3) / 1e9
+        out[name] = {"ms": round(ms, 4), "achieved_gbs": round(gbs, 1), "frac": round(gbs / peak, 4),
+                     "bytes_per_token_head": bytes_per[name]}
+    return out
+
+
 def run_decode(args, tla, inputs, dev, stream, lib, peaks, barrier, max_over_ranks, ws_n):
     dw = inputs.DECODE
     if args.decode_batch:   # profiling option: fewer sequences of the same shape
@@ -675,6 +715,7 @@ def main():
     ap.add_argument("--no-decode", action="store_true")
     ap.add_argument("--no-packed", action="store_true")
     ap.add_argument("--no-variants", action="store_true")
+    ap.add_argument("--no-layer", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--ref-tokens", type=int, default=1024,
