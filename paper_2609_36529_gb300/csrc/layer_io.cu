@@ -17,9 +17,8 @@ namespace tla {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kFwdTok = 16;    // tokens per CTA of the prologue forward
+constexpr int kFwdRun = 128;   // tokens per CTA of the prologue forward
 constexpr int kSeg = 256;      // tokens per CTA of the prologue backward
-constexpr int kSub = 8;        // tokens per sub-block of the prologue backward
 constexpr int kGateRows = 256; // (token, head) rows per CTA of the output gate
 
 __device__ __forceinline__ float sigm(float x) { return 1.f / (1.f + expf(-x)); }
@@ -51,58 +50,216 @@ __device__ __forceinline__ Groups groups(int dk, int dv, int E) {
 // normalised group index (q, k, q', k' -> 0..3) or -1 for v
 __device__ __forceinline__ int norm_slot(int g) { return g < 2 ? g : (g == 2 ? -1 : g - 1); }
 
-template <typename Tin>
-__global__ void __launch_bounds__(kThreads)
-prologue_fwd_kernel(const tla_prologue_args a) {
-    extern __shared__ float sm[];
+// Four consecutive channels of one token as fp32: one 8-byte (bf16) or 16-byte (fp32)
+// access when VEC (rows and channel offsets multiples of four), else four scalar ones.
+template <bool VEC>
+__device__ __forceinline__ void ld4(const __nv_bfloat16* p, float* v) {
+    if constexpr (VEC) {
+        const uint2 u = *reinterpret_cast<const uint2*>(p);
+        const float2 lo = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.x));
+        const float2 hi = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.y));
+        v[0] = lo.x; v[1] = lo.y; v[2] = hi.x; v[3] = hi.y;
+    } else {
+#pragma unroll
+        for (int u = 0; u < 4; ++u) v[u] = __bfloat162float(p[u]);
+    }
+}
+template <bool VEC>
+__device__ __forceinline__ void ld4(const float* p, float* v) {
+    if constexpr (VEC) {
+        const float4 f = *reinterpret_cast<const float4*>(p);
+        v[0] = f.x; v[1] = f.y; v[2] = f.z; v[3] = f.w;
+    } else {
+#pragma unroll
+        for (int u = 0; u < 4; ++u) v[u] = p[u];
+    }
+}
+template <bool VEC>
+__device__ __forceinline__ void st4(__nv_bfloat16* p, const float* v) {
+    if constexpr (VEC) {
+        __nv_bfloat162 lo = __floats2bfloat162_rn(v[0], v[1]), hi = __floats2bfloat162_rn(v[2], v[3]);
+        *reinterpret_cast<uint2*>(p) = make_uint2(*reinterpret_cast<uint32_t*>(&lo), *reinterpret_cast<uint32_t*>(&hi));
+    } else {
+#pragma unroll
+        for (int u = 0; u < 4; ++u) p[u] = __float2bfloat16_rn(v[u]);
+    }
+}
+template <bool VEC>
+__device__ __forceinline__ void st4(float* p, const float* v) {
+    if constexpr (VEC) {
+        *reinterpret_cast<float4*>(p) = make_float4(v[0], v[1], v[2], v[3]);
+    } else {
+#pragma unroll
+        for (int u = 0; u < 4; ++u) p[u] = v[u];
+    }
+}
+
+__device__ __forceinline__ float warp_sum(float x) {
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+    return x;
+}
+
+// Layout of the prologue kernels: a CTA of four warps takes one run of tokens of one
+// (b, h); warp 0 the q channels, warp 1 k, warp 2 v (four channels per lane), warp 3 the
+// q' and k' channels (one or two per lane) together with the gates and beta.  Each norm
+// is then a reduction inside one warp, so the warps never wait on one another.  A warp
+// walks its run token by token, keeping the last three projection rows (and, backward,
+// the last three pre-activation gradients) in registers: the width-K convolution uses
+// K <= 4 taps padded on the left to four with zero weights, so every projection row is
+// loaded once plus a halo of three tokens per run.  Tokens are taken four at a time, all
+// four loads issued before the first use.
+constexpr int kPrWarps = 4;
+
+struct ChanMap {   // the channels of one lane of a q, k or v warp
+    int base, width, c;
+    bool act;
+};
+__device__ __forceinline__ ChanMap chan_map(int g, int dk, int dv, int lane) {
+    ChanMap m;
+    m.base = g == 2 ? 2 * dk : g * dk;
+    m.width = g == 2 ? dv : dk;
+    m.c = m.base + 4 * lane;
+    m.act = 4 * lane < m.width;
+    return m;
+}
+
+template <typename Tin, bool VEC>
+__device__ __forceinline__ void prologue_fwd_qkv(const tla_prologue_args& a, int g, int b, int h,
+                                                 int t0, int t1) {
+    const int lane = threadIdx.x & 31;
     const int dk = a.dk, dv = a.dv, E = a.E, K = a.K, T = a.T, H = a.H;
     const int C = 2 * dk + dv + 2 * E;
-    const Groups G = groups(dk, dv, E);
-    const int t0 = blockIdx.x * kFwdTok, h = blockIdx.y, b = blockIdx.z;
-    const int nt = min(kFwdTok, T - t0);
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    float* ys = sm;                       // [kFwdTok][C] activations
-    float* sc = sm + kFwdTok * C;         // [kFwdTok][4] 1 / norm
-    for (int c = tid; c < C; c += kThreads) {
-        float w[4];
-        for (int j = 0; j < K; ++j) w[j] = a.conv_w[(size_t(h) * C + c) * K + j];
-        const int g = G.of(c);
-        for (int i = 0; i < nt; ++i) {
-            const int t = t0 + i;
-            float acc = 0.f;
-            for (int j = 0; j < K; ++j) {
-                const int ts = t - K + 1 + j;
-                if (ts >= 0) acc = fmaf(w[j], ld<Tin>(a.P, tok_idx(b, ts, h, c, T, H, C)), acc);
+    const ChanMap m = chan_map(g, dk, dv, lane);
+    float w[4][4];   // [padded tap][channel]
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+            w[j][u] = (m.act && j >= 4 - K) ? a.conv_w[(size_t(h) * C + m.c + u) * K + j - (4 - K)] : 0.f;
+    const size_t sP = size_t(H) * C, sD = size_t(H) * m.width;
+    const Tin* pP = static_cast<const Tin*>(a.P) + (size_t(b) * T * H + h) * C + m.c;
+    Tin* pD = static_cast<Tin*>(g == 0 ? a.q : g == 1 ? a.k : a.v) + (size_t(b) * T * H + h) * m.width + 4 * lane;
+    float pw[3][4];
+#pragma unroll
+    for (int i = 0; i < 3; ++i) {
+        const int t = t0 - 3 + i;
+        if (m.act && t >= 0) ld4<VEC>(pP + t * sP, pw[i]);
+        else pw[i][0] = pw[i][1] = pw[i][2] = pw[i][3] = 0.f;
+    }
+    for (int tb = t0; tb < t1; tb += 4) {
+        float xb[4][4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            if (m.act && tb + i < t1) ld4<VEC>(pP + (tb + i) * sP, xb[i]);
+            else xb[i][0] = xb[i][1] = xb[i][2] = xb[i][3] = 0.f;
+        }
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            float y[4], ss = 0.f;
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                float x = w[0][u] * pw[0][u];
+                x = fmaf(w[1][u], pw[1][u], x);
+                x = fmaf(w[2][u], pw[2][u], x);
+                x = fmaf(w[3][u], xb[i][u], x);
+                y[u] = x * sigm(x);
+                ss = fmaf(y[u], y[u], ss);
+                pw[0][u] = pw[1][u]; pw[1][u] = pw[2][u]; pw[2][u] = xb[i][u];
             }
-            ys[i * C + c] = g >= 3 ? softplus(acc) : acc * sigm(acc);
+            if (g != 2) {
+                const float r = rsqrtf(warp_sum(ss) + a.eps);
+#pragma unroll
+                for (int u = 0; u < 4; ++u) y[u] *= r;
+            }
+            if (m.act && tb + i < t1) st4<VEC>(pD + (tb + i) * sD, y);
         }
     }
-    __syncthreads();
-    for (int task = warp; task < nt * 4; task += kThreads / 32) {
-        const int i = task >> 2, s = task & 3, g = s < 2 ? s : s + 1;
-        float ss = 0.f;
-        for (int c = G.off[g] + lane; c < G.off[g + 1]; c += 32) ss = fmaf(ys[i * C + c], ys[i * C + c], ss);
+}
+
+template <typename Tin>
+__device__ __forceinline__ void prologue_fwd_small(const tla_prologue_args& a, int b, int h,
+                                                   int t0, int t1) {
+    const int lane = threadIdx.x & 31;
+    const int dk = a.dk, dv = a.dv, E = a.E, K = a.K, T = a.T, H = a.H;
+    const int C = 2 * dk + dv + 2 * E, off = 2 * dk + dv;
+    // channel slots cc = lane, lane + 32 of the 2E channels [q' | k']
+    bool act[2];
+    int col[2];
+    float w[4][2];
 #pragma unroll
-        for (int o = 16; o >= 1; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
-        if (lane == 0) sc[i * 4 + s] = rsqrtf(ss + a.eps);
+    for (int s = 0; s < 2; ++s) {
+        const int cc = lane + 32 * s;
+        act[s] = cc < 2 * E;
+        col[s] = cc < E ? cc : cc - E;
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+            w[j][s] = (act[s] && j >= 4 - K) ? a.conv_w[(size_t(h) * C + off + cc) * K + j - (4 - K)] : 0.f;
     }
-    __syncthreads();
-    void* dst[5] = {a.q, a.k, a.v, a.q2, a.k2};
-    for (int idx = tid; idx < nt * C; idx += kThreads) {
-        const int i = idx / C, c = idx - i * C, g = G.of(c), s = norm_slot(g);
-        const int width = G.off[g + 1] - G.off[g];
-        const float y = ys[idx] * (s >= 0 ? sc[i * 4 + s] : 1.f);
-        st<Tin>(dst[g], tok_idx(b, t0 + i, h, c - G.off[g], T, H, width), y);
+    const size_t sP = size_t(H) * C, sE = size_t(H) * E;
+    const Tin* pP = static_cast<const Tin*>(a.P) + (size_t(b) * T * H + h) * C + off + lane;
+    const size_t rowE = (size_t(b) * T * H + h) * E;
+    float pw[3][2];
+#pragma unroll
+    for (int i = 0; i < 3; ++i)
+#pragma unroll
+        for (int s = 0; s < 2; ++s) {
+            const int t = t0 - 3 + i;
+            pw[i][s] = (act[s] && t >= 0) ? to_f(pP[t * sP + 32 * s]) : 0.f;
+        }
+    for (int tb = t0; tb < t1; tb += 4) {
+        float xb[4][2];
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+#pragma unroll
+            for (int s = 0; s < 2; ++s)
+                xb[i][s] = (act[s] && tb + i < t1) ? to_f(pP[(tb + i) * sP + 32 * s]) : 0.f;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            float y[2], sq = 0.f, sk = 0.f;
+#pragma unroll
+            for (int s = 0; s < 2; ++s) {
+                float x = w[0][s] * pw[0][s];
+                x = fmaf(w[1][s], pw[1][s], x);
+                x = fmaf(w[2][s], pw[2][s], x);
+                x = fmaf(w[3][s], xb[i][s], x);
+                y[s] = act[s] ? softplus(x) : 0.f;
+                if (lane + 32 * s < E) sq = fmaf(y[s], y[s], sq);
+                else sk = fmaf(y[s], y[s], sk);
+                pw[0][s] = pw[1][s]; pw[1][s] = pw[2][s]; pw[2][s] = xb[i][s];
+            }
+            const float rq = rsqrtf(warp_sum(sq) + a.eps), rk = rsqrtf(warp_sum(sk) + a.eps);
+            if (tb + i < t1) {
+                const size_t o = rowE + (tb + i) * sE;
+#pragma unroll
+                for (int s = 0; s < 2; ++s)
+                    if (act[s]) {
+                        const bool isq = lane + 32 * s < E;
+                        st<Tin>(isq ? a.q2 : a.k2, o + col[s], y[s] * (isq ? rq : rk));
+                    }
+            }
+        }
     }
-    for (int idx = tid; idx < nt * E; idx += kThreads) {
+    const int n = t1 - t0;
+    for (int idx = lane; idx < n * E; idx += 32) {   // log gates
         const int i = idx / E, e = idx - i * E;
-        const size_t o = tok_idx(b, t0 + i, h, e, T, H, E);
+        const size_t o = rowE + (t0 + i) * sE + e;
         a.g[o] = -expf(a.A_log[h * E + e]) * softplus(a.gate_in[o] + a.gate_bias[h * E + e]);
     }
-    if (a.beta_in && tid < nt) {
-        const size_t o = (size_t(b) * T + t0 + tid) * H + h;
-        a.beta[o] = sigm(a.beta_in[o]);
-    }
+    if (a.beta_in)
+        for (int t = t0 + lane; t < t1; t += 32) {
+            const size_t o = (size_t(b) * T + t) * H + h;
+            a.beta[o] = sigm(a.beta_in[o]);
+        }
+}
+
+template <typename Tin, bool VEC>
+__global__ void __launch_bounds__(kPrWarps * 32)
+prologue_fwd_kernel(const tla_prologue_args a) {
+    const int t0 = blockIdx.x * kFwdRun, t1 = min(a.T, t0 + kFwdRun);
+    const int g = threadIdx.x >> 5, h = blockIdx.y, b = blockIdx.z;
+    if (g < 3) prologue_fwd_qkv<Tin, VEC>(a, g, b, h, t0, t1);
+    else prologue_fwd_small<Tin>(a, b, h, t0, t1);
 }
 
 struct PrologueGrads {
@@ -113,133 +270,255 @@ struct PrologueGrads {
     float* part;   // per CTA: [C*K] conv-weight partials, then [E] gate-bias, [E] A_log partials
 };
 
-// One CTA per (segment of kSeg tokens, h, b); sub-blocks of kSub tokens, each recomputing
-// the activations of its tokens and of the K-1 tokens after them (the transposed
-// convolution of a token reads the K-1 following pre-activation gradients).
-template <typename Tin, typename Tg>
-__global__ void __launch_bounds__(kThreads)
-prologue_bwd_kernel(const tla_prologue_args a, const PrologueGrads gr) {
-    extern __shared__ float sm[];
+// Backward of one q, k or v warp over tokens [t0, t1): the pre-activation gradients of
+// tokens t0 .. t1 + 2 (the transposed convolution of token t reads those of t .. t + 3;
+// zero past T), dP of the run's own tokens, and the conv-weight sums over them.
+template <typename Tin, typename Tg, bool VEC>
+__device__ __forceinline__ void prologue_bwd_qkv(const tla_prologue_args& a, const PrologueGrads& gr,
+                                                 int g, int b, int h, int t0, int t1, float* part) {
+    const int lane = threadIdx.x & 31;
     const int dk = a.dk, dv = a.dv, E = a.E, K = a.K, T = a.T, H = a.H;
     const int C = 2 * dk + dv + 2 * E;
-    const Groups G = groups(dk, dv, E);
-    const int seg = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    constexpr int NE = kSub + 3;            // sub-block tokens + up to K - 1 = 3 after them
-    float* ys = sm;                         // [NE][C] activations (then scaled: u = y / n)
-    float* das = ys + NE * C;               // [NE][C] pre-activation gradients
-    float* inv = das + NE * C;              // [NE][4] 1 / n
-    float* udy = inv + NE * 4;              // [NE][4] u . dy
-    void* gsrc[5];
-    gsrc[0] = const_cast<void*>(gr.dq); gsrc[1] = const_cast<void*>(gr.dk);
-    gsrc[2] = const_cast<void*>(gr.dv); gsrc[3] = const_cast<void*>(gr.dq2);
-    gsrc[4] = const_cast<void*>(gr.dk2);
-    // per-thread partial sums of the conv-weight gradient (channels tid, tid + 256)
-    float dwp[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
-    float gbp = 0.f, gap = 0.f;              // gate-bias and A_log partials (threads < E)
-    const int tbeg = seg * kSeg, tend = min(T, tbeg + kSeg);
-    for (int t0 = tbeg; t0 < tend; t0 += kSub) {
-        const int nt = min(kSub, tend - t0);
-        const int ne = min(nt + K - 1, T - t0);   // tokens whose gradients this block needs
-        // pre-activations and activations of tokens t0 .. t0 + ne - 1
-        for (int idx = tid; idx < ne * C; idx += kThreads) {
-            const int i = idx / C, c = idx - i * C, t = t0 + i;
-            float acc = 0.f;
-            for (int j = 0; j < K; ++j) {
-                const int ts = t - K + 1 + j;
-                if (ts >= 0)
-                    acc = fmaf(a.conv_w[(size_t(h) * C + c) * K + j],
-                               ld<Tin>(a.P, tok_idx(b, ts, h, c, T, H, C)), acc);
-            }
-            das[idx] = acc;   // pre-activation, replaced by its gradient below
-            ys[idx] = G.of(c) >= 3 ? softplus(acc) : acc * sigm(acc);
+    const ChanMap m = chan_map(g, dk, dv, lane);
+    float w[4][4], dw[4][4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            w[j][u] = (m.act && j >= 4 - K) ? a.conv_w[(size_t(h) * C + m.c + u) * K + j - (4 - K)] : 0.f;
+            dw[j][u] = 0.f;
         }
-        __syncthreads();
-        for (int task = warp; task < ne * 4; task += kThreads / 32) {   // norms and u . dy
-            const int i = task >> 2, s = task & 3, g = s < 2 ? s : s + 1;
-            const int width = G.off[g + 1] - G.off[g];
-            float ss = 0.f, yd = 0.f;
-            for (int c = G.off[g] + lane; c < G.off[g + 1]; c += 32) {
-                const float y = ys[i * C + c];
-                ss = fmaf(y, y, ss);
-                yd = fmaf(y, ld<Tg>(gsrc[g], tok_idx(b, t0 + i, h, c - G.off[g], T, H, width)), yd);
+    const size_t sP = size_t(H) * C, sG = size_t(H) * m.width;
+    const size_t rowP = (size_t(b) * T * H + h) * C + m.c;
+    const Tin* pP = static_cast<const Tin*>(a.P) + rowP;
+    Tin* pdP = static_cast<Tin*>(gr.dP) + rowP;
+    const Tg* pG = static_cast<const Tg*>(g == 0 ? gr.dq : g == 1 ? gr.dk : gr.dv) +
+                   (size_t(b) * T * H + h) * m.width + 4 * lane;
+    float pw[3][4], dxw[3][4];   // projection rows and pre-activation gradients of t-3 .. t-1
+#pragma unroll
+    for (int i = 0; i < 3; ++i) {
+        const int t = t0 - 3 + i;
+        if (m.act && t >= 0) ld4<VEC>(pP + t * sP, pw[i]);
+        else pw[i][0] = pw[i][1] = pw[i][2] = pw[i][3] = 0.f;
+        dxw[i][0] = dxw[i][1] = dxw[i][2] = dxw[i][3] = 0.f;
+    }
+    const int tl = t1 + 3, tv = min(tl, T), te = min(t1, T);
+    for (int tb = t0; tb < tl; tb += 4) {
+        float xb[4][4], gb[4][4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            if (m.act && tb + i < tv) {
+                ld4<VEC>(pP + (tb + i) * sP, xb[i]);
+                ld4<VEC>(pG + (tb + i) * sG, gb[i]);
+            } else {
+#pragma unroll
+                for (int u = 0; u < 4; ++u) xb[i][u] = gb[i][u] = 0.f;
+            }
+        }
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int t = tb + i;
+            float dx[4] = {0.f, 0.f, 0.f, 0.f};
+            if (t < tv) {
+                float x[4], sg[4], y[4], ss = 0.f, yd = 0.f;
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    float v = w[0][u] * pw[0][u];
+                    v = fmaf(w[1][u], pw[1][u], v);
+                    v = fmaf(w[2][u], pw[2][u], v);
+                    v = fmaf(w[3][u], xb[i][u], v);
+                    x[u] = v;
+                    sg[u] = sigm(v);
+                    y[u] = v * sg[u];
+                    ss = fmaf(y[u], y[u], ss);
+                    yd = fmaf(y[u], gb[i][u], yd);
+                }
+                float dy[4] = {gb[i][0], gb[i][1], gb[i][2], gb[i][3]};
+                if (g != 2) {   // through u = y / n:  (dy - u (u . dy)) / n
+                    const float r = rsqrtf(warp_sum(ss) + a.eps), kk = r * r * warp_sum(yd);
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) dy[u] = (dy[u] - y[u] * kk) * r;
+                }
+#pragma unroll
+                for (int u = 0; u < 4; ++u) dx[u] = dy[u] * sg[u] * (1.f + x[u] * (1.f - sg[u]));
+                if (t < t1) {
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                        dw[0][u] = fmaf(dx[u], pw[0][u], dw[0][u]);
+                        dw[1][u] = fmaf(dx[u], pw[1][u], dw[1][u]);
+                        dw[2][u] = fmaf(dx[u], pw[2][u], dw[2][u]);
+                        dw[3][u] = fmaf(dx[u], xb[i][u], dw[3][u]);
+                    }
+                }
+            }
+            const int tp = t - 3;   // dP of token t - 3 reads dx of t - 3 .. t
+            if (m.act && tp >= t0 && tp < te) {
+                float d[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    float v = w[0][u] * dx[u];
+                    v = fmaf(w[1][u], dxw[2][u], v);
+                    v = fmaf(w[2][u], dxw[1][u], v);
+                    v = fmaf(w[3][u], dxw[0][u], v);
+                    d[u] = v;
+                }
+                st4<VEC>(pdP + tp * sP, d);
             }
 #pragma unroll
-            for (int o = 16; o >= 1; o >>= 1) {
-                ss += __shfl_xor_sync(0xffffffffu, ss, o);
-                yd += __shfl_xor_sync(0xffffffffu, yd, o);
-            }
-            if (lane == 0) {
-                const float r = rsqrtf(ss + a.eps);
-                inv[i * 4 + s] = r;
-                udy[i * 4 + s] = yd * r;
+            for (int u = 0; u < 4; ++u) {
+                pw[0][u] = pw[1][u]; pw[1][u] = pw[2][u]; pw[2][u] = xb[i][u];
+                dxw[0][u] = dxw[1][u]; dxw[1][u] = dxw[2][u]; dxw[2][u] = dx[u];
             }
         }
-        __syncthreads();
-        for (int idx = tid; idx < ne * C; idx += kThreads) {   // pre-activation gradients
-            const int i = idx / C, c = idx - i * C, g = G.of(c), s = norm_slot(g);
-            const int width = G.off[g + 1] - G.off[g];
-            const float dy = ld<Tg>(gsrc[g], tok_idx(b, t0 + i, h, c - G.off[g], T, H, width));
-            float dx = dy;
-            if (s >= 0) {   // d(y / n) = (dy - u (u . dy)) / n
-                const float r = inv[i * 4 + s];
-                dx = (dy - ys[idx] * r * udy[i * 4 + s]) * r;
-            }
-            const float x = das[idx], sg = sigm(x);
-            das[idx] = dx * (g >= 3 ? sg : sg * (1.f + x * (1.f - sg)));
+    }
+    if (m.act)
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+                if (j >= 4 - K) part[(m.c + u) * K + j - (4 - K)] = dw[j][u];
+}
+
+template <typename Tin, typename Tg>
+__device__ __forceinline__ void prologue_bwd_small(const tla_prologue_args& a, const PrologueGrads& gr,
+                                                   int b, int h, int t0, int t1, float* part) {
+    const int lane = threadIdx.x & 31;
+    const int dk = a.dk, dv = a.dv, E = a.E, K = a.K, T = a.T, H = a.H;
+    const int C = 2 * dk + dv + 2 * E, off = 2 * dk + dv;
+    bool act[2], isq[2];
+    int col[2];
+    float w[4][2], dw[4][2];
+#pragma unroll
+    for (int s = 0; s < 2; ++s) {
+        const int cc = lane + 32 * s;
+        act[s] = cc < 2 * E;
+        isq[s] = cc < E;
+        col[s] = cc < E ? cc : cc - E;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            w[j][s] = (act[s] && j >= 4 - K) ? a.conv_w[(size_t(h) * C + off + cc) * K + j - (4 - K)] : 0.f;
+            dw[j][s] = 0.f;
         }
-        __syncthreads();
-        // dP of the block's own tokens (transposed convolution) and conv-weight partials
-        for (int cc = 0; cc < 2; ++cc) {
-            const int c = tid + cc * kThreads;
-            if (c >= C) break;
-            float w[4];
-            for (int j = 0; j < K; ++j) w[j] = a.conv_w[(size_t(h) * C + c) * K + j];
-            for (int i = 0; i < nt; ++i) {
-                const int t = t0 + i;
-                float acc = 0.f;
-                for (int j = 0; j < K; ++j) {
-                    const int td = i + K - 1 - j;   // token t + K - 1 - j, local index
-                    if (t + K - 1 - j < T) acc = fmaf(w[j], das[td * C + c], acc);
+    }
+    const size_t sP = size_t(H) * C, sE = size_t(H) * E;
+    const size_t rowP = (size_t(b) * T * H + h) * C + off + lane;
+    const Tin* pP = static_cast<const Tin*>(a.P) + rowP;
+    Tin* pdP = static_cast<Tin*>(gr.dP) + rowP;
+    const size_t rowE = (size_t(b) * T * H + h) * E;
+    const Tg* gq = static_cast<const Tg*>(gr.dq2);
+    const Tg* gk = static_cast<const Tg*>(gr.dk2);
+    float pw[3][2], dxw[3][2];
+#pragma unroll
+    for (int i = 0; i < 3; ++i)
+#pragma unroll
+        for (int s = 0; s < 2; ++s) {
+            const int t = t0 - 3 + i;
+            pw[i][s] = (act[s] && t >= 0) ? to_f(pP[t * sP + 32 * s]) : 0.f;
+            dxw[i][s] = 0.f;
+        }
+    const int tl = t1 + 3, tv = min(tl, T), te = min(t1, T);
+    for (int tb = t0; tb < tl; tb += 4) {
+        float xb[4][2], gb[4][2];
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+#pragma unroll
+            for (int s = 0; s < 2; ++s) {
+                const bool ok = act[s] && tb + i < tv;
+                const size_t o = rowE + (tb + i) * sE + col[s];
+                xb[i][s] = ok ? to_f(pP[(tb + i) * sP + 32 * s]) : 0.f;
+                gb[i][s] = ok ? to_f(isq[s] ? gq[o] : gk[o]) : 0.f;
+            }
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int t = tb + i;
+            float dx[2] = {0.f, 0.f};
+            if (t < tv) {
+                float x[2], y[2], sq = 0.f, sk = 0.f, dq = 0.f, dkk = 0.f;
+#pragma unroll
+                for (int s = 0; s < 2; ++s) {
+                    float v = w[0][s] * pw[0][s];
+                    v = fmaf(w[1][s], pw[1][s], v);
+                    v = fmaf(w[2][s], pw[2][s], v);
+                    v = fmaf(w[3][s], xb[i][s], v);
+                    x[s] = v;
+                    y[s] = act[s] ? softplus(v) : 0.f;
+                    if (isq[s]) { sq = fmaf(y[s], y[s], sq); dq = fmaf(y[s], gb[i][s], dq); }
+                    else { sk = fmaf(y[s], y[s], sk); dkk = fmaf(y[s], gb[i][s], dkk); }
                 }
-                st<Tin>(gr.dP, tok_idx(b, t, h, c, T, H, C), acc);
-                const float dai = das[i * C + c];
-                for (int j = 0; j < K; ++j) {
-                    const int ts = t - K + 1 + j;
-                    if (ts >= 0) dwp[cc][j] = fmaf(dai, ld<Tin>(a.P, tok_idx(b, ts, h, c, T, H, C)), dwp[cc][j]);
+                const float rq = rsqrtf(warp_sum(sq) + a.eps), rk = rsqrtf(warp_sum(sk) + a.eps);
+                const float kq = rq * rq * warp_sum(dq), kk = rk * rk * warp_sum(dkk);
+#pragma unroll
+                for (int s = 0; s < 2; ++s) {
+                    const float r = isq[s] ? rq : rk, k2 = isq[s] ? kq : kk;
+                    dx[s] = act[s] ? (gb[i][s] - y[s] * k2) * r * sigm(x[s]) : 0.f;
                 }
+                if (t < t1)
+#pragma unroll
+                    for (int s = 0; s < 2; ++s) {
+                        dw[0][s] = fmaf(dx[s], pw[0][s], dw[0][s]);
+                        dw[1][s] = fmaf(dx[s], pw[1][s], dw[1][s]);
+                        dw[2][s] = fmaf(dx[s], pw[2][s], dw[2][s]);
+                        dw[3][s] = fmaf(dx[s], xb[i][s], dw[3][s]);
+                    }
+            }
+            const int tp = t - 3;
+            if (tp >= t0 && tp < te)
+#pragma unroll
+                for (int s = 0; s < 2; ++s)
+                    if (act[s]) {
+                        float v = w[0][s] * dx[s];
+                        v = fmaf(w[1][s], dxw[2][s], v);
+                        v = fmaf(w[2][s], dxw[1][s], v);
+                        v = fmaf(w[3][s], dxw[0][s], v);
+                        pdP[tp * sP + 32 * s] = from_f<Tin>(v);
+                    }
+#pragma unroll
+            for (int s = 0; s < 2; ++s) {
+                pw[0][s] = pw[1][s]; pw[1][s] = pw[2][s]; pw[2][s] = xb[i][s];
+                dxw[0][s] = dxw[1][s]; dxw[1][s] = dxw[2][s]; dxw[2][s] = dx[s];
             }
         }
-        // gates and beta of the block's own tokens
-        if (tid < E) {
-            const int e = tid;
-            const float sA = -expf(a.A_log[h * E + e]);
-            for (int i = 0; i < nt; ++i) {
-                const size_t o = tok_idx(b, t0 + i, h, e, T, H, E);
-                const float z = a.gate_in[o] + a.gate_bias[h * E + e];
-                const float dz = gr.dg[o] * sA * sigm(z);
-                gr.dgate_in[o] = dz;
-                gbp += dz;
-                gap = fmaf(gr.dg[o], sA * softplus(z), gap);
-            }
+    }
+#pragma unroll
+    for (int s = 0; s < 2; ++s)
+        if (act[s])
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+                if (j >= 4 - K) part[(off + lane + 32 * s) * K + j - (4 - K)] = dw[j][s];
+    // log gates (lane e sums over the run's tokens in order) and beta
+    if (lane < E) {
+        const int e = lane;
+        const float sA = -expf(a.A_log[h * E + e]), bias = a.gate_bias[h * E + e];
+        float gbp = 0.f, gap = 0.f;
+#pragma unroll 4
+        for (int t = t0; t < te; ++t) {
+            const size_t o = rowE + t * sE + e;
+            const float z = a.gate_in[o] + bias, dgv = gr.dg[o];
+            const float dz = dgv * sA * sigm(z);
+            gr.dgate_in[o] = dz;
+            gbp += dz;
+            gap = fmaf(dgv, sA * softplus(z), gap);
         }
-        if (a.beta_in && tid >= 64 && tid < 64 + nt) {
-            const size_t o = (size_t(b) * T + t0 + tid - 64) * H + h;
+        part[C * K + e] = gbp;
+        part[C * K + E + e] = gap;
+    }
+    if (a.beta_in)
+        for (int t = t0 + lane; t < te; t += 32) {
+            const size_t o = (size_t(b) * T + t) * H + h;
             const float s = sigm(a.beta_in[o]);
             gr.dbeta_in[o] = gr.dbeta[o] * s * (1.f - s);
         }
-        __syncthreads();
-    }
-    float* part = gr.part + ((size_t(b) * gridDim.x + seg) * H + h) * (size_t(C) * K + 2 * E);
-    for (int cc = 0; cc < 2; ++cc) {
-        const int c = tid + cc * kThreads;
-        if (c < C)
-            for (int j = 0; j < K; ++j) part[c * K + j] = dwp[cc][j];
-    }
-    if (tid < E) {
-        part[C * K + tid] = gbp;
-        part[C * K + E + tid] = gap;
-    }
+}
+
+template <typename Tin, typename Tg, bool VEC>
+__global__ void __launch_bounds__(kPrWarps * 32)
+prologue_bwd_kernel(const tla_prologue_args a, const PrologueGrads gr) {
+    const int seg = blockIdx.x, h = blockIdx.y, b = blockIdx.z, g = threadIdx.x >> 5;
+    const int t0 = seg * kSeg, t1 = min(a.T, t0 + kSeg);
+    const int C = 2 * a.dk + a.dv + 2 * a.E;
+    float* part = gr.part + ((size_t(b) * gridDim.x + seg) * a.H + h) * (size_t(C) * a.K + 2 * a.E);
+    if (g < 3) prologue_bwd_qkv<Tin, Tg, VEC>(a, gr, g, b, h, t0, t1, part);
+    else prologue_bwd_small<Tin, Tg>(a, gr, b, h, t0, t1, part);
 }
 
 // Fixed-order sums of the per-CTA partials: out[h][x] = sum_{b, seg} part[b][seg][h][x].
@@ -386,11 +665,16 @@ extern "C" tla_status tla_layer_prologue(const tla_prologue_args* a, void* strea
     if (st0 != TLA_OK) return st0;
     cudaStream_t s = (cudaStream_t)stream;
     const int C = 2 * a->dk + a->dv + 2 * a->E;
-    const size_t smem = (size_t(kFwdTok) * C + kFwdTok * 4) * sizeof(float);
-    dim3 grid((a->T + kFwdTok - 1) / kFwdTok, a->H, a->B);
+    dim3 grid((a->T + kFwdRun - 1) / kFwdRun, a->H, a->B);
+    const bool vec = (C % 4) == 0;   // every row and channel group starts on four channels
     prof_before("layer_prologue", s);
-    if (a->dtype == TLA_BF16) prologue_fwd_kernel<__nv_bfloat16><<<grid, kThreads, smem, s>>>(*a);
-    else prologue_fwd_kernel<float><<<grid, kThreads, smem, s>>>(*a);
+    if (a->dtype == TLA_BF16) {
+        if (vec) prologue_fwd_kernel<__nv_bfloat16, true><<<grid, kPrWarps * 32, 0, s>>>(*a);
+        else prologue_fwd_kernel<__nv_bfloat16, false><<<grid, kPrWarps * 32, 0, s>>>(*a);
+    } else {
+        if (vec) prologue_fwd_kernel<float, true><<<grid, kPrWarps * 32, 0, s>>>(*a);
+        else prologue_fwd_kernel<float, false><<<grid, kPrWarps * 32, 0, s>>>(*a);
+    }
     prof_after(s);
     return cuda_status(cudaGetLastError());
 }
@@ -425,20 +709,22 @@ extern "C" tla_status tla_layer_prologue_bwd(const tla_prologue_args* a, int gra
     cudaStream_t s = (cudaStream_t)stream;
     const int C = 2 * a->dk + a->dv + 2 * a->E;
     PrologueGrads gr{dq, dk, dv, dq2, dk2, dg, dbeta, dP, dgate_in, dbeta_in, (float*)workspace};
-    const size_t smem = (2 * size_t(kSub + 3) * C + 8 * (kSub + 3)) * sizeof(float);
     dim3 grid(n_segments(a), a->H, a->B);
+    const bool vec = (C % 4) == 0;
     prof_before("layer_prologue_bwd", s);
+#define TLA_PROLOGUE_BWD(TI, TG)                                                        \
+    do {                                                                                \
+        if (vec) prologue_bwd_kernel<TI, TG, true><<<grid, kPrWarps * 32, 0, s>>>(*a, gr); \
+        else prologue_bwd_kernel<TI, TG, false><<<grid, kPrWarps * 32, 0, s>>>(*a, gr);    \
+    } while (0)
     if (a->dtype == TLA_BF16) {
-        if (grad_dtype == TLA_BF16)
-            prologue_bwd_kernel<__nv_bfloat16, __nv_bfloat16><<<grid, kThreads, smem, s>>>(*a, gr);
-        else
-            prologue_bwd_kernel<__nv_bfloat16, float><<<grid, kThreads, smem, s>>>(*a, gr);
+        if (grad_dtype == TLA_BF16) TLA_PROLOGUE_BWD(__nv_bfloat16, __nv_bfloat16);
+        else TLA_PROLOGUE_BWD(__nv_bfloat16, float);
     } else {
-        if (grad_dtype == TLA_BF16)
-            prologue_bwd_kernel<float, __nv_bfloat16><<<grid, kThreads, smem, s>>>(*a, gr);
-        else
-            prologue_bwd_kernel<float, float><<<grid, kThreads, smem, s>>>(*a, gr);
+        if (grad_dtype == TLA_BF16) TLA_PROLOGUE_BWD(float, __nv_bfloat16);
+        else TLA_PROLOGUE_BWD(float, float);
     }
+#undef TLA_PROLOGUE_BWD
     prof_after(s);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return TLA_ERR_CUDA;

@@ -34,7 +34,8 @@ def close(name, got, ref, tol=1e-4, rounded=False):
     assert excess <= 0, f"{name}: exceeds the bound by {excess:.3e} (RMS {rms:.3e})"
 
 
-SHAPES = [(128, 128, 4, 4), (64, 64, 8, 3), (32, 128, 32, 1)]
+# the last shape has an odd channel count C (E odd): the scalar-access path of the prologue
+SHAPES = [(128, 128, 4, 4), (64, 64, 8, 3), (32, 128, 32, 1), (16, 32, 3, 2)]
 ARGS = ("P", "conv_w", "gate_in", "gate_bias", "A_log", "beta_in")
 
 
@@ -66,6 +67,27 @@ def test_prologue_backward(dtype, dk, dv, E, K):
                                    dk, dv, E)
     for n in ref:
         close(n, got[n], ref[n], rounded=(n == "dP" and dtype == "bf16"))
+
+
+@pytest.mark.parametrize("T", [1, 2, 5])
+def test_prologue_sequences_shorter_than_the_window(T):
+    """Fewer tokens than the convolution's K = 4 taps, forward and backward."""
+    dk, dv, E, K, B, H = 32, 32, 4, 4, 2, 2
+    x = inputs.layer_inputs(B, T, H, dk, dv, E, K, dtype="fp32", device="cuda", seed=T)
+    got = tla.layer_prologue(*(x[n] for n in ARGS), dk, dv, E)
+    gen = torch.Generator("cuda").manual_seed(T)
+    grads = {n: torch.randn(B, T, H, w, device="cuda", generator=gen)
+             for n, w in (("dq", dk), ("dk", dk), ("dv", dv), ("dq2", E), ("dk2", E), ("dg", E))}
+    grads["dbeta"] = torch.randn(B, T, H, device="cuda", generator=gen)
+    gotb = tla.layer_prologue_bwd(*(x[n] for n in ARGS), dk, dv, E, grads)
+    torch.cuda.synchronize()
+    ref = oracle.prologue(*(_np(x[n]) for n in ARGS), dk, dv, E)
+    for n in ("q", "k", "v", "q2", "k2", "g", "beta"):
+        close(n, got[n], ref[n])
+    refb = oracle.prologue_backward(*(_np(x[n]) for n in ARGS), {n: _np(t) for n, t in grads.items()},
+                                    dk, dv, E)
+    for n in refb:
+        close(n, gotb[n], refb[n])
 
 
 @pytest.mark.parametrize("zdtype", ["fp32", "bf16"])
