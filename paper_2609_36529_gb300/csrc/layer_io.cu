@@ -21,7 +21,7 @@ constexpr int kFwdRun = 128;   // tokens per CTA of the prologue forward
 constexpr int kSeg = 256;      // tokens per CTA of the prologue backward
 constexpr int kGateRows = 256; // (token, head) rows per CTA of the output gate
 
-__device__ __forceinline__ float sigm(float x) { return 1.f / (1.f + expf(-x)); }
+__device__ __forceinline__ float sigm(float x) { return __fdividef(1.f, 1.f + __expf(-x)); }
 __device__ __forceinline__ float softplus(float x) { return x > 20.f ? x : log1pf(expf(x)); }
 
 template <typename T> __device__ __forceinline__ float ld(const void* p, size_t i) {
@@ -241,15 +241,32 @@ __device__ __forceinline__ void prologue_fwd_small(const tla_prologue_args& a, i
         }
     }
     const int n = t1 - t0;
-    for (int idx = lane; idx < n * E; idx += 32) {   // log gates
-        const int i = idx / E, e = idx - i * E;
-        const size_t o = rowE + (t0 + i) * sE + e;
-        a.g[o] = -expf(a.A_log[h * E + e]) * softplus(a.gate_in[o] + a.gate_bias[h * E + e]);
+    for (int i0 = lane; i0 < n * E; i0 += 32 * 4) {   // log gates, four loads ahead
+        float z[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int idx = i0 + 32 * u, i = idx / E, e = idx - i * E;
+            z[u] = idx < n * E ? a.gate_in[rowE + (t0 + i) * sE + e] + a.gate_bias[h * E + e] : 0.f;
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int idx = i0 + 32 * u, i = idx / E, e = idx - i * E;
+            if (idx < n * E) a.g[rowE + (t0 + i) * sE + e] = -expf(a.A_log[h * E + e]) * softplus(z[u]);
+        }
     }
     if (a.beta_in)
-        for (int t = t0 + lane; t < t1; t += 32) {
-            const size_t o = (size_t(b) * T + t) * H + h;
-            a.beta[o] = sigm(a.beta_in[o]);
+        for (int tb = t0 + lane; tb < t1; tb += 32 * 4) {
+            float bi[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int t = tb + 32 * u;
+                bi[u] = t < t1 ? a.beta_in[(size_t(b) * T + t) * H + h] : 0.f;
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int t = tb + 32 * u;
+                if (t < t1) a.beta[(size_t(b) * T + t) * H + h] = sigm(bi[u]);
+            }
         }
 }
 
@@ -485,33 +502,69 @@ __device__ __forceinline__ void prologue_bwd_small(const tla_prologue_args& a, c
 #pragma unroll
             for (int j = 0; j < 4; ++j)
                 if (j >= 4 - K) part[(off + lane + 32 * s) * K + j - (4 - K)] = dw[j][s];
-    // log gates (lane e sums over the run's tokens in order) and beta
-    if (lane < E) {
-        const int e = lane;
+    // log gates: lane p * E + e takes gate e of tokens t0 + p, t0 + p + NP, ... (NP = 32 / E
+    // phases), eight tokens' loads at a time; the phases' sums are added in order after.
+    __shared__ float red[2][32];
+    const int NP = 32 / E, p = lane / E, e = lane - p * E;
+    float gbp = 0.f, gap = 0.f;
+    if (p < NP) {
         const float sA = -expf(a.A_log[h * E + e]), bias = a.gate_bias[h * E + e];
-        float gbp = 0.f, gap = 0.f;
-#pragma unroll 4
-        for (int t = t0; t < te; ++t) {
-            const size_t o = rowE + t * sE + e;
-            const float z = a.gate_in[o] + bias, dgv = gr.dg[o];
-            const float dz = dgv * sA * sigm(z);
-            gr.dgate_in[o] = dz;
-            gbp += dz;
-            gap = fmaf(dgv, sA * softplus(z), gap);
+        for (int tb = t0 + p; tb < te; tb += 8 * NP) {
+            float z[8], dgv[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                const int t = tb + i * NP;
+                const size_t o = rowE + t * sE + e;
+                z[i] = t < te ? a.gate_in[o] + bias : 0.f;
+                dgv[i] = t < te ? gr.dg[o] : 0.f;
+            }
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                const int t = tb + i * NP;
+                if (t < te) {
+                    const float dz = dgv[i] * sA * sigm(z[i]);
+                    gr.dgate_in[rowE + t * sE + e] = dz;
+                    gbp += dz;
+                    gap = fmaf(dgv[i], sA * softplus(z[i]), gap);
+                }
+            }
         }
-        part[C * K + e] = gbp;
-        part[C * K + E + e] = gap;
+    }
+    red[0][lane] = gbp;
+    red[1][lane] = gap;
+    __syncwarp();
+    if (lane < E) {
+        float sb = 0.f, sa = 0.f;
+        for (int q = 0; q < NP; ++q) {
+            sb += red[0][q * E + lane];
+            sa += red[1][q * E + lane];
+        }
+        part[C * K + lane] = sb;
+        part[C * K + E + lane] = sa;
     }
     if (a.beta_in)
-        for (int t = t0 + lane; t < te; t += 32) {
-            const size_t o = (size_t(b) * T + t) * H + h;
-            const float s = sigm(a.beta_in[o]);
-            gr.dbeta_in[o] = gr.dbeta[o] * s * (1.f - s);
+        for (int tb = t0 + lane; tb < te; tb += 32 * 8) {
+            float bi[8], db[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                const int t = tb + 32 * i;
+                const size_t o = (size_t(b) * T + t) * H + h;
+                bi[i] = t < te ? a.beta_in[o] : 0.f;
+                db[i] = t < te ? gr.dbeta[o] : 0.f;
+            }
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                const int t = tb + 32 * i;
+                if (t < te) {
+                    const float s = sigm(bi[i]);
+                    gr.dbeta_in[(size_t(b) * T + t) * H + h] = db[i] * s * (1.f - s);
+                }
+            }
         }
 }
 
 template <typename Tin, typename Tg, bool VEC>
-__global__ void __launch_bounds__(kPrWarps * 32)
+__global__ void __launch_bounds__(kPrWarps * 32, 4)
 prologue_bwd_kernel(const tla_prologue_args a, const PrologueGrads gr) {
     const int seg = blockIdx.x, h = blockIdx.y, b = blockIdx.z, g = threadIdx.x >> 5;
     const int t0 = seg * kSeg, t1 = min(a.T, t0 + kSeg);
