@@ -588,78 +588,130 @@ __global__ void reduce_partials_kernel(const float* __restrict__ part, int nblk,
     else dA[h * E + x - CK - E] = acc;
 }
 
-// Output gate: one warp per (token, head) row, kGateRows rows per CTA.
+// Output gate: one warp per (token, head) row, four channels per lane (dv <= 128 and a
+// multiple of 16, so every row starts on a 16-byte boundary), four consecutive rows'
+// loads issued before the first is used.
 template <typename To, typename Tz>
 __global__ void __launch_bounds__(kThreads)
 gate_fwd_kernel(const tla_gate_args a, long long rows) {
     const int dv = a.dv, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    for (long long r = blockIdx.x * (long long)kGateRows + warp; r < min(rows, (blockIdx.x + 1LL) * kGateRows);
-         r += kThreads / 32) {
-        const size_t base = size_t(r) * dv;
-        float ss = 0.f;
-        for (int c = lane; c < dv; c += 32) {
-            const float x = ld<To>(a.o, base + c);
-            ss = fmaf(x, x, ss);
+    const bool act = 4 * lane < dv;
+    float wn[4] = {0.f, 0.f, 0.f, 0.f};
+    if (act) ld4<true>(a.w_norm + 4 * lane, wn);
+    const long long r0 = blockIdx.x * (long long)kGateRows, r1 = min(rows, r0 + kGateRows);
+    const To* po = static_cast<const To*>(a.o) + 4 * lane;
+    const Tz* pz = static_cast<const Tz*>(a.z) + 4 * lane;
+    Tz* py = static_cast<Tz*>(a.y) + 4 * lane;
+    for (long long rb = r0 + warp * 4; rb < r1; rb += (kThreads / 32) * 4) {
+        float o[4][4], z[4][4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            if (act && rb + i < r1) {
+                ld4<true>(po + (rb + i) * dv, o[i]);
+                ld4<true>(pz + (rb + i) * dv, z[i]);
+            } else {
+#pragma unroll
+                for (int u = 0; u < 4; ++u) o[i][u] = z[i][u] = 0.f;
+            }
         }
 #pragma unroll
-        for (int o = 16; o >= 1; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
-        const float rr = rsqrtf(ss / dv + a.eps);
-        for (int c = lane; c < dv; c += 32)
-            st<Tz>(a.y, base + c, ld<To>(a.o, base + c) * rr * a.w_norm[c] * sigm(ld<Tz>(a.z, base + c)));
+        for (int i = 0; i < 4; ++i) {
+            float ss = 0.f;
+#pragma unroll
+            for (int u = 0; u < 4; ++u) ss = fmaf(o[i][u], o[i][u], ss);
+            const float rr = rsqrtf(warp_sum(ss) / dv + a.eps);
+            float y[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) y[u] = o[i][u] * rr * wn[u] * sigm(z[i][u]);
+            if (act && rb + i < r1) st4<true>(py + (rb + i) * dv, y);
+        }
     }
 }
 
+// Backward of the output gate over the rows [blk * rpb, (blk + 1) * rpb); the w_norm
+// gradient is summed per lane, then over the CTA's warps in order into part[blk][dv].
 template <typename To, typename Tz>
 __global__ void __launch_bounds__(kThreads)
-gate_bwd_kernel(const tla_gate_args a, long long rows, const void* dy, void* d_o, void* dz,
-                float* part) {
-    extern __shared__ float sm[];   // [kThreads / 32][dv] dw_norm partials per warp
+gate_bwd_kernel(const tla_gate_args a, long long rows, long long rpb, const void* dy, void* d_o,
+                void* dz, float* part) {
+    __shared__ float wsm[kThreads / 32][128];
     const int dv = a.dv, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    float* wp = sm + warp * dv;
-    for (int c = lane; c < dv; c += 32) wp[c] = 0.f;
-    for (long long r = blockIdx.x * (long long)kGateRows + warp; r < min(rows, (blockIdx.x + 1LL) * kGateRows);
-         r += kThreads / 32) {
-        const size_t base = size_t(r) * dv;
-        float ss = 0.f;
-        for (int c = lane; c < dv; c += 32) {
-            const float x = ld<To>(a.o, base + c);
-            ss = fmaf(x, x, ss);
+    const bool act = 4 * lane < dv;
+    float wn[4] = {0.f, 0.f, 0.f, 0.f}, wacc[4] = {0.f, 0.f, 0.f, 0.f};
+    if (act) ld4<true>(a.w_norm + 4 * lane, wn);
+    const long long r0 = blockIdx.x * rpb, r1 = min(rows, r0 + rpb);
+    const To* po = static_cast<const To*>(a.o) + 4 * lane;
+    const Tz* pz = static_cast<const Tz*>(a.z) + 4 * lane;
+    const Tz* pg = static_cast<const Tz*>(dy) + 4 * lane;
+    To* pdo = static_cast<To*>(d_o) + 4 * lane;
+    Tz* pdz = static_cast<Tz*>(dz) + 4 * lane;
+    const float inv_dv = 1.f / dv;
+    for (long long rb = r0 + warp * 4; rb < r1; rb += (kThreads / 32) * 4) {
+        float o[4][4], z[4][4], g[4][4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            if (act && rb + i < r1) {
+                ld4<true>(po + (rb + i) * dv, o[i]);
+                ld4<true>(pz + (rb + i) * dv, z[i]);
+                ld4<true>(pg + (rb + i) * dv, g[i]);
+            } else {
+#pragma unroll
+                for (int u = 0; u < 4; ++u) o[i][u] = z[i][u] = g[i][u] = 0.f;
+            }
         }
 #pragma unroll
-        for (int o = 16; o >= 1; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
-        const float rr = rsqrtf(ss / dv + a.eps);
-        float dot = 0.f;
-        for (int c = lane; c < dv; c += 32) {
-            const float nh = ld<To>(a.o, base + c) * rr, s = sigm(ld<Tz>(a.z, base + c));
-            const float g = ld<Tz>(dy, base + c);
-            const float dnh = g * a.w_norm[c] * s;
-            st<Tz>(dz, base + c, g * nh * a.w_norm[c] * s * (1.f - s));
-            wp[c] = fmaf(g * s, nh, wp[c]);
-            dot = fmaf(dnh, nh, dot);
-        }
+        for (int i = 0; i < 4; ++i) {
+            float ss = 0.f;
 #pragma unroll
-        for (int o = 16; o >= 1; o >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o);
-        for (int c = lane; c < dv; c += 32) {
-            const float nh = ld<To>(a.o, base + c) * rr, s = sigm(ld<Tz>(a.z, base + c));
-            const float dnh = ld<Tz>(dy, base + c) * a.w_norm[c] * s;
-            st<To>(d_o, base + c, rr * (dnh - nh * dot / dv));
+            for (int u = 0; u < 4; ++u) ss = fmaf(o[i][u], o[i][u], ss);
+            const float rr = rsqrtf(warp_sum(ss) * inv_dv + a.eps);
+            float nh[4], dnh[4], dzv[4], dot = 0.f;
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const float sg = sigm(z[i][u]);
+                nh[u] = o[i][u] * rr;
+                dnh[u] = g[i][u] * wn[u] * sg;
+                dzv[u] = g[i][u] * nh[u] * wn[u] * sg * (1.f - sg);
+                if (rb + i < r1) wacc[u] = fmaf(g[i][u] * sg, nh[u], wacc[u]);
+                dot = fmaf(dnh[u], nh[u], dot);
+            }
+            dot = warp_sum(dot) * inv_dv;
+            float dov[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) dov[u] = rr * (dnh[u] - nh[u] * dot);
+            if (act && rb + i < r1) {
+                st4<true>(pdz + (rb + i) * dv, dzv);
+                st4<true>(pdo + (rb + i) * dv, dov);
+            }
         }
     }
+    if (act)
+#pragma unroll
+        for (int u = 0; u < 4; ++u) wsm[warp][4 * lane + u] = wacc[u];
     __syncthreads();
     for (int c = threadIdx.x; c < dv; c += kThreads) {
         float acc = 0.f;
-        for (int w = 0; w < kThreads / 32; ++w) acc += sm[w * dv + c];
+        for (int w = 0; w < kThreads / 32; ++w) acc += wsm[w][c];
         part[size_t(blockIdx.x) * dv + c] = acc;
     }
 }
 
-__global__ void reduce_columns_kernel(const float* __restrict__ part, int nblk, int n,
-                                      float* __restrict__ out) {
-    const int c = blockIdx.x * blockDim.x + threadIdx.x;
-    if (c >= n) return;
+// Fixed-order column sums out[c] = sum_i part[i][c]: block of 8 warps per 32 columns,
+// warp w summing the rows i = w, w + 8, ...; the eight sums then added in order.
+__global__ void __launch_bounds__(256) reduce_columns_kernel(const float* __restrict__ part, int nblk,
+                                                             int n, float* __restrict__ out) {
+    __shared__ float sm[8][32];
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, c = blockIdx.x * 32 + lane;
     float acc = 0.f;
-    for (int i = 0; i < nblk; ++i) acc += part[size_t(i) * n + c];
-    out[c] = acc;
+    if (c < n)
+        for (int i = w; i < nblk; i += 8) acc += part[size_t(i) * n + c];
+    sm[w][lane] = acc;
+    __syncthreads();
+    if (w == 0 && c < n) {
+        float t = 0.f;
+        for (int j = 0; j < 8; ++j) t += sm[j][lane];
+        out[c] = t;
+    }
 }
 
 bool al16(const void* p) { return ((uintptr_t)p & 15) == 0; }
@@ -700,6 +752,16 @@ tla_status check_gate(const tla_gate_args* a) {
 int n_segments(const tla_prologue_args* a) { return (a->T + kSeg - 1) / kSeg; }
 long long gate_blocks(const tla_gate_args* a) {
     return ((long long)a->B * a->T * a->H + kGateRows - 1) / kGateRows;
+}
+// backward: at most 8 CTAs per SM of 152, each over a contiguous range of rows
+long long gate_bwd_rows_per_block(const tla_gate_args* a) {
+    const long long rows = (long long)a->B * a->T * a->H;
+    const long long per = (rows + 152 * 8 - 1) / (152 * 8);
+    return std::max(32LL, (per + 31) / 32 * 32);
+}
+long long gate_bwd_blocks(const tla_gate_args* a) {
+    const long long rows = (long long)a->B * a->T * a->H, rpb = gate_bwd_rows_per_block(a);
+    return (rows + rpb - 1) / rpb;
 }
 size_t prologue_part_bytes(const tla_prologue_args* a) {
     const int C = 2 * a->dk + a->dv + 2 * a->E;
@@ -811,7 +873,7 @@ extern "C" tla_status tla_output_gate(const tla_gate_args* a, void* stream) {
 
 extern "C" size_t tla_output_gate_bwd_workspace_bytes(const tla_gate_args* a) {
     if (check_gate(a) != TLA_OK) return 0;
-    return ((size_t)gate_blocks(a) * a->dv * sizeof(float) + 255) & ~size_t(255);
+    return ((size_t)gate_bwd_blocks(a) * a->dv * sizeof(float) + 255) & ~size_t(255);
 }
 
 extern "C" tla_status tla_output_gate_bwd(const tla_gate_args* a, const void* dy, void* d_o,
@@ -825,29 +887,29 @@ extern "C" tla_status tla_output_gate_bwd(const tla_gate_args* a, const void* dy
         for (const void* p : ptrs)
             if (!al16(p)) return TLA_ERR_INVALID_ARG;
     }
-    const long long nblk = gate_blocks(a);
+    const long long nblk = gate_bwd_blocks(a), rpb = gate_bwd_rows_per_block(a);
     if (!workspace || workspace_bytes < (size_t)nblk * a->dv * sizeof(float)) return TLA_ERR_WORKSPACE;
     cudaStream_t s = (cudaStream_t)stream;
     const long long rows = (long long)a->B * a->T * a->H;
-    const size_t smem = (kThreads / 32) * a->dv * sizeof(float);
     float* part = (float*)workspace;
+    const unsigned g = (unsigned)nblk;
     prof_before("output_gate_bwd", s);
     if (a->o_dtype == TLA_FP32) {
         if (a->dtype == TLA_FP32)
-            gate_bwd_kernel<float, float><<<(unsigned)nblk, kThreads, smem, s>>>(*a, rows, dy, d_o, dz, part);
+            gate_bwd_kernel<float, float><<<g, kThreads, 0, s>>>(*a, rows, rpb, dy, d_o, dz, part);
         else
-            gate_bwd_kernel<float, __nv_bfloat16><<<(unsigned)nblk, kThreads, smem, s>>>(*a, rows, dy, d_o, dz, part);
+            gate_bwd_kernel<float, __nv_bfloat16><<<g, kThreads, 0, s>>>(*a, rows, rpb, dy, d_o, dz, part);
     } else {
         if (a->dtype == TLA_FP32)
-            gate_bwd_kernel<__nv_bfloat16, float><<<(unsigned)nblk, kThreads, smem, s>>>(*a, rows, dy, d_o, dz, part);
+            gate_bwd_kernel<__nv_bfloat16, float><<<g, kThreads, 0, s>>>(*a, rows, rpb, dy, d_o, dz, part);
         else
-            gate_bwd_kernel<__nv_bfloat16, __nv_bfloat16><<<(unsigned)nblk, kThreads, smem, s>>>(*a, rows, dy, d_o, dz, part);
+            gate_bwd_kernel<__nv_bfloat16, __nv_bfloat16><<<g, kThreads, 0, s>>>(*a, rows, rpb, dy, d_o, dz, part);
     }
     prof_after(s);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return TLA_ERR_CUDA;
     prof_before("output_gate_reduce", s);
-    reduce_columns_kernel<<<(a->dv + 127) / 128, 128, 0, s>>>(part, (int)nblk, a->dv, dw_norm);
+    reduce_columns_kernel<<<(a->dv + 31) / 32, 256, 0, s>>>(part, (int)nblk, a->dv, dw_norm);
     prof_after(s);
     return cuda_status(cudaGetLastError());
 }
