@@ -269,6 +269,17 @@ tla_status tla_output_gate_bwd(const tla_gate_args *a, const void *dy, void *d_o
 tla_status tla_last_device_status(void *stream);
 
 /*
+ * Self-test of the failure-detection path.  Launches one CTA whose threads wait on
+ * an mbarrier that nothing ever arrives at, with the same bounded wait the
+ * tensor-core kernels use but a limit of `timeout_ns` nanoseconds of GPU global
+ * time (1 .. 10^9).  The wait expires, the CTA records TLA_ERR_TIMEOUT in the
+ * device error word and returns, so the next tla_last_device_status() reports
+ * TLA_ERR_TIMEOUT and the context stays usable.  Returns TLA_ERR_INVALID_ARG for a
+ * limit outside the range, else the launch status.
+ */
+tla_status tla_selftest_bounded_wait(unsigned long long timeout_ns, void *stream);
+
+/*
  * Kernel timing (tracing).  After tla_profile_begin(), every kernel the library
  * launches is bracketed by CUDA events recorded on its launch stream (event
  * objects are created on first use and reused; no device memory is allocated).

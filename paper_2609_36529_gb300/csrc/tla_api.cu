@@ -8,6 +8,7 @@
 
 #include "common.cuh"
 #include "internal.h"
+#include "sm100.cuh"
 
 namespace tla {
 
@@ -46,6 +47,19 @@ static tla_status validate(const tla_problem* p) {
     return TLA_OK;
 }
 
+
+// Waits on a barrier that nothing arrives at: the bounded wait must give up after
+// timeout_ns and leave its record in the error word.
+static __global__ void selftest_wait_kernel(unsigned long long timeout_ns, int* err) {
+    __shared__ __align__(8) uint64_t bar;
+    if (threadIdx.x == 0) {
+        sm100::mbar_init(&bar, 1);
+        sm100::fence_barrier_init();
+    }
+    __syncthreads();
+    const bool ok = sm100::mbar_wait(&bar, 0, timeout_ns);
+    if (!ok && threadIdx.x == 0) record_device_error(err, TLA_ERR_TIMEOUT);
+}
 
 // Address of the error word on the current device (looked up once per device).
 static int* device_error_word() {
@@ -292,6 +306,14 @@ const char* tla_status_string(int status) {
         case TLA_ERR_WORKSPACE: return "TLA_ERR_WORKSPACE";
         default: return "TLA_UNKNOWN_STATUS";
     }
+}
+
+tla_status tla_selftest_bounded_wait(unsigned long long timeout_ns, void* stream) {
+    if (timeout_ns < 1 || timeout_ns > 1000000000ull) return TLA_ERR_INVALID_ARG;
+    int* err = device_error_word();
+    if (!err) return TLA_ERR_CUDA;
+    selftest_wait_kernel<<<1, 32, 0, (cudaStream_t)stream>>>(timeout_ns, err);
+    return cudaGetLastError() == cudaSuccess ? TLA_OK : TLA_ERR_CUDA;
 }
 
 tla_status tla_last_device_status(void* stream) {

@@ -24,7 +24,7 @@ EXPORTED = ("tla_fwd_workspace_bytes", "tla_chunk_fwd", "tla_bwd_workspace_bytes
             "tla_version", "tla_chunk_fwd_noalloc", "tla_noalloc_scratch_bytes",
             "tla_layer_prologue", "tla_layer_prologue_bwd_workspace_bytes",
             "tla_layer_prologue_bwd", "tla_output_gate", "tla_output_gate_bwd_workspace_bytes",
-            "tla_output_gate_bwd")
+            "tla_output_gate_bwd", "tla_selftest_bounded_wait")
 
 
 class TlaError(RuntimeError):
@@ -89,6 +89,8 @@ def lib():
         L.tla_status_string.restype = ctypes.c_char_p
         L.tla_last_device_status.argtypes = [vp]
         L.tla_last_device_status.restype = i
+        L.tla_selftest_bounded_wait.argtypes = [ctypes.c_ulonglong, vp]
+        L.tla_selftest_bounded_wait.restype = i
         L.tla_version.restype = ctypes.c_char_p
         L.tla_chunk_fwd_noalloc.argtypes = [P, vp]
         L.tla_chunk_fwd_noalloc.restype = i
@@ -266,6 +268,11 @@ def tla_decode_step(state, q, k, v, q2, k2, g, beta=None, use_delta=True, o=None
 
 def tla_last_device_status() -> int:
     return lib().tla_last_device_status(_stream())
+
+
+def tla_selftest_bounded_wait(timeout_ns: int) -> None:
+    """Launch the failure-detection self-test (a bounded wait that must expire)."""
+    _check("tla_selftest_bounded_wait", lib().tla_selftest_bounded_wait(int(timeout_ns), _stream()))
 
 
 def tla_version() -> str:

@@ -191,3 +191,9 @@ def test_layer_io_validation(tla):
     need = L.tla_output_gate_bwd_workspace_bytes(ctypes.byref(g))
     assert need > 0
     assert L.tla_output_gate_bwd(ctypes.byref(g), f, f, f, f, None, need, None) == -5
+
+
+def test_selftest_limit_checked_on_host(tla):
+    L = tla.lib()
+    for bad in (0, 1_000_000_001, 2 ** 63):
+        assert L.tla_selftest_bounded_wait(bad, None) == -1
