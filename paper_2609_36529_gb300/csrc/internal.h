@@ -29,9 +29,9 @@ struct FwdPlan {
     size_t BT;           // bf16 [B,H,NT,4,64,64] A^T, T^T hi/lo (tensor-core backward)
     int tcb;             // 1: the backward recurrence runs on tensor cores
     int ck_tiles;        // 1: state checkpoints (forward S, backward dS) are stored as bf16
-                         //    hi/lo pairs in the chunk-gradient kernel's operand layout:
-                         //    per (b,h,chunk,e) a [dk][dv] hi tile then a lo tile, 128-byte
-                         //    swizzled K-major (same 4 bytes per element as fp32); U, Res
+                         //    hi/lo pairs: per (b,h,chunk,e) a row-major [dk][dv] hi matrix
+                         //    then the lo matrix (same 4 bytes per element as fp32), written
+                         //    and read by TMA (tma_host.h: make_ckpt_map); U, Res
                          //    and the backward's dU, -dRes are then token tiles: per
                          //    (b,h,chunk) 64 rows x dv bf16 hi then lo, SW128 K-major 64-row
                          //    blocks, rows past T zero

@@ -111,6 +111,26 @@ __device__ __forceinline__ void tma_load_4d(void* dst, const CUtensorMap* map, u
         : "memory");
 }
 
+// Hint: bring the box at the given coordinates of a 4-d tensor map into L2 (no
+// shared memory, no barrier); a later TMA load of the same box then hits L2.
+__device__ __forceinline__ void tma_prefetch_l2_4d(const CUtensorMap* map, int x, int y, int z, int w) {
+    asm volatile("cp.async.bulk.prefetch.tensor.4d.L2.global.tile [%0, {%1, %2, %3, %4}];" ::"l"(
+                     reinterpret_cast<uint64_t>(map)),
+                 "r"(x), "r"(y), "r"(z), "r"(w)
+                 : "memory");
+}
+
+// TMA tensor store shared -> global of the box at (x, y, z, w) of a 4-d tensor map, in the
+// issuing thread's current bulk async-group (x * element size a multiple of 16 bytes).
+__device__ __forceinline__ void tma_store_4d(const CUtensorMap* map, const void* src, int x, int y,
+                                             int z, int w) {
+    asm volatile(
+        "cp.async.bulk.tensor.4d.global.shared::cta.bulk_group [%0, {%1, %2, %3, %4}], [%5];" ::"l"(
+            reinterpret_cast<uint64_t>(map)),
+        "r"(x), "r"(y), "r"(z), "r"(w), "r"(smem_u32(src))
+        : "memory");
+}
+
 // Plain bulk copy global -> shared (16-byte aligned addresses, size multiple of 16).
 __device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
     asm volatile(
@@ -119,6 +139,15 @@ __device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t b
         "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(smem_u32(bar))
         : "memory");
 }
+
+// Close the issuing thread's current bulk async-group (TMA stores).
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// Wait until every committed bulk store of this thread has read its shared-memory source
+// (the source may then be overwritten) / has completed its global writes.
+__device__ __forceinline__ void bulk_wait_read_all() {
+    asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+}
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
 // Hint: bring `bytes` of global memory into L2 (16-byte aligned, size multiple of 16).
 __device__ __forceinline__ void bulk_prefetch_l2(const void* src, uint32_t bytes) {
@@ -150,6 +179,10 @@ __device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
 // in 32-45, the fixed version bits 46-48 = 0b001, base offset 0 (atoms are
 // 1024-byte aligned), swizzle mode in 61-63 (2 = 128-byte swizzle).
 constexpr uint64_t kSwizzle128 = 2;
+// Swizzle-mode code of a row width of 32, 64 or 128 bytes.
+__host__ __device__ constexpr uint64_t swizzle_code(int width_bytes) {
+    return width_bytes == 128 ? 2u : width_bytes == 64 ? 4u : 6u;
+}
 __device__ __forceinline__ uint64_t smem_desc(uint32_t saddr, uint32_t lbo, uint32_t sbo,
                                               uint64_t swizzle = kSwizzle128) {
     return uint64_t((saddr & 0x3FFFF) >> 4) | (uint64_t((lbo >> 4) & 0x3FFF) << 16) |

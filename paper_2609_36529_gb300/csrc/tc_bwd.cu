@@ -20,7 +20,10 @@
 //           pre-scaled by gamma^C of the previous chunk.
 // Layout of the M=64 products in TMEM: row r sits on lane 32 * (r / 16) + r % 16,
 // so lanes 0-15 of each warp own the row work and lanes 16-31 prepare dO.
-// Precision, TMA prefetch and bounded waits as in the forward kernel.
+// Precision, TMA prefetch, bounded waits, the slice-block layout of the state
+// operand and the TMA-stored checkpoints as in the forward kernel.
+#include <cstring>
+
 #include "common.cuh"
 #include "internal.h"
 #include "sm100.cuh"
@@ -54,7 +57,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                          const __grid_constant__ CUtensorMap map_q,
                          const __grid_constant__ CUtensorMap map_do,
-                         const __grid_constant__ CUtensorMap map_bt, const TcBwdArgs p) {
+                         const __grid_constant__ CUtensorMap map_bt,
+                         const __grid_constant__ CUtensorMap map_ck, const TcBwdArgs p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
@@ -63,7 +67,7 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     uint8_t* sKQ = sm;                       // 2 blocks x [K rows | Q rows] x 128 B
     uint8_t* sBT = sKQ + 4 * kBoxBytes;      // A^T hi, A^T lo, T^T hi, T^T lo (64 x 64 each)
     uint8_t* sReg = sBT + 4 * kBoxBytes;     // NE * 512 bytes, reused:
-    uint8_t* sDh = sReg;                     //   dS' [dk][NE] hi / lo, MN-major (MMA-A')
+    uint8_t* sDh = sReg;                     //   dS' hi / lo: E blocks [dk][TV] (MMA-A')
     uint8_t* sDl = sReg + NE * 256;
     uint8_t* sUh = sReg;                     //   dU^T [TV][64] hi / lo (MMA-B')
     uint8_t* sUl = sReg + TV * 128;
@@ -81,6 +85,7 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     const int n0 = nb * TV;
     const int T = p.T, H = p.H, dv = p.dv, NT = p.NT;
     const uint32_t tcols = (2 * NE + TV <= 256) ? 256u : 512u;
+    constexpr uint64_t kSwz = swizzle_code(2 * TV);
     // token batch, first token, tokens, chunks and first chunk (in the workspaces) of this state
     int b = sb, tbeg = 0, tlen = T, nct = NT, cb = 0;
     if (p.dtab) {
@@ -113,6 +118,7 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         tma_prefetch_desc(&map_q);
         tma_prefetch_desc(&map_do);
         tma_prefetch_desc(&map_bt);
+        if (p.ck_tiles) tma_prefetch_desc(&map_ck);
     }
     tc_fence_before();
     __syncthreads();
@@ -161,17 +167,10 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                 tmem_wait_ld();
             }
 #pragma unroll
-            for (int n = 0; n < TV; n += 8) st8_split(sDh, sDl, sw128_offset(d, e * TV + n, kDk), v + n);
-            {
+            for (int n = 0; n < TV; n += 8) st8_split(sDh, sDl, e * blk_bytes<TV>() + blk_offset<TV>(d, n), v + n);
+            if (!p.ck_tiles) {   // fp32 checkpoint (tile checkpoints: issue_ckpt)
                 const size_t slab = (((size_t(b) * H + h) * NT + cb + c) * E + e) * kDk * dv;
-                if (p.ck_tiles) {   // bf16 hi/lo tiles in the gradient kernel's layout
-                    uint8_t* hi = reinterpret_cast<uint8_t*>(p.dSck + slab);
-                    uint8_t* lo = hi + kDk * dv * 2;
-#pragma unroll
-                    for (int n = 0; n < TV; n += 8) st8_split(hi, lo, sw128_offset(d, n0 + n, kDk), v + n);
-                } else {
-                    store_f32_row(p.dSck + slab + size_t(d) * dv + n0, v, TV);
-                }
+                store_f32_row(p.dSck + slab + size_t(d) * dv + n0, v, TV);
             }
             const float g = gc[e];
 #pragma unroll
@@ -180,6 +179,14 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             for (int j = 0; j < TV; j += 16) tmem_st16(tmem_lane_addr(tS, warp, e * TV + j), v + j);
         }
         tmem_wait_st();
+    };
+
+    // Checkpoint of dS' at the end of chunk c: this CTA's columns of the slice blocks,
+    // stored by TMA (thread 0, once prepare(c) is complete in shared memory).
+    auto issue_ckpt = [&](int c) {
+        if (!p.ck_tiles) return;
+        tma_store_4d(&map_ck, sDh, n0, 0, ((b * H + h) * NT + cb + c) * E, 0);   // [hi|lo][E][dk][TV]
+        bulk_commit();
     };
 
     bool failed = false;
@@ -206,6 +213,12 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         const float* ae = cf;
         const float* be = cf + 64 * E;
         const float* we = cf + 128 * E;
+        // previous chunk's key and query boxes into L2 (their TMA load waits for MMA-C')
+        if (tid == 0 && c > 0)
+            for (int j = 0; j < 2; ++j) {
+                tma_prefetch_l2_4d(&map_k, 64 * j, h, tbeg + (c - 1) * 64, b);
+                tma_prefetch_l2_4d(&map_q, 64 * j, h, tbeg + (c - 1) * 64, b);
+            }
         bool ok = mbar_wait(&bar_kq, it & 1);
         if (__syncthreads_or(!ok)) { failed = true; break; }
         tc_fence_after();
@@ -237,9 +250,10 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             for (int ks = 0; ks < kDk / 16; ++ks) {
                 const int blk = ks >> 2, kk = (ks & 3) * 16;
                 const uint64_t ad = smem_desc(smem_u32(sKQ) + blk * 2 * kBoxBytes + kk * 2, 16, 1024);
-                umma_bf16(tP, ad, smem_desc(smem_u32(sDh) + ks * 2048, kDk * 128, 1024), ida,
+                const uint32_t ko = ks * 32 * TV;   // 16 rows of the slice blocks per K step
+                umma_bf16(tP, ad, smem_desc(smem_u32(sDh) + ko, blk_bytes<TV>(), 16 * TV, kSwz), ida,
                           ks > 0 ? 1u : 0u);
-                umma_bf16(tP, ad, smem_desc(smem_u32(sDl) + ks * 2048, kDk * 128, 1024), ida, 1u);
+                umma_bf16(tP, ad, smem_desc(smem_u32(sDl) + ko, blk_bytes<TV>(), 16 * TV, kSwz), ida, 1u);
             }
             const uint32_t id0 = idesc_bf16_f32(64, TV, 0, 0);
 #pragma unroll
@@ -249,10 +263,12 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                 umma_bf16(tY, smem_desc(smem_u32(sBT) + kBoxBytes + ks * 32, 16, 1024), bd, id0, 1u);
             }
             umma_commit(&bar_mma);
+            issue_ckpt(c);   // the dS' blocks were completed by prepare(c) before the last barrier
         }
         pending_mma = 1;
         ok = mbar_wait(&bar_mma, mma_phase);
         mma_phase ^= 1;
+        if (tid == 0) bulk_wait_read_all();   // the dS' blocks are rewritten next
         if (__syncthreads_or(!ok)) { failed = true; break; }
         pending_mma = 0;
         tc_fence_after();
@@ -393,6 +409,7 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         record_device_error(p.err, TLA_ERR_TIMEOUT);
         if (pending_mma) mbar_wait(&bar_mma, mma_phase ^ 1);
     }
+    if (tid == 0) bulk_wait_all();
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -409,12 +426,16 @@ template <int TV>
 cudaError_t launch_tv(const tla_problem& p, const FwdPlan& fp, const char* fws, const BwdPlan& bp,
                       char* bws, const void* dO, const float* dht, void* dv, float* dh0, int* err,
                       cudaStream_t s) {
-    CUtensorMap mk, mq, mo, mb;
+    CUtensorMap mk, mq, mo, mb, mc;
     const int NT = fp.NT;
     if (!make_token_map(&mk, p.k, p.B, p.T, p.H, kDk, 64, 64, true) ||
         !make_token_map(&mq, p.q, p.B, p.T, p.H, kDk, 64, 64, true) ||
         !make_token_map(&mo, dO, p.B, p.T, p.H, p.dv, TV, 64, false) ||
         !make_matrix_map(&mb, fws + fp.BT, (long long)p.B * p.H * NT * 256, 64, 64, 64))
+        return cudaErrorInvalidValue;
+    memset(&mc, 0, sizeof(mc));   // unused unless the checkpoints are tiles
+    if (fp.ck_tiles &&
+        !make_ckpt_map(&mc, bws + bp.dS, (long long)p.B * p.H * NT * p.E, p.dv, TV, p.E, 2 * TV))
         return cudaErrorInvalidValue;
     TcBwdArgs a;
     a.coef = (const float*)(fws + fp.coef);
@@ -434,7 +455,7 @@ cudaError_t launch_tv(const tla_problem& p, const FwdPlan& fp, const char* fws, 
     cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     dim3 grid(p.dv / TV, p.H, fp.nseq);
     prof_before("bwd_recurrence_tc", s);
-    kern<<<grid, kThreads, smem, s>>>(mk, mq, mo, mb, a);
+    kern<<<grid, kThreads, smem, s>>>(mk, mq, mo, mb, mc, a);
     prof_after(s);
     return cudaGetLastError();
 }

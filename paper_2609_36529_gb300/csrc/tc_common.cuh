@@ -39,6 +39,22 @@ __device__ __forceinline__ void st_split(uint8_t* tile_hi, uint8_t* tile_lo, uin
 }
 
 
+// State operand blocks.  For a block of TV value columns, each slice e of the state
+// (or of its gradient) is a [128 rows][TV] bf16 block of 256 * TV bytes whose rows
+// are 2 * TV bytes wide, with the tensor cores' swizzle of that width (16-byte chunks
+// XOR-ed with the row's position in its 8-row group: 32-, 64- or 128-byte swizzle for
+// TV = 16, 32, 64), which is also the shared-memory layout of a TMA box of TV columns
+// with that swizzle.  The recurrences use the blocks of all slices as the MN-major
+// operand [dk][E * TV] (one swizzle atom of TV columns per slice) and store each
+// block by TMA into the row-major checkpoint of its value columns.
+template <int TV>
+__host__ __device__ __forceinline__ uint32_t blk_offset(int row, int col) {
+    const uint32_t o = uint32_t(row) * (2 * TV) + uint32_t(col) * 2;
+    return o ^ (((o >> 7) & (TV / 8 - 1)) << 4);
+}
+template <int TV>
+__host__ __device__ constexpr uint32_t blk_bytes() { return 256u * TV; }
+
 // Token tile of one chunk: 64 rows x dv as bf16 hi (64*dv*2 bytes) then bf16 lo, each in
 // SW128 K-major 64-row blocks of 64 columns -- the operand layout of the chunk-gradient
 // kernel, which copies a tile into shared memory as is.  Writes columns n0..n0+cnt of row r

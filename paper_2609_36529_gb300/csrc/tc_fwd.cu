@@ -23,12 +23,16 @@
 // accuracy: with a single bf16 rounding of those operands the error of o and of
 // the state reaches the 2e-2 x RMS parity bound.
 // The state and Ut operands are stored MN-major (one row per thread, 16-byte
-// stores), so each thread writes the TMEM row it read.  Key, query, value
+// stores), so each thread writes the TMEM row it read.  The state operand is kept
+// as one swizzled [dk][TV] block per slice (tc_common.cuh); a chunk's checkpoint
+// leaves shared memory as one TMA tensor store of those blocks into the row-major
+// [dk][dv] hi and lo matrices of its slices (tma_host.h).  Key, query, value
 // tiles, the [T; A T] tiles and the coefficient block arrive by TMA, prefetched
 // one chunk ahead as soon as their buffers are free.  Every mbarrier wait is
 // bounded by the GPU global timer; on expiry the CTA records TLA_ERR_TIMEOUT and
 // leaves after a bounded drain of its outstanding work.
 #include <algorithm>
+#include <cstring>
 
 #include "common.cuh"
 #include "internal.h"
@@ -63,7 +67,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                          const __grid_constant__ CUtensorMap map_q,
                          const __grid_constant__ CUtensorMap map_v,
-                         const __grid_constant__ CUtensorMap map_a2, const TcFwdArgs p) {
+                         const __grid_constant__ CUtensorMap map_a2,
+                         const __grid_constant__ CUtensorMap map_ck, const TcFwdArgs p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
@@ -72,7 +77,7 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     uint8_t* sKQ = sm;                         // 2 blocks x [K rows 0-63 | Q rows 64-127] x 128 B
     uint8_t* sA2 = sKQ + 4 * kBoxBytes;        // [T; A T] 128 x 64 bf16: hi tile, lo tile
     uint8_t* sReg = sA2 + 4 * kBoxBytes;       // shared region, NE * 512 bytes:
-    uint8_t* sSh = sReg;                       //   S_all [dk][NE] hi, MN-major (MMA-A operand)
+    uint8_t* sSh = sReg;                       //   S_all hi: E blocks [dk][TV] (MMA-A operand)
     uint8_t* sSl = sReg + NE * 256;            //   S_all lo
     uint8_t* sRh = sReg;                       //   Res^T [TV][64] hi, lo (after MMA-A)
     uint8_t* sRl = sReg + TV * 128;
@@ -89,6 +94,7 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     const int n0 = nb * TV;
     const int T = p.T, H = p.H, dv = p.dv, NT = p.NT;
     const uint32_t tcols = (2 * NE <= 256) ? 256u : 512u;
+    constexpr uint64_t kSwz = swizzle_code(2 * TV);
     // token batch, first token, tokens, chunks and first chunk (in the workspace) of this state
     int b = sb, tbeg = 0, tlen = T, nct = NT, cb = 0;
     if (p.dtab) {
@@ -118,6 +124,7 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         tma_prefetch_desc(&map_q);
         tma_prefetch_desc(&map_v);
         tma_prefetch_desc(&map_a2);
+        if (p.save && p.ck_tiles) tma_prefetch_desc(&map_ck);
     }
     tc_fence_before();
     __syncthreads();
@@ -165,8 +172,15 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                 tmem_wait_ld();
             }
 #pragma unroll
-            for (int n = 0; n < TV; n += 8) st8_split(sSh, sSl, sw128_offset(d, e * TV + n, kDk), v + n);
+            for (int n = 0; n < TV; n += 8) st8_split(sSh, sSl, e * blk_bytes<TV>() + blk_offset<TV>(d, n), v + n);
         }
+    };
+    // Checkpoint of S_{[c]} (bf16 hi/lo) for the backward: this CTA's columns of the
+    // slice blocks, stored by TMA (thread 0, after the operand is complete).
+    auto issue_ckpt = [&](int c) {
+        if (!(p.save && p.ck_tiles)) return;
+        tma_store_4d(&map_ck, sSh, n0, 0, ((b * H + h) * NT + cb + c) * E, 0);   // [hi|lo][E][dk][TV]
+        bulk_commit();
     };
     // Row d of S_{[c]}: checkpoint for the backward, and the gamma^C_c-scaled copy in
     // TMEM that chunk c's state update accumulates onto.  Runs while MMA-A(c) executes.
@@ -193,16 +207,9 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                 for (int j = 0; j < TV; j += 16) tmem_ld16(tmem_lane_addr(tS, warp, e * TV + j), v + j);
                 tmem_wait_ld();
             }
-            if (p.save) {
+            if (p.save && !p.ck_tiles) {   // fp32 checkpoint (tile checkpoints: issue_ckpt)
                 const size_t slab = (((size_t(b) * H + h) * NT + cb + c) * E + e) * kDk * dv;
-                if (p.ck_tiles) {   // bf16 hi/lo tiles in the gradient kernel's layout
-                    uint8_t* hi = reinterpret_cast<uint8_t*>(p.Sck + slab);
-                    uint8_t* lo = hi + kDk * dv * 2;
-#pragma unroll
-                    for (int n = 0; n < TV; n += 8) st8_split(hi, lo, sw128_offset(d, n0 + n, kDk), v + n);
-                } else {
-                    store_f32_row(p.Sck + slab + size_t(d) * dv + n0, v, TV);
-                }
+                store_f32_row(p.Sck + slab + size_t(d) * dv + n0, v, TV);
             }
             const float g = gc[e];
 #pragma unroll
@@ -219,9 +226,12 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         for (int ks = 0; ks < kDk / 16; ++ks) {
             const int blk = ks >> 2, kk = (ks & 3) * 16;
             const uint64_t ad = smem_desc(smem_u32(sKQ) + blk * 2 * kBoxBytes + kk * 2, 16, 1024);
-            umma_bf16(tP, ad, smem_desc(smem_u32(sSh) + ks * 2048, kDk * 128, 1024), idesc,
+            // B = the slice blocks: 16 rows (two 8-row groups) per K step, one TV-column
+            // swizzle atom per slice
+            const uint32_t ko = ks * 32 * TV;
+            umma_bf16(tP, ad, smem_desc(smem_u32(sSh) + ko, blk_bytes<TV>(), 16 * TV, kSwz), idesc,
                       ks > 0 ? 1u : 0u);
-            umma_bf16(tP, ad, smem_desc(smem_u32(sSl) + ks * 2048, kDk * 128, 1024), idesc, 1u);
+            umma_bf16(tP, ad, smem_desc(smem_u32(sSl) + ko, blk_bytes<TV>(), 16 * TV, kSwz), idesc, 1u);
         }
         umma_commit(&bar_mma);
     };
@@ -243,7 +253,10 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         if (__syncthreads_or(!ok)) failed = true;
         tc_fence_after();
         if (!failed) {
-            if (tid == 0) issue_mma_a();
+            if (tid == 0) {
+                issue_mma_a();
+                issue_ckpt(0);
+            }
             pending_mma = 1;
             finish_state(0, true);
         }
@@ -255,9 +268,18 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         const float* ae = cf;
         const float* be = cf + 64 * E;
         const float* we = cf + 128 * E;
-        // ---- wait for MMA-A(c) (issued at the end of the previous step)
+        // next chunk's key and query boxes into L2: their TMA load is issued only once
+        // MMA-C(c) has released the tile, and then waits on the chain
+        if (tid == 0 && c + 1 < nct)
+            for (int j = 0; j < 2; ++j) {
+                tma_prefetch_l2_4d(&map_k, 64 * j, h, tbeg + (c + 1) * 64, b);
+                tma_prefetch_l2_4d(&map_q, 64 * j, h, tbeg + (c + 1) * 64, b);
+            }
+        // ---- wait for MMA-A(c) (issued at the end of the previous step); the operand
+        // region is rewritten next, so the checkpoint copies must have read it
         bool ok = mbar_wait(&bar_mma, mma_phase);
         mma_phase ^= 1;
+        if (tid == 0) bulk_wait_read_all();
         tc_fence_before();
         if (__syncthreads_or(!ok)) { failed = true; break; }
         pending_mma = 0;
@@ -403,7 +425,10 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             ok = mbar_wait(&bar_kq, (c + 1) & 1);
             if (__syncthreads_or(!ok)) { failed = true; break; }
             tc_fence_after();
-            if (tid == 0) issue_mma_a();
+            if (tid == 0) {
+                issue_mma_a();
+                issue_ckpt(c + 1);
+            }
             pending_mma = 1;
             finish_state(c + 1, false);
         } else if (p.ht) {
@@ -426,6 +451,7 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             if (pending_mma) mbar_wait(&bar_mma, mma_phase ^ 1);
         }
     }
+    if (tid == 0) bulk_wait_all();
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -441,12 +467,16 @@ size_t tc_fwd_smem(int E) {
 template <int TV>
 cudaError_t launch_tv(const tla_problem& p, const FwdPlan& fp, char* ws, int save, int* err,
                       cudaStream_t s) {
-    CUtensorMap mk, mq, mv, ma;
+    CUtensorMap mk, mq, mv, ma, mc;
     const int NT = fp.NT;
     if (!make_token_map(&mk, p.k, p.B, p.T, p.H, kDk, 64, 64, true) ||
         !make_token_map(&mq, p.q, p.B, p.T, p.H, kDk, 64, 64, true) ||
         !make_token_map(&mv, p.v, p.B, p.T, p.H, p.dv, TV, 64, false) ||
         !make_matrix_map(&ma, ws + fp.A2, (long long)p.B * p.H * NT * 256, 64, 64, 128))
+        return cudaErrorInvalidValue;
+    memset(&mc, 0, sizeof(mc));   // unused unless tile checkpoints are saved
+    if (save && fp.ck_tiles &&
+        !make_ckpt_map(&mc, ws + fp.S, (long long)p.B * p.H * NT * p.E, p.dv, TV, p.E, 2 * TV))
         return cudaErrorInvalidValue;
     TcFwdArgs a;
     a.coef = (const float*)(ws + fp.coef);
@@ -466,7 +496,7 @@ cudaError_t launch_tv(const tla_problem& p, const FwdPlan& fp, char* ws, int sav
     cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     dim3 grid(p.dv / TV, p.H, fp.nseq);
     prof_before("fwd_recurrence_tc", s);
-    kern<<<grid, kThreads, smem, s>>>(mk, mq, mv, ma, a);
+    kern<<<grid, kThreads, smem, s>>>(mk, mq, mv, ma, mc, a);
     prof_after(s);
     return cudaGetLastError();
 }

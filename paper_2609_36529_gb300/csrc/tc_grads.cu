@@ -146,7 +146,9 @@ template <int OUT_F32, bool PACKED>
 __global__ void __launch_bounds__(kThreads, 1)
 bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                           const __grid_constant__ CUtensorMap map_q,
-                          const __grid_constant__ CUtensorMap map_do, const TcGradArgs p) {
+                          const __grid_constant__ CUtensorMap map_do,
+                          const __grid_constant__ CUtensorMap map_s,
+                          const __grid_constant__ CUtensorMap map_ds, const TcGradArgs p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
@@ -191,7 +193,6 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
 
     const size_t sbase = ((size_t(b) * H + h) * NT + c) * E;   // this chunk's first slab
     const uint32_t slab_bytes = uint32_t(kDk) * dv * 4;        // hi tile + lo tile
-    const uint32_t LO = uint32_t(kDk) * dv * 2;                // lo tile offset in a slab
     const uint8_t* gS = reinterpret_cast<const uint8_t*>(p.Sck);
     const uint8_t* gD = reinterpret_cast<const uint8_t*>(p.dSck);
 
@@ -590,8 +591,9 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     mph ^= 1;
     tc_fence_after();
 
-    // ---- phase 2: per slice.  S_e and dS'_e (bf16 hi/lo, operand layout) arrive by bulk copy,
-    // one 64-column half per quarter of the work region with its own barrier.  Thread 0 issues
+    // ---- phase 2: per slice.  S_e and dS'_e (bf16 hi/lo, row-major checkpoints) arrive by TMA
+    // in the operand layout, one 64-column half per quarter of the work region with its own
+    // barrier.  Thread 0 issues
     // the slice's products (it is held for about their execution time) and, once they and the
     // Frobenius sum of warps 1-7 are done, the next slice's copies; slice e-1's epilogue runs
     // on all warps meanwhile (D1/D2 double-buffered in TMEM).
@@ -601,11 +603,9 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         for (int j = 0; j < nb; ++j)
             for (int which = 0; which < 2; ++which) {
                 uint8_t* dst = quarter(which, j);
-                const uint8_t* src = (which ? gD : gS) + (sbase + e) * slab_bytes + j * 16384;
                 uint64_t* bar = &bar_q[2 * j + which];
-                mbar_arrive_expect_tx(bar, 32768);
-                bulk_load(dst, src, 16384, bar);
-                bulk_load(dst + 16384, src + LO, 16384, bar);
+                mbar_arrive_expect_tx(bar, 32768);   // [hi | lo][128][64 columns]
+                tma_load_4d(dst, which ? &map_ds : &map_s, bar, 64 * j, 0, int(sbase + e), 0);
                 pend |= 1u << (2 * j + which);
             }
         if (e + 1 < E) {
@@ -869,10 +869,13 @@ cudaError_t launch_bwd_chunk_grads_tc(const tla_problem& p, const FwdPlan& fp, c
                                       const BwdPlan& bp, const char* bws, const void* dO,
                                       void* dq, void* dk, void* dq2, void* dk2, float* dbeta,
                                       float* dg, int* err, cudaStream_t s) {
-    CUtensorMap mk, mq, mo;
+    CUtensorMap mk, mq, mo, ms, md;
+    const long long nslab = (long long)p.B * p.H * fp.NT * p.E;
     if (!make_token_map(&mk, p.k, p.B, p.T, p.H, kDk, 64, 64, true) ||
         !make_token_map(&mq, p.q, p.B, p.T, p.H, kDk, 64, 64, true) ||
-        !make_token_map(&mo, dO, p.B, p.T, p.H, p.dv, 64, 64, true))
+        !make_token_map(&mo, dO, p.B, p.T, p.H, p.dv, 64, 64, true) ||
+        !make_ckpt_map(&ms, fws + fp.S, nslab, p.dv, 64, 1, 128) ||
+        !make_ckpt_map(&md, bws + bp.dS, nslab, p.dv, 64, 1, 128))
         return cudaErrorInvalidValue;
     TcGradArgs a;
     a.q2 = (const __nv_bfloat16*)p.q2;
@@ -897,7 +900,7 @@ cudaError_t launch_bwd_chunk_grads_tc(const tla_problem& p, const FwdPlan& fp, c
     cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     dim3 grid(fp.NT, p.H, p.B);
     prof_before("bwd_chunk_grads_tc", s);
-    kern<<<grid, kThreads, smem, s>>>(mk, mq, mo, a);
+    kern<<<grid, kThreads, smem, s>>>(mk, mq, mo, ms, md, a);
     prof_after(s);
     return cudaGetLastError();
 }

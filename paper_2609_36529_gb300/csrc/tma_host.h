@@ -39,9 +39,10 @@ inline bool make_token_map(CUtensorMap* m, const void* base, int B, int T, int H
     return r == CUDA_SUCCESS;
 }
 
-// bf16 row-major matrix [rows][cols] as 2-D (cols, rows); box (box_c, box_r), 128-byte swizzle.
+// bf16 row-major matrix [rows][cols] as 2-D (cols, rows); box (box_c, box_r); shared-memory
+// side swizzled by swizzle_bytes (32, 64 or 128; box_c * 2 must not exceed it).
 inline bool make_matrix_map(CUtensorMap* m, const void* base, long long rows, int cols, int box_c,
-                            int box_r) {
+                            int box_r, int swizzle_bytes = 128) {
     auto enc = tensor_map_encoder();
     if (!enc) return false;
     cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
@@ -49,7 +50,32 @@ inline bool make_matrix_map(CUtensorMap* m, const void* base, long long rows, in
     cuuint32_t box[2] = {(cuuint32_t)box_c, (cuuint32_t)box_r};
     cuuint32_t es[2] = {1, 1};
     CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
-                     box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                     swizzle_bytes == 32   ? CU_TENSOR_MAP_SWIZZLE_32B
+                     : swizzle_bytes == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                           : CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+// State checkpoints of the tensor-core path: per slab s = ((b * H + h) * NT + chunk) * E + e
+// a row-major [128][dv] bf16 hi matrix then the lo matrix.  Viewed as 4-D (column, row,
+// slab, hi/lo) with the hi/lo stride inside the slab stride, a box of (box_c, 128, box_s, 2)
+// lands in shared memory as [hi/lo][box_s][128][box_c]: the hi blocks of box_s slabs, then
+// their lo blocks.  swizzle_bytes: the shared-memory swizzle (box_c * 2 bytes wide).
+inline bool make_ckpt_map(CUtensorMap* m, const void* base, long long nslab, int dv, int box_c,
+                          int box_s, int swizzle_bytes) {
+    auto enc = tensor_map_encoder();
+    if (!enc) return false;
+    cuuint64_t dims[4] = {(cuuint64_t)dv, 128, (cuuint64_t)nslab, 2};
+    cuuint64_t strides[3] = {(cuuint64_t)dv * 2, (cuuint64_t)dv * 2 * 256, (cuuint64_t)dv * 2 * 128};
+    cuuint32_t box[4] = {(cuuint32_t)box_c, 128, (cuuint32_t)box_s, 2};
+    cuuint32_t es[4] = {1, 1, 1, 1};
+    CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides,
+                     box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                     swizzle_bytes == 32   ? CU_TENSOR_MAP_SWIZZLE_32B
+                     : swizzle_bytes == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                           : CU_TENSOR_MAP_SWIZZLE_128B,
                      CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS;
 }
