@@ -188,7 +188,7 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     float* red = scl + 384;                    // [3][4][64] row-dot partials per lane quarter
     float* frw = red + 768;                    // [2][8] Frobenius partials per warp (slice parity)
 
-    __shared__ __align__(8) uint64_t bar_ld, bar_mma, bar_fro, bar_q[4];
+    __shared__ __align__(8) uint64_t bar_ld, bar_mma, bar_q[4], bar_mh[2], bar_fh[2];
     __shared__ uint32_t tmem_slot;
 
     const size_t sbase = ((size_t(b) * H + h) * NT + c) * E;   // this chunk's first slab
@@ -204,7 +204,10 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         mbar_init(&bar_ld, 1);
         mbar_init(&bar_mma, 1);
         for (int q = 0; q < 4; ++q) mbar_init(&bar_q[q], 1);
-        mbar_init(&bar_fro, kThreads / 32 - 1);   // one arrival per warp 1..7
+        for (int j = 0; j < 2; ++j) {
+            mbar_init(&bar_mh[j], 1);
+            mbar_init(&bar_fh[j], kThreads / 32 - 1);   // one arrival per warp 1..7
+        }
         fence_barrier_init();
         const size_t ci = (size_t(b) * H + h) * NT + c;
         const uint32_t tt = 2 * T64;   // one token tile: hi then lo
@@ -395,7 +398,7 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
 #pragma unroll
             for (int c2 = 0; c2 < 4; ++c2) {
                 // exp of a non-positive difference (entries above the diagonal are discarded)
-                const float gam = expf(fminf(gr - gs[c2], 0.f));
+                const float gam = __expf(fminf(gr - gs[c2], 0.f));
                 const float ks2 = (R0 + a >= S0 + c2) ? ksv[c2] * gam : 0.f;
                 Rv[a][c2] = fmaf(kr, ks2, Rv[a][c2]);
                 Rq[a][c2] = fmaf(qr, ks2, Rq[a][c2]);
@@ -508,7 +511,7 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             float dk2v = 0.f, dq2v = 0.f, dGv = 0.f;
 #pragma unroll 4
             for (int s = 0; s <= x; ++s) {
-                const float gam = expf(gx - Gs[s * E + e]);
+                const float gam = __expf(gx - Gs[s * E + e]);
                 const float ks = __bfloat162float(k2s[s * E + e]);
                 const float dR = dRm[x * MP + s], dRq = dRqm[x * MP + s];
                 dk2v = fmaf(dR * ks, gam, dk2v);
@@ -517,7 +520,7 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             }
 #pragma unroll 4
             for (int r = x; r < 64; ++r) {
-                const float gam = expf(Gs[r * E + e] - gx);
+                const float gam = __expf(Gs[r * E + e] - gx);
                 const float dR = dRm[r * MP + x], dRq = dRqm[r * MP + x];
                 const float t = (dR * __bfloat162float(k2s[r * E + e]) +
                                  dRq * __bfloat162float(q2s[r * E + e])) * gam;
@@ -592,72 +595,73 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     tc_fence_after();
 
     // ---- phase 2: per slice.  S_e and dS'_e (bf16 hi/lo, row-major checkpoints) arrive by TMA
-    // in the operand layout, one 64-column half per quarter of the work region with its own
-    // barrier.  Thread 0 issues
-    // the slice's products (it is held for about their execution time) and, once they and the
-    // Frobenius sum of warps 1-7 are done, the next slice's copies; slice e-1's epilogue runs
-    // on all warps meanwhile (D1/D2 double-buffered in TMEM).
-    uint32_t qph = 0, pend = 0, fph = 0;   // quarter phases, loads in flight (thread 0), bar_fro phase
+    // in the operand layout, one 64-column half of each per quarter of the work region, with a
+    // barrier per quarter.  The slice is pipelined by halves: thread 0 issues half j's products
+    // as soon as its quarters land (committed to bar_mh[j]); warps 1-7 take half j's part of the
+    // Frobenius sum (bar_fh[j]); once both are done the half's quarters take the next slice's
+    // copies, while the other half is still being multiplied.  Slice e-1's epilogue runs on all
+    // warps meanwhile (D1/D2 double-buffered in TMEM).  Every barrier of this phase completes
+    // once per slice, so the parity of slice e is e & 1.
+    uint32_t pend = 0, mpend = 0;   // thread 0: quarters with copies in flight, halves with products
+    int pend_slice = 0;             // thread 0: the slice those copies belong to
     auto quarter = [&](int which, int j) { return W + (2 * j + which) * 32768; };   // 0: S, 1: dS'
-    auto issue_slice = [&](int e) {
-        for (int j = 0; j < nb; ++j)
-            for (int which = 0; which < 2; ++which) {
-                uint8_t* dst = quarter(which, j);
-                uint64_t* bar = &bar_q[2 * j + which];
-                mbar_arrive_expect_tx(bar, 32768);   // [hi | lo][128][64 columns]
-                tma_load_4d(dst, which ? &map_ds : &map_s, bar, 64 * j, 0, int(sbase + e), 0);
-                pend |= 1u << (2 * j + which);
-            }
-        if (e + 1 < E) {
+    auto issue_half = [&](int e, int j) {
+        for (int which = 0; which < 2; ++which) {
+            uint64_t* bar = &bar_q[2 * j + which];
+            mbar_arrive_expect_tx(bar, 32768);   // [hi | lo][128][64 columns]
+            tma_load_4d(quarter(which, j), which ? &map_ds : &map_s, bar, 64 * j, 0, int(sbase + e), 0);
+            pend |= 1u << (2 * j + which);
+        }
+        pend_slice = e;
+        if (j == 0 && e + 1 < E) {
             bulk_prefetch_l2(gS + (sbase + e + 1) * slab_bytes, slab_bytes);
             bulk_prefetch_l2(gD + (sbase + e + 1) * slab_bytes, slab_bytes);
         }
     };
-    auto fail = [&](bool mma) {   // timeout: record it, drain this CTA's copies and products
+    auto fail = [&](int e) {   // timeout: record it, drain this CTA's copies and products
         if (tid == 0) {
             record_device_error(p.err, TLA_ERR_TIMEOUT);
             for (int q = 0; q < 4; ++q)
-                if ((pend >> q) & 1) mbar_wait(&bar_q[q], (qph >> q) & 1);
-            if (mma) mbar_wait(&bar_mma, mph);
+                if ((pend >> q) & 1) mbar_wait(&bar_q[q], pend_slice & 1);
+            for (int j = 0; j < 2; ++j)
+                if ((mpend >> j) & 1) mbar_wait(&bar_mh[j], e & 1);
         }
         tc_fence_before();
         __syncthreads();
         if (warp == 0) tmem_dealloc(tmem, 512);
     };
-    if (tid == 0) issue_slice(0);
+    if (tid == 0)
+        for (int j = 0; j < nb; ++j) issue_half(0, j);
     float acq[32], ack[32];
 #pragma unroll
     for (int j = 0; j < 32; ++j) acq[j] = ack[j] = 0.f;
-    const uint32_t qmask = nb == 2 ? 15u : 3u;
     for (int e = 0; e <= E; ++e) {   // e == E only finishes slice E-1
         const bool act = e < E;
         const int pb = e & 1;
+        const uint32_t par = e & 1;
         bool ok = true;
+        // the row-dot partials of slice e-2 have been read (end of the last iteration)
+        tc_fence_before();
+        __syncthreads();
+        tc_fence_after();
         if (act) {
             if (tid < 192) {   // b_e, a_e, w_e of the 64 tokens
                 const int r = tid & 63, i = r * E + e;
                 float sv;
-                if (tid < 64) sv = __bfloat162float(q2s[i]) * expf(Gs[i]);
-                else if (tid < 128) sv = __bfloat162float(k2s[i]) * expf(Gs[i]);
-                else sv = __bfloat162float(k2s[i]) * expf(Gs[(n - 1) * E + e] - Gs[i]);
+                if (tid < 64) sv = __bfloat162float(q2s[i]) * __expf(Gs[i]);
+                else if (tid < 128) sv = __bfloat162float(k2s[i]) * __expf(Gs[i]);
+                else sv = __bfloat162float(k2s[i]) * __expf(Gs[(n - 1) * E + e] - Gs[i]);
                 scl[pb * 192 + tid] = sv;
             }
-            for (int q = 0; q < 4; ++q)
-                if ((qmask >> q) & 1) ok = mbar_wait(&bar_q[q], (qph >> q) & 1) && ok;
-            tc_fence_before();
-            if (__syncthreads_or(!ok)) {
-                fail(false);
-                return;
-            }
-            qph ^= qmask;
-            pend &= ~qmask;
-            tc_fence_after();
             if (warp == 0) {
-                if (lane == 0) {   // D1 = S_e [dO; -dRes]^T, D2 = dS'_e U^T
+                if (lane == 0) {   // D1 = S_e [dO; -dRes]^T, D2 = dS'_e U^T, by halves of K = dv
                     const uint32_t d1 = pb ? tmem + 320 : tmem + 128, d2 = pb ? tmem + 448 : tmem + 256;
                     const uint32_t id128 = idesc_bf16_f32(128, 128, 0, 0);
                     const uint32_t id64 = idesc_bf16_f32(128, 64, 0, 0);
-                    for (int j = 0; j < nb; ++j) {
+                    for (int j = 0; j < nb && ok; ++j) {
+                        ok = mbar_wait(&bar_q[2 * j], par) && mbar_wait(&bar_q[2 * j + 1], par);
+                        if (!ok) break;
+                        pend &= ~(3u << (2 * j));
                         const uint32_t qs = smem_u32(quarter(0, j)), qd = smem_u32(quarter(1, j));
                         for (int kk = 0; kk < 4; ++kk) {
                             const uint32_t k32 = kk * 32, acc = (j > 0 || kk > 0) ? 1u : 0u;
@@ -676,34 +680,41 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                             umma_bf16(d2, dl, uh, id64, 1u);
                             umma_bf16(d2, dh, ul, id64, 1u);
                         }
+                        umma_commit(&bar_mh[j]);
+                        mpend |= 1u << j;
                     }
-                    umma_commit(&bar_mma);
-                    // the slabs are free once the products and the Frobenius sum have read them
-                    ok = mbar_wait(&bar_mma, mph) && mbar_wait(&bar_fro, fph);
-                    if (ok && e + 1 < E) issue_slice(e + 1);
+                    // a half's quarters are free once its products and Frobenius part have read them
+                    for (int j = 0; j < nb && ok; ++j) {
+                        ok = mbar_wait(&bar_mh[j], par) && mbar_wait(&bar_fh[j], par);
+                        if (!ok) break;
+                        mpend &= ~(1u << j);
+                        if (e + 1 < E) issue_half(e + 1, j);
+                    }
                 }
                 __syncwarp();
             } else {   // <dS'_e, S_e> (hi + lo reproduces each value to ~2^-16), warps 1..7
                 float fro = 0.f;
                 for (int j = 0; j < nb; ++j) {
-                    const uint8_t* qsb = quarter(0, j);
-                    const uint8_t* qdb = quarter(1, j);
-                    for (uint32_t o = (tid - 32) * 16; o < 16384; o += (kThreads - 32) * 16) {
-                        float sh[8], sl[8], dh[8], dl[8];
-                        load_bf16x8(qsb + o, sh);
-                        load_bf16x8(qsb + 16384 + o, sl);
-                        load_bf16x8(qdb + o, dh);
-                        load_bf16x8(qdb + 16384 + o, dl);
+                    ok = ok && mbar_wait(&bar_q[2 * j], par) && mbar_wait(&bar_q[2 * j + 1], par);
+                    if (ok) {
+                        const uint8_t* qsb = quarter(0, j);
+                        const uint8_t* qdb = quarter(1, j);
+                        for (uint32_t o = (tid - 32) * 16; o < 16384; o += (kThreads - 32) * 16) {
+                            float sh[8], sl[8], dh[8], dl[8];
+                            load_bf16x8(qsb + o, sh);
+                            load_bf16x8(qsb + 16384 + o, sl);
+                            load_bf16x8(qdb + o, dh);
+                            load_bf16x8(qdb + 16384 + o, dl);
 #pragma unroll
-                        for (int u = 0; u < 8; ++u) fro = fmaf(dh[u] + dl[u], sh[u] + sl[u], fro);
+                            for (int u = 0; u < 8; ++u) fro = fmaf(dh[u] + dl[u], sh[u] + sl[u], fro);
+                        }
                     }
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&bar_fh[j]);   // also on failure: thread 0's wait stays bounded
                 }
 #pragma unroll
                 for (int sft = 16; sft >= 1; sft >>= 1) fro += __shfl_xor_sync(0xffffffffu, fro, sft);
-                if (lane == 0) {
-                    frw[pb * 8 + warp] = fro;
-                    mbar_arrive(&bar_fro);
-                }
+                if (lane == 0) frw[pb * 8 + warp] = fro;
             }
         }
         if (e > 0) {   // epilogue of slice e-1 (its D1/D2 and scales)
@@ -744,14 +755,10 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         }
         tc_fence_before();
         if (__syncthreads_or(!ok)) {
-            fail(act);
+            fail(e);
             return;
         }
         tc_fence_after();
-        if (act) {
-            mph ^= 1;
-            fph ^= 1;
-        }
         if (e > 0) {   // slice e-1's row dots -> dq2, dk2, dG (a_e = k2 gamma, b_e = q2 gamma, w_e)
             const int es = e - 1;
             if (tid < 64) {
@@ -763,8 +770,8 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                     da += red[(1 * 4 + q) * 64 + tid];
                     dw += red[(2 * 4 + q) * 64 + tid];
                 }
-                const float gam = expf(Gs[i]);
-                const float wdec = expf(Gs[(n - 1) * E + es] - Gs[i]);
+                const float gam = __expf(Gs[i]);
+                const float wdec = __expf(Gs[(n - 1) * E + es] - Gs[i]);
                 const float k2v = __bfloat162float(k2s[i]), q2v = __bfloat162float(q2s[i]);
                 dk2a[i] += da * gam + dw * wdec;
                 dq2a[i] += db * gam;
@@ -817,10 +824,10 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         const float gl = Gs[(n - 1) * E + e];
         float dGC = 0.f;
         for (int r = lane; r < n; r += 32)
-            dGC = fmaf(dwk[r * E + e], __bfloat162float(k2s[r * E + e]) * expf(gl - Gs[r * E + e]), dGC);
+            dGC = fmaf(dwk[r * E + e], __bfloat162float(k2s[r * E + e]) * __expf(gl - Gs[r * E + e]), dGC);
 #pragma unroll
         for (int s = 16; s >= 1; s >>= 1) dGC += __shfl_xor_sync(0xffffffffu, dGC, s);
-        dGC = fmaf(dgc[e], expf(gl), dGC);
+        dGC = fmaf(dgc[e], __expf(gl), dGC);
         const int r0 = 2 * lane, r1 = r0 + 1;
         const float a0 = r0 < n ? dGa[r0 * E + e] + (r0 == n - 1 ? dGC : 0.f) : 0.f;
         const float a1 = r1 < n ? dGa[r1 * E + e] + (r1 == n - 1 ? dGC : 0.f) : 0.f;

@@ -193,7 +193,7 @@ chunk_prep_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                 for (int c2 = 0; c2 < 4; ++c2) {
                     // exp of a non-positive log-decay difference (Eq. joint-gram); the
                     // clamp only matters above the diagonal, where the entry is discarded
-                    const float ks2 = ks[c2] * expf(fminf(gr - gs[c2], 0.f));
+                    const float ks2 = ks[c2] * __expf(fminf(gr - gs[c2], 0.f));
                     R[a][c2] = fmaf(kr, ks2, R[a][c2]);
                     Rq[a][c2] = fmaf(qr, ks2, Rq[a][c2]);
                 }
@@ -355,12 +355,12 @@ chunk_prep_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     for (int i = tid; i < 64 * E; i += kThreads) {
         const int e = i - (i / E) * E;
         const float Gr = Gs[i], GC = Gs[(n - 1) * E + e];
-        const float gam = expf(Gr);
+        const float gam = __expf(Gr);
         cf[i] = k2s[i] * gam;
         cf[64 * E + i] = q2s[i] * gam;
-        cf[128 * E + i] = k2s[i] * expf(GC - Gr);
+        cf[128 * E + i] = k2s[i] * __expf(GC - Gr);
     }
-    if (tid < 16) cf[192 * E + tid] = tid < E ? expf(Gs[(n - 1) * E + tid]) : 0.f;
+    if (tid < 16) cf[192 * E + tid] = tid < E ? __expf(Gs[(n - 1) * E + tid]) : 0.f;
 }
 
 size_t prep_tc_smem(int E) { return 1024 + size_t(5) * kSlot * 4 + (3 * 64 * E + 64) * 4; }
