@@ -58,7 +58,8 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                          const __grid_constant__ CUtensorMap map_q,
                          const __grid_constant__ CUtensorMap map_do,
                          const __grid_constant__ CUtensorMap map_bt,
-                         const __grid_constant__ CUtensorMap map_ck, const TcBwdArgs p) {
+                         const __grid_constant__ CUtensorMap map_ck,
+                         const __grid_constant__ CUtensorMap map_dv, const TcBwdArgs p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
@@ -75,7 +76,8 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     uint8_t* sBl = sReg + NE * 256;
     uint8_t* sOT = sReg + NE * 512;          // dO^T [TV][64] bf16 (MMA-0)
     __nv_bfloat16* sdO = reinterpret_cast<__nv_bfloat16*>(sOT + TV * 128);   // [64][TV] (TMA)
-    float* sCoef = reinterpret_cast<float*>(sOT + TV * 128 + 64 * TV * 2);   // 2 x CB
+    uint8_t* sDvo = sOT + TV * 128 + 64 * TV * 2;                           // dv tile [64][TV] (TMA store)
+    float* sCoef = reinterpret_cast<float*>(sDvo + 64 * TV * 4);             // 2 x CB
 
     __shared__ __align__(8) uint64_t bar_kq, bar_av, bar_mma;
     __shared__ uint32_t tmem_slot;
@@ -209,6 +211,9 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     for (int c = nct - 1; c >= 0 && !failed; --c) {
         const int it = nct - 1 - c;                // iteration index (barrier phases)
         const int t0 = tbeg + c * 64, n = min(64, tlen - c * 64);
+        // dv leaves as one TMA store of the chunk's tile, except for a packed document's partial
+        // last chunk, whose tile rows past its end belong to the next document
+        const bool tma_dv = !p.dtab || n == 64;
         const float* cf = sCoef + (c & 1) * CB;
         const float* ae = cf;
         const float* be = cf + 64 * E;
@@ -330,10 +335,14 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             for (int j = 0; j < TV; j += 16) tmem_ld16(tmem_lane_addr(tY, warp, j), dr + j);
             tmem_wait_ld();
             if (row_thread) {
+                if (tma_dv) {   // row of the dv tile; thread 0 stores the tile after the barrier
+                    if (p.out_f32) store_f32_row(reinterpret_cast<float*>(sDvo) + r64 * TV, dr, TV);
+                    else store_row(sDvo, size_t(r64) * TV, dr, TV, 0);
+                }
                 if (r64 < n) {
                     const size_t off = tok_idx(b, t0 + r64, h, n0, T, H, dv);
                     if (!p.ck_tiles) store_f32_row(p.dRbuf + off, dr, TV);
-                    store_row(p.dv_out, off, dr, TV, p.out_f32);
+                    if (!tma_dv) store_row(p.dv_out, off, dr, TV, p.out_f32);
                 }
                 if (p.ck_tiles && p.use_delta) {   // -dRes, the operand sign the gradient kernel uses
                     float ndr[TV];
@@ -377,6 +386,10 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                 umma_bf16(tS, ad, smem_desc(smem_u32(sBl) + ks * 2048, 128 * 128, 1024), idc, 1u);
             }
             umma_commit(&bar_mma);
+            if (tma_dv) {   // rows past T are skipped by the store
+                tma_store_4d(&map_dv, sDvo, n0, h, t0, b);
+                bulk_commit();
+            }
         }
         pending_mma = 1;
         ok = mbar_wait(&bar_mma, mma_phase);
@@ -419,19 +432,22 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
 template <int TV>
 size_t tc_bwd_smem(int E) {
     const int NE = E * TV;
-    return 1024 + 8 * kBoxBytes + NE * 512 + TV * 128 + 64 * TV * 2 + 2 * (3 * 64 * E + 16) * 4;
+    return 1024 + 8 * kBoxBytes + NE * 512 + TV * 128 + 64 * TV * 2 + 64 * TV * 4 +
+           2 * (3 * 64 * E + 16) * 4;
 }
 
 template <int TV>
 cudaError_t launch_tv(const tla_problem& p, const FwdPlan& fp, const char* fws, const BwdPlan& bp,
                       char* bws, const void* dO, const float* dht, void* dv, float* dh0, int* err,
                       cudaStream_t s) {
-    CUtensorMap mk, mq, mo, mb, mc;
+    CUtensorMap mk, mq, mo, mb, mc, mdv;
     const int NT = fp.NT;
     if (!make_token_map(&mk, p.k, p.B, p.T, p.H, kDk, 64, 64, true) ||
         !make_token_map(&mq, p.q, p.B, p.T, p.H, kDk, 64, 64, true) ||
         !make_token_map(&mo, dO, p.B, p.T, p.H, p.dv, TV, 64, false) ||
-        !make_matrix_map(&mb, fws + fp.BT, (long long)p.B * p.H * NT * 256, 64, 64, 64))
+        !make_matrix_map(&mb, fws + fp.BT, (long long)p.B * p.H * NT * 256, 64, 64, 64) ||
+        !make_token_map(&mdv, dv, p.B, p.T, p.H, p.dv, TV, 64, false,
+                        p.out_dtype == TLA_FP32 ? 4 : 2))
         return cudaErrorInvalidValue;
     memset(&mc, 0, sizeof(mc));   // unused unless the checkpoints are tiles
     if (fp.ck_tiles &&
@@ -455,7 +471,7 @@ cudaError_t launch_tv(const tla_problem& p, const FwdPlan& fp, const char* fws, 
     cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     dim3 grid(p.dv / TV, p.H, fp.nseq);
     prof_before("bwd_recurrence_tc", s);
-    kern<<<grid, kThreads, smem, s>>>(mk, mq, mo, mb, mc, a);
+    kern<<<grid, kThreads, smem, s>>>(mk, mq, mo, mb, mc, mdv, a);
     prof_after(s);
     return cudaGetLastError();
 }

@@ -13,8 +13,8 @@
 //   epi-B  O = Oi + Oa;  Ut_e = diag(w_e) U
 //   MMA-C  S_all += K^T [Ut_1 .. Ut_E] (M=dk=128, K=64, N=NE; K^T read MN-major
 //                                      straight from the TMA-loaded key tile)
-//   epi-C  S_{[c+1]} from TMEM -> operand of the next MMA-A, checkpoint, and
-//          pre-scaled by gamma^C of the next chunk for its MMA-C.
+//   epi-C  S_{[c+1]} from TMEM in one pass: operand of the next MMA-A (also the
+//          checkpoint), and pre-scaled by gamma^C of the next chunk for its MMA-C.
 // Accumulation is fp32 in TMEM.  Keys and queries are bf16 inputs and enter the
 // products exactly; every other operand (the state, Res, T, A T, Ut) is carried
 // as a pair of bf16 values hi + lo (lo = bf16 of the rounding remainder), and
@@ -68,7 +68,8 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                          const __grid_constant__ CUtensorMap map_q,
                          const __grid_constant__ CUtensorMap map_v,
                          const __grid_constant__ CUtensorMap map_a2,
-                         const __grid_constant__ CUtensorMap map_ck, const TcFwdArgs p) {
+                         const __grid_constant__ CUtensorMap map_ck,
+                         const __grid_constant__ CUtensorMap map_o, const TcFwdArgs p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
@@ -84,7 +85,8 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     uint8_t* sUh = sReg + TV * 256;            //   Ut [64][NE] hi, lo, MN-major (after MMA-B)
     uint8_t* sUl = sUh + NE * 128;
     __nv_bfloat16* sV = reinterpret_cast<__nv_bfloat16*>(sReg + NE * 512);  // [64][TV]
-    float* sCoef = reinterpret_cast<float*>(sReg + NE * 512 + 64 * TV * 2);  // 2 x CB
+    uint8_t* sOo = sReg + NE * 512 + 64 * TV * 2;                             // o tile [64][TV] (TMA store)
+    float* sCoef = reinterpret_cast<float*>(sOo + 64 * TV * 4);               // 2 x CB
 
     __shared__ __align__(8) uint64_t bar_kq, bar_av, bar_mma;
     __shared__ uint32_t tmem_slot;
@@ -148,43 +150,10 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         tma_load_4d(sV, &map_v, &bar_av, n0, h, tbeg + c * 64, b);
         bulk_load(sCoef + (c & 1) * CB, p.coef + idx * CB, CB * 4, &bar_av);
     };
-    // Row d = tid of S_{[c]} (from h0 or from TMEM) as the bf16 hi/lo operand of MMA-A.
-    auto write_operand = [&](bool from_h0) {
-        const int d = tid;
-        for (int e = 0; e < E; ++e) {
-            float v[TV];
-            if (from_h0) {
-                if (p.h0) {
-                    const float4* src = reinterpret_cast<const float4*>(
-                        p.h0 + ((size_t(sb * H + h) * E + e) * kDk + d) * dv + n0);
-#pragma unroll
-                    for (int i = 0; i < TV / 4; ++i) {
-                        float4 x = src[i];
-                        v[4 * i] = x.x; v[4 * i + 1] = x.y; v[4 * i + 2] = x.z; v[4 * i + 3] = x.w;
-                    }
-                } else {
-#pragma unroll
-                    for (int i = 0; i < TV; ++i) v[i] = 0.f;
-                }
-            } else {
-#pragma unroll
-                for (int j = 0; j < TV; j += 16) tmem_ld16(tmem_lane_addr(tS, warp, e * TV + j), v + j);
-                tmem_wait_ld();
-            }
-#pragma unroll
-            for (int n = 0; n < TV; n += 8) st8_split(sSh, sSl, e * blk_bytes<TV>() + blk_offset<TV>(d, n), v + n);
-        }
-    };
-    // Checkpoint of S_{[c]} (bf16 hi/lo) for the backward: this CTA's columns of the
-    // slice blocks, stored by TMA (thread 0, after the operand is complete).
-    auto issue_ckpt = [&](int c) {
-        if (!(p.save && p.ck_tiles)) return;
-        tma_store_4d(&map_ck, sSh, n0, 0, ((b * H + h) * NT + cb + c) * E, 0);   // [hi|lo][E][dk][TV]
-        bulk_commit();
-    };
-    // Row d of S_{[c]}: checkpoint for the backward, and the gamma^C_c-scaled copy in
-    // TMEM that chunk c's state update accumulates onto.  Runs while MMA-A(c) executes.
-    auto finish_state = [&](int c, bool from_h0) {
+    // Row d = tid of S_{[c]} (from h0 or from TMEM), in one pass: the bf16 hi/lo operand of
+    // MMA-A, the fp32 checkpoint when checkpoints are not tiles (tiles: issue_ckpt), and the
+    // gamma^C_c-scaled copy in TMEM that chunk c's state update accumulates onto.
+    auto stage_state = [&](int c, bool from_h0) {
         const int d = tid;
         const float* gc = sCoef + (c & 1) * CB + 3 * 64 * E;
         for (int e = 0; e < E; ++e) {
@@ -207,7 +176,9 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                 for (int j = 0; j < TV; j += 16) tmem_ld16(tmem_lane_addr(tS, warp, e * TV + j), v + j);
                 tmem_wait_ld();
             }
-            if (p.save && !p.ck_tiles) {   // fp32 checkpoint (tile checkpoints: issue_ckpt)
+#pragma unroll
+            for (int n = 0; n < TV; n += 8) st8_split(sSh, sSl, e * blk_bytes<TV>() + blk_offset<TV>(d, n), v + n);
+            if (p.save && !p.ck_tiles) {
                 const size_t slab = (((size_t(b) * H + h) * NT + cb + c) * E + e) * kDk * dv;
                 store_f32_row(p.Sck + slab + size_t(d) * dv + n0, v, TV);
             }
@@ -218,6 +189,13 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             for (int j = 0; j < TV; j += 16) tmem_st16(tmem_lane_addr(tS, warp, e * TV + j), v + j);
         }
         tmem_wait_st();
+    };
+    // Checkpoint of S_{[c]} (bf16 hi/lo) for the backward: this CTA's columns of the
+    // slice blocks, stored by TMA (thread 0, after the operand is complete).
+    auto issue_ckpt = [&](int c) {
+        if (!(p.save && p.ck_tiles)) return;
+        tma_store_4d(&map_ck, sSh, n0, 0, ((b * H + h) * NT + cb + c) * E, 0);   // [hi|lo][E][dk][TV]
+        bulk_commit();
     };
     // MMA-A: P = [K; Q] S_all    (B = S_all, MN-major, hi and lo)
     auto issue_mma_a = [&]() {
@@ -246,7 +224,7 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     if (!mbar_wait(&bar_av, 0)) failed = true;
     if (__syncthreads_or(failed)) failed = true;
     if (!failed) {
-        write_operand(true);
+        stage_state(0, true);
         fence_proxy_async_smem();
         tc_fence_before();
         const bool ok = mbar_wait(&bar_kq, 0);
@@ -258,12 +236,14 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                 issue_ckpt(0);
             }
             pending_mma = 1;
-            finish_state(0, true);
         }
     }
 
     for (int c = 0; c < nct && !failed; ++c) {
         const int t0 = tbeg + c * 64, n = min(64, tlen - c * 64);
+        // o leaves as one TMA store of the chunk's tile, except for a packed document's partial
+        // last chunk, whose tile rows past its end belong to the next document
+        const bool tma_o = !p.dtab || n == 64;
         const float* cf = sCoef + (c & 1) * CB;
         const float* ae = cf;
         const float* be = cf + 64 * E;
@@ -380,6 +360,11 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         } else {
 #pragma unroll
             for (int i = 0; i < TV; ++i) d2[i] += oi[i];
+            if (tma_o) {   // row of the o tile; thread 0 stores the tile after the barrier
+                const int r = tid - 64;
+                if (p.out_f32) store_f32_row(reinterpret_cast<float*>(sOo) + r * TV, d2, TV);
+                else store_row(sOo, size_t(r) * TV, d2, TV, 0);
+            }
         }
         fence_proxy_async_smem();
         tc_fence_before();
@@ -396,6 +381,10 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                 umma_bf16(tS, ad, smem_desc(smem_u32(sUl) + ks * 2048, 64 * 128, 1024), idesc, 1u);
             }
             umma_commit(&bar_mma);
+            if (tma_o) {   // rows past T are skipped by the store
+                tma_store_4d(&map_o, sOo, n0, h, t0, b);
+                bulk_commit();
+            }
         }
         pending_mma = 1;
         {   // while MMA-C runs: U (key rows) and o (query rows) to global memory
@@ -405,7 +394,7 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                     if (p.ck_tiles) store_tok_tile(p.Ubuf, (size_t(b) * H + h) * NT + cb + c, dv, r, n0, d2, TV, r < n);
                     else if (r < n) store_f32_row(p.Ubuf + tok_idx(b, t0 + r, h, n0, T, H, dv), d2, TV);
                 }
-            } else if (r < n) {
+            } else if (!tma_o && r < n) {
                 store_row(p.o, tok_idx(b, t0 + r, h, n0, T, H, dv), d2, TV, p.out_f32);
             }
         }
@@ -417,9 +406,9 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         tc_fence_after();
         if (tid == 0 && c + 1 < nct) issue_kq(c + 1);   // key/query buffer is free
 
-        // ---- epi-C: next chunk's operand, MMA-A(c+1), then checkpoint and scaling
+        // ---- epi-C: next chunk's state (operand, scaled TMEM copy), MMA-A(c+1), checkpoint
         if (c + 1 < nct) {
-            write_operand(false);
+            stage_state(c + 1, false);
             fence_proxy_async_smem();
             tc_fence_before();
             ok = mbar_wait(&bar_kq, (c + 1) & 1);
@@ -430,7 +419,6 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                 issue_ckpt(c + 1);
             }
             pending_mma = 1;
-            finish_state(c + 1, false);
         } else if (p.ht) {
             const int d = tid;
             for (int e = 0; e < E; ++e) {
@@ -461,18 +449,20 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
 template <int TV>
 size_t tc_fwd_smem(int E) {
     const int NE = E * TV;
-    return 1024 + 4 * kBoxBytes + 4 * kBoxBytes + NE * 512 + 64 * TV * 2 + 2 * (3 * 64 * E + 16) * 4;
+    return 1024 + 4 * kBoxBytes + 4 * kBoxBytes + NE * 512 + 64 * TV * 2 + 64 * TV * 4 +
+           2 * (3 * 64 * E + 16) * 4;
 }
 
 template <int TV>
 cudaError_t launch_tv(const tla_problem& p, const FwdPlan& fp, char* ws, int save, int* err,
                       cudaStream_t s) {
-    CUtensorMap mk, mq, mv, ma, mc;
+    CUtensorMap mk, mq, mv, ma, mc, mo;
     const int NT = fp.NT;
     if (!make_token_map(&mk, p.k, p.B, p.T, p.H, kDk, 64, 64, true) ||
         !make_token_map(&mq, p.q, p.B, p.T, p.H, kDk, 64, 64, true) ||
         !make_token_map(&mv, p.v, p.B, p.T, p.H, p.dv, TV, 64, false) ||
-        !make_matrix_map(&ma, ws + fp.A2, (long long)p.B * p.H * NT * 256, 64, 64, 128))
+        !make_matrix_map(&ma, ws + fp.A2, (long long)p.B * p.H * NT * 256, 64, 64, 128) ||
+        !make_token_map(&mo, p.o, p.B, p.T, p.H, p.dv, TV, 64, false, p.out_dtype == TLA_FP32 ? 4 : 2))
         return cudaErrorInvalidValue;
     memset(&mc, 0, sizeof(mc));   // unused unless tile checkpoints are saved
     if (save && fp.ck_tiles &&
@@ -496,7 +486,7 @@ cudaError_t launch_tv(const tla_problem& p, const FwdPlan& fp, char* ws, int sav
     cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     dim3 grid(p.dv / TV, p.H, fp.nseq);
     prof_before("fwd_recurrence_tc", s);
-    kern<<<grid, kThreads, smem, s>>>(mk, mq, mv, ma, mc, a);
+    kern<<<grid, kThreads, smem, s>>>(mk, mq, mv, ma, mc, mo, a);
     prof_after(s);
     return cudaGetLastError();
 }

@@ -22,17 +22,20 @@ inline PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
     return fn;
 }
 
-// bf16 token tensor [B, T, H, D] viewed as 4-D (D, H, T, B); box (box_d, 1, box_t, 1).
-// Rows past T read as zero.  swizzle128: 128-byte swizzle (box_d * 2 must be 128).
+// Token tensor [B, T, H, D] of bf16 (elem_bytes 2) or fp32 (4) viewed as 4-D (D, H, T, B);
+// box (box_d, 1, box_t, 1).  Loads read rows past T as zero, stores skip them.  swizzle128:
+// 128-byte swizzle (box_d * elem_bytes must be 128).
 inline bool make_token_map(CUtensorMap* m, const void* base, int B, int T, int H, int D, int box_d,
-                           int box_t, bool swizzle128) {
+                           int box_t, bool swizzle128, int elem_bytes = 2) {
     auto enc = tensor_map_encoder();
     if (!enc) return false;
     cuuint64_t dims[4] = {(cuuint64_t)D, (cuuint64_t)H, (cuuint64_t)T, (cuuint64_t)B};
-    cuuint64_t strides[3] = {(cuuint64_t)D * 2, (cuuint64_t)H * D * 2, (cuuint64_t)T * H * D * 2};
+    const cuuint64_t eb = (cuuint64_t)elem_bytes;
+    cuuint64_t strides[3] = {(cuuint64_t)D * eb, (cuuint64_t)H * D * eb, (cuuint64_t)T * H * D * eb};
     cuuint32_t box[4] = {(cuuint32_t)box_d, 1, (cuuint32_t)box_t, 1};
     cuuint32_t es[4] = {1, 1, 1, 1};
-    CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides,
+    CUresult r = enc(m, elem_bytes == 4 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
+                     4, const_cast<void*>(base), dims, strides,
                      box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
                      swizzle128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
                      CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
