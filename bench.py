@@ -81,17 +81,66 @@ def flops_per_token_head(kernel, E, dk, dv, C=CHUNK):
     return 0.0
 
 
+def bytes_per_token_head(kernel, E, dk, dv, C=CHUNK, in_b=2, out_b=4, delta=True):
+    """Algorithmic HBM bytes of one token of one head for each kernel of the tensor-core path.
+
+    Every tensor a kernel reads or writes is counted once (re-reads that the design leaves to
+    L2, e.g. the key/query tiles shared by a head's value blocks, are not counted).  bf16
+    hi/lo operands take 4 bytes per element; per-chunk matrices are divided by C tokens.
+      gate cumsum:  log gates in, chunk-local cumsum out (fp32).
+      chunk prep:   k, q, k', q', G, beta in; N (delta rule), [T; A T] and [A^T; T^T] hi/lo
+                    tiles (2 x 128 x 64 and 4 x 64 x 64 bf16 per chunk), coefficient block out.
+      forward:      k, q, v, [T; A T], coefficients in; o, the chunk-start state checkpoint
+                    (E dk dv hi/lo per chunk), U and Res token tiles out.
+      backward:     k, q, dO, [A^T; T^T], coefficients in; dv, the state-gradient checkpoint,
+                    dU and -dRes token tiles out.
+      gradients:    k, q, dO, U, Res, dU, -dRes, both checkpoints, N, G, k', q', beta in;
+                    dq, dk, dq', dk', dg, dbeta out.
+    """
+    ck = E * dk * dv * 4 / C
+    coef = (3 * C * E + 16) * 4 / C
+    tiles = 8 * C                  # a 2 x 128 x 64 or 4 x 64 x 64 bf16 tile pair per chunk
+    name = kernel
+    if name.startswith("gate_cumsum"):
+        return 8 * E
+    if name.startswith("chunk_prep"):
+        return (2 * dk * in_b + 2 * E * in_b + 4 * E + 4) + (4 * C if delta else 0) + 2 * tiles + coef
+    if name.startswith("fwd_recurrence"):
+        return (in_b * (2 * dk + dv) + tiles + coef) + (dv * out_b + ck + 4 * dv * 2)
+    if name.startswith("bwd_recurrence"):
+        return (in_b * (2 * dk + dv) + tiles + coef) + (dv * out_b + ck + 4 * dv * (2 if delta else 1))
+    if name.startswith("bwd_chunk_grads"):
+        return (in_b * (2 * dk + dv) + 4 * dv * (4 if delta else 3) + 2 * ck + (4 * C if delta else 0)
+                + 4 * E + 2 * E * in_b + 4) + (2 * dk * out_b + 2 * E * out_b + 4 * E + 4)
+    return 0.0
+
+
 def kernel_source_hash(kernel):
-    """Hash of the source file that defines a kernel (to invalidate stale ncu traffic)."""
+    """Hash of the source that builds a kernel: the .cu files that define it and every local
+    header they include, recursively (to invalidate stale ncu traffic)."""
     csrc = os.path.join(ROOT, "paper_2609_36529_gb300", "csrc")
-    h = hashlib.sha256()
+    files, todo = set(), []
     for fn in sorted(os.listdir(csrc)):
         path = os.path.join(csrc, fn)
+        if fn.endswith(".cu"):
+            with open(path, "rb") as f:
+                if kernel.encode() in f.read():
+                    todo.append(path)
+    while todo:
+        path = os.path.normpath(todo.pop())
+        if path in files or not os.path.exists(path):
+            continue
+        files.add(path)
+        with open(path) as f:
+            for line in f:
+                line = line.strip()
+                if line.startswith("#include \""):
+                    todo.append(os.path.join(os.path.dirname(path), line.split('"')[1]))
+    h = hashlib.sha256()
+    for path in sorted(files):
+        h.update(os.path.relpath(path, ROOT).encode())
         with open(path, "rb") as f:
-            data = f.read()
-        if kernel.encode() in data or fn.endswith((".cuh", ".h")):
-            h.update(fn.encode())
-            h.update(data)
+            h.update(f.read())
     return h.hexdigest()[:16]
 
 
@@ -294,25 +343,45 @@ def run_ours(args):
     peaks = load_peaks()
     units = w.B * w.T * w.H  # token-heads per launch
     kernels = {}
+    peak = peaks["bf16_tflops_sustained"]
+    hbm = peaks["hbm_gbs"]
     for name, r in prof.items():
         f = flops_per_token_head(name, w.E, w.dk, w.dv) * units
+        by = bytes_per_token_head(name, w.E, w.dk, w.dv) * units
         avg_ms = r["ms"] / max(r["launches"], 1)
+        # the binding roofline: the larger of the tensor-core time and the HBM time
+        t_tc = f / (peak * 1e12) if f else 0.0
+        t_hbm = by / (hbm * 1e9) if by else 0.0
         kernels[name] = {"launches": r["launches"], "avg_ms": round(avg_ms, 4),
                          "share": round(r["ms"] / max(sum(v["ms"] for v in prof.values()), 1e-9), 4),
-                         "tflops": round(f / (avg_ms / 1e3) / 1e12, 2) if f else None}
+                         "tflops": round(f / (avg_ms / 1e3) / 1e12, 2) if f else None,
+                         "gbs": round(by / (avg_ms / 1e3) / 1e9, 1) if by else None,
+                         "bound": "hbm" if t_hbm >= t_tc else "tensor",
+                         "roofline_ms": round(max(t_tc, t_hbm) * 1e3, 4)}
     top = max(prof, key=lambda n: prof[n]["ms"])
-    top_flops = flops_per_token_head(top, w.E, w.dk, w.dv) * units
     top_avg_s = prof[top]["ms"] / prof[top]["launches"] / 1e3
-    achieved = top_flops / top_avg_s / 1e12
-    peak = peaks["bf16_tflops_sustained"]
     traffic = ncu_traffic(top, units)
-    roofline = {"kernel": top, "bound": "tensor", "achieved": round(achieved, 3),
-                "peak": peak, "unit": "TFLOP/s", "frac": round(achieved / peak, 5),
-                "traffic": traffic,
-                "peak_source": f"bf16 dense sustained, {peaks['source']} (MEASURED_PEAKS.json)"
-                if peaks["source"] == "measured" else "bf16 dense sustained, fallback"}
+    if kernels[top]["bound"] == "hbm":
+        top_bytes = bytes_per_token_head(top, w.E, w.dk, w.dv) * units
+        achieved = top_bytes / top_avg_s / 1e9
+        roofline = {"kernel": top, "bound": "hbm", "achieved": round(achieved, 1), "peak": hbm,
+                    "unit": "GB/s", "frac": round(achieved / hbm, 4), "traffic": traffic,
+                    "algorithmic_bytes": int(top_bytes),
+                    "peak_source": f"HBM copy bandwidth, {peaks['source']} (MEASURED_PEAKS.json)"
+                    if peaks["source"] == "measured" else "HBM copy bandwidth, fallback"}
+    else:
+        top_flops = flops_per_token_head(top, w.E, w.dk, w.dv) * units
+        achieved = top_flops / top_avg_s / 1e12
+        roofline = {"kernel": top, "bound": "tensor", "achieved": round(achieved, 3),
+                    "peak": peak, "unit": "TFLOP/s", "frac": round(achieved / peak, 5),
+                    "traffic": traffic,
+                    "peak_source": f"bf16 dense sustained, {peaks['source']} (MEASURED_PEAKS.json)"
+                    if peaks["source"] == "measured" else "bf16 dense sustained, fallback"}
     total_flops = sum(flops_per_token_head(n, w.E, w.dk, w.dv) * units * prof[n]["launches"]
                       for n in prof) / args.steps
+    total_bytes = sum(bytes_per_token_head(n, w.E, w.dk, w.dv) * units * prof[n]["launches"]
+                      for n in prof) / args.steps
+    roofline_ms_step = sum(v["roofline_ms"] * v["launches"] for v in kernels.values()) / args.steps
     gpu_launches = sum(r["launches"] for r in prof.values())
 
     # ---- end to end through the public API from pinned host buffers
@@ -361,6 +430,10 @@ def run_ours(args):
                        "l2": "inputs larger than L2 (q,k,v,dO 268 MB each per GPU)"},
             "tflops": round(total_flops / (ms_step / 1e3) / 1e12, 3),
             "tflops_frac": round(total_flops / (ms_step / 1e3) / 1e12 / peak, 5),
+            "step_hbm": {"algorithmic_gb": round(total_bytes / 1e9, 3),
+                         "achieved_gbs": round(total_bytes / (ms_step / 1e3) / 1e9, 1),
+                         "frac": round(total_bytes / (ms_step / 1e3) / 1e9 / hbm, 4),
+                         "roofline_ms": round(roofline_ms_step, 4)},
             "roofline": roofline, "kernels": kernels, "gpu_launches": gpu_launches,
             "clocks": ck, "clocks_remeasured": remeasured,
             "e2e": e2e, "packed": packed, "variants": variants, "layer_io": layer, "decode": decode, "cpu_baseline": cpu, "impl": "ours",

@@ -36,6 +36,7 @@ struct FwdPlan {
                          //    (b,h,chunk) 64 rows x dv bf16 hi then lo, SW128 K-major 64-row
                          //    blocks, rows past T zero
     int tc_tv;           // value columns per CTA of the tensor-core recurrence (0: SIMT)
+    int need_A;          // 1: the fp32 A matrices are read (a CUDA-core recurrence follows)
     size_t bytes;        // total
 };
 

@@ -216,7 +216,8 @@ chunk_prep_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     const size_t mat = ((size_t(b) * H + h) * NT + c) * (64 * 64);
 #pragma unroll
     for (int a = 0; a < 4; ++a) {
-        *reinterpret_cast<float4*>(p.Aout + mat + (R0 + a) * 64 + S0) = make_float4(Av[a][0], Av[a][1], Av[a][2], Av[a][3]);
+        if (p.Aout)
+            *reinterpret_cast<float4*>(p.Aout + mat + (R0 + a) * 64 + S0) = make_float4(Av[a][0], Av[a][1], Av[a][2], Av[a][3]);
     }
 #pragma unroll
     for (int c2 = 0; c2 < 4; ++c2) {
@@ -378,7 +379,7 @@ cudaError_t launch_chunk_prep_tc(const tla_problem& p, const FwdPlan& fp, char* 
     a.k2 = (const __nv_bfloat16*)p.k2;
     a.G = (const float*)(ws + fp.G);
     a.beta = p.beta;
-    a.Aout = (float*)(ws + fp.A);
+    a.Aout = fp.need_A ? (float*)(ws + fp.A) : nullptr;   // read only by the CUDA-core backward
     a.Nout = p.use_delta ? (float*)(ws + fp.N) : nullptr;
     a.A2out = (__nv_bfloat16*)(ws + fp.A2);
     a.BTout = fp.tcb ? (__nv_bfloat16*)(ws + fp.BT) : nullptr;

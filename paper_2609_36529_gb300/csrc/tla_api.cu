@@ -109,6 +109,9 @@ FwdPlan plan_fwd(const tla_problem& p, int save) {
         f.ck_tiles = (f.tcb && tc_grads_shape_ok(p)) ? 1 : 0;
         if (f.tcb) { f.BT = off; off = align256(off + 2 * mats); }
     }
+    // A feeds the CUDA-core recurrences only: the forward without tensor cores, or the
+    // backward recurrence when it cannot run on tensor cores
+    f.need_A = (!f.tc_tv || (save && !f.tcb)) ? 1 : 0;
     if (save) {
         f.S = off; off = align256(off + states);
         f.U = off; off = align256(off + tokV);

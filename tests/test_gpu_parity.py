@@ -260,6 +260,30 @@ def test_decode_steps(dtype, use_delta, dk, dv, E):
         close(f"state step {step}", state, ref_state, 1e-4)
 
 
+@pytest.mark.parametrize("dtype", ["fp32", "bf16"])
+@pytest.mark.parametrize("use_delta", [True, False])
+def test_decode_many_heads(dtype, use_delta):
+    """Enough (b, h, 16-column) slabs that each CTA of the persistent decode walks several of
+    them through its shared-memory ring (dv = 48: three column blocks; E*dk = 512 rows)."""
+    B, H, dk, dv, E = 40, 4, 128, 48, 4
+    gen = torch.Generator("cuda").manual_seed(77)
+    state = 0.1 * torch.randn(B, H, E, dk, dv, device="cuda", generator=gen)
+    ref_state = _np(state)
+    for step in range(3):
+        d = inputs.decode_inputs(B, H, dk, dv, E, dtype=dtype, device="cuda", gen=gen)
+        o = tla.tla_decode_step(state, d["q"], d["k"], d["v"], d["q2"], d["k2"], d["g"], d["beta"],
+                                use_delta=use_delta)
+        torch.cuda.synchronize()
+        c = {n: _np(t) for n, t in d.items()}
+        ro, ref_state = oracle.decode_step(ref_state, c["q"], c["k"], c["v"], c["q2"], c["k2"],
+                                           c["g"], c["beta"], use_delta=use_delta)
+        if dtype == "fp32":
+            close(f"o step {step}", o, ro, TOL["fp32"])
+        else:   # bf16-stored o: the tolerance plus its own rounding
+            close_rounded(f"o step {step}", o, ro, TOL["bf16"])
+        close(f"state step {step}", state, ref_state, 1e-4)
+
+
 def test_decode_after_chunk_prefill_matches_token_recurrence():
     """Prefill by the chunk forward, then decode: equals the oracle's recurrence over all tokens."""
     x = inputs.chunk_inputs(2, 70, 2, 64, 64, 4, dtype="fp32", with_beta=True, device="cuda",
