@@ -263,8 +263,8 @@ def test_decode_steps(dtype, use_delta, dk, dv, E):
 @pytest.mark.parametrize("dtype", ["fp32", "bf16"])
 @pytest.mark.parametrize("use_delta", [True, False])
 def test_decode_many_heads(dtype, use_delta):
-    """Enough (b, h, 16-column) slabs that each CTA of the persistent decode walks several of
-    them through its shared-memory ring (dv = 48: three column blocks; E*dk = 512 rows)."""
+    """Many (b, h, 16-column) slabs, several waves of CTAs (dv = 48: three column blocks;
+    E*dk = 512 rows), every output checked."""
     B, H, dk, dv, E = 40, 4, 128, 48, 4
     gen = torch.Generator("cuda").manual_seed(77)
     state = 0.1 * torch.randn(B, H, E, dk, dv, device="cuda", generator=gen)
