@@ -38,6 +38,17 @@ import torch  # noqa: E402
 
 HEADLINE_METRIC = "tokens/s triadic GDN fwd+bwd (T=8K, E=4); TFLOP/s and decode GB/s vs GB300 peak"
 CHUNK = 64
+OUT_DTYPE = torch.float32    # o, dq, dk, dv, dq', dk' (fp32, the accumulation precision); dg, dbeta fp32
+
+
+def make_grads(x, out_dtype, dev):
+    """Gradient buffers: dq, dk, dv, dq', dk' in out_dtype; dg and dbeta fp32."""
+    od = dict(dtype=out_dtype, device=dev)
+    return {"dq": torch.empty(x["q"].shape, **od), "dk": torch.empty(x["k"].shape, **od),
+            "dv": torch.empty(x["v"].shape, **od), "dq2": torch.empty(x["q2"].shape, **od),
+            "dk2": torch.empty(x["k2"].shape, **od),
+            "dg": torch.empty(x["g"].shape, dtype=torch.float32, device=dev),
+            "dbeta": torch.empty(x["beta"].shape, dtype=torch.float32, device=dev)}
 
 
 # ----------------------------------------------------------------------------- helpers
@@ -285,17 +296,14 @@ def run_ours(args):
     x = inputs.workload_inputs(w, device=dev, seed=rank)
     stream = torch.cuda.current_stream(dev)
 
-    # preallocated outputs and workspaces (allocation is outside the timed region)
-    o = torch.empty(w.B, w.T, w.H, w.dv, dtype=torch.float32, device=dev)   # fp32 results
+    # preallocated outputs and workspaces (allocation is outside the timed region): o and every
+    # gradient fp32 (the kernels accumulate in fp32; bf16 results are a variant below)
+    o = torch.empty(w.B, w.T, w.H, w.dv, dtype=OUT_DTYPE, device=dev)
     p = tla.make_problem(x["q"], x["k"], x["v"], x["q2"], x["k2"], x["g"], x["beta"], None, o,
                          None, use_delta=True)
     fws = torch.empty(tla.fwd_workspace_bytes(p, True), dtype=torch.uint8, device=dev)
     bws = torch.empty(tla.bwd_workspace_bytes(p), dtype=torch.uint8, device=dev)
-    f32 = dict(dtype=torch.float32, device=dev)
-    grads = {"dq": torch.empty(x["q"].shape, **f32), "dk": torch.empty(x["k"].shape, **f32),
-             "dv": torch.empty(x["v"].shape, **f32), "dq2": torch.empty(x["q2"].shape, **f32),
-             "dk2": torch.empty(x["k2"].shape, **f32), "dg": torch.empty_like(x["g"]),
-             "dbeta": torch.empty_like(x["beta"])}
+    grads = make_grads(x, OUT_DTYPE, dev)
 
     def step(xx):
         tla.tla_chunk_fwd(xx["q"], xx["k"], xx["v"], xx["q2"], xx["k2"], xx["g"], xx["beta"],
@@ -426,7 +434,8 @@ def run_ours(args):
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": {"workload": w.name, "B": w.B, "T": w.T, "H": w.H, "dk": w.dk, "dv": w.dv,
                        "E": w.E, "chunk": CHUNK, "variant": "triadic GDN (joint-key delta rule)",
-                       "state": "fp32", "outputs": "fp32 o and gradients", "parallelism": f"replicas x{ws_n} (independent sequences)",
+                       "state": "fp32", "outputs": "fp32 o and gradients",
+                       "parallelism": f"replicas x{ws_n} (independent sequences)",
                        "l2": "inputs larger than L2 (q,k,v,dO 268 MB each per GPU)"},
             "tflops": round(total_flops / (ms_step / 1e3) / 1e12, 3),
             "tflops_frac": round(total_flops / (ms_step / 1e3) / 1e12 / peak, 5),
@@ -518,16 +527,12 @@ def run_packed(args, tla, inputs, w, dev, stream, barrier, max_over_ranks, ws_n,
     lens = inputs.packed_lengths(total, 1000, seed=rank)
     x, cu = inputs.packed_inputs(lens, w.H, w.dk, w.dv, w.E, dtype=w.dtype, backward=True,
                                  device=dev, seed=100 + rank)
-    o = torch.empty(1, total, w.H, w.dv, dtype=torch.float32, device=dev)
+    o = torch.empty(1, total, w.H, w.dv, dtype=OUT_DTYPE, device=dev)
     p = tla.make_problem(x["q"], x["k"], x["v"], x["q2"], x["k2"], x["g"], x["beta"], None, o,
                          None, use_delta=True, cu_seqlens=cu)
     fws = torch.empty(tla.fwd_workspace_bytes(p, True), dtype=torch.uint8, device=dev)
     bws = torch.empty(tla.bwd_workspace_bytes(p), dtype=torch.uint8, device=dev)
-    f32 = dict(dtype=torch.float32, device=dev)
-    grads = {"dq": torch.empty(x["q"].shape, **f32), "dk": torch.empty(x["k"].shape, **f32),
-             "dv": torch.empty(x["v"].shape, **f32), "dq2": torch.empty(x["q2"].shape, **f32),
-             "dk2": torch.empty(x["k2"].shape, **f32), "dg": torch.empty_like(x["g"]),
-             "dbeta": torch.empty_like(x["beta"])}
+    grads = make_grads(x, OUT_DTYPE, dev)
 
     def step():
         tla.tla_chunk_fwd(x["q"], x["k"], x["v"], x["q2"], x["k2"], x["g"], x["beta"], None,
@@ -579,25 +584,25 @@ def _time_steps(step, k, warm, stream, barrier, max_over_ranks):
 def run_variants(args, tla, inputs, w, dev, stream, barrier, max_over_ranks, ws_n, rank,
                  headline):
     """Forward + backward tokens/s of the shape/gate variants: one log gate per head on the
-    headline workload (tensor-core path), and E = 32 slices with d_k = 64 (Table 4's
-    iso-state variant; CUDA-core path) on one 8192-token sequence."""
+    headline workload (tensor-core path), the headline with o and the input gradients in
+    bf16 (the input dtype), and E = 32 slices with d_k = 64 (Table 4's iso-state variant;
+    CUDA-core path) on one 8192-token sequence."""
     out = {}
     cases = [("gate_per_head", w.B, w.T, w.H, w.dk, w.dv, w.E, True),
+             ("bf16_outputs", w.B, w.T, w.H, w.dk, w.dv, w.E, False),
              ("E32_dk64", 1, w.T, w.H, 64, w.dv, 32, False)]
     for name, B, T, H, dk, dv, E, per_head in cases:
+        out_dtype = torch.bfloat16 if name == "bf16_outputs" else OUT_DTYPE
         x = inputs.chunk_inputs(B, T, H, dk, dv, E, dtype=w.dtype, with_beta=True,
                                 backward=True, device=dev, seed=200 + rank)
         if per_head:
             x["g"] = x["g"][..., 0].contiguous()
-        o = torch.empty(B, T, H, dv, dtype=torch.float32, device=dev)
+        o = torch.empty(B, T, H, dv, dtype=out_dtype, device=dev)
         p = tla.make_problem(x["q"], x["k"], x["v"], x["q2"], x["k2"], x["g"], x["beta"], None,
                              o, None, use_delta=True)
         fws = torch.empty(tla.fwd_workspace_bytes(p, True), dtype=torch.uint8, device=dev)
         bws = torch.empty(tla.bwd_workspace_bytes(p), dtype=torch.uint8, device=dev)
-        f32 = dict(dtype=torch.float32, device=dev)
-        grads = {n: torch.empty(x[k].shape, **f32) for n, k in
-                 (("dq", "q"), ("dk", "k"), ("dv", "v"), ("dq2", "q2"), ("dk2", "k2"),
-                  ("dg", "g"), ("dbeta", "beta"))}
+        grads = make_grads(x, out_dtype, dev)
 
         def step():
             tla.tla_chunk_fwd(x["q"], x["k"], x["v"], x["q2"], x["k2"], x["g"], x["beta"], None,
@@ -609,10 +614,11 @@ def run_variants(args, tla, inputs, w, dev, stream, barrier, max_over_ranks, ws_
         ms = _time_steps(step, 3, 3, stream, barrier, max_over_ranks)
         val = ws_n * B * T / (ms / 1e3)
         out[name] = {"config": {"B": B, "T": T, "H": H, "dk": dk, "dv": dv, "E": E,
-                                "gate": "per head [B,T,H]" if per_head else "per slice"},
+                                "gate": "per head [B,T,H]" if per_head else "per slice",
+                                "outputs": "fp32" if out_dtype == torch.float32 else "bf16"},
                      "value": round(val, 1), "unit": "tokens/s", "ms_per_step": round(ms, 4),
                      "path": "tensor cores" if dk == 128 else "CUDA cores (fp32 SIMT)"}
-        if per_head:
+        if B == w.B and T == w.T:
             out[name]["vs_headline"] = round(val / headline, 4)
         del x, fws, bws, grads, o
     if tla.tla_last_device_status() != 0:
