@@ -109,6 +109,6 @@ cudaError_t launch_sum_slices(const float* src, float* dst, long long n, int E, 
 cudaError_t launch_decode_step(int B, int H, int dk, int dv, int E, int use_delta, int dtype,
                                const void* q, const void* k, const void* v, const void* q2,
                                const void* k2, const float* g, const float* beta,
-                               float* state, void* o, cudaStream_t s);
+                               float* state, void* o, int* err, cudaStream_t s);
 
 }  // namespace tla

@@ -296,7 +296,7 @@ tla_status tla_decode_step(int B, int H, int dk, int dv, int E, int use_delta, i
     if (!dims_ok(dk) || !dims_ok(dv) || E > 32 || E * dk > 2048) return TLA_ERR_UNSUPPORTED;
     if ((long long)B * H > 65535) return TLA_ERR_UNSUPPORTED;  // grid.y
     return cuda_status(launch_decode_step(B, H, dk, dv, E, use_delta, dtype, q, k, v, q2, k2, g,
-                                          beta, state, o, (cudaStream_t)stream));
+                                          beta, state, o, device_error_word(), (cudaStream_t)stream));
 }
 
 const char* tla_status_string(int status) {
