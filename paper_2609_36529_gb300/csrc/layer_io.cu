@@ -22,7 +22,13 @@ constexpr int kSeg = 256;      // tokens per CTA of the prologue backward
 constexpr int kGateRows = 256; // (token, head) rows per CTA of the output gate
 
 __device__ __forceinline__ float sigm(float x) { return __fdividef(1.f, 1.f + __expf(-x)); }
-__device__ __forceinline__ float softplus(float x) { return x > 20.f ? x : log1pf(expf(x)); }
+// softplus(x) = log(1 + e^x) with fast intrinsics; for e^x < 2^-10 the series e (1 - e/2)
+// keeps the relative accuracy that log(1 + e) in fp32 would lose.
+__device__ __forceinline__ float softplus(float x) {
+    if (x > 20.f) return x;
+    const float e = __expf(x);
+    return e < 0.0009765625f ? e * fmaf(-0.5f, e, 1.f) : __logf(1.f + e);
+}
 
 template <typename T> __device__ __forceinline__ float ld(const void* p, size_t i) {
     return to_f(static_cast<const T*>(p)[i]);
@@ -101,8 +107,8 @@ __device__ __forceinline__ float warp_sum(float x) {
 }
 
 // Layout of the prologue kernels: a CTA of four warps takes one run of tokens of one
-// (b, h); warp 0 the q channels, warp 1 k, warp 2 v (four channels per lane), warp 3 the
-// q' and k' channels (one or two per lane) together with the gates and beta.  Each norm
+// (b, h); warp 0 the q channels, warp 1 k, warp 2 v (four channels per lane) and then the
+// gates and beta (v needs no norm), warp 3 the q' and k' channels (one or two per lane).  Each norm
 // is then a reduction inside one warp, so the warps never wait on one another.  A warp
 // walks its run token by token, keeping the last three projection rows (and, backward,
 // the last three pre-activation gradients) in registers: the width-K convolution uses
@@ -240,6 +246,15 @@ __device__ __forceinline__ void prologue_fwd_small(const tla_prologue_args& a, i
             }
         }
     }
+}
+
+// Log gates and beta of tokens [t0, t1) of (b, h) (the v warp, whose channels need no norm).
+__device__ __forceinline__ void prologue_fwd_gates(const tla_prologue_args& a, int b, int h, int t0,
+                                                   int t1) {
+    const int lane = threadIdx.x & 31;
+    const int E = a.E, T = a.T, H = a.H;
+    const size_t sE = size_t(H) * E;
+    const size_t rowE = (size_t(b) * T * H + h) * E;
     const int n = t1 - t0;
     for (int i0 = lane; i0 < n * E; i0 += 32 * 4) {   // log gates, four loads ahead
         float z[4];
@@ -251,7 +266,7 @@ __device__ __forceinline__ void prologue_fwd_small(const tla_prologue_args& a, i
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
             const int idx = i0 + 32 * u, i = idx / E, e = idx - i * E;
-            if (idx < n * E) a.g[rowE + (t0 + i) * sE + e] = -expf(a.A_log[h * E + e]) * softplus(z[u]);
+            if (idx < n * E) a.g[rowE + (t0 + i) * sE + e] = -__expf(a.A_log[h * E + e]) * softplus(z[u]);
         }
     }
     if (a.beta_in)
@@ -277,6 +292,7 @@ prologue_fwd_kernel(const tla_prologue_args a) {
     const int g = threadIdx.x >> 5, h = blockIdx.y, b = blockIdx.z;
     if (g < 3) prologue_fwd_qkv<Tin, VEC>(a, g, b, h, t0, t1);
     else prologue_fwd_small<Tin>(a, b, h, t0, t1);
+    if (g == 2) prologue_fwd_gates(a, b, h, t0, t1);
 }
 
 struct PrologueGrads {
@@ -502,13 +518,25 @@ __device__ __forceinline__ void prologue_bwd_small(const tla_prologue_args& a, c
 #pragma unroll
             for (int j = 0; j < 4; ++j)
                 if (j >= 4 - K) part[(off + lane + 32 * s) * K + j - (4 - K)] = dw[j][s];
+}
+
+// Gradients through the log gates and beta of tokens [t0, t1) of (b, h), with the gate-bias
+// and A_log partials of this CTA (the v warp, whose channels need no norm).
+__device__ __forceinline__ void prologue_bwd_gates(const tla_prologue_args& a, const PrologueGrads& gr,
+                                                   int b, int h, int t0, int t1, float* part) {
+    const int lane = threadIdx.x & 31;
+    const int dk = a.dk, dv = a.dv, E = a.E, K = a.K, T = a.T, H = a.H;
+    const int C = 2 * dk + dv + 2 * E;
+    const size_t sE = size_t(H) * E;
+    const size_t rowE = (size_t(b) * T * H + h) * E;
+    const int te = min(t1, T);
     // log gates: lane p * E + e takes gate e of tokens t0 + p, t0 + p + NP, ... (NP = 32 / E
     // phases), eight tokens' loads at a time; the phases' sums are added in order after.
     __shared__ float red[2][32];
     const int NP = 32 / E, p = lane / E, e = lane - p * E;
     float gbp = 0.f, gap = 0.f;
     if (p < NP) {
-        const float sA = -expf(a.A_log[h * E + e]), bias = a.gate_bias[h * E + e];
+        const float sA = -__expf(a.A_log[h * E + e]), bias = a.gate_bias[h * E + e];
         for (int tb = t0 + p; tb < te; tb += 8 * NP) {
             float z[8], dgv[8];
 #pragma unroll
@@ -572,6 +600,7 @@ prologue_bwd_kernel(const tla_prologue_args a, const PrologueGrads gr) {
     float* part = gr.part + ((size_t(b) * gridDim.x + seg) * a.H + h) * (size_t(C) * a.K + 2 * a.E);
     if (g < 3) prologue_bwd_qkv<Tin, Tg, VEC>(a, gr, g, b, h, t0, t1, part);
     else prologue_bwd_small<Tin, Tg>(a, gr, b, h, t0, t1, part);
+    if (g == 2) prologue_bwd_gates(a, gr, b, h, t0, t1, part);
 }
 
 // Fixed-order sums of the per-CTA partials: out[h][x] = sum_{b, seg} part[b][seg][h][x].
