@@ -174,7 +174,10 @@ tla_status tla_chunk_bwd(const tla_problem *p, const void *fwd_ws, size_t fwd_ws
  *   state [B,H,E,dk,dv] fp32, updated in place; o [B,H,dv] dtype (written).
  * Supported: dk, dv multiples of 16 up to 128, 1 <= E <= 32 with E*dk <= 2048,
  * B*H <= 65535.  A per-head gate is passed as E equal values of g.
- * No workspace.
+ * No workspace.  Each (b, h, 16 value columns) slab of the state is read once
+ * and written once (through shared memory by TMA when E*dk <= 1024 and is a
+ * multiple of 64); a bounded wait on that copy that expires records
+ * TLA_ERR_TIMEOUT for tla_last_device_status().
  */
 tla_status tla_decode_step(int B, int H, int dk, int dv, int E, int use_delta, int dtype,
                            const void *q, const void *k, const void *v,
