@@ -127,15 +127,15 @@ def bytes_per_token_head(kernel, E, dk, dv, C=CHUNK, in_b=2, out_b=4, delta=True
 
 
 def kernel_source_hash(kernel):
-    """Hash of the source that builds a kernel: the .cu files that define it and every local
-    header they include, recursively (to invalidate stale ncu traffic)."""
+    """Hash of the source that builds a kernel: the .cu files that define it (`<name>_kernel`)
+    and every local header they include, recursively (to invalidate stale ncu traffic)."""
     csrc = os.path.join(ROOT, "paper_2609_36529_gb300", "csrc")
     files, todo = set(), []
     for fn in sorted(os.listdir(csrc)):
         path = os.path.join(csrc, fn)
         if fn.endswith(".cu"):
             with open(path, "rb") as f:
-                if kernel.encode() in f.read():
+                if (kernel + "_kernel").encode() in f.read():
                     todo.append(path)
     while todo:
         path = os.path.normpath(todo.pop())

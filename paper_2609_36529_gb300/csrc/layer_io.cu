@@ -12,14 +12,20 @@
 
 #include "common.cuh"
 #include "internal.h"
+#include "sm100.cuh"
 
 namespace tla {
+
+// Address of the library's device error word on the current device (tla_api.cu): kernels
+// with bounded waits record TLA_ERR_TIMEOUT there.
+int* device_error_word();
+
 namespace {
 
 constexpr int kThreads = 256;
 constexpr int kFwdRun = 128;   // tokens per CTA of the prologue forward
 constexpr int kSeg = 256;      // tokens per CTA of the prologue backward
-constexpr int kGateRows = 256; // (token, head) rows per CTA of the output gate
+constexpr int kGateTile = 64;  // (token, head) rows per CTA of the output gate
 
 __device__ __forceinline__ float sigm(float x) { return __fdividef(1.f, 1.f + __expf(-x)); }
 // softplus(x) = log(1 + e^x) with fast intrinsics; for e^x < 2^-10 the series e (1 - e/2)
@@ -617,101 +623,163 @@ __global__ void reduce_partials_kernel(const float* __restrict__ part, int nblk,
     else dA[h * E + x - CK - E] = acc;
 }
 
-// Output gate: one warp per (token, head) row, four channels per lane (dv <= 128 and a
-// multiple of 16, so every row starts on a 16-byte boundary), four consecutive rows'
-// loads issued before the first is used.
+// Bulk copy shared -> global (16-byte aligned addresses, size a multiple of 16) in the issuing
+// thread's bulk async-group.
+__device__ __forceinline__ void bulk_store_g(void* dst, const void* src, uint32_t bytes) {
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(
+                     reinterpret_cast<uint64_t>(dst)),
+                 "r"(sm100::smem_u32(src)), "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit_g() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read_g() {
+    asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+}
+
+// Output gate through shared memory (dv <= 128 and a multiple of 16): the kGateTile
+// consecutive (token, head) rows of a CTA are contiguous in o, z and y, so they arrive by one
+// bulk copy per tensor; one warp per row (four channels per lane) normalises and gates in
+// shared memory, y over z in place, and y leaves by one bulk copy.  With little register
+// state several CTAs' copies are in flight on an SM.
 template <typename To, typename Tz>
 __global__ void __launch_bounds__(kThreads)
-gate_fwd_kernel(const tla_gate_args a, long long rows) {
+gate_fwd_kernel(const tla_gate_args a, long long rows, int* err) {
+    using namespace sm100;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 127) & ~uintptr_t(127));
+    __shared__ __align__(8) uint64_t bar;
     const int dv = a.dv, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const long long r0 = blockIdx.x * (long long)kGateTile;
+    const int nr = (int)min((long long)kGateTile, rows - r0);
+    To* so = reinterpret_cast<To*>(sm);
+    Tz* sz = reinterpret_cast<Tz*>(sm + size_t(kGateTile) * dv * sizeof(To));
+    const uint32_t bo = uint32_t(nr) * dv * sizeof(To), bz = uint32_t(nr) * dv * sizeof(Tz);
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        fence_barrier_init();
+        mbar_arrive_expect_tx(&bar, bo + bz);
+        bulk_load(so, static_cast<const To*>(a.o) + r0 * dv, bo, &bar);
+        bulk_load(sz, static_cast<const Tz*>(a.z) + r0 * dv, bz, &bar);
+    }
     const bool act = 4 * lane < dv;
     float wn[4] = {0.f, 0.f, 0.f, 0.f};
     if (act) ld4<true>(a.w_norm + 4 * lane, wn);
-    const long long r0 = blockIdx.x * (long long)kGateRows, r1 = min(rows, r0 + kGateRows);
-    const To* po = static_cast<const To*>(a.o) + 4 * lane;
-    const Tz* pz = static_cast<const Tz*>(a.z) + 4 * lane;
-    Tz* py = static_cast<Tz*>(a.y) + 4 * lane;
-    for (long long rb = r0 + warp * 4; rb < r1; rb += (kThreads / 32) * 4) {
-        float o[4][4], z[4][4];
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            if (act && rb + i < r1) {
-                ld4<true>(po + (rb + i) * dv, o[i]);
-                ld4<true>(pz + (rb + i) * dv, z[i]);
-            } else {
-#pragma unroll
-                for (int u = 0; u < 4; ++u) o[i][u] = z[i][u] = 0.f;
-            }
+    __syncthreads();
+    const bool ok = mbar_wait(&bar, 0);
+    if (__syncthreads_or(!ok)) {
+        if (threadIdx.x == 0) {
+            record_device_error(err, TLA_ERR_TIMEOUT);
+            mbar_wait(&bar, 0);   // bounded drain of the copies
         }
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            float ss = 0.f;
-#pragma unroll
-            for (int u = 0; u < 4; ++u) ss = fmaf(o[i][u], o[i][u], ss);
-            const float rr = rsqrtf(warp_sum(ss) / dv + a.eps);
-            float y[4];
-#pragma unroll
-            for (int u = 0; u < 4; ++u) y[u] = o[i][u] * rr * wn[u] * sigm(z[i][u]);
-            if (act && rb + i < r1) st4<true>(py + (rb + i) * dv, y);
+        return;
+    }
+    for (int r = warp; r < nr; r += kThreads / 32) {
+        float o[4] = {0.f, 0.f, 0.f, 0.f}, z[4] = {0.f, 0.f, 0.f, 0.f};
+        if (act) {
+            ld4<true>(so + r * dv + 4 * lane, o);
+            ld4<true>(sz + r * dv + 4 * lane, z);
         }
+        float ss = 0.f;
+#pragma unroll
+        for (int u = 0; u < 4; ++u) ss = fmaf(o[u], o[u], ss);
+        const float rr = rsqrtf(warp_sum(ss) / dv + a.eps);
+        float y[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) y[u] = o[u] * rr * wn[u] * sigm(z[u]);
+        if (act) st4<true>(sz + r * dv + 4 * lane, y);
+    }
+    fence_proxy_async_smem();
+    __syncthreads();
+    if (threadIdx.x == 0) {   // the CTA's shared memory must outlive the copy's read
+        bulk_store_g(static_cast<Tz*>(a.y) + r0 * dv, sz, bz);
+        bulk_commit_g();
+        bulk_wait_read_g();
     }
 }
 
-// Backward of the output gate over the rows [blk * rpb, (blk + 1) * rpb); the w_norm
-// gradient is summed per lane, then over the CTA's warps in order into part[blk][dv].
+// Backward of the output gate through shared memory, kGateBwdTiles tiles of kGateTile rows per
+// CTA in turn: a tile's rows of o, z and dy arrive by one bulk copy each; do and dz are written
+// in place over o and z and leave by one bulk copy each; the w_norm gradient is summed per lane
+// over the CTA's rows, then over its warps in order into part[blk][dv].
+constexpr int kGateBwdTiles = 4;
 template <typename To, typename Tz>
 __global__ void __launch_bounds__(kThreads)
-gate_bwd_kernel(const tla_gate_args a, long long rows, long long rpb, const void* dy, void* d_o,
-                void* dz, float* part) {
+gate_bwd_kernel(const tla_gate_args a, long long rows, const void* dy, void* d_o, void* dz,
+                float* part, int* err) {
+    using namespace sm100;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 127) & ~uintptr_t(127));
+    __shared__ __align__(8) uint64_t bar;
     __shared__ float wsm[kThreads / 32][128];
     const int dv = a.dv, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    To* so = reinterpret_cast<To*>(sm);                                          // o, then do
+    Tz* sz = reinterpret_cast<Tz*>(sm + size_t(kGateTile) * dv * sizeof(To));    // z, then dz
+    Tz* sg = sz + size_t(kGateTile) * dv;                                        // dy
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        fence_barrier_init();
+    }
     const bool act = 4 * lane < dv;
     float wn[4] = {0.f, 0.f, 0.f, 0.f}, wacc[4] = {0.f, 0.f, 0.f, 0.f};
     if (act) ld4<true>(a.w_norm + 4 * lane, wn);
-    const long long r0 = blockIdx.x * rpb, r1 = min(rows, r0 + rpb);
-    const To* po = static_cast<const To*>(a.o) + 4 * lane;
-    const Tz* pz = static_cast<const Tz*>(a.z) + 4 * lane;
-    const Tz* pg = static_cast<const Tz*>(dy) + 4 * lane;
-    To* pdo = static_cast<To*>(d_o) + 4 * lane;
-    Tz* pdz = static_cast<Tz*>(dz) + 4 * lane;
     const float inv_dv = 1.f / dv;
-    for (long long rb = r0 + warp * 4; rb < r1; rb += (kThreads / 32) * 4) {
-        float o[4][4], z[4][4], g[4][4];
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            if (act && rb + i < r1) {
-                ld4<true>(po + (rb + i) * dv, o[i]);
-                ld4<true>(pz + (rb + i) * dv, z[i]);
-                ld4<true>(pg + (rb + i) * dv, g[i]);
-            } else {
-#pragma unroll
-                for (int u = 0; u < 4; ++u) o[i][u] = z[i][u] = g[i][u] = 0.f;
-            }
+    __syncthreads();
+    for (int j = 0; j < kGateBwdTiles; ++j) {
+        const long long r0 = (blockIdx.x * (long long)kGateBwdTiles + j) * kGateTile;
+        if (r0 >= rows) break;
+        const int nr = (int)min((long long)kGateTile, rows - r0);
+        const uint32_t bo = uint32_t(nr) * dv * sizeof(To), bz = uint32_t(nr) * dv * sizeof(Tz);
+        if (threadIdx.x == 0) {
+            mbar_arrive_expect_tx(&bar, bo + 2 * bz);
+            bulk_load(so, static_cast<const To*>(a.o) + r0 * dv, bo, &bar);
+            bulk_load(sz, static_cast<const Tz*>(a.z) + r0 * dv, bz, &bar);
+            bulk_load(sg, static_cast<const Tz*>(dy) + r0 * dv, bz, &bar);
         }
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
+        const bool ok = mbar_wait(&bar, uint32_t(j) & 1u);
+        if (__syncthreads_or(!ok)) {
+            if (threadIdx.x == 0) {
+                record_device_error(err, TLA_ERR_TIMEOUT);
+                mbar_wait(&bar, uint32_t(j) & 1u);   // bounded drain of the copies
+            }
+            return;
+        }
+        for (int r = warp; r < nr; r += kThreads / 32) {
+            float o[4] = {0.f, 0.f, 0.f, 0.f}, z[4] = {0.f, 0.f, 0.f, 0.f}, g[4] = {0.f, 0.f, 0.f, 0.f};
+            if (act) {
+                ld4<true>(so + r * dv + 4 * lane, o);
+                ld4<true>(sz + r * dv + 4 * lane, z);
+                ld4<true>(sg + r * dv + 4 * lane, g);
+            }
             float ss = 0.f;
 #pragma unroll
-            for (int u = 0; u < 4; ++u) ss = fmaf(o[i][u], o[i][u], ss);
+            for (int u = 0; u < 4; ++u) ss = fmaf(o[u], o[u], ss);
             const float rr = rsqrtf(warp_sum(ss) * inv_dv + a.eps);
             float nh[4], dnh[4], dzv[4], dot = 0.f;
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
-                const float sg = sigm(z[i][u]);
-                nh[u] = o[i][u] * rr;
-                dnh[u] = g[i][u] * wn[u] * sg;
-                dzv[u] = g[i][u] * nh[u] * wn[u] * sg * (1.f - sg);
-                if (rb + i < r1) wacc[u] = fmaf(g[i][u] * sg, nh[u], wacc[u]);
+                const float sgm = sigm(z[u]);
+                nh[u] = o[u] * rr;
+                dnh[u] = g[u] * wn[u] * sgm;
+                dzv[u] = g[u] * nh[u] * wn[u] * sgm * (1.f - sgm);
+                wacc[u] = fmaf(g[u] * sgm, nh[u], wacc[u]);
                 dot = fmaf(dnh[u], nh[u], dot);
             }
             dot = warp_sum(dot) * inv_dv;
             float dov[4];
 #pragma unroll
             for (int u = 0; u < 4; ++u) dov[u] = rr * (dnh[u] - nh[u] * dot);
-            if (act && rb + i < r1) {
-                st4<true>(pdz + (rb + i) * dv, dzv);
-                st4<true>(pdo + (rb + i) * dv, dov);
+            if (act) {
+                st4<true>(sz + r * dv + 4 * lane, dzv);
+                st4<true>(so + r * dv + 4 * lane, dov);
             }
+        }
+        fence_proxy_async_smem();
+        __syncthreads();
+        if (threadIdx.x == 0) {   // the next tile's copies overwrite these buffers
+            bulk_store_g(static_cast<To*>(d_o) + r0 * dv, so, bo);
+            bulk_store_g(static_cast<Tz*>(dz) + r0 * dv, sz, bz);
+            bulk_commit_g();
+            bulk_wait_read_g();
         }
     }
     if (act)
@@ -779,18 +847,14 @@ tla_status check_gate(const tla_gate_args* a) {
 }
 
 int n_segments(const tla_prologue_args* a) { return (a->T + kSeg - 1) / kSeg; }
+// forward: one CTA per kGateTile (token, head) rows; backward: kGateBwdTiles such tiles per
+// CTA, each CTA writing one partial w_norm gradient
 long long gate_blocks(const tla_gate_args* a) {
-    return ((long long)a->B * a->T * a->H + kGateRows - 1) / kGateRows;
-}
-// backward: at most 8 CTAs per SM of 152, each over a contiguous range of rows
-long long gate_bwd_rows_per_block(const tla_gate_args* a) {
-    const long long rows = (long long)a->B * a->T * a->H;
-    const long long per = (rows + 152 * 8 - 1) / (152 * 8);
-    return std::max(32LL, (per + 31) / 32 * 32);
+    return ((long long)a->B * a->T * a->H + kGateTile - 1) / kGateTile;
 }
 long long gate_bwd_blocks(const tla_gate_args* a) {
-    const long long rows = (long long)a->B * a->T * a->H, rpb = gate_bwd_rows_per_block(a);
-    return (rows + rpb - 1) / rpb;
+    const long long per = (long long)kGateTile * kGateBwdTiles;
+    return ((long long)a->B * a->T * a->H + per - 1) / per;
 }
 size_t prologue_part_bytes(const tla_prologue_args* a) {
     const int C = 2 * a->dk + a->dv + 2 * a->E;
@@ -888,14 +952,24 @@ extern "C" tla_status tla_output_gate(const tla_gate_args* a, void* stream) {
     cudaStream_t s = (cudaStream_t)stream;
     const long long rows = (long long)a->B * a->T * a->H;
     const unsigned blocks = (unsigned)gate_blocks(a);
+    const size_t so = a->o_dtype == TLA_FP32 ? 4 : 2, sz = a->dtype == TLA_FP32 ? 4 : 2;
+    const size_t smem = 128 + size_t(kGateTile) * a->dv * (so + sz);
+    int* err = device_error_word();
     prof_before("output_gate", s);
+#define TLA_GATE_LAUNCH(TO, TZ)                                                                    \
+    do {                                                                                           \
+        auto kern = gate_fwd_kernel<TO, TZ>;                                                       \
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);        \
+        kern<<<blocks, kThreads, smem, s>>>(*a, rows, err);                                        \
+    } while (0)
     if (a->o_dtype == TLA_FP32) {
-        if (a->dtype == TLA_FP32) gate_fwd_kernel<float, float><<<blocks, kThreads, 0, s>>>(*a, rows);
-        else gate_fwd_kernel<float, __nv_bfloat16><<<blocks, kThreads, 0, s>>>(*a, rows);
+        if (a->dtype == TLA_FP32) TLA_GATE_LAUNCH(float, float);
+        else TLA_GATE_LAUNCH(float, __nv_bfloat16);
     } else {
-        if (a->dtype == TLA_FP32) gate_fwd_kernel<__nv_bfloat16, float><<<blocks, kThreads, 0, s>>>(*a, rows);
-        else gate_fwd_kernel<__nv_bfloat16, __nv_bfloat16><<<blocks, kThreads, 0, s>>>(*a, rows);
+        if (a->dtype == TLA_FP32) TLA_GATE_LAUNCH(__nv_bfloat16, float);
+        else TLA_GATE_LAUNCH(__nv_bfloat16, __nv_bfloat16);
     }
+#undef TLA_GATE_LAUNCH
     prof_after(s);
     return cuda_status(cudaGetLastError());
 }
@@ -916,24 +990,30 @@ extern "C" tla_status tla_output_gate_bwd(const tla_gate_args* a, const void* dy
         for (const void* p : ptrs)
             if (!al16(p)) return TLA_ERR_INVALID_ARG;
     }
-    const long long nblk = gate_bwd_blocks(a), rpb = gate_bwd_rows_per_block(a);
+    const long long nblk = gate_bwd_blocks(a);
     if (!workspace || workspace_bytes < (size_t)nblk * a->dv * sizeof(float)) return TLA_ERR_WORKSPACE;
     cudaStream_t s = (cudaStream_t)stream;
     const long long rows = (long long)a->B * a->T * a->H;
     float* part = (float*)workspace;
     const unsigned g = (unsigned)nblk;
+    const size_t so = a->o_dtype == TLA_FP32 ? 4 : 2, sz = a->dtype == TLA_FP32 ? 4 : 2;
+    const size_t smem = 128 + size_t(kGateTile) * a->dv * (so + 2 * sz);
+    int* err = device_error_word();
     prof_before("output_gate_bwd", s);
+#define TLA_GATE_BWD_LAUNCH(TO, TZ)                                                                \
+    do {                                                                                           \
+        auto kern = gate_bwd_kernel<TO, TZ>;                                                       \
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);        \
+        kern<<<g, kThreads, smem, s>>>(*a, rows, dy, d_o, dz, part, err);                          \
+    } while (0)
     if (a->o_dtype == TLA_FP32) {
-        if (a->dtype == TLA_FP32)
-            gate_bwd_kernel<float, float><<<g, kThreads, 0, s>>>(*a, rows, rpb, dy, d_o, dz, part);
-        else
-            gate_bwd_kernel<float, __nv_bfloat16><<<g, kThreads, 0, s>>>(*a, rows, rpb, dy, d_o, dz, part);
+        if (a->dtype == TLA_FP32) TLA_GATE_BWD_LAUNCH(float, float);
+        else TLA_GATE_BWD_LAUNCH(float, __nv_bfloat16);
     } else {
-        if (a->dtype == TLA_FP32)
-            gate_bwd_kernel<__nv_bfloat16, float><<<g, kThreads, 0, s>>>(*a, rows, rpb, dy, d_o, dz, part);
-        else
-            gate_bwd_kernel<__nv_bfloat16, __nv_bfloat16><<<g, kThreads, 0, s>>>(*a, rows, rpb, dy, d_o, dz, part);
+        if (a->dtype == TLA_FP32) TLA_GATE_BWD_LAUNCH(__nv_bfloat16, float);
+        else TLA_GATE_BWD_LAUNCH(__nv_bfloat16, __nv_bfloat16);
     }
+#undef TLA_GATE_BWD_LAUNCH
     prof_after(s);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return TLA_ERR_CUDA;

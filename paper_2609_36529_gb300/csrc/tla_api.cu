@@ -62,7 +62,7 @@ static __global__ void selftest_wait_kernel(unsigned long long timeout_ns, int* 
 }
 
 // Address of the error word on the current device (looked up once per device).
-static int* device_error_word() {
+int* device_error_word() {
     static int* ptr[64] = {nullptr};
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
