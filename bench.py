@@ -60,6 +60,30 @@ def dist_env():
     return ws, rank, local
 
 
+def rank_ops(ws_n, device):
+    """barrier() and max_over_ranks(x) of a run with ws_n ranks.  With one rank both are no-ops;
+    with more, a process-group barrier and an all-reduce MAX of one float64 on `device`: the
+    run's only collectives, on timings, never on data (ranks process independent sequences)."""
+    def barrier():
+        if ws_n > 1:
+            torch.distributed.barrier()
+
+    def max_over_ranks(x):
+        if ws_n == 1:
+            return x
+        t = torch.tensor([x], dtype=torch.float64, device=device)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        return float(t.item())
+
+    return barrier, max_over_ranks
+
+
+def job_tokens_per_s(ws_n, tokens_per_rank_step, ms_step_max):
+    """Whole-job throughput under weak scaling: each of ws_n ranks processes its own
+    tokens_per_rank_step per step, and the job's step takes the slowest rank's time."""
+    return ws_n * tokens_per_rank_step / (ms_step_max / 1e3)
+
+
 def load_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -279,16 +303,7 @@ def run_ours(args):
                                     ctypes.c_int]
     lib.tla_profile_end.restype = ctypes.c_int
 
-    def barrier():
-        if ws_n > 1:
-            torch.distributed.barrier()
-
-    def max_over_ranks(x):
-        if ws_n == 1:
-            return x
-        t = torch.tensor([x], dtype=torch.float64, device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        return float(t.item())
+    barrier, max_over_ranks = rank_ops(ws_n, dev)
 
     w = inputs.GDN_FWDBWD_BF16
     if args.batch:   # profiling option: fewer sequences of the same shape
@@ -344,7 +359,7 @@ def run_ours(args):
         remeasured = True
     ms_step = max_over_ranks(ms_total / args.steps)
     tokens_step = w.B * w.T
-    value = ws_n * tokens_step / (ms_step / 1e3)
+    value = job_tokens_per_s(ws_n, tokens_step, ms_step)
     if tla.tla_last_device_status() != 0:
         raise RuntimeError("device status not OK after timed loop")
 
