@@ -10,7 +10,13 @@ GDN after a 512-token chunked prefill) and reported under "decode", and the
 same step with the headline's tokens packed into documents of log-normal length
 around 1000 tokens (cu_seqlens, each document from its own state) under "packed";
 the per-head-gate and E = 32 / d_k = 64 variants under "variants"; the layer's
-fused input path and output gate (GB/s) under "layer_io".
+fused input path and output gate (GB/s) under "layer_io"; the forward-only
+workloads (GDN bf16 B=4 H=16 T=4096 E=8, long-context GDN B=1 H=32 T=65536
+E=16, fp32 sGLA B=1 H=2 T=256 d=32 E=4) under "fwd_workloads".  Every call is
+also set against the method's algorithmic flops and bytes ("s8d": the larger of
+its tensor-core and HBM times at the measured peaks, as a fraction of the
+measured time); the bytes this implementation moves are reported separately
+("impl_bytes").
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
@@ -116,7 +122,7 @@ def flops_per_token_head(kernel, E, dk, dv, C=CHUNK):
     return 0.0
 
 
-def bytes_per_token_head(kernel, E, dk, dv, C=CHUNK, in_b=2, out_b=4, delta=True):
+def bytes_per_token_head(kernel, E, dk, dv, C=CHUNK, in_b=2, out_b=4, delta=True, save=True):
     """Algorithmic HBM bytes of one token of one head for each kernel of the tensor-core path.
 
     Every tensor a kernel reads or writes is counted once (re-reads that the design leaves to
@@ -124,9 +130,11 @@ def bytes_per_token_head(kernel, E, dk, dv, C=CHUNK, in_b=2, out_b=4, delta=True
     hi/lo operands take 4 bytes per element; per-chunk matrices are divided by C tokens.
       gate cumsum:  log gates in, chunk-local cumsum out (fp32).
       chunk prep:   k, q, k', q', G, beta in; N (delta rule), [T; A T] and [A^T; T^T] hi/lo
-                    tiles (2 x 128 x 64 and 4 x 64 x 64 bf16 per chunk), coefficient block out.
+                    tiles (2 x 128 x 64 and 4 x 64 x 64 bf16 per chunk), coefficient block out
+                    (without a backward to follow, only [T; A T] and the coefficients).
       forward:      k, q, v, [T; A T], coefficients in; o, the chunk-start state checkpoint
-                    (E dk dv hi/lo per chunk), U and Res token tiles out.
+                    (E dk dv hi/lo per chunk), U and Res token tiles out (without a backward
+                    to follow, o alone).
       backward:     k, q, dO, [A^T; T^T], coefficients in; dv, the state-gradient checkpoint,
                     dU and -dRes token tiles out.
       gradients:    k, q, dO, U, Res, dU, -dRes, both checkpoints, N, G, k', q', beta in;
@@ -139,8 +147,11 @@ def bytes_per_token_head(kernel, E, dk, dv, C=CHUNK, in_b=2, out_b=4, delta=True
     if name.startswith("gate_cumsum"):
         return 8 * E
     if name.startswith("chunk_prep"):
-        return (2 * dk * in_b + 2 * E * in_b + 4 * E + 4) + (4 * C if delta else 0) + 2 * tiles + coef
+        return ((2 * dk * in_b + 2 * E * in_b + 4 * E + 4) + (4 * C if delta and save else 0)
+                + (2 if save else 1) * tiles + coef)
     if name.startswith("fwd_recurrence"):
+        if not save:   # no checkpoints and no token tiles for a backward
+            return (in_b * (2 * dk + dv) + tiles + coef) + dv * out_b
         return (in_b * (2 * dk + dv) + tiles + coef) + (dv * out_b + ck + 4 * dv * 2)
     if name.startswith("bwd_recurrence"):
         return (in_b * (2 * dk + dv) + tiles + coef) + (dv * out_b + ck + 4 * dv * (2 if delta else 1))
@@ -148,6 +159,46 @@ def bytes_per_token_head(kernel, E, dk, dv, C=CHUNK, in_b=2, out_b=4, delta=True
         return (in_b * (2 * dk + dv) + 4 * dv * (4 if delta else 3) + 2 * ck + (4 * C if delta else 0)
                 + 4 * E + 2 * E * in_b + 4) + (2 * dk * out_b + 2 * E * out_b + 4 * E + 4)
     return 0.0
+
+
+def s8d_flops_per_token_head(E, dk, dv, backward, C=CHUNK):
+    """Algorithmic flops of the method per token-head, counted on the chunk form (dense
+    contractions only): forward 6 E dk dv + 4 C (dk + dv) + C^2 / 3 (state reads and update,
+    the intra-chunk products, the triangular solve); forward + backward
+    18 E dk dv + 12 C (dk + dv) (the backward doubles the forward's contractions)."""
+    if backward:
+        return 18 * E * dk * dv + 12 * C * (dk + dv)
+    return 6 * E * dk * dv + 4 * C * (dk + dv) + C * C / 3
+
+
+def s8d_bytes_per_token_head(E, dk, dv, backward, in_b=2, out_b=2, ckpt_b=2, C=CHUNK):
+    """Algorithmic HBM bytes of the method per token-head: every input read once and every
+    output written once (q, k, v, q', k' and o in bf16; log gates and beta fp32); with the
+    backward also dO in and dq, dk, dv, dq', dk' (bf16), dg, dbeta (fp32) out, plus one bf16
+    chunk-start state per chunk written by the forward and read by the backward."""
+    inputs_b = in_b * (2 * dk + dv + 2 * E) + 4 * E + 4
+    fwd = inputs_b + out_b * dv
+    if not backward:
+        return fwd
+    bwd = inputs_b + in_b * dv + out_b * (2 * dk + dv + 2 * E) + 4 * E + 4
+    return fwd + bwd + 2 * ckpt_b * E * dk * dv / C
+
+
+def s8d_roofline(E, dk, dv, backward, units, ms, peaks):
+    """The whole call against its algorithmic work: achieved TFLOP/s and GB/s, the fraction of
+    the measured peaks, and the call's roofline time (the larger of the tensor and HBM times)."""
+    f = s8d_flops_per_token_head(E, dk, dv, backward) * units
+    b = s8d_bytes_per_token_head(E, dk, dv, backward) * units
+    t_tc = f / (peaks["bf16_tflops_sustained"] * 1e12)
+    t_hbm = b / (peaks["hbm_gbs"] * 1e9)
+    s = ms / 1e3
+    return {"flop": f, "bytes": b, "tflops": round(f / s / 1e12, 3),
+            "tensor_frac": round(f / s / 1e12 / peaks["bf16_tflops_sustained"], 5),
+            "gbs": round(b / s / 1e9, 1), "hbm_frac": round(b / s / 1e9 / peaks["hbm_gbs"], 5),
+            "bound": "tensor" if t_tc >= t_hbm else "hbm",
+            "roofline_ms": round(max(t_tc, t_hbm) * 1e3, 4),
+            "frac": round(max(t_tc, t_hbm) / s, 5),
+            "peaks": "bf16 dense sustained and HBM copy bandwidth, " + peaks["source"]}
 
 
 def kernel_source_hash(kernel):
@@ -365,46 +416,33 @@ def run_ours(args):
 
     peaks = load_peaks()
     units = w.B * w.T * w.H  # token-heads per launch
-    kernels = {}
-    peak = peaks["bf16_tflops_sustained"]
-    hbm = peaks["hbm_gbs"]
-    for name, r in prof.items():
-        f = flops_per_token_head(name, w.E, w.dk, w.dv) * units
-        by = bytes_per_token_head(name, w.E, w.dk, w.dv) * units
-        avg_ms = r["ms"] / max(r["launches"], 1)
-        # the binding roofline: the larger of the tensor-core time and the HBM time
-        t_tc = f / (peak * 1e12) if f else 0.0
-        t_hbm = by / (hbm * 1e9) if by else 0.0
-        kernels[name] = {"launches": r["launches"], "avg_ms": round(avg_ms, 4),
-                         "share": round(r["ms"] / max(sum(v["ms"] for v in prof.values()), 1e-9), 4),
-                         "tflops": round(f / (avg_ms / 1e3) / 1e12, 2) if f else None,
-                         "gbs": round(by / (avg_ms / 1e3) / 1e9, 1) if by else None,
-                         "bound": "hbm" if t_hbm >= t_tc else "tensor",
-                         "roofline_ms": round(max(t_tc, t_hbm) * 1e3, 4)}
+    kernels = kernel_table(prof, w, units, peaks)
     top = max(prof, key=lambda n: prof[n]["ms"])
     top_avg_s = prof[top]["ms"] / prof[top]["launches"] / 1e3
-    traffic = ncu_traffic(top, units)
-    if kernels[top]["bound"] == "hbm":
-        top_bytes = bytes_per_token_head(top, w.E, w.dk, w.dv) * units
-        achieved = top_bytes / top_avg_s / 1e9
-        roofline = {"kernel": top, "bound": "hbm", "achieved": round(achieved, 1), "peak": hbm,
-                    "unit": "GB/s", "frac": round(achieved / hbm, 4), "traffic": traffic,
-                    "algorithmic_bytes": int(top_bytes),
-                    "peak_source": f"HBM copy bandwidth, {peaks['source']} (MEASURED_PEAKS.json)"
-                    if peaks["source"] == "measured" else "HBM copy bandwidth, fallback"}
-    else:
-        top_flops = flops_per_token_head(top, w.E, w.dk, w.dv) * units
-        achieved = top_flops / top_avg_s / 1e12
-        roofline = {"kernel": top, "bound": "tensor", "achieved": round(achieved, 3),
-                    "peak": peak, "unit": "TFLOP/s", "frac": round(achieved / peak, 5),
-                    "traffic": traffic,
-                    "peak_source": f"bf16 dense sustained, {peaks['source']} (MEASURED_PEAKS.json)"
-                    if peaks["source"] == "measured" else "bf16 dense sustained, fallback"}
+    peak = peaks["bf16_tflops_sustained"]
+    hbm = peaks["hbm_gbs"]
+    # The dominant kernel against its share of the method's algorithmic flops (the chunk
+    # kernels' work is dense contractions; its algorithmic bytes are far below its flops at
+    # the measured peaks).  The bytes this design moves (bf16 hi/lo checkpoints and token
+    # tiles, coefficient blocks) are reported beside it as impl_bytes, a different quantity.
+    top_flops = flops_per_token_head(top, w.E, w.dk, w.dv) * units
+    top_impl_bytes = bytes_per_token_head(top, w.E, w.dk, w.dv) * units
+    achieved = top_flops / top_avg_s / 1e12
+    roofline = {"kernel": top, "bound": "tensor", "achieved": round(achieved, 3), "peak": peak,
+                "unit": "TFLOP/s", "frac": round(achieved / peak, 5),
+                "traffic": ncu_traffic(top, units), "algorithmic_flops": int(top_flops),
+                "avg_ms": round(top_avg_s * 1e3, 4),
+                "peak_source": f"bf16 dense sustained, {peaks['source']} (MEASURED_PEAKS.json)"
+                if peaks["source"] == "measured" else "bf16 dense sustained, fallback",
+                "impl_bytes": int(top_impl_bytes),
+                "impl_bytes_gbs": round(top_impl_bytes / top_avg_s / 1e9, 1),
+                "impl_bytes_frac": round(top_impl_bytes / top_avg_s / 1e9 / hbm, 4)}
     total_flops = sum(flops_per_token_head(n, w.E, w.dk, w.dv) * units * prof[n]["launches"]
                       for n in prof) / args.steps
     total_bytes = sum(bytes_per_token_head(n, w.E, w.dk, w.dv) * units * prof[n]["launches"]
                       for n in prof) / args.steps
-    roofline_ms_step = sum(v["roofline_ms"] * v["launches"] for v in kernels.values()) / args.steps
+    step_s8d = s8d_roofline(w.E, w.dk, w.dv, True, units, ms_step, peaks)
+    roofline["frac_s8d"] = step_s8d["frac"]
     gpu_launches = sum(r["launches"] for r in prof.values())
 
     # ---- end to end through the public API from pinned host buffers
@@ -413,7 +451,11 @@ def run_ours(args):
         e2e = run_e2e(args, tla, x, w, dev, stream, o, fws, bws, grads, barrier, max_over_ranks,
                       ws_n)
 
-    # ---- decode workload
+    # ---- the forward-only workloads (bf16 E=8 T=4096, long-context E=16 T=65536, fp32 sGLA)
+    fwd_loads = None
+    if not args.no_fwd_workloads:
+        fwd_loads = run_fwd_workloads(args, tla, inputs, dev, stream, lib, peaks, barrier,
+                                      max_over_ranks, ws_n, rank)
     packed = None
     if not args.no_packed:
         packed = run_packed(args, tla, inputs, w, dev, stream, barrier, max_over_ranks, ws_n, rank)
@@ -454,17 +496,91 @@ def run_ours(args):
                        "l2": "inputs larger than L2 (q,k,v,dO 268 MB each per GPU)"},
             "tflops": round(total_flops / (ms_step / 1e3) / 1e12, 3),
             "tflops_frac": round(total_flops / (ms_step / 1e3) / 1e12 / peak, 5),
-            "step_hbm": {"algorithmic_gb": round(total_bytes / 1e9, 3),
-                         "achieved_gbs": round(total_bytes / (ms_step / 1e3) / 1e9, 1),
-                         "frac": round(total_bytes / (ms_step / 1e3) / 1e9 / hbm, 4),
-                         "roofline_ms": round(roofline_ms_step, 4)},
+            "s8d": step_s8d,
+            "step_impl_bytes": {"gb": round(total_bytes / 1e9, 3),
+                                "achieved_gbs": round(total_bytes / (ms_step / 1e3) / 1e9, 1),
+                                "frac": round(total_bytes / (ms_step / 1e3) / 1e9 / hbm, 4),
+                                "note": "bytes this design moves (hi/lo checkpoints, token "
+                                        "tiles, coefficient blocks), not the method's"},
             "roofline": roofline, "kernels": kernels, "gpu_launches": gpu_launches,
             "clocks": ck, "clocks_remeasured": remeasured,
-            "e2e": e2e, "packed": packed, "variants": variants, "layer_io": layer, "decode": decode, "cpu_baseline": cpu, "impl": "ours",
+            "e2e": e2e, "fwd_workloads": fwd_loads, "packed": packed, "variants": variants,
+            "layer_io": layer, "decode": decode, "cpu_baseline": cpu, "impl": "ours",
         }
         print(json.dumps(line), flush=True)
     if ws_n > 1:
         torch.distributed.destroy_process_group()
+
+
+def kernel_table(prof, w, units, peaks):
+    """Per kernel of a profiled loop: launches, mean device time, share of the loop, achieved
+    TFLOP/s on its algorithmic flops (fraction of the sustained bf16 peak) and the GB/s of the
+    bytes this design moves through it (impl_gbs, fraction of the HBM copy bandwidth)."""
+    tot = max(sum(v["ms"] for v in prof.values()), 1e-9)
+    out = {}
+    for name, r in prof.items():
+        f = flops_per_token_head(name, w.E, w.dk, w.dv) * units
+        by = bytes_per_token_head(name, w.E, w.dk, w.dv, delta=w.use_delta, save=w.backward) * units
+        avg_s = r["ms"] / max(r["launches"], 1) / 1e3
+        out[name] = {"launches": r["launches"], "avg_ms": round(avg_s * 1e3, 4),
+                     "share": round(r["ms"] / tot, 4),
+                     "tflops": round(f / avg_s / 1e12, 2) if f else None,
+                     "tensor_frac": round(f / avg_s / 1e12 / peaks["bf16_tflops_sustained"], 4)
+                     if f else None,
+                     "impl_gbs": round(by / avg_s / 1e9, 1) if by else None,
+                     "impl_hbm_frac": round(by / avg_s / 1e9 / peaks["hbm_gbs"], 4) if by else None}
+    return out
+
+
+def run_fwd_workloads(args, tla, inputs, dev, stream, lib, peaks, barrier, max_over_ranks, ws_n,
+                      rank):
+    """The forward-only workloads: triadic GDN forward bf16 B=4 H=16 T=4096 E=8 (zero initial
+    state), the long-context forward B=1 H=32 T=65536 E=16 (initial state ~ N(0, 0.01)), both
+    returning o (fp32) and the final state, and the fp32 sGLA forward B=1 H=2 T=256 d=32 E=4
+    (latency-bound; time only).  Each: tokens/s, per-kernel shares from the library's own event
+    timing, and the whole call against the algorithmic flops and bytes of the forward."""
+    out = {}
+    for w in (inputs.GDN_FWD_BF16, inputs.GDN_LONG_BF16, inputs.SGLA_FWD_FP32):
+        x = inputs.workload_inputs(w, device=dev, seed=rank)
+        o = torch.empty(w.B, w.T, w.H, w.dv, dtype=torch.float32, device=dev)
+        ht = torch.empty(w.B, w.H, w.E, w.dk, w.dv, dtype=torch.float32, device=dev)
+        p = tla.make_problem(x["q"], x["k"], x["v"], x["q2"], x["k2"], x["g"], x["beta"],
+                             x["h0"], o, ht, use_delta=w.use_delta)
+        fws = torch.empty(tla.fwd_workspace_bytes(p, False), dtype=torch.uint8, device=dev)
+
+        def step():
+            tla.tla_chunk_fwd(x["q"], x["k"], x["v"], x["q2"], x["k2"], x["g"], x["beta"],
+                              x["h0"], use_delta=w.use_delta, save_for_bwd=False, o=o, ht=ht,
+                              workspace=fws)
+
+        k = 20 if w.B * w.T <= 4096 else 5
+        for _ in range(3):
+            step()
+        torch.cuda.synchronize()
+        barrier()
+        lib.tla_profile_begin()
+        ms = _time_steps(step, k, 0, stream, barrier, max_over_ranks)
+        prof = profile_read(lib, stream.cuda_stream)
+        if tla.tla_last_device_status() != 0:
+            raise RuntimeError(f"device status not OK after {w.name}")
+        units = w.B * w.T * w.H
+        rec = {"value": round(ws_n * w.B * w.T / (ms / 1e3), 1), "unit": "tokens/s",
+               "ms": round(ms, 4), "steps": k,
+               "config": {"B": w.B, "T": w.T, "H": w.H, "dk": w.dk, "dv": w.dv, "E": w.E,
+                          "dtype": w.dtype, "delta_rule": w.use_delta,
+                          "h0": f"N(0, {w.h0_std ** 2:g})" if w.h0_std else "zero",
+                          "outputs": "fp32 o and final state"},
+               "kernels": kernel_table(prof, w, units, peaks)}
+        if w.dtype == "bf16":
+            rec["s8d"] = s8d_roofline(w.E, w.dk, w.dv, False, units, ms, peaks)
+            rec["l2"] = ("inputs and outputs larger than L2" if units * (2 * (2 * w.dk + w.dv) + 4 * w.dv)
+                         > 129e6 else "working set within L2")
+        else:
+            rec["bound"] = "latency (tiny problem: one CTA per head and value block)"
+        out[w.name] = rec
+        del x, o, ht, fws
+        torch.cuda.empty_cache()
+    return out
 
 
 def run_e2e(args, tla, x, w, dev, stream, o, fws, bws, grads, barrier, max_over_ranks, ws_n):
@@ -810,6 +926,7 @@ def main():
     ap.add_argument("--no-packed", action="store_true")
     ap.add_argument("--no-variants", action="store_true")
     ap.add_argument("--no-layer", action="store_true")
+    ap.add_argument("--no-fwd-workloads", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--ref-tokens", type=int, default=1024,

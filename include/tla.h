@@ -31,9 +31,10 @@
  *  - `stream` is a cudaStream_t passed as void*; NULL means the legacy default
  *    stream.  Calls only enqueue work: they never synchronise the device.
  *  - Argument errors are detected on the host before anything is launched and
- *    return a negative status; nothing is written in that case.  Launch errors
- *    return TLA_ERR_CUDA.  Device-side bounded waits that expire record an
- *    error word that tla_last_device_status() reports (TLA_ERR_TIMEOUT).
+ *    return a negative status; nothing is written in that case.  Launch errors,
+ *    and a failed lookup of the device error word below, return TLA_ERR_CUDA.
+ *    Device-side bounded waits that expire record an error word that
+ *    tla_last_device_status() reports (TLA_ERR_TIMEOUT).
  *  - Results are deterministic: no floating-point atomics (Appendix A, Kernels).
  */
 #ifndef TLA_H
@@ -268,6 +269,12 @@ tla_status tla_output_gate_bwd(const tla_gate_args *a, const void *dy, void *d_o
  * Synchronises `stream`, then returns TLA_ERR_TIMEOUT if a device-side bounded
  * wait of any kernel launched since the previous call expired (and clears that
  * record), TLA_ERR_CUDA if the stream reports an error, else TLA_OK.
+ * The record is ONE word per device, shared by every stream and host thread
+ * that uses the library on that device: only `stream` is synchronised, so a
+ * timeout in a kernel still running on another stream may be reported by a
+ * later call, and a timeout on another stream is reported (and cleared) by
+ * whichever call reads the word first.  Callers with several streams should
+ * synchronise all of them before reading the status.
  */
 tla_status tla_last_device_status(void *stream);
 

@@ -955,6 +955,7 @@ extern "C" tla_status tla_output_gate(const tla_gate_args* a, void* stream) {
     const size_t so = a->o_dtype == TLA_FP32 ? 4 : 2, sz = a->dtype == TLA_FP32 ? 4 : 2;
     const size_t smem = 128 + size_t(kGateTile) * a->dv * (so + sz);
     int* err = device_error_word();
+    if (!err) return TLA_ERR_CUDA;
     prof_before("output_gate", s);
 #define TLA_GATE_LAUNCH(TO, TZ)                                                                    \
     do {                                                                                           \
@@ -999,6 +1000,7 @@ extern "C" tla_status tla_output_gate_bwd(const tla_gate_args* a, const void* dy
     const size_t so = a->o_dtype == TLA_FP32 ? 4 : 2, sz = a->dtype == TLA_FP32 ? 4 : 2;
     const size_t smem = 128 + size_t(kGateTile) * a->dv * (so + 2 * sz);
     int* err = device_error_word();
+    if (!err) return TLA_ERR_CUDA;
     prof_before("output_gate_bwd", s);
 #define TLA_GATE_BWD_LAUNCH(TO, TZ)                                                                \
     do {                                                                                           \

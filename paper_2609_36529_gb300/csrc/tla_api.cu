@@ -61,12 +61,19 @@ static __global__ void selftest_wait_kernel(unsigned long long timeout_ns, int* 
     if (!ok && threadIdx.x == 0) record_device_error(err, TLA_ERR_TIMEOUT);
 }
 
-// Address of the error word on the current device (looked up once per device).
+// Address of the error word on the current device, looked up once per device (a
+// std::once_flag per device orders concurrent first calls); nullptr if the lookup
+// failed, which every entry point reports as TLA_ERR_CUDA before launching anything.
+constexpr int kMaxDevices = 64;
 int* device_error_word() {
-    static int* ptr[64] = {nullptr};
+    static std::once_flag once[kMaxDevices];
+    static int* ptr[kMaxDevices] = {nullptr};
     int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
-    if (!ptr[dev]) cudaGetSymbolAddress((void**)&ptr[dev], g_device_error);
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+    std::call_once(once[dev], [dev]() {
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_device_error) == cudaSuccess) ptr[dev] = (int*)p;
+    });
     return ptr[dev];
 }
 
@@ -203,10 +210,12 @@ tla_status tla_chunk_fwd(const tla_problem* p, void* workspace, size_t workspace
     FwdPlan fp = plan_fwd(*p, save);
     if (!workspace || workspace_bytes < fp.bytes || ((uintptr_t)workspace & 255))
         return TLA_ERR_WORKSPACE;
+    if (p->cu_seqlens && !fp.tc_tv) return TLA_ERR_UNSUPPORTED;   // packed: tensor-core path only
+    int* err = device_error_word();
+    if (!err) return TLA_ERR_CUDA;
     cudaStream_t s = (cudaStream_t)stream;
     char* ws = (char*)workspace;
-    if (p->cu_seqlens) {   // packed documents: tensor-core path only; chunk and document tables
-        if (!fp.tc_tv) return TLA_ERR_UNSUPPORTED;
+    if (p->cu_seqlens) {   // packed documents: chunk and document tables
         std::vector<int2> ct(fp.NT);
         std::vector<int4> dt(p->n_docs);
         int g = 0;
@@ -226,7 +235,7 @@ tla_status tla_chunk_fwd(const tla_problem* p, void* workspace, size_t workspace
     cudaError_t e = launch_gate_cumsum(*p, fp, ws, (float*)(ws + fp.G), s);
     if (e == cudaSuccess) {
         if (fp.tc_tv)
-            e = launch_chunk_prep_tc(*p, fp, ws, device_error_word(), s);
+            e = launch_chunk_prep_tc(*p, fp, ws, err, s);
         else
             e = launch_chunk_prep(*p, (const float*)(ws + fp.G), (float*)(ws + fp.A),
                                   p->use_delta ? (float*)(ws + fp.N) : nullptr, nullptr, nullptr,
@@ -234,7 +243,7 @@ tla_status tla_chunk_fwd(const tla_problem* p, void* workspace, size_t workspace
     }
     if (e == cudaSuccess) {
         if (fp.tc_tv)
-            e = launch_fwd_recurrence_tc(*p, fp, ws, save, device_error_word(), s);
+            e = launch_fwd_recurrence_tc(*p, fp, ws, save, err, s);
         else e = launch_fwd_recurrence(*p, fp, ws, save, s);
     }
     return cuda_status(e);
@@ -260,17 +269,19 @@ tla_status tla_chunk_bwd(const tla_problem* p, const void* fwd_ws, size_t fwd_ws
     if (!fwd_ws || fwd_ws_bytes < fp.bytes || ((uintptr_t)fwd_ws & 255)) return TLA_ERR_WORKSPACE;
     if (!workspace || workspace_bytes < bp.bytes || ((uintptr_t)workspace & 255))
         return TLA_ERR_WORKSPACE;
+    int* err = device_error_word();
+    if (!err) return TLA_ERR_CUDA;
     cudaStream_t s = (cudaStream_t)stream;
     const char* fws = (const char*)fwd_ws;
     char* bws = (char*)workspace;
     float* dgs = p->gate_per_head ? (float*)(bws + bp.dgE) : dg;   // per-slice gate gradient
     cudaError_t e = fp.tcb ? launch_bwd_recurrence_tc(*p, fp, fws, bp, bws, dO, dht, dv, dh0,
-                                                      device_error_word(), s)
+                                                      err, s)
                            : launch_bwd_recurrence(*p, fp, fws, bp, bws, dO, dht, dv, dh0, s);
     if (e == cudaSuccess) {
         if (tc_grads_ok(*p, fp))
             e = launch_bwd_chunk_grads_tc(*p, fp, fws, bp, bws, dO, dq, dk, dq2, dk2, dbeta, dgs,
-                                          device_error_word(), s);
+                                          err, s);
         else
             e = launch_bwd_chunk_grads(*p, fp, fws, bp, bws, dO, dq, dk, dq2, dk2, dbeta, dgs, s);
     }
@@ -295,8 +306,10 @@ tla_status tla_decode_step(int B, int H, int dk, int dv, int E, int use_delta, i
     }
     if (!dims_ok(dk) || !dims_ok(dv) || E > 32 || E * dk > 2048) return TLA_ERR_UNSUPPORTED;
     if ((long long)B * H > 65535) return TLA_ERR_UNSUPPORTED;  // grid.y
+    int* err = device_error_word();
+    if (!err) return TLA_ERR_CUDA;
     return cuda_status(launch_decode_step(B, H, dk, dv, E, use_delta, dtype, q, k, v, q2, k2, g,
-                                          beta, state, o, device_error_word(), (cudaStream_t)stream));
+                                          beta, state, o, err, (cudaStream_t)stream));
 }
 
 const char* tla_status_string(int status) {

@@ -18,6 +18,8 @@
 // ordering) race on it.  The first call on each device looks up the buffer's
 // device address (cudaGetSymbolAddress) with that device current; make that
 // first call before capturing the stream into a CUDA graph.
+#include <mutex>
+
 #include "common.cuh"
 #include "internal.h"
 
@@ -28,16 +30,19 @@ constexpr size_t kNoAllocScratchBytes = size_t(64) << 20;
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
 // Device address of the scratch array on the current device (host code must not
-// use the array's name as a device pointer).
+// use the array's name as a device pointer).  Looked up once per device with that
+// device current; a std::once_flag per device orders concurrent first calls.
+constexpr int kMaxDevices = 64;
 static tla_status noalloc_scratch(void** out) {
-    static void* addr[64] = {nullptr};
+    static std::once_flag once[kMaxDevices];
+    static void* addr[kMaxDevices] = {nullptr};
     int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return TLA_ERR_CUDA;
-    if (!addr[dev]) {
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return TLA_ERR_CUDA;
+    std::call_once(once[dev], [dev]() {
         void* p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return TLA_ERR_CUDA;
-        addr[dev] = p;
-    }
+        if (cudaGetSymbolAddress(&p, g_noalloc_scratch) == cudaSuccess) addr[dev] = p;
+    });
+    if (!addr[dev]) return TLA_ERR_CUDA;
     *out = addr[dev];
     return TLA_OK;
 }

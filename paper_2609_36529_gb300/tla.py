@@ -203,16 +203,21 @@ def tla_chunk_fwd(q, k, v, q2, k2, g, beta=None, h0=None, use_delta=True, save_f
     return o, ht, workspace
 
 
-def tla_chunk_fwd_noalloc(q, k, v, q2, k2, g, beta=None, h0=None, use_delta=True, o=None,
-                          ht=None, cu_seqlens=None):
+def tla_chunk_fwd_noalloc(q, k, v, q2, k2, g, beta=None, h0=None, use_delta=True,
+                          want_ht=True, o=None, ht=None, out_dtype=torch.float32,
+                          cu_seqlens=None):
     """Forward through the entry point that allocates nothing (built-in scratch).
 
-    o and ht must be preallocated by the caller when it cannot allocate; when they
-    are None they are allocated here with PyTorch for convenience."""
+    Same defaults and results as tla_chunk_fwd(save_for_bwd=False).  A caller that
+    cannot allocate passes o (and ht) preallocated; when they are None they are
+    allocated here with PyTorch for convenience.  Returns (o, ht or None)."""
     B, T, H, _ = q.shape
     E, dv = q2.shape[-1], v.shape[-1]
     if o is None:
-        o = torch.empty(B, T, H, dv, dtype=torch.float32, device=q.device)
+        o = torch.empty(B, T, H, dv, dtype=out_dtype, device=q.device)
+    if ht is None and want_ht:
+        ht = torch.empty(_n_states(q, cu_seqlens), H, E, q.shape[-1], dv, dtype=torch.float32,
+                         device=q.device)
     p = make_problem(q, k, v, q2, k2, g, beta, h0, o, ht, use_delta, cu_seqlens=cu_seqlens)
     _check("tla_chunk_fwd_noalloc", lib().tla_chunk_fwd_noalloc(ctypes.byref(p), _stream()))
     return o, ht
