@@ -247,6 +247,47 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const float* v) {
         "r"(__float_as_uint(v[15]))
         : "memory");
 }
+__device__ __forceinline__ void tmem_ld8(uint32_t taddr, float* v) {
+    uint32_t r[8];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7])
+        : "r"(taddr));
+#pragma unroll
+    for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(r[i]);
+}
+__device__ __forceinline__ void tmem_st8(uint32_t taddr, const float* v) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"r"(taddr),
+        "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])),
+        "r"(__float_as_uint(v[3])), "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])),
+        "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7]))
+        : "memory");
+}
+// N consecutive columns (N a multiple of 8) of this thread's TMEM lane, without waiting.
+template <int N>
+__device__ __forceinline__ void tmem_ld(uint32_t taddr, float* v) {
+    static_assert(N % 8 == 0, "tmem_ld: N must be a multiple of 8");
+    if constexpr (N % 16 == 0) {
+#pragma unroll
+        for (int j = 0; j < N; j += 16) tmem_ld16(taddr + j, v + j);
+    } else {
+#pragma unroll
+        for (int j = 0; j < N; j += 8) tmem_ld8(taddr + j, v + j);
+    }
+}
+template <int N>
+__device__ __forceinline__ void tmem_st(uint32_t taddr, const float* v) {
+    static_assert(N % 8 == 0, "tmem_st: N must be a multiple of 8");
+    if constexpr (N % 16 == 0) {
+#pragma unroll
+        for (int j = 0; j < N; j += 16) tmem_st16(taddr + j, v + j);
+    } else {
+#pragma unroll
+        for (int j = 0; j < N; j += 8) tmem_st8(taddr + j, v + j);
+    }
+}
 __device__ __forceinline__ void tmem_wait_ld() {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }

@@ -7,19 +7,21 @@
 //   dU   = A^T dO + sum_e diag(w_e) K dS'_e
 //   dRes = T^T dU                                   (= dV)
 //   dS_e = gamma^C_e dS'_e + Q^T diag(b_e) dO - K^T diag(a_e) dRes
-// One CTA of 4 warps per (b, h, block of TV value columns) keeps dS for its
+// One CTA of 8 warps per (b, h, block of TV value columns) keeps dS for its
 // value columns in TMEM.  Per chunk:
 //   MMA-A'  P' = K dS'_all              (M=64, N=NE, K=dk; dS' MN-major hi/lo)
-//   MMA-0   Y  = A^T dO                 (M=64, N=TV, K=64; A^T hi/lo, dO exact bf16)
-//   epi     dU = Y + sum_e w_e (.) P'_e  -> dU^T hi/lo operand, dU to the workspace
+//   MMA-0   Y  = A^T dO                 (M=64, N=TV, K=64; A^T hi/lo, dO exact bf16,
+//                                        MN-major as the TMA loads it)
+//   epi     dU = Y + sum_e w_e (.) P'_e  -> dU hi/lo operand, dU to the workspace
 //   MMA-B'  dRes = T^T dU               (M=64, N=TV, K=64; both hi/lo)
 //   epi     dRes -> workspace and dv; operand rows [-a_e (.) dRes ; b_e (.) dO]
 //   MMA-C'  dS_all += [K^T | Q^T] [-a (.) dRes ; b (.) dO]   (M=dk=128, K=128, N=NE;
 //           K^T and Q^T read MN-major from the TMA key/query tile)
-//   epi     dS_{[c]} from TMEM -> operand of the previous chunk, checkpoint, and
-//           pre-scaled by gamma^C of the previous chunk.
+//   epi     dS_{[c]} from TMEM -> operand of the previous chunk and checkpoint; once the
+//           previous chunk's MMA-A' is issued, the slab is rescaled in place by its gamma^C.
 // Layout of the M=64 products in TMEM: row r sits on lane 32 * (r / 16) + r % 16,
-// so lanes 0-15 of each warp own the row work and lanes 16-31 prepare dO.
+// so lanes 0-15 of each warp own the row work and lanes 16-31 the dO rows.
+// Warps 0-3 / 4-7 take the first / second half of each slice's TV value columns.
 // Precision, TMA prefetch, bounded waits, the slice-block layout of the state
 // operand and the TMA-stored checkpoints as in the forward kernel.
 #include <cstring>
@@ -35,7 +37,7 @@ using namespace sm100;
 
 namespace {
 
-constexpr int kThreads = 128;
+constexpr int kThreads = 256;
 constexpr int kDk = 128;
 constexpr int kBoxBytes = 64 * 64 * 2;
 
@@ -52,14 +54,17 @@ struct TcBwdArgs {
     int T, H, dv, E, NT, use_delta, out_f32, ck_tiles;
 };
 
+// Two CTAs per SM (at most 128 registers a thread), except for 64-column blocks.
 template <int TV>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kThreads, TV == 64 ? 1 : 2)
 bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                          const __grid_constant__ CUtensorMap map_q,
                          const __grid_constant__ CUtensorMap map_do,
                          const __grid_constant__ CUtensorMap map_bt,
                          const __grid_constant__ CUtensorMap map_ck,
                          const __grid_constant__ CUtensorMap map_dv, const TcBwdArgs p) {
+    constexpr int TVH = TV / 2;                      // value columns per thread
+    constexpr int GRP = TVH >= 32 ? 1 : 32 / TVH;    // slices per batch of TMEM loads
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
@@ -70,19 +75,20 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     uint8_t* sReg = sBT + 4 * kBoxBytes;     // NE * 512 bytes, reused:
     uint8_t* sDh = sReg;                     //   dS' hi / lo: E blocks [dk][TV] (MMA-A')
     uint8_t* sDl = sReg + NE * 256;
-    uint8_t* sUh = sReg;                     //   dU^T [TV][64] hi / lo (MMA-B')
+    uint8_t* sUh = sReg;                     //   dU [64][TV] hi / lo, MN-major (MMA-B')
     uint8_t* sUl = sReg + TV * 128;
     uint8_t* sBh = sReg;                     //   [-a dRes ; b dO] [128][NE] hi / lo (MMA-C')
     uint8_t* sBl = sReg + NE * 256;
-    uint8_t* sOT = sReg + NE * 512;          // dO^T [TV][64] bf16 (MMA-0)
-    __nv_bfloat16* sdO = reinterpret_cast<__nv_bfloat16*>(sOT + TV * 128);   // [64][TV] (TMA)
-    uint8_t* sDvo = sOT + TV * 128 + 64 * TV * 2;                           // dv tile [64][TV] (TMA store)
-    float* sCoef = reinterpret_cast<float*>(sDvo + 64 * TV * 4);             // 2 x CB
+    uint8_t* sdO = sReg + NE * 512;          // dO [64][TV] bf16, MN-major operand (TMA, swizzled)
+    uint8_t* sDvo = sdO + 64 * TV * 2;       // dv tile [64][TV] (TMA store)
+    float* sCoef = reinterpret_cast<float*>(sDvo + 64 * TV * 4);   // 2 x CB
 
     __shared__ __align__(8) uint64_t bar_kq, bar_av, bar_mma;
     __shared__ uint32_t tmem_slot;
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int r = tid & 127;                 // TMEM lane of the dS slab: row d
+    const int cofs = (tid >> 7) * TVH;       // this thread's first column within a slice
     const int nb = blockIdx.x, h = blockIdx.y, sb = blockIdx.z;   // sb: sequence or document
     const int n0 = nb * TV;
     const int T = p.T, H = p.H, dv = p.dv, NT = p.NT;
@@ -97,15 +103,15 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     if (nct == 0) {   // empty document: the gradient of the initial state is that of the final one
         if (p.dh0)
             for (int e = 0; e < E; ++e)
-                for (int n = 0; n < TV; ++n) {
-                    const size_t o = ((size_t(sb * H + h) * E + e) * kDk + tid) * dv + n0 + n;
+                for (int n = cofs; n < cofs + TVH; ++n) {
+                    const size_t o = ((size_t(sb * H + h) * E + e) * kDk + r) * dv + n0 + n;
                     p.dh0[o] = p.dht ? p.dht[o] : 0.f;
                 }
         return;
     }
-    // M=64 row owned by this thread (lanes 0-15) or prepared by it (lanes 16-31)
+    // M=64 row owned by this thread (lanes 0-15) or whose dO part it prepares (lanes 16-31)
     const bool row_thread = lane < 16;
-    const int r64 = 16 * warp + (lane & 15);
+    const int r64 = 16 * (warp & 3) + (lane & 15);
 
     if (warp == 0) {
         tmem_alloc(&tmem_slot, tcols);
@@ -143,48 +149,73 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         tma_load_4d(sdO, &map_do, &bar_av, n0, h, tbeg + c * 64, b);
         bulk_load(sCoef + (c & 1) * CB, p.coef + idx * CB, CB * 4, &bar_av);
     };
-    // Row d = tid of the gradient at the end of chunk c: operand of MMA-A'(c),
-    // checkpoint for the chunk-parallel gradients, and gamma^C_c-scaled copy in TMEM.
-    auto prepare = [&](int c, bool from_dht) {
-        const int d = tid;
+    // This thread's part (row r, TVH columns) of slice e of the gradient at the end of chunk
+    // c -> the operand of MMA-A'(c), and the fp32 checkpoint when checkpoints are not tiles
+    auto put_operand = [&](int c, int e, const float* v) {
+#pragma unroll
+        for (int n = 0; n < TVH; n += 8)
+            st8_split(sDh, sDl, e * blk_bytes<TV>() + blk_offset<TV>(r, cofs + n), v + n);
+        if (!p.ck_tiles) {
+            const size_t slab = (((size_t(b) * H + h) * NT + cb + c) * E + e) * kDk * dv;
+            store_f32_row(p.dSck + slab + size_t(r) * dv + n0 + cofs, v, TVH);
+        }
+    };
+    auto stage_operand = [&](int c) {
+        for (int e0 = 0; e0 < E; e0 += GRP) {
+            float v[GRP * TVH];
+#pragma unroll
+            for (int g = 0; g < GRP; ++g) tmem_ld<TVH>(tmem_lane_addr(tS, warp, (e0 + g) * TV + cofs), v + g * TVH);
+            tmem_wait_ld();
+#pragma unroll
+            for (int g = 0; g < GRP; ++g) put_operand(c, e0 + g, v + g * TVH);
+        }
+    };
+    // The slab rescaled in place by gamma^C_c: chunk c's MMA-C' accumulates onto it.
+    auto scale_state = [&](int c) {
+        const float* gc = sCoef + (c & 1) * CB + 3 * 64 * E;
+        for (int e0 = 0; e0 < E; e0 += GRP) {
+            float v[GRP * TVH];
+#pragma unroll
+            for (int g = 0; g < GRP; ++g) tmem_ld<TVH>(tmem_lane_addr(tS, warp, (e0 + g) * TV + cofs), v + g * TVH);
+            tmem_wait_ld();
+#pragma unroll
+            for (int g = 0; g < GRP; ++g) {
+                const float gm = gc[e0 + g];
+#pragma unroll
+                for (int i = 0; i < TVH; ++i) v[g * TVH + i] *= gm;
+                tmem_st<TVH>(tmem_lane_addr(tS, warp, (e0 + g) * TV + cofs), v + g * TVH);
+            }
+        }
+        tmem_wait_st();
+    };
+    // Gradient of the final state (dht or zero): operand of MMA-A'(nct-1) and the scaled slab.
+    auto stage_dht = [&](int c) {
         const float* gc = sCoef + (c & 1) * CB + 3 * 64 * E;
         for (int e = 0; e < E; ++e) {
-            float v[TV];
-            if (from_dht) {
-                if (p.dht) {
-                    const float4* src = reinterpret_cast<const float4*>(
-                        p.dht + ((size_t(sb * H + h) * E + e) * kDk + d) * dv + n0);
+            float v[TVH];
+            if (p.dht) {
+                const float4* src = reinterpret_cast<const float4*>(
+                    p.dht + ((size_t(sb * H + h) * E + e) * kDk + r) * dv + n0 + cofs);
 #pragma unroll
-                    for (int i = 0; i < TV / 4; ++i) {
-                        float4 x = src[i];
-                        v[4 * i] = x.x; v[4 * i + 1] = x.y; v[4 * i + 2] = x.z; v[4 * i + 3] = x.w;
-                    }
-                } else {
-#pragma unroll
-                    for (int i = 0; i < TV; ++i) v[i] = 0.f;
+                for (int i = 0; i < TVH / 4; ++i) {
+                    const float4 x = src[i];
+                    v[4 * i] = x.x; v[4 * i + 1] = x.y; v[4 * i + 2] = x.z; v[4 * i + 3] = x.w;
                 }
             } else {
 #pragma unroll
-                for (int j = 0; j < TV; j += 16) tmem_ld16(tmem_lane_addr(tS, warp, e * TV + j), v + j);
-                tmem_wait_ld();
+                for (int i = 0; i < TVH; ++i) v[i] = 0.f;
             }
+            put_operand(c, e, v);
+            const float gm = gc[e];
 #pragma unroll
-            for (int n = 0; n < TV; n += 8) st8_split(sDh, sDl, e * blk_bytes<TV>() + blk_offset<TV>(d, n), v + n);
-            if (!p.ck_tiles) {   // fp32 checkpoint (tile checkpoints: issue_ckpt)
-                const size_t slab = (((size_t(b) * H + h) * NT + cb + c) * E + e) * kDk * dv;
-                store_f32_row(p.dSck + slab + size_t(d) * dv + n0, v, TV);
-            }
-            const float g = gc[e];
-#pragma unroll
-            for (int n = 0; n < TV; ++n) v[n] *= g;
-#pragma unroll
-            for (int j = 0; j < TV; j += 16) tmem_st16(tmem_lane_addr(tS, warp, e * TV + j), v + j);
+            for (int i = 0; i < TVH; ++i) v[i] *= gm;
+            tmem_st<TVH>(tmem_lane_addr(tS, warp, e * TV + cofs), v);
         }
         tmem_wait_st();
     };
 
     // Checkpoint of dS' at the end of chunk c: this CTA's columns of the slice blocks,
-    // stored by TMA (thread 0, once prepare(c) is complete in shared memory).
+    // stored by TMA (thread 0, once the operand of chunk c is complete in shared memory).
     auto issue_ckpt = [&](int c) {
         if (!p.ck_tiles) return;
         tma_store_4d(&map_ck, sDh, n0, 0, ((b * H + h) * NT + cb + c) * E, 0);   // [hi|lo][E][dk][TV]
@@ -194,6 +225,7 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     bool failed = false;
     uint32_t mma_phase = 0;
     int pending_mma = 0;
+    bool scaled = true;   // the slab already holds gamma^C-scaled values for the current chunk
     if (tid == 0) {
         issue_kq(nct - 1);
         issue_av(nct - 1);
@@ -201,7 +233,7 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     if (!mbar_wait(&bar_av, 0)) failed = true;
     if (__syncthreads_or(failed)) failed = true;
     if (!failed) {
-        prepare(nct - 1, true);
+        stage_dht(nct - 1);
         fence_proxy_async_smem();
         tc_fence_before();
         __syncthreads();
@@ -228,26 +260,6 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         if (__syncthreads_or(!ok)) { failed = true; break; }
         tc_fence_after();
 
-        // ---- step 1 (lanes 16-31): dO row -> registers and dO^T operand of MMA-0
-        float dorow[TV];
-        if (!row_thread) {
-            const uint4* src = reinterpret_cast<const uint4*>(sdO + r64 * TV);
-#pragma unroll
-            for (int i = 0; i < TV / 8; ++i) {
-                uint4 u = src[i];
-                const __nv_bfloat16* pb = reinterpret_cast<const __nv_bfloat16*>(&u);
-#pragma unroll
-                for (int j = 0; j < 8; ++j) {
-                    *reinterpret_cast<__nv_bfloat16*>(sOT + sw128_offset(8 * i + j, r64, TV)) = pb[j];
-                    dorow[8 * i + j] = __bfloat162float(pb[j]);
-                }
-            }
-        }
-        fence_proxy_async_smem();
-        tc_fence_before();
-        __syncthreads();
-        tc_fence_after();
-
         // ---- MMA-A' (P' = K dS') and MMA-0 (Y = A^T dO)
         if (tid == 0) {
             const uint32_t ida = idesc_bf16_f32(64, NE, 0, 1);
@@ -260,17 +272,35 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                           ks > 0 ? 1u : 0u);
                 umma_bf16(tP, ad, smem_desc(smem_u32(sDl) + ko, blk_bytes<TV>(), 16 * TV, kSwz), ida, 1u);
             }
-            const uint32_t id0 = idesc_bf16_f32(64, TV, 0, 0);
+            const uint32_t id0 = idesc_bf16_f32(64, TV, 0, 1);
 #pragma unroll
             for (int ks = 0; ks < 4; ++ks) {
-                const uint64_t bd = smem_desc(smem_u32(sOT) + ks * 32, 16, 1024);
+                const uint64_t bd = smem_desc(smem_u32(sdO) + ks * 32 * TV, blk_bytes<TV>(), 16 * TV, kSwz);
                 umma_bf16(tY, smem_desc(smem_u32(sBT) + ks * 32, 16, 1024), bd, id0, ks > 0 ? 1u : 0u);
                 umma_bf16(tY, smem_desc(smem_u32(sBT) + kBoxBytes + ks * 32, 16, 1024), bd, id0, 1u);
             }
             umma_commit(&bar_mma);
-            issue_ckpt(c);   // the dS' blocks were completed by prepare(c) before the last barrier
+            issue_ckpt(c);   // the dS' blocks were completed before the last barrier
         }
         pending_mma = 1;
+        // while the products run: the slab rescaled by this chunk's gamma^C (MMA-C' of this
+        // chunk accumulates onto it), and the dO row of this thread's M=64 row (lanes 16-31)
+        if (!scaled) scale_state(c);
+        scaled = false;
+        float dorow[TVH];
+        if (!row_thread) {
+#pragma unroll
+            for (int i = 0; i < TVH; i += 8) {
+                const uint4 u = *reinterpret_cast<const uint4*>(sdO + blk_offset<TV>(r64, cofs + i));
+                const __nv_bfloat162* pb = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    const float2 f = __bfloat1622float2(pb[j]);
+                    dorow[i + 2 * j] = f.x;
+                    dorow[i + 2 * j + 1] = f.y;
+                }
+            }
+        }
         ok = mbar_wait(&bar_mma, mma_phase);
         mma_phase ^= 1;
         if (tid == 0) bulk_wait_read_all();   // the dS' blocks are rewritten next
@@ -278,26 +308,27 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         pending_mma = 0;
         tc_fence_after();
 
-        // ---- dU = Y + sum_e w_e (.) P'_e   (row threads)
+        // ---- dU = Y + sum_e w_e (.) P'_e   (row threads; the loads are warp-wide)
         {
-            float du[TV];
+            float du[TVH];
+            tmem_ld<TVH>(tmem_lane_addr(tY, warp, cofs), du);
+            for (int e0 = 0; e0 < E; e0 += GRP) {
+                float pv[GRP * TVH];
 #pragma unroll
-            for (int j = 0; j < TV; j += 16) tmem_ld16(tmem_lane_addr(tY, warp, j), du + j);
-            tmem_wait_ld();
-            for (int e = 0; e < E; ++e) {
-                float pv[TV];
-#pragma unroll
-                for (int j = 0; j < TV; j += 16) tmem_ld16(tmem_lane_addr(tP, warp, e * TV + j), pv + j);
+                for (int g = 0; g < GRP; ++g) tmem_ld<TVH>(tmem_lane_addr(tP, warp, (e0 + g) * TV + cofs), pv + g * TVH);
                 tmem_wait_ld();
-                const float wv = row_thread ? we[r64 * E + e] : 0.f;
 #pragma unroll
-                for (int i = 0; i < TV; ++i) du[i] = fmaf(wv, pv[i], du[i]);
+                for (int g = 0; g < GRP; ++g) {
+                    const float wv = row_thread ? we[r64 * E + e0 + g] : 0.f;
+#pragma unroll
+                    for (int i = 0; i < TVH; ++i) du[i] = fmaf(wv, pv[g * TVH + i], du[i]);
+                }
             }
             if (row_thread) {
 #pragma unroll
-                for (int i = 0; i < TV; ++i) st_split(sUh, sUl, sw128_offset(i, r64, TV), du[i]);
-                if (p.ck_tiles) store_tok_tile(p.dUbuf, (size_t(b) * H + h) * NT + cb + c, dv, r64, n0, du, TV, r64 < n);
-                else if (r64 < n) store_f32_row(p.dUbuf + tok_idx(b, t0 + r64, h, n0, T, H, dv), du, TV);
+                for (int i = 0; i < TVH; i += 8) st8_split(sUh, sUl, blk_offset<TV>(r64, cofs + i), du + i);
+                if (p.ck_tiles) store_tok_tile(p.dUbuf, (size_t(b) * H + h) * NT + cb + c, dv, r64, n0 + cofs, du, TVH, r64 < n);
+                else if (r64 < n) store_f32_row(p.dUbuf + tok_idx(b, t0 + r64, h, n0 + cofs, T, H, dv), du, TVH);
             }
         }
         fence_proxy_async_smem();
@@ -305,15 +336,16 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         __syncthreads();
         tc_fence_after();
 
-        // ---- MMA-B': dRes = T^T dU   (into tY)
+        // ---- MMA-B': dRes = T^T dU   (into tY; dU MN-major)
         if (tid == 0) {
-            const uint32_t idb = idesc_bf16_f32(64, TV, 0, 0);
+            const uint32_t idb = idesc_bf16_f32(64, TV, 0, 1);
 #pragma unroll
             for (int ks = 0; ks < 4; ++ks) {
                 const uint64_t th = smem_desc(smem_u32(sBT) + 2 * kBoxBytes + ks * 32, 16, 1024);
                 const uint64_t tl = smem_desc(smem_u32(sBT) + 3 * kBoxBytes + ks * 32, 16, 1024);
-                const uint64_t uh = smem_desc(smem_u32(sUh) + ks * 32, 16, 1024);
-                const uint64_t ul = smem_desc(smem_u32(sUl) + ks * 32, 16, 1024);
+                const uint32_t ko = ks * 32 * TV;
+                const uint64_t uh = smem_desc(smem_u32(sUh) + ko, blk_bytes<TV>(), 16 * TV, kSwz);
+                const uint64_t ul = smem_desc(smem_u32(sUl) + ko, blk_bytes<TV>(), 16 * TV, kSwz);
                 umma_bf16(tY, th, uh, idb, ks > 0 ? 1u : 0u);
                 umma_bf16(tY, th, ul, idb, 1u);
                 umma_bf16(tY, tl, uh, idb, 1u);
@@ -330,45 +362,45 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
 
         // ---- operand rows of MMA-C': [-a_e (.) dRes ; b_e (.) dO]
         {
-            float dr[TV];
-#pragma unroll
-            for (int j = 0; j < TV; j += 16) tmem_ld16(tmem_lane_addr(tY, warp, j), dr + j);
+            float dr[TVH];
+            tmem_ld<TVH>(tmem_lane_addr(tY, warp, cofs), dr);
             tmem_wait_ld();
             if (row_thread) {
                 if (tma_dv) {   // row of the dv tile; thread 0 stores the tile after the barrier
-                    if (p.out_f32) store_f32_row(reinterpret_cast<float*>(sDvo) + r64 * TV, dr, TV);
-                    else store_row(sDvo, size_t(r64) * TV, dr, TV, 0);
+                    if (p.out_f32) store_f32_row(reinterpret_cast<float*>(sDvo) + r64 * TV + cofs, dr, TVH);
+                    else store_row(sDvo, size_t(r64) * TV + cofs, dr, TVH, 0);
                 }
                 if (r64 < n) {
-                    const size_t off = tok_idx(b, t0 + r64, h, n0, T, H, dv);
-                    if (!p.ck_tiles) store_f32_row(p.dRbuf + off, dr, TV);
-                    if (!tma_dv) store_row(p.dv_out, off, dr, TV, p.out_f32);
+                    const size_t off = tok_idx(b, t0 + r64, h, n0 + cofs, T, H, dv);
+                    if (!p.ck_tiles) store_f32_row(p.dRbuf + off, dr, TVH);
+                    if (!tma_dv) store_row(p.dv_out, off, dr, TVH, p.out_f32);
                 }
                 if (p.ck_tiles && p.use_delta) {   // -dRes, the operand sign the gradient kernel uses
-                    float ndr[TV];
+                    float ndr[TVH];
 #pragma unroll
-                    for (int i = 0; i < TV; ++i) ndr[i] = -dr[i];
-                    store_tok_tile(p.dRbuf, (size_t(b) * H + h) * NT + cb + c, dv, r64, n0, ndr, TV, r64 < n);
+                    for (int i = 0; i < TVH; ++i) ndr[i] = -dr[i];
+                    store_tok_tile(p.dRbuf, (size_t(b) * H + h) * NT + cb + c, dv, r64, n0 + cofs, ndr, TVH, r64 < n);
                 }
                 if (p.use_delta) {
                     for (int e = 0; e < E; ++e) {
                         const float a = -ae[r64 * E + e];
-                        float x[TV];
+                        float x[TVH];
 #pragma unroll
-                        for (int i = 0; i < TV; ++i) x[i] = a * dr[i];
+                        for (int i = 0; i < TVH; ++i) x[i] = a * dr[i];
 #pragma unroll
-                        for (int i = 0; i < TV; i += 8) st8_split(sBh, sBl, sw128_offset(r64, e * TV + i, 128), x + i);
+                        for (int i = 0; i < TVH; i += 8)
+                            st8_split(sBh, sBl, sw128_offset(r64, e * TV + cofs + i, 128), x + i);
                     }
                 }
             } else {
                 for (int e = 0; e < E; ++e) {
                     const float bq = be[r64 * E + e];
-                    float x[TV];
+                    float x[TVH];
 #pragma unroll
-                    for (int i = 0; i < TV; ++i) x[i] = bq * dorow[i];
+                    for (int i = 0; i < TVH; ++i) x[i] = bq * dorow[i];
 #pragma unroll
-                    for (int i = 0; i < TV; i += 8)
-                        st8_split(sBh, sBl, sw128_offset(64 + r64, e * TV + i, 128), x + i);
+                    for (int i = 0; i < TVH; i += 8)
+                        st8_split(sBh, sBl, sw128_offset(64 + r64, e * TV + cofs + i, 128), x + i);
                 }
             }
         }
@@ -401,15 +433,17 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         if (tid == 0 && c > 0) issue_kq(c - 1);
 
         if (c > 0) {
-            prepare(c - 1, false);
+            stage_operand(c - 1);   // its gamma^C scaling follows the next MMA-A' issue
         } else if (p.dh0) {
-            const int d = tid;
-            for (int e = 0; e < E; ++e) {
-                float v[TV];
+            for (int e0 = 0; e0 < E; e0 += GRP) {
+                float v[GRP * TVH];
 #pragma unroll
-                for (int j = 0; j < TV; j += 16) tmem_ld16(tmem_lane_addr(tS, warp, e * TV + j), v + j);
+                for (int g = 0; g < GRP; ++g) tmem_ld<TVH>(tmem_lane_addr(tS, warp, (e0 + g) * TV + cofs), v + g * TVH);
                 tmem_wait_ld();
-                store_f32_row(p.dh0 + ((size_t(sb * H + h) * E + e) * kDk + d) * dv + n0, v, TV);
+#pragma unroll
+                for (int g = 0; g < GRP; ++g)
+                    store_f32_row(p.dh0 + ((size_t(sb * H + h) * E + e0 + g) * kDk + r) * dv + n0 + cofs,
+                                  v + g * TVH, TVH);
             }
         }
         fence_proxy_async_smem();
@@ -432,8 +466,7 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
 template <int TV>
 size_t tc_bwd_smem(int E) {
     const int NE = E * TV;
-    return 1024 + 8 * kBoxBytes + NE * 512 + TV * 128 + 64 * TV * 2 + 64 * TV * 4 +
-           2 * (3 * 64 * E + 16) * 4;
+    return 1024 + 8 * kBoxBytes + NE * 512 + 64 * TV * 2 + 64 * TV * 4 + 2 * (3 * 64 * E + 16) * 4;
 }
 
 template <int TV>
@@ -444,7 +477,7 @@ cudaError_t launch_tv(const tla_problem& p, const FwdPlan& fp, const char* fws, 
     const int NT = fp.NT;
     if (!make_token_map(&mk, p.k, p.B, p.T, p.H, kDk, 64, 64, true) ||
         !make_token_map(&mq, p.q, p.B, p.T, p.H, kDk, 64, 64, true) ||
-        !make_token_map(&mo, dO, p.B, p.T, p.H, p.dv, TV, 64, false) ||
+        !make_token_map_sw(&mo, dO, p.B, p.T, p.H, p.dv, TV, 64) ||
         !make_matrix_map(&mb, fws + fp.BT, (long long)p.B * p.H * NT * 256, 64, 64, 64) ||
         !make_token_map(&mdv, dv, p.B, p.T, p.H, p.dv, TV, 64, false,
                         p.out_dtype == TLA_FP32 ? 4 : 2))

@@ -1,6 +1,6 @@
 // Tensor-core (tcgen05) forward recurrence over chunks, Appendix A, Eq. joint-chunk.
 //
-// One CTA of 4 warps per (b, h, block of TV value columns); value columns never
+// One CTA of 8 warps per (b, h, block of TV value columns); value columns never
 // interact (Section 2.5, Eq. slices), so each CTA carries its own E x dk x TV
 // slab of the fp32 state in tensor memory for the whole sequence.  Per chunk of
 // C = 64 positions, with a_e = k'_e (.) gamma_e, b_e = q'_e (.) gamma_e and
@@ -13,8 +13,9 @@
 //   epi-B  O = Oi + Oa;  Ut_e = diag(w_e) U
 //   MMA-C  S_all += K^T [Ut_1 .. Ut_E] (M=dk=128, K=64, N=NE; K^T read MN-major
 //                                      straight from the TMA-loaded key tile)
-//   epi-C  S_{[c+1]} from TMEM in one pass: operand of the next MMA-A (also the
-//          checkpoint), and pre-scaled by gamma^C of the next chunk for its MMA-C.
+//   epi-C  S_{[c+1]} from TMEM: operand of the next MMA-A (also the checkpoint);
+//          once that product is issued, the TMEM slab is rescaled in place by
+//          gamma^C of the next chunk for its MMA-C (off the critical path).
 // Accumulation is fp32 in TMEM.  Keys and queries are bf16 inputs and enter the
 // products exactly; every other operand (the state, Res, T, A T, Ut) is carried
 // as a pair of bf16 values hi + lo (lo = bf16 of the rounding remainder), and
@@ -22,15 +23,19 @@
 // the other side is an exact key or query).  This keeps the products near fp32
 // accuracy: with a single bf16 rounding of those operands the error of o and of
 // the state reaches the 2e-2 x RMS parity bound.
-// The state and Ut operands are stored MN-major (one row per thread, 16-byte
-// stores), so each thread writes the TMEM row it read.  The state operand is kept
-// as one swizzled [dk][TV] block per slice (tc_common.cuh); a chunk's checkpoint
-// leaves shared memory as one TMA tensor store of those blocks into the row-major
-// [dk][dv] hi and lo matrices of its slices (tma_host.h).  Key, query, value
-// tiles, the [T; A T] tiles and the coefficient block arrive by TMA, prefetched
-// one chunk ahead as soon as their buffers are free.  Every mbarrier wait is
-// bounded by the GPU global timer; on expiry the CTA records TLA_ERR_TIMEOUT and
-// leaves after a bounded drain of its outstanding work.
+// Thread layout: warp w reads TMEM lanes 32 (w % 4) .. +31 (the rows of every
+// product), and warps 0-3 / 4-7 take the first / second half of each slice's TV
+// value columns, so every epilogue is split over 256 threads; TMEM loads of
+// several slices are issued before one wait.  The state, Res and Ut operands
+// are stored MN-major (value columns contiguous: 16-byte stores of a thread's
+// row).  The state operand is kept as one swizzled [dk][TV] block per slice
+// (tc_common.cuh); a chunk's checkpoint leaves shared memory as one TMA tensor
+// store of those blocks into the row-major [dk][dv] hi and lo matrices of its
+// slices (tma_host.h).  Key, query, value tiles, the [T; A T] tiles and the
+// coefficient block arrive by TMA, prefetched one chunk ahead as soon as their
+// buffers are free.  Every mbarrier wait is bounded by the GPU global timer; on
+// expiry the CTA records TLA_ERR_TIMEOUT and leaves after a bounded drain of
+// its outstanding work.
 #include <algorithm>
 #include <cstring>
 
@@ -45,7 +50,7 @@ using namespace sm100;
 
 namespace {
 
-constexpr int kThreads = 128;
+constexpr int kThreads = 256;
 constexpr int kDk = 128;
 constexpr int kBoxBytes = 64 * 64 * 2;  // one 64 x 64 bf16 TMA box
 
@@ -62,14 +67,18 @@ struct TcFwdArgs {
     int T, H, dv, E, NT, use_delta, save, out_f32, ck_tiles;
 };
 
+// Two CTAs per SM (at most 128 registers a thread), except for 64-column blocks (E = 1, 3),
+// whose 32 columns per thread need more registers.
 template <int TV>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kThreads, TV == 64 ? 1 : 2)
 fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                          const __grid_constant__ CUtensorMap map_q,
                          const __grid_constant__ CUtensorMap map_v,
                          const __grid_constant__ CUtensorMap map_a2,
                          const __grid_constant__ CUtensorMap map_ck,
                          const __grid_constant__ CUtensorMap map_o, const TcFwdArgs p) {
+    constexpr int TVH = TV / 2;             // value columns per thread
+    constexpr int GRP = TVH >= 32 ? 1 : 32 / TVH;   // slices per batch of TMEM loads
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
@@ -80,7 +89,7 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     uint8_t* sReg = sA2 + 4 * kBoxBytes;       // shared region, NE * 512 bytes:
     uint8_t* sSh = sReg;                       //   S_all hi: E blocks [dk][TV] (MMA-A operand)
     uint8_t* sSl = sReg + NE * 256;            //   S_all lo
-    uint8_t* sRh = sReg;                       //   Res^T [TV][64] hi, lo (after MMA-A)
+    uint8_t* sRh = sReg;                       //   Res [64][TV] hi, lo, MN-major (after MMA-A)
     uint8_t* sRl = sReg + TV * 128;
     uint8_t* sUh = sReg + TV * 256;            //   Ut [64][NE] hi, lo, MN-major (after MMA-B)
     uint8_t* sUl = sUh + NE * 128;
@@ -92,6 +101,8 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     __shared__ uint32_t tmem_slot;
 
     const int tid = threadIdx.x, warp = tid >> 5;
+    const int r = tid & 127;                   // TMEM lane: row of every product
+    const int cofs = (tid >> 7) * TVH;         // this thread's first column within a slice
     const int nb = blockIdx.x, h = blockIdx.y, sb = blockIdx.z;   // sb: sequence or document
     const int n0 = nb * TV;
     const int T = p.T, H = p.H, dv = p.dv, NT = p.NT;
@@ -106,8 +117,8 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     if (nct == 0) {   // empty document: the final state is the initial one
         if (p.ht)
             for (int e = 0; e < E; ++e)
-                for (int n = 0; n < TV; ++n) {
-                    const size_t o = ((size_t(sb * H + h) * E + e) * kDk + tid) * dv + n0 + n;
+                for (int n = cofs; n < cofs + TVH; ++n) {
+                    const size_t o = ((size_t(sb * H + h) * E + e) * kDk + r) * dv + n0 + n;
                     p.ht[o] = p.h0 ? p.h0[o] : 0.f;
                 }
         return;
@@ -150,48 +161,74 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         tma_load_4d(sV, &map_v, &bar_av, n0, h, tbeg + c * 64, b);
         bulk_load(sCoef + (c & 1) * CB, p.coef + idx * CB, CB * 4, &bar_av);
     };
-    // Row d = tid of S_{[c]} (from h0 or from TMEM), in one pass: the bf16 hi/lo operand of
-    // MMA-A, the fp32 checkpoint when checkpoints are not tiles (tiles: issue_ckpt), and the
-    // gamma^C_c-scaled copy in TMEM that chunk c's state update accumulates onto.
-    auto stage_state = [&](int c, bool from_h0) {
-        const int d = tid;
+    // This thread's part (row r, TVH columns) of slice e of S_{[c]} -> the bf16 hi/lo
+    // operand block of MMA-A, and the fp32 checkpoint when checkpoints are not tiles (tiles:
+    // issue_ckpt stores the operand blocks).
+    auto put_operand = [&](int c, int e, const float* v) {
+#pragma unroll
+        for (int n = 0; n < TVH; n += 8)
+            st8_split(sSh, sSl, e * blk_bytes<TV>() + blk_offset<TV>(r, cofs + n), v + n);
+        if (p.save && !p.ck_tiles) {
+            const size_t slab = (((size_t(b) * H + h) * NT + cb + c) * E + e) * kDk * dv;
+            store_f32_row(p.Sck + slab + size_t(r) * dv + n0 + cofs, v, TVH);
+        }
+    };
+    // Operand of MMA-A(c) from the state slab in TMEM (S_{[c]}, the result of MMA-C(c-1)).
+    auto stage_operand = [&](int c) {
+        for (int e0 = 0; e0 < E; e0 += GRP) {
+            float v[GRP * TVH];
+#pragma unroll
+            for (int g = 0; g < GRP; ++g) tmem_ld<TVH>(tmem_lane_addr(tS, warp, (e0 + g) * TV + cofs), v + g * TVH);
+            tmem_wait_ld();
+#pragma unroll
+            for (int g = 0; g < GRP; ++g) put_operand(c, e0 + g, v + g * TVH);
+        }
+    };
+    // The slab rescaled in place by gamma^C_c: chunk c's state update accumulates onto it.
+    auto scale_state = [&](int c) {
         const float* gc = sCoef + (c & 1) * CB + 3 * 64 * E;
-        for (int e = 0; e < E; ++e) {
-            float v[TV];
-            if (from_h0) {
-                if (p.h0) {
-                    const float4* src = reinterpret_cast<const float4*>(
-                        p.h0 + ((size_t(sb * H + h) * E + e) * kDk + d) * dv + n0);
+        for (int e0 = 0; e0 < E; e0 += GRP) {
+            float v[GRP * TVH];
 #pragma unroll
-                    for (int i = 0; i < TV / 4; ++i) {
-                        float4 x = src[i];
-                        v[4 * i] = x.x; v[4 * i + 1] = x.y; v[4 * i + 2] = x.z; v[4 * i + 3] = x.w;
-                    }
-                } else {
+            for (int g = 0; g < GRP; ++g) tmem_ld<TVH>(tmem_lane_addr(tS, warp, (e0 + g) * TV + cofs), v + g * TVH);
+            tmem_wait_ld();
 #pragma unroll
-                    for (int i = 0; i < TV; ++i) v[i] = 0.f;
-                }
-            } else {
+            for (int g = 0; g < GRP; ++g) {
+                const float gm = gc[e0 + g];
 #pragma unroll
-                for (int j = 0; j < TV; j += 16) tmem_ld16(tmem_lane_addr(tS, warp, e * TV + j), v + j);
-                tmem_wait_ld();
+                for (int i = 0; i < TVH; ++i) v[g * TVH + i] *= gm;
+                tmem_st<TVH>(tmem_lane_addr(tS, warp, (e0 + g) * TV + cofs), v + g * TVH);
             }
-#pragma unroll
-            for (int n = 0; n < TV; n += 8) st8_split(sSh, sSl, e * blk_bytes<TV>() + blk_offset<TV>(d, n), v + n);
-            if (p.save && !p.ck_tiles) {
-                const size_t slab = (((size_t(b) * H + h) * NT + cb + c) * E + e) * kDk * dv;
-                store_f32_row(p.Sck + slab + size_t(d) * dv + n0, v, TV);
-            }
-            const float g = gc[e];
-#pragma unroll
-            for (int n = 0; n < TV; ++n) v[n] *= g;
-#pragma unroll
-            for (int j = 0; j < TV; j += 16) tmem_st16(tmem_lane_addr(tS, warp, e * TV + j), v + j);
         }
         tmem_wait_st();
     };
-    // Checkpoint of S_{[c]} (bf16 hi/lo) for the backward: this CTA's columns of the
-    // slice blocks, stored by TMA (thread 0, after the operand is complete).
+    // Initial state (h0 or zero): the operand of MMA-A(0) and the gamma^C_0-scaled slab.
+    auto stage_h0 = [&]() {
+        const float* gc = sCoef + 3 * 64 * E;
+        for (int e = 0; e < E; ++e) {
+            float v[TVH];
+            if (p.h0) {
+                const float4* src = reinterpret_cast<const float4*>(
+                    p.h0 + ((size_t(sb * H + h) * E + e) * kDk + r) * dv + n0 + cofs);
+#pragma unroll
+                for (int i = 0; i < TVH / 4; ++i) {
+                    const float4 x = src[i];
+                    v[4 * i] = x.x; v[4 * i + 1] = x.y; v[4 * i + 2] = x.z; v[4 * i + 3] = x.w;
+                }
+            } else {
+#pragma unroll
+                for (int i = 0; i < TVH; ++i) v[i] = 0.f;
+            }
+            put_operand(0, e, v);
+            const float gm = gc[e];
+#pragma unroll
+            for (int i = 0; i < TVH; ++i) v[i] *= gm;
+            tmem_st<TVH>(tmem_lane_addr(tS, warp, e * TV + cofs), v);
+        }
+        tmem_wait_st();
+    };
+    // Checkpoint of S_{[c]} (bf16 hi/lo) for the backward: this CTA's columns of the slice
+    // blocks, stored by TMA (thread 0, after the operand is complete).
     auto issue_ckpt = [&](int c) {
         if (!(p.save && p.ck_tiles)) return;
         tma_store_4d(&map_ck, sSh, n0, 0, ((b * H + h) * NT + cb + c) * E, 0);   // [hi|lo][E][dk][TV]
@@ -224,7 +261,7 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     if (!mbar_wait(&bar_av, 0)) failed = true;
     if (__syncthreads_or(failed)) failed = true;
     if (!failed) {
-        stage_state(0, true);
+        stage_h0();
         fence_proxy_async_smem();
         tc_fence_before();
         const bool ok = mbar_wait(&bar_kq, 0);
@@ -266,13 +303,12 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         tc_fence_after();
 
         // ---- epi-A: Res (key rows) and the inter-chunk read (query rows)
-        float oi[TV], res[TV];
-        if (warp < 2) {
-            const int r = tid;
+        float oi[TVH], res[TVH];
+        if (r < 64) {
             {
-                const uint4* vrow = reinterpret_cast<const uint4*>(sV + r * TV);
+                const uint4* vrow = reinterpret_cast<const uint4*>(sV + r * TV + cofs);
 #pragma unroll
-                for (int i = 0; i < TV / 8; ++i) {
+                for (int i = 0; i < TVH / 8; ++i) {
                     uint4 u = vrow[i];
                     const __nv_bfloat162* pr = reinterpret_cast<const __nv_bfloat162*>(&u);
 #pragma unroll
@@ -284,30 +320,36 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                 }
             }
             if (p.use_delta) {
-                for (int e = 0; e < E; ++e) {
-                    float pv[TV];
+                for (int e0 = 0; e0 < E; e0 += GRP) {
+                    float pv[GRP * TVH];
 #pragma unroll
-                    for (int j = 0; j < TV; j += 16) tmem_ld16(tmem_lane_addr(tP, warp, e * TV + j), pv + j);
+                    for (int g = 0; g < GRP; ++g) tmem_ld<TVH>(tmem_lane_addr(tP, warp, (e0 + g) * TV + cofs), pv + g * TVH);
                     tmem_wait_ld();
-                    const float a = ae[r * E + e];
 #pragma unroll
-                    for (int i = 0; i < TV; ++i) res[i] = fmaf(-a, pv[i], res[i]);
+                    for (int g = 0; g < GRP; ++g) {
+                        const float a = ae[r * E + e0 + g];
+#pragma unroll
+                        for (int i = 0; i < TVH; ++i) res[i] = fmaf(-a, pv[g * TVH + i], res[i]);
+                    }
                 }
             }
 #pragma unroll
-            for (int i = 0; i < TV; ++i) st_split(sRh, sRl, sw128_offset(i, r, TV), res[i]);
+            for (int i = 0; i < TVH; i += 8) st8_split(sRh, sRl, blk_offset<TV>(r, cofs + i), res + i);
         } else {
-            const int r = tid - 64;
+            const int rq = r - 64;
 #pragma unroll
-            for (int i = 0; i < TV; ++i) oi[i] = 0.f;
-            for (int e = 0; e < E; ++e) {
-                float pv[TV];
+            for (int i = 0; i < TVH; ++i) oi[i] = 0.f;
+            for (int e0 = 0; e0 < E; e0 += GRP) {
+                float pv[GRP * TVH];
 #pragma unroll
-                for (int j = 0; j < TV; j += 16) tmem_ld16(tmem_lane_addr(tP, warp, e * TV + j), pv + j);
+                for (int g = 0; g < GRP; ++g) tmem_ld<TVH>(tmem_lane_addr(tP, warp, (e0 + g) * TV + cofs), pv + g * TVH);
                 tmem_wait_ld();
-                const float bq = be[r * E + e];
 #pragma unroll
-                for (int i = 0; i < TV; ++i) oi[i] = fmaf(bq, pv[i], oi[i]);
+                for (int g = 0; g < GRP; ++g) {
+                    const float bq = be[rq * E + e0 + g];
+#pragma unroll
+                    for (int i = 0; i < TVH; ++i) oi[i] = fmaf(bq, pv[g * TVH + i], oi[i]);
+                }
             }
         }
         fence_proxy_async_smem();
@@ -315,15 +357,16 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         __syncthreads();
         tc_fence_after();
 
-        // ---- MMA-B: [U; Oa] = [T; A T] Res  (into columns [0, TV))
+        // ---- MMA-B: [U; Oa] = [T; A T] Res  (into columns [0, TV); Res MN-major)
         if (tid == 0) {
-            const uint32_t idesc = idesc_bf16_f32(128, TV, 0, 0);
+            const uint32_t idesc = idesc_bf16_f32(128, TV, 0, 1);
 #pragma unroll
             for (int ks = 0; ks < 4; ++ks) {
                 const uint64_t ah = smem_desc(smem_u32(sA2) + ks * 32, 16, 1024);
                 const uint64_t al = smem_desc(smem_u32(sA2) + 2 * kBoxBytes + ks * 32, 16, 1024);
-                const uint64_t bh = smem_desc(smem_u32(sRh) + ks * 32, 16, 1024);
-                const uint64_t bl = smem_desc(smem_u32(sRl) + ks * 32, 16, 1024);
+                const uint32_t ko = ks * 32 * TV;
+                const uint64_t bh = smem_desc(smem_u32(sRh) + ko, blk_bytes<TV>(), 16 * TV, kSwz);
+                const uint64_t bl = smem_desc(smem_u32(sRl) + ko, blk_bytes<TV>(), 16 * TV, kSwz);
                 umma_bf16(tP, ah, bh, idesc, ks > 0 ? 1u : 0u);
                 umma_bf16(tP, ah, bl, idesc, 1u);
                 umma_bf16(tP, al, bh, idesc, 1u);
@@ -331,9 +374,9 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             umma_commit(&bar_mma);
         }
         pending_mma = 1;
-        if (warp < 2 && p.Rbuf) {   // while MMA-B runs
-            if (p.ck_tiles) store_tok_tile(p.Rbuf, (size_t(b) * H + h) * NT + cb + c, dv, tid, n0, res, TV, tid < n);
-            else if (tid < n) store_f32_row(p.Rbuf + tok_idx(b, t0 + tid, h, n0, T, H, dv), res, TV);
+        if (r < 64 && p.Rbuf) {   // while MMA-B runs
+            if (p.ck_tiles) store_tok_tile(p.Rbuf, (size_t(b) * H + h) * NT + cb + c, dv, r, n0 + cofs, res, TVH, r < n);
+            else if (r < n) store_f32_row(p.Rbuf + tok_idx(b, t0 + r, h, n0 + cofs, T, H, dv), res, TVH);
         }
         ok = mbar_wait(&bar_mma, mma_phase);
         mma_phase ^= 1;
@@ -343,27 +386,25 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         if (tid == 0 && c + 1 < nct) issue_av(c + 1);   // [T; A T], V and the other coef buffer are free
 
         // ---- epi-B: Ut operand (key rows); O = Oi + Oa (query rows)
-        float d2[TV];
-#pragma unroll
-        for (int j = 0; j < TV; j += 16) tmem_ld16(tmem_lane_addr(tP, warp, j), d2 + j);
+        float d2[TVH];
+        tmem_ld<TVH>(tmem_lane_addr(tP, warp, cofs), d2);
         tmem_wait_ld();
-        if (warp < 2) {
-            const int r = tid;
+        if (r < 64) {
             for (int e = 0; e < E; ++e) {
                 const float wv = we[r * E + e];
-                float u[TV];
+                float u[TVH];
 #pragma unroll
-                for (int i = 0; i < TV; ++i) u[i] = wv * d2[i];
+                for (int i = 0; i < TVH; ++i) u[i] = wv * d2[i];
 #pragma unroll
-                for (int i = 0; i < TV; i += 8) st8_split(sUh, sUl, sw128_offset(r, e * TV + i, 64), u + i);
+                for (int i = 0; i < TVH; i += 8) st8_split(sUh, sUl, sw128_offset(r, e * TV + cofs + i, 64), u + i);
             }
         } else {
 #pragma unroll
-            for (int i = 0; i < TV; ++i) d2[i] += oi[i];
+            for (int i = 0; i < TVH; ++i) d2[i] += oi[i];
             if (tma_o) {   // row of the o tile; thread 0 stores the tile after the barrier
-                const int r = tid - 64;
-                if (p.out_f32) store_f32_row(reinterpret_cast<float*>(sOo) + r * TV, d2, TV);
-                else store_row(sOo, size_t(r) * TV, d2, TV, 0);
+                const int rq = r - 64;
+                if (p.out_f32) store_f32_row(reinterpret_cast<float*>(sOo) + rq * TV + cofs, d2, TVH);
+                else store_row(sOo, size_t(rq) * TV + cofs, d2, TVH, 0);
             }
         }
         fence_proxy_async_smem();
@@ -388,14 +429,13 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         }
         pending_mma = 1;
         {   // while MMA-C runs: U (key rows) and o (query rows) to global memory
-            const int r = warp < 2 ? tid : tid - 64;
-            if (warp < 2) {
+            if (r < 64) {
                 if (p.save) {
-                    if (p.ck_tiles) store_tok_tile(p.Ubuf, (size_t(b) * H + h) * NT + cb + c, dv, r, n0, d2, TV, r < n);
-                    else if (r < n) store_f32_row(p.Ubuf + tok_idx(b, t0 + r, h, n0, T, H, dv), d2, TV);
+                    if (p.ck_tiles) store_tok_tile(p.Ubuf, (size_t(b) * H + h) * NT + cb + c, dv, r, n0 + cofs, d2, TVH, r < n);
+                    else if (r < n) store_f32_row(p.Ubuf + tok_idx(b, t0 + r, h, n0 + cofs, T, H, dv), d2, TVH);
                 }
-            } else if (!tma_o && r < n) {
-                store_row(p.o, tok_idx(b, t0 + r, h, n0, T, H, dv), d2, TV, p.out_f32);
+            } else if (!tma_o && r - 64 < n) {
+                store_row(p.o, tok_idx(b, t0 + r - 64, h, n0 + cofs, T, H, dv), d2, TVH, p.out_f32);
             }
         }
         ok = mbar_wait(&bar_mma, mma_phase);
@@ -406,9 +446,10 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         tc_fence_after();
         if (tid == 0 && c + 1 < nct) issue_kq(c + 1);   // key/query buffer is free
 
-        // ---- epi-C: next chunk's state (operand, scaled TMEM copy), MMA-A(c+1), checkpoint
+        // ---- epi-C: next chunk's state operand, MMA-A(c+1) and its checkpoint, then the
+        // gamma^C-scaled slab for MMA-C(c+1)
         if (c + 1 < nct) {
-            stage_state(c + 1, false);
+            stage_operand(c + 1);
             fence_proxy_async_smem();
             tc_fence_before();
             ok = mbar_wait(&bar_kq, (c + 1) & 1);
@@ -419,14 +460,17 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                 issue_ckpt(c + 1);
             }
             pending_mma = 1;
+            scale_state(c + 1);   // ordered before MMA-C(c+1) by the barriers in between
         } else if (p.ht) {
-            const int d = tid;
-            for (int e = 0; e < E; ++e) {
-                float v[TV];
+            for (int e0 = 0; e0 < E; e0 += GRP) {
+                float v[GRP * TVH];
 #pragma unroll
-                for (int j = 0; j < TV; j += 16) tmem_ld16(tmem_lane_addr(tS, warp, e * TV + j), v + j);
+                for (int g = 0; g < GRP; ++g) tmem_ld<TVH>(tmem_lane_addr(tS, warp, (e0 + g) * TV + cofs), v + g * TVH);
                 tmem_wait_ld();
-                store_f32_row(p.ht + ((size_t(sb * H + h) * E + e) * kDk + d) * dv + n0, v, TV);
+#pragma unroll
+                for (int g = 0; g < GRP; ++g)
+                    store_f32_row(p.ht + ((size_t(sb * H + h) * E + e0 + g) * kDk + r) * dv + n0 + cofs,
+                                  v + g * TVH, TVH);
             }
         }
     }

@@ -42,6 +42,27 @@ inline bool make_token_map(CUtensorMap* m, const void* base, int B, int T, int H
     return r == CUDA_SUCCESS;
 }
 
+// Token tensor as above (bf16), box (box_d, 1, box_t, 1), the shared-memory side swizzled by
+// swizzle_bytes = 2 * box_d (32, 64 or 128): the rows land as the MN-major operand layout of a
+// [box_t][box_d] block (tc_common.cuh: blk_offset).
+inline bool make_token_map_sw(CUtensorMap* m, const void* base, int B, int T, int H, int D,
+                              int box_d, int box_t) {
+    auto enc = tensor_map_encoder();
+    if (!enc) return false;
+    const int sw = 2 * box_d;
+    if (sw != 32 && sw != 64 && sw != 128) return false;
+    cuuint64_t dims[4] = {(cuuint64_t)D, (cuuint64_t)H, (cuuint64_t)T, (cuuint64_t)B};
+    cuuint64_t strides[3] = {(cuuint64_t)D * 2, (cuuint64_t)H * D * 2, (cuuint64_t)T * H * D * 2};
+    cuuint32_t box[4] = {(cuuint32_t)box_d, 1, (cuuint32_t)box_t, 1};
+    cuuint32_t es[4] = {1, 1, 1, 1};
+    CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides,
+                     box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                     sw == 32 ? CU_TENSOR_MAP_SWIZZLE_32B
+                     : sw == 64 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
 // bf16 row-major matrix [rows][cols] as 2-D (cols, rows); box (box_c, box_r); shared-memory
 // side swizzled by swizzle_bytes (32, 64 or 128; box_c * 2 must not exceed it).
 inline bool make_matrix_map(CUtensorMap* m, const void* base, long long rows, int cols, int box_c,
