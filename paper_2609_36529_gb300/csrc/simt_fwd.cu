@@ -155,16 +155,16 @@ chunk_prep_kernel(const Tin* __restrict__ q, const Tin* __restrict__ k, const Ti
     }
     if (coef_out) {
         // Per-row coefficients of the tensor-core recurrence, one block per chunk:
-        // [k'_e gamma_e | q'_e gamma_e | k'_e gamma^C_e / gamma_e] as [64][E] each, then gamma^C_e
-        // (padded to 16).  Decays are exponentials of non-positive log differences.
+        // [k'_e gamma_e | q'_e gamma_e | k'_e gamma^C_e / gamma_e] as [E][64] each (slice-major),
+        // then gamma^C_e (padded to 16).  Decays are exponentials of non-positive log differences.
         float* cf = coef_out + ((size_t(b) * H + h) * NT + c) * (3 * kChunk * E + 16);
         for (int i = tid; i < kChunk * E; i += blockDim.x) {
-            const int e = i % E;
-            const float Gr = Gs[i], GC = Gs[(n - 1) * E + e];
+            const int e = i / kChunk, r = i % kChunk, ir = r * E + e;
+            const float Gr = Gs[ir], GC = Gs[(n - 1) * E + e];
             const float gam = expf(Gr);
-            cf[i] = k2s[i] * gam;
-            cf[kChunk * E + i] = q2s[i] * gam;
-            cf[2 * kChunk * E + i] = k2s[i] * expf(GC - Gr);
+            cf[i] = k2s[ir] * gam;
+            cf[kChunk * E + i] = q2s[ir] * gam;
+            cf[2 * kChunk * E + i] = k2s[ir] * expf(GC - Gr);
         }
         if (tid < 16) cf[3 * kChunk * E + tid] = tid < E ? expf(Gs[(n - 1) * E + tid]) : 0.f;
     }

@@ -21,7 +21,9 @@
 //           previous chunk's MMA-A' is issued, the slab is rescaled in place by its gamma^C.
 // Layout of the M=64 products in TMEM: row r sits on lane 32 * (r / 16) + r % 16,
 // so lanes 0-15 of each warp own the row work and lanes 16-31 the dO rows.
-// Warps 0-3 / 4-7 take the first / second half of each slice's TV value columns.
+// Warps 0-3 / 4-7 take the first / second half of each slice's TV value columns.  E is a
+// compile-time parameter (per-slice loops unroll; each thread keeps its row's coefficients,
+// read from the slice-major coefficient block, in registers).
 // Precision, TMA prefetch, bounded waits, the slice-block layout of the state
 // operand and the TMA-stored checkpoints as in the forward kernel.
 #include <cstring>
@@ -54,9 +56,20 @@ struct TcBwdArgs {
     int T, H, dv, E, NT, use_delta, out_f32, ck_tiles;
 };
 
-// Two CTAs per SM (at most 128 registers a thread), except for 64-column blocks.
 template <int TV>
-__global__ void __launch_bounds__(kThreads, TV == 64 ? 1 : 2)
+__host__ __device__ constexpr size_t tc_bwd_smem_c(int E) {
+    return 1024 + 8 * kBoxBytes + size_t(E) * TV * 512 + 64 * TV * 2 + 64 * TV * 4 +
+           2 * (3 * 64 * E + 16) * 4;
+}
+// CTAs per SM the launch bounds plan for: two (at most 128 registers a thread) when two fit
+// in shared memory, else one.
+template <int TV, int E>
+__host__ __device__ constexpr int bwd_min_blocks() {
+    return tc_bwd_smem_c<TV>(E) <= 113 * 1024 ? 2 : 1;
+}
+
+template <int TV, int E>
+__global__ void __launch_bounds__(kThreads, (bwd_min_blocks<TV, E>()))
 bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                          const __grid_constant__ CUtensorMap map_q,
                          const __grid_constant__ CUtensorMap map_do,
@@ -64,12 +77,14 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                          const __grid_constant__ CUtensorMap map_ck,
                          const __grid_constant__ CUtensorMap map_dv, const TcBwdArgs p) {
     constexpr int TVH = TV / 2;                      // value columns per thread
-    constexpr int GRP = TVH >= 32 ? 1 : 32 / TVH;    // slices per batch of TMEM loads
+    constexpr int GRP0 = TVH >= 32 ? 1 : 32 / TVH;
+    constexpr int GRP = GRP0 < E ? GRP0 : E;         // slices per batch of TMEM loads
+    static_assert(E % GRP == 0, "slices per batch must divide E");
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
-    const int E = p.E, NE = E * TV;
-    const int CB = 3 * 64 * E + 16;
+    constexpr int NE = E * TV;
+    constexpr int CB = 3 * 64 * E + 16;
     uint8_t* sKQ = sm;                       // 2 blocks x [K rows | Q rows] x 128 B
     uint8_t* sBT = sKQ + 4 * kBoxBytes;      // A^T hi, A^T lo, T^T hi, T^T lo (64 x 64 each)
     uint8_t* sReg = sBT + 4 * kBoxBytes;     // NE * 512 bytes, reused:
@@ -92,7 +107,7 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     const int nb = blockIdx.x, h = blockIdx.y, sb = blockIdx.z;   // sb: sequence or document
     const int n0 = nb * TV;
     const int T = p.T, H = p.H, dv = p.dv, NT = p.NT;
-    const uint32_t tcols = (2 * NE + TV <= 256) ? 256u : 512u;
+    constexpr uint32_t tcols = (2 * NE + TV <= 256) ? 256u : 512u;
     constexpr uint64_t kSwz = swizzle_code(2 * TV);
     // token batch, first token, tokens, chunks and first chunk (in the workspaces) of this state
     int b = sb, tbeg = 0, tlen = T, nct = NT, cb = 0;
@@ -161,6 +176,7 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         }
     };
     auto stage_operand = [&](int c) {
+        #pragma unroll
         for (int e0 = 0; e0 < E; e0 += GRP) {
             float v[GRP * TVH];
 #pragma unroll
@@ -173,6 +189,7 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     // The slab rescaled in place by gamma^C_c: chunk c's MMA-C' accumulates onto it.
     auto scale_state = [&](int c) {
         const float* gc = sCoef + (c & 1) * CB + 3 * 64 * E;
+        #pragma unroll
         for (int e0 = 0; e0 < E; e0 += GRP) {
             float v[GRP * TVH];
 #pragma unroll
@@ -191,6 +208,7 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     // Gradient of the final state (dht or zero): operand of MMA-A'(nct-1) and the scaled slab.
     auto stage_dht = [&](int c) {
         const float* gc = sCoef + (c & 1) * CB + 3 * 64 * E;
+        #pragma unroll
         for (int e = 0; e < E; ++e) {
             float v[TVH];
             if (p.dht) {
@@ -310,19 +328,20 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
 
         // ---- dU = Y + sum_e w_e (.) P'_e   (row threads; the loads are warp-wide)
         {
-            float du[TVH];
+            float du[TVH], wr[E];
+#pragma unroll
+            for (int e = 0; e < E; ++e) wr[e] = row_thread ? we[e * 64 + r64] : 0.f;
             tmem_ld<TVH>(tmem_lane_addr(tY, warp, cofs), du);
+#pragma unroll
             for (int e0 = 0; e0 < E; e0 += GRP) {
                 float pv[GRP * TVH];
 #pragma unroll
                 for (int g = 0; g < GRP; ++g) tmem_ld<TVH>(tmem_lane_addr(tP, warp, (e0 + g) * TV + cofs), pv + g * TVH);
                 tmem_wait_ld();
 #pragma unroll
-                for (int g = 0; g < GRP; ++g) {
-                    const float wv = row_thread ? we[r64 * E + e0 + g] : 0.f;
+                for (int g = 0; g < GRP; ++g)
 #pragma unroll
-                    for (int i = 0; i < TVH; ++i) du[i] = fmaf(wv, pv[g * TVH + i], du[i]);
-                }
+                    for (int i = 0; i < TVH; ++i) du[i] = fmaf(wr[e0 + g], pv[g * TVH + i], du[i]);
             }
             if (row_thread) {
 #pragma unroll
@@ -362,7 +381,9 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
 
         // ---- operand rows of MMA-C': [-a_e (.) dRes ; b_e (.) dO]
         {
-            float dr[TVH];
+            float dr[TVH], cr[E];   // -a_e (row threads) or b_e (dO rows) of this thread's row
+#pragma unroll
+            for (int e = 0; e < E; ++e) cr[e] = row_thread ? -ae[e * 64 + r64] : be[e * 64 + r64];
             tmem_ld<TVH>(tmem_lane_addr(tY, warp, cofs), dr);
             tmem_wait_ld();
             if (row_thread) {
@@ -382,8 +403,9 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                     store_tok_tile(p.dRbuf, (size_t(b) * H + h) * NT + cb + c, dv, r64, n0 + cofs, ndr, TVH, r64 < n);
                 }
                 if (p.use_delta) {
+#pragma unroll
                     for (int e = 0; e < E; ++e) {
-                        const float a = -ae[r64 * E + e];
+                        const float a = cr[e];
                         float x[TVH];
 #pragma unroll
                         for (int i = 0; i < TVH; ++i) x[i] = a * dr[i];
@@ -393,8 +415,9 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                     }
                 }
             } else {
+#pragma unroll
                 for (int e = 0; e < E; ++e) {
-                    const float bq = be[r64 * E + e];
+                    const float bq = cr[e];
                     float x[TVH];
 #pragma unroll
                     for (int i = 0; i < TVH; ++i) x[i] = bq * dorow[i];
@@ -435,6 +458,7 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         if (c > 0) {
             stage_operand(c - 1);   // its gamma^C scaling follows the next MMA-A' issue
         } else if (p.dh0) {
+            #pragma unroll
             for (int e0 = 0; e0 < E; e0 += GRP) {
                 float v[GRP * TVH];
 #pragma unroll
@@ -463,16 +487,11 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     if (warp == 0) tmem_dealloc(tmem_slot, tcols);
 }
 
-template <int TV>
-size_t tc_bwd_smem(int E) {
-    const int NE = E * TV;
-    return 1024 + 8 * kBoxBytes + NE * 512 + 64 * TV * 2 + 64 * TV * 4 + 2 * (3 * 64 * E + 16) * 4;
-}
-
-template <int TV>
+template <int TV, int E>
 cudaError_t launch_tv(const tla_problem& p, const FwdPlan& fp, const char* fws, const BwdPlan& bp,
                       char* bws, const void* dO, const float* dht, void* dv, float* dh0, int* err,
                       cudaStream_t s) {
+    if (p.E != E || fp.tc_tv != TV) return cudaErrorInvalidValue;
     CUtensorMap mk, mq, mo, mb, mc, mdv;
     const int NT = fp.NT;
     if (!make_token_map(&mk, p.k, p.B, p.T, p.H, kDk, 64, 64, true) ||
@@ -499,8 +518,8 @@ cudaError_t launch_tv(const tla_problem& p, const FwdPlan& fp, const char* fws, 
     a.use_delta = p.use_delta; a.out_f32 = p.out_dtype == TLA_FP32;
     a.ck_tiles = fp.ck_tiles;
     a.dtab = p.cu_seqlens ? (const int4*)(fws + fp.dtab) : nullptr;
-    const size_t smem = tc_bwd_smem<TV>(p.E);
-    auto kern = bwd_recurrence_tc_kernel<TV>;
+    const size_t smem = tc_bwd_smem_c<TV>(E);
+    auto kern = bwd_recurrence_tc_kernel<TV, E>;
     cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     dim3 grid(p.dv / TV, p.H, fp.nseq);
     prof_before("bwd_recurrence_tc", s);
@@ -518,8 +537,8 @@ int tc_bwd_ok(const tla_problem& p, int tv) {
     if (tv == 0) return 0;
     const int ne = p.E * tv;
     if (2 * ne + tv > 512) return 0;
-    const size_t smem = tv == 16 ? tc_bwd_smem<16>(p.E) : tv == 32 ? tc_bwd_smem<32>(p.E)
-                                                                   : tc_bwd_smem<64>(p.E);
+    const size_t smem = tv == 16 ? tc_bwd_smem_c<16>(p.E)
+                                 : tv == 32 ? tc_bwd_smem_c<32>(p.E) : tc_bwd_smem_c<64>(p.E);
     return smem <= 227 * 1024 ? 1 : 0;
 }
 
@@ -527,10 +546,16 @@ cudaError_t launch_bwd_recurrence_tc(const tla_problem& p, const FwdPlan& fp, co
                                      const BwdPlan& bp, char* bws, const void* dO,
                                      const float* dht, void* dv, float* dh0, int* err,
                                      cudaStream_t s) {
-    switch (fp.tc_tv) {
-        case 16: return launch_tv<16>(p, fp, fws, bp, bws, dO, dht, dv, dh0, err, s);
-        case 32: return launch_tv<32>(p, fp, fws, bp, bws, dO, dht, dv, dh0, err, s);
-        default: return launch_tv<64>(p, fp, fws, bp, bws, dO, dht, dv, dh0, err, s);
+    // one instance per slice count the tensor-core path takes (tc_fwd_tv, tc_bwd_ok)
+    switch (p.E) {
+        case 1: return launch_tv<64, 1>(p, fp, fws, bp, bws, dO, dht, dv, dh0, err, s);
+        case 2: return launch_tv<32, 2>(p, fp, fws, bp, bws, dO, dht, dv, dh0, err, s);
+        case 3: return launch_tv<64, 3>(p, fp, fws, bp, bws, dO, dht, dv, dh0, err, s);
+        case 4: return launch_tv<16, 4>(p, fp, fws, bp, bws, dO, dht, dv, dh0, err, s);
+        case 6: return launch_tv<32, 6>(p, fp, fws, bp, bws, dO, dht, dv, dh0, err, s);
+        case 8: return launch_tv<16, 8>(p, fp, fws, bp, bws, dO, dht, dv, dh0, err, s);
+        case 12: return launch_tv<16, 12>(p, fp, fws, bp, bws, dO, dht, dv, dh0, err, s);
+        default: return cudaErrorInvalidValue;
     }
 }
 

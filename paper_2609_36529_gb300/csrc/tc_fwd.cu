@@ -26,7 +26,9 @@
 // Thread layout: warp w reads TMEM lanes 32 (w % 4) .. +31 (the rows of every
 // product), and warps 0-3 / 4-7 take the first / second half of each slice's TV
 // value columns, so every epilogue is split over 256 threads; TMEM loads of
-// several slices are issued before one wait.  The state, Res and Ut operands
+// several slices are issued before one wait.  E is a compile-time parameter, so the
+// per-slice loops unroll and each thread holds its row's coefficients (read from the
+// slice-major coefficient block, conflict-free) in registers.  The state, Res and Ut operands
 // are stored MN-major (value columns contiguous: 16-byte stores of a thread's
 // row).  The state operand is kept as one swizzled [dk][TV] block per slice
 // (tc_common.cuh); a chunk's checkpoint leaves shared memory as one TMA tensor
@@ -67,10 +69,20 @@ struct TcFwdArgs {
     int T, H, dv, E, NT, use_delta, save, out_f32, ck_tiles;
 };
 
-// Two CTAs per SM (at most 128 registers a thread), except for 64-column blocks (E = 1, 3),
-// whose 32 columns per thread need more registers.
 template <int TV>
-__global__ void __launch_bounds__(kThreads, TV == 64 ? 1 : 2)
+__host__ __device__ constexpr size_t tc_fwd_smem_c(int E) {
+    return 1024 + 4 * kBoxBytes + 4 * kBoxBytes + size_t(E) * TV * 512 + 64 * TV * 2 + 64 * TV * 4 +
+           2 * (3 * 64 * E + 16) * 4;
+}
+// CTAs per SM the launch bounds plan for: two (at most 128 registers a thread) when two fit
+// in shared memory, else one.
+template <int TV, int E>
+__host__ __device__ constexpr int fwd_min_blocks() {
+    return tc_fwd_smem_c<TV>(E) <= 113 * 1024 ? 2 : 1;
+}
+
+template <int TV, int E>
+__global__ void __launch_bounds__(kThreads, (fwd_min_blocks<TV, E>()))
 fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                          const __grid_constant__ CUtensorMap map_q,
                          const __grid_constant__ CUtensorMap map_v,
@@ -78,12 +90,14 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                          const __grid_constant__ CUtensorMap map_ck,
                          const __grid_constant__ CUtensorMap map_o, const TcFwdArgs p) {
     constexpr int TVH = TV / 2;             // value columns per thread
-    constexpr int GRP = TVH >= 32 ? 1 : 32 / TVH;   // slices per batch of TMEM loads
+    constexpr int GRP0 = TVH >= 32 ? 1 : 32 / TVH;
+    constexpr int GRP = GRP0 < E ? GRP0 : E;   // slices per batch of TMEM loads
+    static_assert(E % GRP == 0, "slices per batch must divide E");
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
-    const int E = p.E, NE = E * TV;
-    const int CB = 3 * 64 * E + 16;            // floats per coefficient block
+    constexpr int NE = E * TV;
+    constexpr int CB = 3 * 64 * E + 16;        // floats per coefficient block
     uint8_t* sKQ = sm;                         // 2 blocks x [K rows 0-63 | Q rows 64-127] x 128 B
     uint8_t* sA2 = sKQ + 4 * kBoxBytes;        // [T; A T] 128 x 64 bf16: hi tile, lo tile
     uint8_t* sReg = sA2 + 4 * kBoxBytes;       // shared region, NE * 512 bytes:
@@ -106,7 +120,7 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     const int nb = blockIdx.x, h = blockIdx.y, sb = blockIdx.z;   // sb: sequence or document
     const int n0 = nb * TV;
     const int T = p.T, H = p.H, dv = p.dv, NT = p.NT;
-    const uint32_t tcols = (2 * NE <= 256) ? 256u : 512u;
+    constexpr uint32_t tcols = (2 * NE <= 256) ? 256u : 512u;
     constexpr uint64_t kSwz = swizzle_code(2 * TV);
     // token batch, first token, tokens, chunks and first chunk (in the workspace) of this state
     int b = sb, tbeg = 0, tlen = T, nct = NT, cb = 0;
@@ -175,6 +189,7 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     };
     // Operand of MMA-A(c) from the state slab in TMEM (S_{[c]}, the result of MMA-C(c-1)).
     auto stage_operand = [&](int c) {
+#pragma unroll
         for (int e0 = 0; e0 < E; e0 += GRP) {
             float v[GRP * TVH];
 #pragma unroll
@@ -187,6 +202,7 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     // The slab rescaled in place by gamma^C_c: chunk c's state update accumulates onto it.
     auto scale_state = [&](int c) {
         const float* gc = sCoef + (c & 1) * CB + 3 * 64 * E;
+#pragma unroll
         for (int e0 = 0; e0 < E; e0 += GRP) {
             float v[GRP * TVH];
 #pragma unroll
@@ -205,6 +221,7 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     // Initial state (h0 or zero): the operand of MMA-A(0) and the gamma^C_0-scaled slab.
     auto stage_h0 = [&]() {
         const float* gc = sCoef + 3 * 64 * E;
+#pragma unroll
         for (int e = 0; e < E; ++e) {
             float v[TVH];
             if (p.h0) {
@@ -302,8 +319,15 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         pending_mma = 0;
         tc_fence_after();
 
-        // ---- epi-A: Res (key rows) and the inter-chunk read (query rows)
-        float oi[TVH], res[TVH];
+        // ---- epi-A: Res (key rows) and the inter-chunk read (query rows).  The per-row
+        // coefficients of this thread's row for every slice come first (slice-major block:
+        // a warp reads 32 consecutive rows of one slice), then the products.
+        float oi[TVH], res[TVH], cr[E];
+        {
+            const float* crow = (r < 64 ? ae + r : be + (r - 64));
+#pragma unroll
+            for (int e = 0; e < E; ++e) cr[e] = crow[e * 64];
+        }
         if (r < 64) {
             {
                 const uint4* vrow = reinterpret_cast<const uint4*>(sV + r * TV + cofs);
@@ -320,36 +344,33 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                 }
             }
             if (p.use_delta) {
+#pragma unroll
                 for (int e0 = 0; e0 < E; e0 += GRP) {
                     float pv[GRP * TVH];
 #pragma unroll
                     for (int g = 0; g < GRP; ++g) tmem_ld<TVH>(tmem_lane_addr(tP, warp, (e0 + g) * TV + cofs), pv + g * TVH);
                     tmem_wait_ld();
 #pragma unroll
-                    for (int g = 0; g < GRP; ++g) {
-                        const float a = ae[r * E + e0 + g];
+                    for (int g = 0; g < GRP; ++g)
 #pragma unroll
-                        for (int i = 0; i < TVH; ++i) res[i] = fmaf(-a, pv[g * TVH + i], res[i]);
-                    }
+                        for (int i = 0; i < TVH; ++i) res[i] = fmaf(-cr[e0 + g], pv[g * TVH + i], res[i]);
                 }
             }
 #pragma unroll
             for (int i = 0; i < TVH; i += 8) st8_split(sRh, sRl, blk_offset<TV>(r, cofs + i), res + i);
         } else {
-            const int rq = r - 64;
 #pragma unroll
             for (int i = 0; i < TVH; ++i) oi[i] = 0.f;
+#pragma unroll
             for (int e0 = 0; e0 < E; e0 += GRP) {
                 float pv[GRP * TVH];
 #pragma unroll
                 for (int g = 0; g < GRP; ++g) tmem_ld<TVH>(tmem_lane_addr(tP, warp, (e0 + g) * TV + cofs), pv + g * TVH);
                 tmem_wait_ld();
 #pragma unroll
-                for (int g = 0; g < GRP; ++g) {
-                    const float bq = be[rq * E + e0 + g];
+                for (int g = 0; g < GRP; ++g)
 #pragma unroll
-                    for (int i = 0; i < TVH; ++i) oi[i] = fmaf(bq, pv[g * TVH + i], oi[i]);
-                }
+                    for (int i = 0; i < TVH; ++i) oi[i] = fmaf(cr[e0 + g], pv[g * TVH + i], oi[i]);
             }
         }
         fence_proxy_async_smem();
@@ -387,11 +408,16 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
 
         // ---- epi-B: Ut operand (key rows); O = Oi + Oa (query rows)
         float d2[TVH];
+        if (r < 64) {
+#pragma unroll
+            for (int e = 0; e < E; ++e) cr[e] = we[e * 64 + r];
+        }
         tmem_ld<TVH>(tmem_lane_addr(tP, warp, cofs), d2);
         tmem_wait_ld();
         if (r < 64) {
+#pragma unroll
             for (int e = 0; e < E; ++e) {
-                const float wv = we[r * E + e];
+                const float wv = cr[e];
                 float u[TVH];
 #pragma unroll
                 for (int i = 0; i < TVH; ++i) u[i] = wv * d2[i];
@@ -462,6 +488,7 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             pending_mma = 1;
             scale_state(c + 1);   // ordered before MMA-C(c+1) by the barriers in between
         } else if (p.ht) {
+#pragma unroll
             for (int e0 = 0; e0 < E; e0 += GRP) {
                 float v[GRP * TVH];
 #pragma unroll
@@ -490,16 +517,10 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     if (warp == 0) tmem_dealloc(tmem_slot, tcols);
 }
 
-template <int TV>
-size_t tc_fwd_smem(int E) {
-    const int NE = E * TV;
-    return 1024 + 4 * kBoxBytes + 4 * kBoxBytes + NE * 512 + 64 * TV * 2 + 64 * TV * 4 +
-           2 * (3 * 64 * E + 16) * 4;
-}
-
-template <int TV>
+template <int TV, int E>
 cudaError_t launch_tv(const tla_problem& p, const FwdPlan& fp, char* ws, int save, int* err,
                       cudaStream_t s) {
+    if (p.E != E || fp.tc_tv != TV) return cudaErrorInvalidValue;
     CUtensorMap mk, mq, mv, ma, mc, mo;
     const int NT = fp.NT;
     if (!make_token_map(&mk, p.k, p.B, p.T, p.H, kDk, 64, 64, true) ||
@@ -525,8 +546,8 @@ cudaError_t launch_tv(const tla_problem& p, const FwdPlan& fp, char* ws, int sav
     a.use_delta = p.use_delta; a.save = save; a.out_f32 = p.out_dtype == TLA_FP32;
     a.ck_tiles = fp.ck_tiles;
     a.dtab = p.cu_seqlens ? (const int4*)(ws + fp.dtab) : nullptr;
-    const size_t smem = tc_fwd_smem<TV>(p.E);
-    auto kern = fwd_recurrence_tc_kernel<TV>;
+    const size_t smem = tc_fwd_smem_c<TV>(E);
+    auto kern = fwd_recurrence_tc_kernel<TV, E>;
     cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     dim3 grid(p.dv / TV, p.H, fp.nseq);
     prof_before("fwd_recurrence_tc", s);
@@ -552,10 +573,17 @@ int tc_fwd_tv(const tla_problem& p) {
 
 cudaError_t launch_fwd_recurrence_tc(const tla_problem& p, const FwdPlan& fp, char* ws,
                                      int save_for_bwd, int* err, cudaStream_t s) {
-    switch (fp.tc_tv) {
-        case 16: return launch_tv<16>(p, fp, ws, save_for_bwd, err, s);
-        case 32: return launch_tv<32>(p, fp, ws, save_for_bwd, err, s);
-        default: return launch_tv<64>(p, fp, ws, save_for_bwd, err, s);
+    // one instance per slice count the tensor-core path takes (tc_fwd_tv)
+    switch (p.E) {
+        case 1: return launch_tv<64, 1>(p, fp, ws, save_for_bwd, err, s);
+        case 2: return launch_tv<32, 2>(p, fp, ws, save_for_bwd, err, s);
+        case 3: return launch_tv<64, 3>(p, fp, ws, save_for_bwd, err, s);
+        case 4: return launch_tv<16, 4>(p, fp, ws, save_for_bwd, err, s);
+        case 6: return launch_tv<32, 6>(p, fp, ws, save_for_bwd, err, s);
+        case 8: return launch_tv<16, 8>(p, fp, ws, save_for_bwd, err, s);
+        case 12: return launch_tv<16, 12>(p, fp, ws, save_for_bwd, err, s);
+        case 16: return launch_tv<16, 16>(p, fp, ws, save_for_bwd, err, s);
+        default: return cudaErrorInvalidValue;
     }
 }
 

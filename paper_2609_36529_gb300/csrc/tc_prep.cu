@@ -9,7 +9,7 @@
 //   T = N diag(beta) (sGLA: diag(beta)), A T
 // and writes A and N (fp32), the bf16 hi/lo tiles [T; A T] (forward recurrence) and
 // [A^T; T^T] (backward recurrence), and the per-row coefficient block
-// [k'_e gamma_e | q'_e gamma_e | k'_e gamma^C_e / gamma_e | gamma^C_e].
+// [k'_e gamma_e | q'_e gamma_e | k'_e gamma^C_e / gamma_e | gamma^C_e] (slice-major).
 #include "common.cuh"
 #include "internal.h"
 #include "sm100.cuh"
@@ -351,15 +351,15 @@ chunk_prep_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             put4(BT + 8192 + o, BT + 12288 + o, Tv[0][c2], Tv[1][c2], Tv[2][c2], Tv[3][c2]);
         }
     }
-    // coefficient block
+    // coefficient block, slice-major: [a | b | w] each [E][64 rows], then gamma^C_e
     float* cf = p.coef + ((size_t(b) * H + h) * NT + c) * (3 * 64 * E + 16);
     for (int i = tid; i < 64 * E; i += kThreads) {
-        const int e = i - (i / E) * E;
-        const float Gr = Gs[i], GC = Gs[(n - 1) * E + e];
+        const int e = i >> 6, r = i & 63, ir = r * E + e;
+        const float Gr = Gs[ir], GC = Gs[(n - 1) * E + e];
         const float gam = __expf(Gr);
-        cf[i] = k2s[i] * gam;
-        cf[64 * E + i] = q2s[i] * gam;
-        cf[128 * E + i] = k2s[i] * __expf(GC - Gr);
+        cf[i] = k2s[ir] * gam;
+        cf[64 * E + i] = q2s[ir] * gam;
+        cf[128 * E + i] = k2s[ir] * __expf(GC - Gr);
     }
     if (tid < 16) cf[192 * E + tid] = tid < E ? __expf(Gs[(n - 1) * E + tid]) : 0.f;
 }
