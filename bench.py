@@ -789,6 +789,26 @@ def run_layer_io(args, tla, inputs, w, dev, stream, barrier, max_over_ranks, ran
         gbs = bytes_per[name] * units / (ms / 1e3) / 1e9
         out[name] = {"ms": round(ms, 4), "achieved_gbs": round(gbs, 1), "frac": round(gbs / peak, 4),
                      "bytes_per_token_head": bytes_per[name]}
+    del x, args_p, grads, dy
+    torch.cuda.empty_cache()
+    # the input projection GEMM with the input path fused into its epilogue, at the paper's
+    # 1.3B-parameter width (d_model 2048, 16 heads of d = 128): tensor-bound
+    Dm = 2048
+    xp = inputs.projection_inputs(B, T, H, dk, dv, E, Dm, K, device=dev, seed=310 + rank)
+    C = 2 * dk + dv + 2 * E
+    call = lambda: tla.layer_projection(xp["u"], xp["W"], xp["conv_w"], xp["gate_in"],  # noqa: E731
+                                        xp["gate_bias"], xp["A_log"], xp["beta_in"], dk, dv, E)
+    ms = _time_steps(call, 3, 3, stream, barrier, max_over_ranks)
+    flops = 2.0 * B * T * Dm * H * C
+    tf = flops / (ms / 1e3) / 1e12
+    out["projection"] = {"ms": round(ms, 4), "tflops": round(tf, 1),
+                         "peak_tflops": peaks["bf16_tflops"],
+                         "frac": round(tf / peaks["bf16_tflops"], 4),
+                         "bound": "tensor", "d_model": Dm, "channels_per_head": C,
+                         "algorithmic_flops": flops,
+                         "peak_source": "bf16 dense burst, " + peaks["source"],
+                         "what": "u W^T (bf16, fp32 accumulation) + causal conv K=4, SiLU/softplus, "
+                                 "L2 norms, log gates, beta in the epilogue; q,k,v,q',k' bf16 out"}
     return out
 
 

@@ -239,6 +239,38 @@ tla_status tla_layer_prologue_bwd(const tla_prologue_args *a, int grad_dtype, co
                                   size_t workspace_bytes, void *stream);
 
 /*
+ * Input projection of Algorithm 4 fused with the input path above (Appendix A, Input
+ * projections: one GEMM produces q, k, v, k', q' of every head, then one causal depthwise
+ * convolution processes them).  From the normalised layer input u:
+ *   P[b,t,h,c] = sum_i u[b,t,i] W[h*C + c, i]      (C = 2 dk + dv + 2 E, [q | k | v | q' | k'])
+ * on the tensor cores, then in the same kernel, per (b, t, h), the prologue of
+ * tla_layer_prologue on P (convolution of width K, SiLU / softplus, L2 normalisation, log
+ * gates from gate_in, beta from beta_in).  P is written only when P != NULL (the backward
+ * of the input path, tla_layer_prologue_bwd, takes it).
+ * Supported: dk, dv in {64, 128}, 1 <= E <= 16, 1 <= K <= 4, Dm a multiple of 64,
+ * bf16 u, W and outputs; all pointers 16-byte aligned.
+ */
+typedef struct {
+    int B, T, H, dk, dv, E;
+    int K;               /* convolution width, 1..4                                  */
+    int Dm;              /* model width (the GEMM's K dimension)                      */
+    float eps;           /* L2-normalisation epsilon                                  */
+    const void *u;       /* [B,T,Dm] bf16 layer input                                 */
+    const void *W;       /* [H*C, Dm] bf16 projection weight (output channel major)   */
+    const float *conv_w; /* [H,C,K]                                                   */
+    const float *gate_in;   /* [B,T,H,E]  W_alpha u                                   */
+    const float *gate_bias; /* [H,E]                                                  */
+    const float *A_log;     /* [H,E]                                                  */
+    const float *beta_in;   /* [B,T,H]  W_beta u, or NULL (then beta is NULL)         */
+    void *q, *k, *v, *q2, *k2;   /* [B,T,H,dk|dk|dv|E|E] bf16 (written)                */
+    float *g;            /* [B,T,H,E] (written)                                       */
+    float *beta;         /* [B,T,H] (written), NULL iff beta_in is NULL               */
+    void *P;             /* [B,T,H,C] bf16 projection output (written), or NULL       */
+} tla_projection_args;
+
+tla_status tla_layer_projection(const tla_projection_args *a, void *stream);
+
+/*
  * Output gate of Algorithm 4: per (b, t, h) over dv channels
  *   y = o / sqrt(mean(o^2) + eps) * w_norm * sigmoid(z).
  */

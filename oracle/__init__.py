@@ -126,6 +126,17 @@ def decode_step(state, q, k, v, q2, k2, g, beta=None, use_delta=True):
     return o, st
 
 
+def projection(u, W, H):
+    """Input projection of Algorithm 4 / Appendix A (Input projections): one GEMM of the
+    layer input u [B,T,Dm] with the weight W [H*C, Dm] (rows: head h's channels
+    [q|k|v|q'|k'] at h*C..h*C+C-1), P[b,t,h,c] = sum_i u[b,t,i] W[h*C+c, i], in float64
+    (the matrix product is the library primitive).  Returns P [B,T,H,C]."""
+    u, W = _f64(u), _f64(W)
+    B, T, Dm = u.shape
+    C = W.shape[0] // H
+    return (u.reshape(B * T, Dm) @ W.T).reshape(B, T, H, C)
+
+
 def prologue(P, conv_w, gate_in, gate_bias, A_log, beta_in, dk, dv, E, eps=1e-6):
     """Layer input path of Algorithm 4: causal depthwise convolution of the projection
     output P [B,T,H,2dk+dv+2E] (per head [q|k|v|q'|k']) with conv_w [H,C,K], SiLU on

@@ -10,6 +10,7 @@
 // partials reduced in a fixed order by a second kernel.
 #include <cuda_bf16.h>
 
+#include "act.cuh"
 #include "common.cuh"
 #include "internal.h"
 #include "sm100.cuh"
@@ -27,14 +28,6 @@ constexpr int kFwdRun = 128;   // tokens per CTA of the prologue forward
 constexpr int kSeg = 256;      // tokens per CTA of the prologue backward
 constexpr int kGateTile = 64;  // (token, head) rows per CTA of the output gate
 
-__device__ __forceinline__ float sigm(float x) { return __fdividef(1.f, 1.f + __expf(-x)); }
-// softplus(x) = log(1 + e^x) with fast intrinsics; for e^x < 2^-10 the series e (1 - e/2)
-// keeps the relative accuracy that log(1 + e) in fp32 would lose.
-__device__ __forceinline__ float softplus(float x) {
-    if (x > 20.f) return x;
-    const float e = __expf(x);
-    return e < 0.0009765625f ? e * fmaf(-0.5f, e, 1.f) : __logf(1.f + e);
-}
 
 template <typename T> __device__ __forceinline__ float ld(const void* p, size_t i) {
     return to_f(static_cast<const T*>(p)[i]);

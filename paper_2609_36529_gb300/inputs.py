@@ -162,6 +162,26 @@ def layer_inputs(B, T, H, dk, dv, E, K=4, dtype="bf16", device="cpu", seed=0):
             "w_norm": 1.0 + 0.1 * randn(dv)}
 
 
+def projection_inputs(B, T, H, dk, dv, E, Dm, K=4, device="cpu", seed=0):
+    """Inputs of the fused input projection (Algorithm 4): the normalised layer input
+    u ~ N(0,1) [B,T,Dm] and the projection weight W ~ N(0, 1/Dm) [H*(2dk+dv+2E), Dm], both
+    bf16, then the parameters of layer_inputs (conv_w, gate_in, gate_bias, A_log, beta_in;
+    fp32) from the same generator."""
+    dev = torch.device(device)
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(seed)
+    C = 2 * dk + dv + 2 * E
+
+    def randn(*shape):
+        return torch.randn(*shape, generator=gen, device=dev, dtype=torch.float32)
+
+    return {"u": randn(B, T, Dm).to(torch.bfloat16),
+            "W": (randn(H * C, Dm) / Dm ** 0.5).to(torch.bfloat16),
+            "conv_w": randn(H, C, K) / K ** 0.5, "gate_in": randn(B, T, H, E),
+            "gate_bias": randn(H, E) + 1.0, "A_log": 0.5 * randn(H, E) - 1.0,
+            "beta_in": randn(B, T, H)}
+
+
 def workload_inputs(w: Workload, device="cpu", seed=0, B=None, T=None, H=None):
     """Inputs of a named workload, optionally with a reduced B/T/H for tests."""
     return chunk_inputs(B or w.B, T or w.T, H or w.H, w.dk, w.dv, w.E, w.dtype, w.with_beta,

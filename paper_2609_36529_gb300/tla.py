@@ -24,7 +24,7 @@ EXPORTED = ("tla_fwd_workspace_bytes", "tla_chunk_fwd", "tla_bwd_workspace_bytes
             "tla_version", "tla_chunk_fwd_noalloc", "tla_noalloc_scratch_bytes",
             "tla_layer_prologue", "tla_layer_prologue_bwd_workspace_bytes",
             "tla_layer_prologue_bwd", "tla_output_gate", "tla_output_gate_bwd_workspace_bytes",
-            "tla_output_gate_bwd", "tla_selftest_bounded_wait")
+            "tla_output_gate_bwd", "tla_selftest_bounded_wait", "tla_layer_projection")
 
 
 class TlaError(RuntimeError):
@@ -54,6 +54,18 @@ class tla_prologue_args(ctypes.Structure):
                 ("beta_in", ctypes.c_void_p), ("q", ctypes.c_void_p), ("k", ctypes.c_void_p),
                 ("v", ctypes.c_void_p), ("q2", ctypes.c_void_p), ("k2", ctypes.c_void_p),
                 ("g", ctypes.c_void_p), ("beta", ctypes.c_void_p)]
+
+
+class tla_projection_args(ctypes.Structure):
+    _fields_ = [("B", ctypes.c_int), ("T", ctypes.c_int), ("H", ctypes.c_int),
+                ("dk", ctypes.c_int), ("dv", ctypes.c_int), ("E", ctypes.c_int),
+                ("K", ctypes.c_int), ("Dm", ctypes.c_int), ("eps", ctypes.c_float),
+                ("u", ctypes.c_void_p), ("W", ctypes.c_void_p), ("conv_w", ctypes.c_void_p),
+                ("gate_in", ctypes.c_void_p), ("gate_bias", ctypes.c_void_p),
+                ("A_log", ctypes.c_void_p), ("beta_in", ctypes.c_void_p),
+                ("q", ctypes.c_void_p), ("k", ctypes.c_void_p), ("v", ctypes.c_void_p),
+                ("q2", ctypes.c_void_p), ("k2", ctypes.c_void_p), ("g", ctypes.c_void_p),
+                ("beta", ctypes.c_void_p), ("P", ctypes.c_void_p)]
 
 
 class tla_gate_args(ctypes.Structure):
@@ -108,6 +120,8 @@ def lib():
         L.tla_output_gate_bwd_workspace_bytes.restype = sz
         L.tla_output_gate_bwd.argtypes = [GA, vp, vp, vp, vp, vp, sz, vp]
         L.tla_output_gate_bwd.restype = i
+        L.tla_layer_projection.argtypes = [ctypes.POINTER(tla_projection_args), vp]
+        L.tla_layer_projection.restype = i
         _lib = L
     return _lib
 
@@ -374,3 +388,36 @@ def output_gate_bwd(o, z, w_norm, dy, eps=1e-6):
         ctypes.byref(a), _ptr(dy), _ptr(out["do"]), _ptr(out["dz"]), _ptr(out["dw_norm"]),
         _ptr(ws), need, _stream()))
     return out
+
+
+# --- input projection GEMM fused with the input path (Algorithm 4)
+
+def layer_projection(u, W, conv_w, gate_in, gate_bias, A_log, beta_in, dk, dv, E, eps=1e-6,
+                     want_P=False):
+    """One tensor-core GEMM P = u W^T (u [B,T,Dm] bf16, W [H*C, Dm] bf16, C = 2dk+dv+2E,
+    per head [q|k|v|q'|k']) with the input path of layer_prologue applied in its epilogue.
+    Returns q, k, v, q2, k2 (bf16), g and beta (fp32), and P (bf16) when want_P."""
+    B, T, Dm = u.shape
+    H = conv_w.shape[0]
+    C = 2 * dk + dv + 2 * E
+    assert W.shape == (H * C, Dm), "W must be [H * (2 dk + dv + 2 E), Dm]"
+    dev, bf = u.device, torch.bfloat16
+    out = {"q": torch.empty(B, T, H, dk, dtype=bf, device=dev),
+           "k": torch.empty(B, T, H, dk, dtype=bf, device=dev),
+           "v": torch.empty(B, T, H, dv, dtype=bf, device=dev),
+           "q2": torch.empty(B, T, H, E, dtype=bf, device=dev),
+           "k2": torch.empty(B, T, H, E, dtype=bf, device=dev),
+           "g": torch.empty(B, T, H, E, dtype=torch.float32, device=dev),
+           "beta": torch.empty(B, T, H, dtype=torch.float32, device=dev)
+           if beta_in is not None else None,
+           "P": torch.empty(B, T, H, C, dtype=bf, device=dev) if want_P else None}
+    a = tla_projection_args()
+    a.B, a.T, a.H, a.dk, a.dv, a.E = B, T, H, dk, dv, E
+    a.K, a.Dm, a.eps = conv_w.shape[-1], Dm, float(eps)
+    for name, t in (("u", u), ("W", W), ("conv_w", conv_w), ("gate_in", gate_in),
+                    ("gate_bias", gate_bias), ("A_log", A_log), ("beta_in", beta_in)):
+        setattr(a, name, _ptr(t))
+    for name in ("q", "k", "v", "q2", "k2", "g", "beta", "P"):
+        setattr(a, name, _ptr(out[name]))
+    _check("tla_layer_projection", lib().tla_layer_projection(ctypes.byref(a), _stream()))
+    return {n: t for n, t in out.items() if t is not None}

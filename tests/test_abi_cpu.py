@@ -197,3 +197,25 @@ def test_selftest_limit_checked_on_host(tla):
     L = tla.lib()
     for bad in (0, 1_000_000_001, 2 ** 63):
         assert L.tla_selftest_bounded_wait(bad, None) == -1
+
+
+def test_projection_validation(tla):
+    """Fused input projection (Algorithm 4): argument checks before any launch."""
+    L = tla.lib()
+    f = ctypes.c_void_p(0x1000)
+
+    def args(**kw):
+        a = tla.tla_projection_args()
+        a.B, a.T, a.H, a.dk, a.dv, a.E, a.K, a.Dm, a.eps = 2, 100, 3, 128, 128, 4, 4, 256, 1e-6
+        for n in ("u", "W", "conv_w", "gate_in", "gate_bias", "A_log", "q", "k", "v", "q2", "k2",
+                  "g"):
+            setattr(a, n, f)
+        for n, v in kw.items():
+            setattr(a, n, v)
+        return a
+
+    cases = [(dict(dk=96), -2), (dict(dv=32), -2), (dict(E=17), -2), (dict(Dm=100), -2),
+             (dict(K=5), -1), (dict(K=0), -1), (dict(eps=0.0), -1), (dict(u=None), -1),
+             (dict(beta_in=f), -1), (dict(q=ctypes.c_void_p(0x1004)), -1), (dict(T=0), -1)]
+    for kw, want in cases:
+        assert L.tla_layer_projection(ctypes.byref(args(**kw)), None) == want, kw

@@ -391,3 +391,23 @@ def test_output_gate_matches_library_form_and_autograd():
     got = oracle.gate_norm_backward(o, z, w, dy)
     for gname, t in (("do", to), ("dz", tz), ("dw_norm", tw)):
         np.testing.assert_allclose(got[gname], t.grad.numpy(), rtol=1e-9, atol=1e-10, err_msg=gname)
+
+
+def test_projection_is_the_per_channel_sum():
+    """Input projection of Algorithm 4 (Appendix A, Input projections): every entry of
+    P[b,t,h,c] is the explicit sum over the model width of u[b,t,i] W[h C + c, i], head h's
+    rows of W in the order [q|k|v|q'|k'] (brute force on a tiny case)."""
+    rng = np.random.default_rng(3)
+    B, T, H, C, Dm = 2, 3, 2, 5, 7
+    u = rng.standard_normal((B, T, Dm))
+    W = rng.standard_normal((H * C, Dm))
+    P = oracle.projection(u, W, H)
+    assert P.shape == (B, T, H, C)
+    for b in range(B):
+        for t in range(T):
+            for h in range(H):
+                for c in range(C):
+                    ref = 0.0
+                    for i in range(Dm):
+                        ref += u[b, t, i] * W[h * C + c, i]
+                    assert abs(P[b, t, h, c] - ref) <= 1e-12 * (1 + abs(ref))
