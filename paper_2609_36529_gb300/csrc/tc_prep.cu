@@ -106,14 +106,25 @@ chunk_prep_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             tma_load_4d(sKQ + j * 2 * kBoxBytes + kBoxBytes, &map_q, &bar_ld, 64 * j, h, t0, b);
         }
     }
-    for (int i = tid; i < 64 * E; i += kThreads) {
-        const int r = i / E, e = i - (i / E) * E;
-        const int rr = r < n ? r : n - 1;
-        Gs[i] = p.G[tok_idx(b, t0 + rr, h, e, T, H, E)];
-        k2s[i] = r < n ? __bfloat162float(p.k2[tok_idx(b, t0 + r, h, e, T, H, E)]) : 0.f;
-        q2s[i] = r < n ? __bfloat162float(p.q2[tok_idx(b, t0 + r, h, e, T, H, E)]) : 0.f;
+    // the chunk's log decays, second keys and queries and beta: loaded into registers now
+    // (token-major, E values of a token side by side), so that their latency overlaps the
+    // key/query copies and the Gram product; stored slice-major ([E][64]) after it
+    float gv[4], kv[4], qv[4], bv = 0.f;
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {   // 64 E <= 1024 values: at most four per thread
+        const int i = tid + u * kThreads;
+        gv[u] = kv[u] = qv[u] = 0.f;
+        if (i < 64 * E) {
+            const int r = i / E, e = i - (i / E) * E;
+            const int rr = r < n ? r : n - 1;
+            gv[u] = p.G[tok_idx(b, t0 + rr, h, e, T, H, E)];
+            if (r < n) {
+                kv[u] = __bfloat162float(p.k2[tok_idx(b, t0 + r, h, e, T, H, E)]);
+                qv[u] = __bfloat162float(p.q2[tok_idx(b, t0 + r, h, e, T, H, E)]);
+            }
+        }
     }
-    if (tid < 64) bs[tid] = tid < n ? (p.beta ? p.beta[(size_t(b) * T + t0 + tid) * H + h] : 1.f) : 0.f;
+    if (tid < 64) bv = tid < n ? (p.beta ? p.beta[(size_t(b) * T + t0 + tid) * H + h] : 1.f) : 0.f;
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -158,6 +169,17 @@ chunk_prep_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             for (int q = 0; q < 4; ++q) st4(dst + j + 4 * q, v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
         }
     }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+        const int i = tid + u * kThreads;
+        if (i < 64 * E) {
+            const int r = i / E, e = i - (i / E) * E;
+            Gs[e * 64 + r] = gv[u];
+            k2s[e * 64 + r] = kv[u];
+            q2s[e * 64 + r] = qv[u];
+        }
+    }
+    if (tid < 64) bs[tid] = bv;
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -180,15 +202,15 @@ chunk_prep_tc_kernel(const __grid_constant__ CUtensorMap map_k,
 #pragma unroll
             for (int c2 = 0; c2 < 4; ++c2) R[a][c2] = Rq[a][c2] = 0.f;
         for (int e = 0; e < E; ++e) {
-            float gs[4], ks[4];
-#pragma unroll
-            for (int c2 = 0; c2 < 4; ++c2) {
-                gs[c2] = Gs[(S0 + c2) * E + e];
-                ks[c2] = k2s[(S0 + c2) * E + e];
-            }
+            float gs[4], ks[4], grv[4], krv[4], qrv[4];
+            ld4(Gs + e * 64 + S0, gs);
+            ld4(k2s + e * 64 + S0, ks);
+            ld4(Gs + e * 64 + R0, grv);
+            ld4(k2s + e * 64 + R0, krv);
+            ld4(q2s + e * 64 + R0, qrv);
 #pragma unroll
             for (int a = 0; a < 4; ++a) {
-                const float gr = Gs[(R0 + a) * E + e], kr = k2s[(R0 + a) * E + e], qr = q2s[(R0 + a) * E + e];
+                const float gr = grv[a], kr = krv[a], qr = qrv[a];
 #pragma unroll
                 for (int c2 = 0; c2 < 4; ++c2) {
                     // exp of a non-positive log-decay difference (Eq. joint-gram); the
@@ -334,34 +356,46 @@ chunk_prep_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                 for (int c2 = 0; c2 < 4; ++c2) ATv[a][c2] = fmaf(av[a], tv[c2], ATv[a][c2]);
         }
     }
-    const size_t m2 = ((size_t(b) * H + h) * NT + c) * (4 * 64 * 64);
-    __nv_bfloat16* A2 = p.A2out + m2;   // [T ; A T] hi (128 x 64), then lo
+    __syncthreads();   // every matrix slot is free from here
+    // images of the two tile blocks in their global layout (bf16 row-major 64-wide rows):
+    // [T; A T] hi (128 x 64) then lo, and [A^T hi, A^T lo, T^T hi, T^T lo] (64 x 64 each),
+    // built in slots 0-3 and written by two bulk copies
+    __nv_bfloat16* stA2 = reinterpret_cast<__nv_bfloat16*>(sm);
+    __nv_bfloat16* stBT = stA2 + 4 * 64 * 64;
 #pragma unroll
     for (int a = 0; a < 4; ++a) {
         const int o = (R0 + a) * 64 + S0;
-        put4(A2 + o, A2 + 8192 + o, Tv[a][0], Tv[a][1], Tv[a][2], Tv[a][3]);
-        put4(A2 + 4096 + o, A2 + 12288 + o, ATv[a][0], ATv[a][1], ATv[a][2], ATv[a][3]);
+        put4(stA2 + o, stA2 + 8192 + o, Tv[a][0], Tv[a][1], Tv[a][2], Tv[a][3]);
+        put4(stA2 + 4096 + o, stA2 + 12288 + o, ATv[a][0], ATv[a][1], ATv[a][2], ATv[a][3]);
     }
-    if (p.BTout) {   // [A^T hi, A^T lo, T^T hi, T^T lo], 64 x 64 each
-        __nv_bfloat16* BT = p.BTout + m2;
+    if (p.BTout) {
 #pragma unroll
         for (int c2 = 0; c2 < 4; ++c2) {
             const int o = (S0 + c2) * 64 + R0;
-            put4(BT + o, BT + 4096 + o, Av[0][c2], Av[1][c2], Av[2][c2], Av[3][c2]);
-            put4(BT + 8192 + o, BT + 12288 + o, Tv[0][c2], Tv[1][c2], Tv[2][c2], Tv[3][c2]);
+            put4(stBT + o, stBT + 4096 + o, Av[0][c2], Av[1][c2], Av[2][c2], Av[3][c2]);
+            put4(stBT + 8192 + o, stBT + 12288 + o, Tv[0][c2], Tv[1][c2], Tv[2][c2], Tv[3][c2]);
         }
+    }
+    fence_proxy_async_smem();
+    __syncthreads();
+    const size_t m2 = ((size_t(b) * H + h) * NT + c) * (4 * 64 * 64);
+    if (tid == 0) {
+        bulk_store(p.A2out + m2, stA2, 4 * 64 * 64 * 2);
+        if (p.BTout) bulk_store(p.BTout + m2, stBT, 4 * 64 * 64 * 2);
+        bulk_commit();
     }
     // coefficient block, slice-major: [a | b | w] each [E][64 rows], then gamma^C_e
     float* cf = p.coef + ((size_t(b) * H + h) * NT + c) * (3 * 64 * E + 16);
     for (int i = tid; i < 64 * E; i += kThreads) {
-        const int e = i >> 6, r = i & 63, ir = r * E + e;
-        const float Gr = Gs[ir], GC = Gs[(n - 1) * E + e];
+        const int e = i >> 6;
+        const float Gr = Gs[i], GC = Gs[e * 64 + n - 1];
         const float gam = __expf(Gr);
-        cf[i] = k2s[ir] * gam;
-        cf[64 * E + i] = q2s[ir] * gam;
-        cf[128 * E + i] = k2s[ir] * __expf(GC - Gr);
+        cf[i] = k2s[i] * gam;
+        cf[64 * E + i] = q2s[i] * gam;
+        cf[128 * E + i] = k2s[i] * __expf(GC - Gr);
     }
-    if (tid < 16) cf[192 * E + tid] = tid < E ? __expf(Gs[(n - 1) * E + tid]) : 0.f;
+    if (tid < 16) cf[192 * E + tid] = tid < E ? __expf(Gs[tid * 64 + n - 1]) : 0.f;
+    if (tid == 0) bulk_wait_read_all();   // the images stay in shared memory until read
 }
 
 size_t prep_tc_smem(int E) { return 1024 + size_t(5) * kSlot * 4 + (3 * 64 * E + 64) * 4; }
