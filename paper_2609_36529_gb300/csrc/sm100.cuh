@@ -198,6 +198,10 @@ __device__ __forceinline__ uint64_t smem_desc(uint32_t saddr, uint32_t lbo, uint
            (uint64_t((sbo >> 4) & 0x3FFF) << 32) | (uint64_t(1) << 46) | (swizzle << 61);
 }
 
+// The descriptor d with its start address advanced by byte_off bytes (a multiple of 16 that
+// keeps the address within the 256 KB the 14-bit field encodes).
+__device__ __forceinline__ uint64_t desc_add(uint64_t d, uint32_t byte_off) { return d + (byte_off >> 4); }
+
 // Instruction descriptor of kind::f16: D fp32 (bits 4-5 = 1), A and B bf16
 // (bits 7-9 = 1, 10-12 = 1), A/B major (bit 15/16: 0 = K-major, 1 = MN-major),
 // N >> 3 in bits 17-22, M >> 4 in bits 24-28.

@@ -281,21 +281,26 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         // ---- MMA-A' (P' = K dS') and MMA-0 (Y = A^T dO)
         if (tid == 0) {
             const uint32_t ida = idesc_bf16_f32(64, NE, 0, 1);
+            // descriptors built once; each K step advances their start addresses
+            const uint64_t a0 = smem_desc(smem_u32(sKQ), 16, 1024);
+            const uint64_t dh0 = smem_desc(smem_u32(sDh), blk_bytes<TV>(), 16 * TV, kSwz);
+            const uint64_t dl0 = smem_desc(smem_u32(sDl), blk_bytes<TV>(), 16 * TV, kSwz);
 #pragma unroll
             for (int ks = 0; ks < kDk / 16; ++ks) {
                 const int blk = ks >> 2, kk = (ks & 3) * 16;
-                const uint64_t ad = smem_desc(smem_u32(sKQ) + blk * 2 * kBoxBytes + kk * 2, 16, 1024);
+                const uint64_t ad = desc_add(a0, blk * 2 * kBoxBytes + kk * 2);
                 const uint32_t ko = ks * 32 * TV;   // 16 rows of the slice blocks per K step
-                umma_bf16(tP, ad, smem_desc(smem_u32(sDh) + ko, blk_bytes<TV>(), 16 * TV, kSwz), ida,
-                          ks > 0 ? 1u : 0u);
-                umma_bf16(tP, ad, smem_desc(smem_u32(sDl) + ko, blk_bytes<TV>(), 16 * TV, kSwz), ida, 1u);
+                umma_bf16(tP, ad, desc_add(dh0, ko), ida, ks > 0 ? 1u : 0u);
+                umma_bf16(tP, ad, desc_add(dl0, ko), ida, 1u);
             }
             const uint32_t id0 = idesc_bf16_f32(64, TV, 0, 1);
+            const uint64_t o0 = smem_desc(smem_u32(sdO), blk_bytes<TV>(), 16 * TV, kSwz);
+            const uint64_t t0d = smem_desc(smem_u32(sBT), 16, 1024);
 #pragma unroll
             for (int ks = 0; ks < 4; ++ks) {
-                const uint64_t bd = smem_desc(smem_u32(sdO) + ks * 32 * TV, blk_bytes<TV>(), 16 * TV, kSwz);
-                umma_bf16(tY, smem_desc(smem_u32(sBT) + ks * 32, 16, 1024), bd, id0, ks > 0 ? 1u : 0u);
-                umma_bf16(tY, smem_desc(smem_u32(sBT) + kBoxBytes + ks * 32, 16, 1024), bd, id0, 1u);
+                const uint64_t bd = desc_add(o0, ks * 32 * TV);
+                umma_bf16(tY, desc_add(t0d, ks * 32), bd, id0, ks > 0 ? 1u : 0u);
+                umma_bf16(tY, desc_add(t0d, kBoxBytes + ks * 32), bd, id0, 1u);
             }
             umma_commit(&bar_mma);
             issue_ckpt(c);   // the dS' blocks were completed before the last barrier
@@ -358,13 +363,15 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         // ---- MMA-B': dRes = T^T dU   (into tY; dU MN-major)
         if (tid == 0) {
             const uint32_t idb = idesc_bf16_f32(64, TV, 0, 1);
+            const uint64_t t0d = smem_desc(smem_u32(sBT), 16, 1024);
+            const uint64_t u0 = smem_desc(smem_u32(sUh), blk_bytes<TV>(), 16 * TV, kSwz);
 #pragma unroll
             for (int ks = 0; ks < 4; ++ks) {
-                const uint64_t th = smem_desc(smem_u32(sBT) + 2 * kBoxBytes + ks * 32, 16, 1024);
-                const uint64_t tl = smem_desc(smem_u32(sBT) + 3 * kBoxBytes + ks * 32, 16, 1024);
+                const uint64_t th = desc_add(t0d, 2 * kBoxBytes + ks * 32);
+                const uint64_t tl = desc_add(t0d, 3 * kBoxBytes + ks * 32);
                 const uint32_t ko = ks * 32 * TV;
-                const uint64_t uh = smem_desc(smem_u32(sUh) + ko, blk_bytes<TV>(), 16 * TV, kSwz);
-                const uint64_t ul = smem_desc(smem_u32(sUl) + ko, blk_bytes<TV>(), 16 * TV, kSwz);
+                const uint64_t uh = desc_add(u0, ko);
+                const uint64_t ul = desc_add(u0, TV * 128 + ko);   // sUl = sUh + TV * 128
                 umma_bf16(tY, th, uh, idb, ks > 0 ? 1u : 0u);
                 umma_bf16(tY, th, ul, idb, 1u);
                 umma_bf16(tY, tl, uh, idb, 1u);
@@ -435,10 +442,13 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         // ---- MMA-C': dS += [K^T | Q^T] [-a dRes ; b dO]   (sGLA: query half only)
         if (tid == 0) {
             const uint32_t idc = idesc_bf16_f32(128, NE, 1, 1);
+            const uint64_t a0 = smem_desc(smem_u32(sKQ), 2 * kBoxBytes, 1024);
+            const uint64_t bh0 = smem_desc(smem_u32(sBh), 128 * 128, 1024);
+            const uint64_t bl0 = smem_desc(smem_u32(sBl), 128 * 128, 1024);
             for (int ks = p.use_delta ? 0 : 4; ks < 8; ++ks) {
-                const uint64_t ad = smem_desc(smem_u32(sKQ) + ks * 2048, 2 * kBoxBytes, 1024);
-                umma_bf16(tS, ad, smem_desc(smem_u32(sBh) + ks * 2048, 128 * 128, 1024), idc, 1u);
-                umma_bf16(tS, ad, smem_desc(smem_u32(sBl) + ks * 2048, 128 * 128, 1024), idc, 1u);
+                const uint64_t ad = desc_add(a0, ks * 2048);
+                umma_bf16(tS, ad, desc_add(bh0, ks * 2048), idc, 1u);
+                umma_bf16(tS, ad, desc_add(bl0, ks * 2048), idc, 1u);
             }
             umma_commit(&bar_mma);
             if (tma_dv) {   // rows past T are skipped by the store

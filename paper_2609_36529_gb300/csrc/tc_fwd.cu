@@ -254,16 +254,19 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     // MMA-A: P = [K; Q] S_all    (B = S_all, MN-major, hi and lo)
     auto issue_mma_a = [&]() {
         const uint32_t idesc = idesc_bf16_f32(128, NE, 0, 1);
+        // descriptors built once; each K step advances their start addresses
+        const uint64_t a0 = smem_desc(smem_u32(sKQ), 16, 1024);
+        const uint64_t bh0 = smem_desc(smem_u32(sSh), blk_bytes<TV>(), 16 * TV, kSwz);
+        const uint64_t bl0 = smem_desc(smem_u32(sSl), blk_bytes<TV>(), 16 * TV, kSwz);
 #pragma unroll
         for (int ks = 0; ks < kDk / 16; ++ks) {
             const int blk = ks >> 2, kk = (ks & 3) * 16;
-            const uint64_t ad = smem_desc(smem_u32(sKQ) + blk * 2 * kBoxBytes + kk * 2, 16, 1024);
+            const uint64_t ad = desc_add(a0, blk * 2 * kBoxBytes + kk * 2);
             // B = the slice blocks: 16 rows (two 8-row groups) per K step, one TV-column
             // swizzle atom per slice
             const uint32_t ko = ks * 32 * TV;
-            umma_bf16(tP, ad, smem_desc(smem_u32(sSh) + ko, blk_bytes<TV>(), 16 * TV, kSwz), idesc,
-                      ks > 0 ? 1u : 0u);
-            umma_bf16(tP, ad, smem_desc(smem_u32(sSl) + ko, blk_bytes<TV>(), 16 * TV, kSwz), idesc, 1u);
+            umma_bf16(tP, ad, desc_add(bh0, ko), idesc, ks > 0 ? 1u : 0u);
+            umma_bf16(tP, ad, desc_add(bl0, ko), idesc, 1u);
         }
         umma_commit(&bar_mma);
     };
@@ -381,13 +384,15 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         // ---- MMA-B: [U; Oa] = [T; A T] Res  (into columns [0, TV); Res MN-major)
         if (tid == 0) {
             const uint32_t idesc = idesc_bf16_f32(128, TV, 0, 1);
+            const uint64_t ah0 = smem_desc(smem_u32(sA2), 16, 1024);
+            const uint64_t bh0 = smem_desc(smem_u32(sRh), blk_bytes<TV>(), 16 * TV, kSwz);
 #pragma unroll
             for (int ks = 0; ks < 4; ++ks) {
-                const uint64_t ah = smem_desc(smem_u32(sA2) + ks * 32, 16, 1024);
-                const uint64_t al = smem_desc(smem_u32(sA2) + 2 * kBoxBytes + ks * 32, 16, 1024);
+                const uint64_t ah = desc_add(ah0, ks * 32);
+                const uint64_t al = desc_add(ah0, 2 * kBoxBytes + ks * 32);
                 const uint32_t ko = ks * 32 * TV;
-                const uint64_t bh = smem_desc(smem_u32(sRh) + ko, blk_bytes<TV>(), 16 * TV, kSwz);
-                const uint64_t bl = smem_desc(smem_u32(sRl) + ko, blk_bytes<TV>(), 16 * TV, kSwz);
+                const uint64_t bh = desc_add(bh0, ko);
+                const uint64_t bl = desc_add(bh0, TV * 128 + ko);   // sRl = sRh + TV * 128
                 umma_bf16(tP, ah, bh, idesc, ks > 0 ? 1u : 0u);
                 umma_bf16(tP, ah, bl, idesc, 1u);
                 umma_bf16(tP, al, bh, idesc, 1u);
@@ -441,11 +446,14 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         // ---- MMA-C: S_all += K^T Ut   (A = K^T MN-major from the key rows; B = Ut MN-major)
         if (tid == 0) {
             const uint32_t idesc = idesc_bf16_f32(128, NE, 1, 1);
+            const uint64_t a0 = smem_desc(smem_u32(sKQ), 2 * kBoxBytes, 1024);
+            const uint64_t uh0 = smem_desc(smem_u32(sUh), 64 * 128, 1024);
+            const uint64_t ul0 = smem_desc(smem_u32(sUl), 64 * 128, 1024);
 #pragma unroll
             for (int ks = 0; ks < 4; ++ks) {
-                const uint64_t ad = smem_desc(smem_u32(sKQ) + ks * 2048, 2 * kBoxBytes, 1024);
-                umma_bf16(tS, ad, smem_desc(smem_u32(sUh) + ks * 2048, 64 * 128, 1024), idesc, 1u);
-                umma_bf16(tS, ad, smem_desc(smem_u32(sUl) + ks * 2048, 64 * 128, 1024), idesc, 1u);
+                const uint64_t ad = desc_add(a0, ks * 2048);
+                umma_bf16(tS, ad, desc_add(uh0, ks * 2048), idesc, 1u);
+                umma_bf16(tS, ad, desc_add(ul0, ks * 2048), idesc, 1u);
             }
             umma_commit(&bar_mma);
             if (tma_o) {   // rows past T are skipped by the store
