@@ -40,6 +40,8 @@ constexpr int kNBytes = 64 * 64 * 4;       // one C x C fp32 matrix in global me
 constexpr int MP = 68;                     // row stride (floats) of the shared C x C matrices
 constexpr int kMat = 64 * MP;              // floats per shared C x C matrix
 constexpr uint32_t kWorkBytes = 131072;    // [K;Q] tiles + phase 0/1 scratch; later two slabs
+constexpr int GP = 68;                     // slice stride of the per-token arrays [E][GP] (float4
+                                           // aligned, and slices fall on different banks)
 
 struct TcGradArgs {
     const __nv_bfloat16* q2;
@@ -115,6 +117,14 @@ __device__ __forceinline__ void load_bf16x8(const uint8_t* src, float* v) {
     }
 }
 
+// Four consecutive bf16 values (8-byte aligned) as fp32.
+__device__ __forceinline__ void load_bf16x4(const __nv_bfloat16* src, float* v) {
+    const uint2 u = *reinterpret_cast<const uint2*>(src);
+    const float2 lo = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.x));
+    const float2 hi = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.y));
+    v[0] = lo.x; v[1] = lo.y; v[2] = hi.x; v[3] = hi.y;
+}
+
 // One halving step of a warp transpose-reduction over 2S values per lane.
 template <int S>
 __device__ __forceinline__ void xreduce_step(float* v, int lane) {
@@ -174,10 +184,11 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     uint8_t* W = sUl + T64;                    // 128 KB work region
     uint8_t* sKQ = W;                          // [K rows | Q rows] per 64-column block (TMA)
     uint8_t* scr = W + 4 * kBoxBytes;          // 96 KB: phase 0 staging, six C x C matrices, A3
+    // per-token log decays, second keys and queries of the chunk, slice-major [E][GP]
     float* Gs = reinterpret_cast<float*>(W + kWorkBytes);
-    __nv_bfloat16* k2s = reinterpret_cast<__nv_bfloat16*>(Gs + 64 * E);
-    __nv_bfloat16* q2s = k2s + 64 * E;
-    float* dk2a = reinterpret_cast<float*>(q2s + 64 * E);
+    __nv_bfloat16* k2s = reinterpret_cast<__nv_bfloat16*>(Gs + GP * E);
+    __nv_bfloat16* q2s = k2s + GP * E;
+    float* dk2a = reinterpret_cast<float*>(q2s + GP * E);
     float* dq2a = dk2a + 64 * E;
     float* dGa = dq2a + 64 * E;
     float* dwk = dGa + 64 * E;
@@ -234,9 +245,9 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     for (int i = tid; i < 64 * E; i += kThreads) {
         const int r = i / E, e = i - (i / E) * E;
         const int rr = r < n ? r : n - 1;
-        Gs[i] = p.G[tok_idx(b, t0 + rr, h, e, T, H, E)];
-        k2s[i] = r < n ? p.k2[tok_idx(b, t0 + r, h, e, T, H, E)] : __float2bfloat16_rn(0.f);
-        q2s[i] = r < n ? p.q2[tok_idx(b, t0 + r, h, e, T, H, E)] : __float2bfloat16_rn(0.f);
+        Gs[e * GP + r] = p.G[tok_idx(b, t0 + rr, h, e, T, H, E)];
+        k2s[e * GP + r] = r < n ? p.k2[tok_idx(b, t0 + r, h, e, T, H, E)] : __float2bfloat16_rn(0.f);
+        q2s[e * GP + r] = r < n ? p.q2[tok_idx(b, t0 + r, h, e, T, H, E)] : __float2bfloat16_rn(0.f);
     }
     if (tid < 64) {
         bs[tid] = tid < n ? (p.beta ? p.beta[(size_t(b) * T + t0 + tid) * H + h] : 1.f) : 0.f;
@@ -384,17 +395,21 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
 #pragma unroll
         for (int c2 = 0; c2 < 4; ++c2) Rv[a][c2] = Rq[a][c2] = 0.f;
     for (int e = 0; e < E; ++e) {
-        float gs[4], ksv[4];
-#pragma unroll
-        for (int c2 = 0; c2 < 4; ++c2) {
-            gs[c2] = Gs[(S0 + c2) * E + e];
-            ksv[c2] = __bfloat162float(k2s[(S0 + c2) * E + e]);
+        float gs[4], ksv[4], grv[4], krv[4], qrv[4];
+        {   // four consecutive tokens of slice e: one 16-byte / 8-byte load each
+            const float4 g4 = *reinterpret_cast<const float4*>(Gs + e * GP + S0);
+            const float4 h4 = *reinterpret_cast<const float4*>(Gs + e * GP + R0);
+            gs[0] = g4.x; gs[1] = g4.y; gs[2] = g4.z; gs[3] = g4.w;
+            grv[0] = h4.x; grv[1] = h4.y; grv[2] = h4.z; grv[3] = h4.w;
+            load_bf16x4(k2s + e * GP + S0, ksv);
+            load_bf16x4(k2s + e * GP + R0, krv);
+            load_bf16x4(q2s + e * GP + R0, qrv);
         }
 #pragma unroll
         for (int a = 0; a < 4; ++a) {
-            const float gr = Gs[(R0 + a) * E + e];
-            const float kr = __bfloat162float(k2s[(R0 + a) * E + e]);
-            const float qr = __bfloat162float(q2s[(R0 + a) * E + e]);
+            const float gr = grv[a];
+            const float kr = krv[a];
+            const float qr = qrv[a];
 #pragma unroll
             for (int c2 = 0; c2 < 4; ++c2) {
                 // exp of a non-positive difference (entries above the diagonal are discarded)
@@ -506,13 +521,13 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         const float* dRqm = Fm;
         for (int i = tid; i < 64 * E; i += kThreads) {
             const int x = i / E, e = i - (i / E) * E;
-            const float gx = Gs[x * E + e];
-            const float kx = __bfloat162float(k2s[x * E + e]), qx = __bfloat162float(q2s[x * E + e]);
+            const float gx = Gs[e * GP + x];
+            const float kx = __bfloat162float(k2s[e * GP + x]), qx = __bfloat162float(q2s[e * GP + x]);
             float dk2v = 0.f, dq2v = 0.f, dGv = 0.f;
 #pragma unroll 4
             for (int s = 0; s <= x; ++s) {
-                const float gam = __expf(gx - Gs[s * E + e]);
-                const float ks = __bfloat162float(k2s[s * E + e]);
+                const float gam = __expf(gx - Gs[e * GP + s]);
+                const float ks = __bfloat162float(k2s[e * GP + s]);
                 const float dR = dRm[x * MP + s], dRq = dRqm[x * MP + s];
                 dk2v = fmaf(dR * ks, gam, dk2v);
                 dq2v = fmaf(dRq * ks, gam, dq2v);
@@ -520,10 +535,10 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             }
 #pragma unroll 4
             for (int r = x; r < 64; ++r) {
-                const float gam = __expf(Gs[r * E + e] - gx);
+                const float gam = __expf(Gs[e * GP + r] - gx);
                 const float dR = dRm[r * MP + x], dRq = dRqm[r * MP + x];
-                const float t = (dR * __bfloat162float(k2s[r * E + e]) +
-                                 dRq * __bfloat162float(q2s[r * E + e])) * gam;
+                const float t = (dR * __bfloat162float(k2s[e * GP + r]) +
+                                 dRq * __bfloat162float(q2s[e * GP + r])) * gam;
                 dk2v += t;
                 dGv = fmaf(-t, kx, dGv);
             }
@@ -646,11 +661,11 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         tc_fence_after();
         if (act) {
             if (tid < 192) {   // b_e, a_e, w_e of the 64 tokens
-                const int r = tid & 63, i = r * E + e;
+                const int r = tid & 63, i = e * GP + r;
                 float sv;
                 if (tid < 64) sv = __bfloat162float(q2s[i]) * __expf(Gs[i]);
                 else if (tid < 128) sv = __bfloat162float(k2s[i]) * __expf(Gs[i]);
-                else sv = __bfloat162float(k2s[i]) * __expf(Gs[(n - 1) * E + e] - Gs[i]);
+                else sv = __bfloat162float(k2s[i]) * __expf(Gs[e * GP + n - 1] - Gs[i]);
                 scl[pb * 192 + tid] = sv;
             }
             if (warp == 0) {
@@ -762,7 +777,7 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         if (e > 0) {   // slice e-1's row dots -> dq2, dk2, dG (a_e = k2 gamma, b_e = q2 gamma, w_e)
             const int es = e - 1;
             if (tid < 64) {
-                const int i = tid * E + es;
+                const int i = tid * E + es, ig = es * GP + tid;
                 float db = 0.f, da = 0.f, dw = 0.f;
 #pragma unroll
                 for (int q = 0; q < 4; ++q) {
@@ -770,9 +785,9 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                     da += red[(1 * 4 + q) * 64 + tid];
                     dw += red[(2 * 4 + q) * 64 + tid];
                 }
-                const float gam = __expf(Gs[i]);
-                const float wdec = __expf(Gs[(n - 1) * E + es] - Gs[i]);
-                const float k2v = __bfloat162float(k2s[i]), q2v = __bfloat162float(q2s[i]);
+                const float gam = __expf(Gs[ig]);
+                const float wdec = __expf(Gs[es * GP + n - 1] - Gs[ig]);
+                const float k2v = __bfloat162float(k2s[ig]), q2v = __bfloat162float(q2s[ig]);
                 dk2a[i] += da * gam + dw * wdec;
                 dq2a[i] += db * gam;
                 dGa[i] += da * (k2v * gam) + db * (q2v * gam) - dw * (k2v * wdec);
@@ -821,10 +836,10 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     __syncthreads();
     if (warp < E) {   // one warp per slice: dgamma^C, then the reverse cumulative sum of dG
         const int e = warp;
-        const float gl = Gs[(n - 1) * E + e];
+        const float gl = Gs[e * GP + n - 1];
         float dGC = 0.f;
         for (int r = lane; r < n; r += 32)
-            dGC = fmaf(dwk[r * E + e], __bfloat162float(k2s[r * E + e]) * __expf(gl - Gs[r * E + e]), dGC);
+            dGC = fmaf(dwk[r * E + e], __bfloat162float(k2s[e * GP + r]) * __expf(gl - Gs[e * GP + r]), dGC);
 #pragma unroll
         for (int s = 16; s >= 1; s >>= 1) dGC += __shfl_xor_sync(0xffffffffu, dGC, s);
         dGC = fmaf(dgc[e], __expf(gl), dGC);
@@ -859,7 +874,8 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
 
 size_t grads_tc_smem(int E, int dv) {
     const size_t T64 = size_t(64) * dv * 2;
-    const size_t small = size_t(64) * E * (4 + 2 + 2 + 4 * 4) + (64 + 64 + 16 + 384 + 768 + 16) * 4;
+    const size_t small = size_t(GP) * E * (4 + 2 + 2) + size_t(64) * E * 4 * 4 +
+                         (64 + 64 + 16 + 384 + 768 + 16) * 4;
     return 1024 + 5 * T64 + kWorkBytes + small;   // small: Gs, k2s, q2s, dk2a, dq2a, dGa, dwk, bs, dba, dgc, scl, red, frw
 }
 
