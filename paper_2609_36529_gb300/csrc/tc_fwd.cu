@@ -6,10 +6,13 @@
 // C = 64 positions, with a_e = k'_e (.) gamma_e, b_e = q'_e (.) gamma_e and
 // w_e = k'_e (.) gamma^C_e / gamma_e (precomputed per chunk by the prep kernel):
 //   MMA-A  P  = [K; Q] S_all          (M=128 rows: 64 key rows, 64 query rows;
-//                                      N = NE = E*TV columns, slice-major; K = dk)
+//                                      N = NE = E*TV columns, slice-major; K = dk; the hi
+//                                      and lo halves of S side by side, N = 2 NE, when
+//                                      that fits one instruction)
 //   epi-A  Res = V - sum_e diag(a_e) P_K,e   (delta rule; sGLA: Res = V)
 //          Oi  = sum_e diag(b_e) P_Q,e       (kept in registers)
-//   MMA-B  [U; Oa] = [T; A T] Res      (M=128, K=64, N=TV; T and A T from the prep kernel)
+//   MMA-B  [U; Oa] = [T; A T] Res      (M=128, K=64; T and A T from the prep kernel; the
+//                                      hi*hi and hi*lo terms in one N = 2 TV product)
 //   epi-B  O = Oi + Oa;  Ut_e = diag(w_e) U
 //   MMA-C  S_all += K^T [Ut_1 .. Ut_E] (M=dk=128, K=64, N=NE; K^T read MN-major
 //                                      straight from the TMA-loaded key tile)
@@ -120,7 +123,11 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     const int nb = blockIdx.x, h = blockIdx.y, sb = blockIdx.z;   // sb: sequence or document
     const int n0 = nb * TV;
     const int T = p.T, H = p.H, dv = p.dv, NT = p.NT;
-    constexpr uint32_t tcols = (2 * NE <= 256) ? 256u : 512u;
+    // hi and lo halves of the state product side by side in one N = 2 NE product (half the
+    // UMMAs on the chain) when N fits one instruction; P then takes 2 NE columns
+    constexpr bool kSide = 2 * NE <= 256;
+    constexpr int kPc = kSide ? 2 * NE : NE;   // TMEM columns of P
+    constexpr uint32_t tcols = (kPc + NE <= 256) ? 256u : 512u;
     constexpr uint64_t kSwz = swizzle_code(2 * TV);
     // token batch, first token, tokens, chunks and first chunk (in the workspace) of this state
     int b = sb, tbeg = 0, tlen = T, nct = NT, cb = 0;
@@ -156,8 +163,9 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    const uint32_t tP = tmem_slot;        // columns [0, NE): P, then [U; Oa] in [0, TV)
-    const uint32_t tS = tmem_slot + NE;   // columns [NE, 2 NE): the state slab
+    const uint32_t tP = tmem_slot;         // columns [0, kPc): P (hi part, then lo part when
+                                           // side by side), then [U; Oa] in [0, 2 TV)
+    const uint32_t tS = tmem_slot + kPc;   // columns [kPc, kPc + NE): the state slab
 
     auto issue_kq = [&](int c) {
         mbar_arrive_expect_tx(&bar_kq, 4 * kBoxBytes);
@@ -253,22 +261,40 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     };
     // MMA-A: P = [K; Q] S_all    (B = S_all, MN-major, hi and lo)
     auto issue_mma_a = [&]() {
-        const uint32_t idesc = idesc_bf16_f32(128, NE, 0, 1);
         // descriptors built once; each K step advances their start addresses
         const uint64_t a0 = smem_desc(smem_u32(sKQ), 16, 1024);
         const uint64_t bh0 = smem_desc(smem_u32(sSh), blk_bytes<TV>(), 16 * TV, kSwz);
         const uint64_t bl0 = smem_desc(smem_u32(sSl), blk_bytes<TV>(), 16 * TV, kSwz);
+        // B = the slice blocks: 16 rows (two 8-row groups) per K step, one TV-column swizzle
+        // atom per slice; the lo blocks follow the hi blocks, so one descriptor spans both
+        const uint32_t idesc = idesc_bf16_f32(128, kSide ? 2 * NE : NE, 0, 1);
 #pragma unroll
         for (int ks = 0; ks < kDk / 16; ++ks) {
             const int blk = ks >> 2, kk = (ks & 3) * 16;
             const uint64_t ad = desc_add(a0, blk * 2 * kBoxBytes + kk * 2);
-            // B = the slice blocks: 16 rows (two 8-row groups) per K step, one TV-column
-            // swizzle atom per slice
             const uint32_t ko = ks * 32 * TV;
             umma_bf16(tP, ad, desc_add(bh0, ko), idesc, ks > 0 ? 1u : 0u);
-            umma_bf16(tP, ad, desc_add(bl0, ko), idesc, 1u);
+            if (!kSide) umma_bf16(tP, ad, desc_add(bl0, ko), idesc, 1u);
         }
         umma_commit(&bar_mma);
+    };
+
+    // this thread's columns of P for slices e0 .. e0 + GRP - 1 (the hi and lo parts summed
+    // when the halves were multiplied side by side)
+    auto load_p = [&](int e0, float* pv) {
+#pragma unroll
+        for (int g = 0; g < GRP; ++g) tmem_ld<TVH>(tmem_lane_addr(tP, warp, (e0 + g) * TV + cofs), pv + g * TVH);
+        if constexpr (kSide) {
+            float pl[GRP * TVH];
+#pragma unroll
+            for (int g = 0; g < GRP; ++g)
+                tmem_ld<TVH>(tmem_lane_addr(tP, warp, NE + (e0 + g) * TV + cofs), pl + g * TVH);
+            tmem_wait_ld();
+#pragma unroll
+            for (int i = 0; i < GRP * TVH; ++i) pv[i] += pl[i];
+        } else {
+            tmem_wait_ld();
+        }
     };
 
     bool failed = false;
@@ -350,9 +376,7 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
 #pragma unroll
                 for (int e0 = 0; e0 < E; e0 += GRP) {
                     float pv[GRP * TVH];
-#pragma unroll
-                    for (int g = 0; g < GRP; ++g) tmem_ld<TVH>(tmem_lane_addr(tP, warp, (e0 + g) * TV + cofs), pv + g * TVH);
-                    tmem_wait_ld();
+                    load_p(e0, pv);
 #pragma unroll
                     for (int g = 0; g < GRP; ++g)
 #pragma unroll
@@ -367,9 +391,7 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
 #pragma unroll
             for (int e0 = 0; e0 < E; e0 += GRP) {
                 float pv[GRP * TVH];
-#pragma unroll
-                for (int g = 0; g < GRP; ++g) tmem_ld<TVH>(tmem_lane_addr(tP, warp, (e0 + g) * TV + cofs), pv + g * TVH);
-                tmem_wait_ld();
+                load_p(e0, pv);
 #pragma unroll
                 for (int g = 0; g < GRP; ++g)
 #pragma unroll
@@ -383,18 +405,18 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
 
         // ---- MMA-B: [U; Oa] = [T; A T] Res  (into columns [0, TV); Res MN-major)
         if (tid == 0) {
+            // [T; A T]_hi [Res_hi | Res_lo] (N = 2 TV: the lo block is the next swizzle atom,
+            // TV * 128 bytes on) into columns [0, 2 TV), and [T; A T]_lo Res_hi into [0, TV)
+            const uint32_t idesc2 = idesc_bf16_f32(128, 2 * TV, 0, 1);
             const uint32_t idesc = idesc_bf16_f32(128, TV, 0, 1);
             const uint64_t ah0 = smem_desc(smem_u32(sA2), 16, 1024);
-            const uint64_t bh0 = smem_desc(smem_u32(sRh), blk_bytes<TV>(), 16 * TV, kSwz);
+            const uint64_t bh0 = smem_desc(smem_u32(sRh), TV * 128, 16 * TV, kSwz);
 #pragma unroll
             for (int ks = 0; ks < 4; ++ks) {
                 const uint64_t ah = desc_add(ah0, ks * 32);
                 const uint64_t al = desc_add(ah0, 2 * kBoxBytes + ks * 32);
-                const uint32_t ko = ks * 32 * TV;
-                const uint64_t bh = desc_add(bh0, ko);
-                const uint64_t bl = desc_add(bh0, TV * 128 + ko);   // sRl = sRh + TV * 128
-                umma_bf16(tP, ah, bh, idesc, ks > 0 ? 1u : 0u);
-                umma_bf16(tP, ah, bl, idesc, 1u);
+                const uint64_t bh = desc_add(bh0, ks * 32 * TV);
+                umma_bf16(tP, ah, bh, idesc2, ks > 0 ? 1u : 0u);
                 umma_bf16(tP, al, bh, idesc, 1u);
             }
             umma_commit(&bar_mma);
@@ -417,8 +439,14 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
 #pragma unroll
             for (int e = 0; e < E; ++e) cr[e] = we[e * 64 + r];
         }
-        tmem_ld<TVH>(tmem_lane_addr(tP, warp, cofs), d2);
-        tmem_wait_ld();
+        {
+            float d2l[TVH];
+            tmem_ld<TVH>(tmem_lane_addr(tP, warp, cofs), d2);
+            tmem_ld<TVH>(tmem_lane_addr(tP, warp, TV + cofs), d2l);
+            tmem_wait_ld();
+#pragma unroll
+            for (int i = 0; i < TVH; ++i) d2[i] += d2l[i];
+        }
         if (r < 64) {
 #pragma unroll
             for (int e = 0; e < E; ++e) {
