@@ -9,11 +9,13 @@
 //   dS_e = gamma^C_e dS'_e + Q^T diag(b_e) dO - K^T diag(a_e) dRes
 // One CTA of 8 warps per (b, h, block of TV value columns) keeps dS for its
 // value columns in TMEM.  Per chunk:
-//   MMA-A'  P' = K dS'_all              (M=64, N=NE, K=dk; dS' MN-major hi/lo)
+//   MMA-A'  P' = K dS'_all              (M=64, N=NE, K=dk; dS' MN-major hi/lo, the two halves
+//                                        side by side, N = 2 NE, when that fits one instruction)
 //   MMA-0   Y  = A^T dO                 (M=64, N=TV, K=64; A^T hi/lo, dO exact bf16,
 //                                        MN-major as the TMA loads it)
 //   epi     dU = Y + sum_e w_e (.) P'_e  -> dU hi/lo operand, dU to the workspace
-//   MMA-B'  dRes = T^T dU               (M=64, N=TV, K=64; both hi/lo)
+//   MMA-B'  dRes = T^T dU               (M=64, K=64; both hi/lo, the hi*hi and hi*lo terms in
+//                                        one N = 2 TV product)
 //   epi     dRes -> workspace and dv; operand rows [-a_e (.) dRes ; b_e (.) dO]
 //   MMA-C'  dS_all += [K^T | Q^T] [-a (.) dRes ; b (.) dO]   (M=dk=128, K=128, N=NE;
 //           K^T and Q^T read MN-major from the TMA key/query tile)
@@ -107,7 +109,11 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     const int nb = blockIdx.x, h = blockIdx.y, sb = blockIdx.z;   // sb: sequence or document
     const int n0 = nb * TV;
     const int T = p.T, H = p.H, dv = p.dv, NT = p.NT;
-    constexpr uint32_t tcols = (2 * NE + TV <= 256) ? 256u : 512u;
+    // hi and lo halves of dS' side by side in one N = 2 NE product K dS' (half the UMMAs on
+    // the chain) when N fits one instruction; dRes takes 2 TV columns (hi*hi + lo*hi, hi*lo)
+    constexpr bool kSide = 2 * NE <= 256;
+    constexpr int kPc = kSide ? 2 * NE : NE;   // TMEM columns of P'
+    constexpr uint32_t tcols = (kPc + 2 * TV + NE <= 256) ? 256u : 512u;
     constexpr uint64_t kSwz = swizzle_code(2 * TV);
     // token batch, first token, tokens, chunks and first chunk (in the workspaces) of this state
     int b = sb, tbeg = 0, tlen = T, nct = NT, cb = 0;
@@ -146,9 +152,9 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    const uint32_t tP = tmem_slot;             // [0, NE): K dS'
-    const uint32_t tY = tmem_slot + NE;        // [NE, NE+TV): A^T dO, then dRes
-    const uint32_t tS = tmem_slot + NE + TV;   // [NE+TV, 2 NE+TV): dS
+    const uint32_t tP = tmem_slot;                   // [0, kPc): K dS' (hi part, lo part)
+    const uint32_t tY = tmem_slot + kPc;             // [kPc, kPc + 2 TV): A^T dO, then dRes
+    const uint32_t tS = tmem_slot + kPc + 2 * TV;    // then NE columns: dS
 
     auto issue_kq = [&](int c) {
         mbar_arrive_expect_tx(&bar_kq, 4 * kBoxBytes);
@@ -280,7 +286,8 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
 
         // ---- MMA-A' (P' = K dS') and MMA-0 (Y = A^T dO)
         if (tid == 0) {
-            const uint32_t ida = idesc_bf16_f32(64, NE, 0, 1);
+            // dS' lo blocks follow the hi blocks: one descriptor spans both when side by side
+            const uint32_t ida = idesc_bf16_f32(64, kSide ? 2 * NE : NE, 0, 1);
             // descriptors built once; each K step advances their start addresses
             const uint64_t a0 = smem_desc(smem_u32(sKQ), 16, 1024);
             const uint64_t dh0 = smem_desc(smem_u32(sDh), blk_bytes<TV>(), 16 * TV, kSwz);
@@ -291,7 +298,7 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                 const uint64_t ad = desc_add(a0, blk * 2 * kBoxBytes + kk * 2);
                 const uint32_t ko = ks * 32 * TV;   // 16 rows of the slice blocks per K step
                 umma_bf16(tP, ad, desc_add(dh0, ko), ida, ks > 0 ? 1u : 0u);
-                umma_bf16(tP, ad, desc_add(dl0, ko), ida, 1u);
+                if (!kSide) umma_bf16(tP, ad, desc_add(dl0, ko), ida, 1u);
             }
             const uint32_t id0 = idesc_bf16_f32(64, TV, 0, 1);
             const uint64_t o0 = smem_desc(smem_u32(sdO), blk_bytes<TV>(), 16 * TV, kSwz);
@@ -342,7 +349,17 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                 float pv[GRP * TVH];
 #pragma unroll
                 for (int g = 0; g < GRP; ++g) tmem_ld<TVH>(tmem_lane_addr(tP, warp, (e0 + g) * TV + cofs), pv + g * TVH);
-                tmem_wait_ld();
+                if constexpr (kSide) {   // the lo part of K dS'
+                    float pl[GRP * TVH];
+#pragma unroll
+                    for (int g = 0; g < GRP; ++g)
+                        tmem_ld<TVH>(tmem_lane_addr(tP, warp, NE + (e0 + g) * TV + cofs), pl + g * TVH);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int i = 0; i < GRP * TVH; ++i) pv[i] += pl[i];
+                } else {
+                    tmem_wait_ld();
+                }
 #pragma unroll
                 for (int g = 0; g < GRP; ++g)
 #pragma unroll
@@ -362,18 +379,18 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
 
         // ---- MMA-B': dRes = T^T dU   (into tY; dU MN-major)
         if (tid == 0) {
+            // T^T_hi [dU_hi | dU_lo] (N = 2 TV: the lo block is the next swizzle atom, TV * 128
+            // bytes on) into tY columns [0, 2 TV), and T^T_lo dU_hi into [0, TV)
+            const uint32_t idb2 = idesc_bf16_f32(64, 2 * TV, 0, 1);
             const uint32_t idb = idesc_bf16_f32(64, TV, 0, 1);
             const uint64_t t0d = smem_desc(smem_u32(sBT), 16, 1024);
-            const uint64_t u0 = smem_desc(smem_u32(sUh), blk_bytes<TV>(), 16 * TV, kSwz);
+            const uint64_t u0 = smem_desc(smem_u32(sUh), TV * 128, 16 * TV, kSwz);
 #pragma unroll
             for (int ks = 0; ks < 4; ++ks) {
                 const uint64_t th = desc_add(t0d, 2 * kBoxBytes + ks * 32);
                 const uint64_t tl = desc_add(t0d, 3 * kBoxBytes + ks * 32);
-                const uint32_t ko = ks * 32 * TV;
-                const uint64_t uh = desc_add(u0, ko);
-                const uint64_t ul = desc_add(u0, TV * 128 + ko);   // sUl = sUh + TV * 128
-                umma_bf16(tY, th, uh, idb, ks > 0 ? 1u : 0u);
-                umma_bf16(tY, th, ul, idb, 1u);
+                const uint64_t uh = desc_add(u0, ks * 32 * TV);
+                umma_bf16(tY, th, uh, idb2, ks > 0 ? 1u : 0u);
                 umma_bf16(tY, tl, uh, idb, 1u);
             }
             umma_commit(&bar_mma);
@@ -391,8 +408,14 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             float dr[TVH], cr[E];   // -a_e (row threads) or b_e (dO rows) of this thread's row
 #pragma unroll
             for (int e = 0; e < E; ++e) cr[e] = row_thread ? -ae[e * 64 + r64] : be[e * 64 + r64];
-            tmem_ld<TVH>(tmem_lane_addr(tY, warp, cofs), dr);
-            tmem_wait_ld();
+            {
+                float drl[TVH];
+                tmem_ld<TVH>(tmem_lane_addr(tY, warp, cofs), dr);
+                tmem_ld<TVH>(tmem_lane_addr(tY, warp, TV + cofs), drl);
+                tmem_wait_ld();
+#pragma unroll
+                for (int i = 0; i < TVH; ++i) dr[i] += drl[i];
+            }
             if (row_thread) {
                 if (tma_dv) {   // row of the dv tile; thread 0 stores the tile after the barrier
                     if (p.out_f32) store_f32_row(reinterpret_cast<float*>(sDvo) + r64 * TV + cofs, dr, TVH);
@@ -546,7 +569,8 @@ cudaError_t launch_tv(const tla_problem& p, const FwdPlan& fp, const char* fws, 
 int tc_bwd_ok(const tla_problem& p, int tv) {
     if (tv == 0) return 0;
     const int ne = p.E * tv;
-    if (2 * ne + tv > 512) return 0;
+    const int pc = 2 * ne <= 256 ? 2 * ne : ne;   // TMEM columns of K dS' (side by side or not)
+    if (pc + 2 * tv + ne > 512) return 0;
     const size_t smem = tv == 16 ? tc_bwd_smem_c<16>(p.E)
                                  : tv == 32 ? tc_bwd_smem_c<32>(p.E) : tc_bwd_smem_c<64>(p.E);
     return smem <= 227 * 1024 ? 1 : 0;
