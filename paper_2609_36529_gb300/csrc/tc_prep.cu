@@ -109,22 +109,26 @@ chunk_prep_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     // the chunk's log decays, second keys and queries and beta: loaded into registers now
     // (token-major, E values of a token side by side), so that their latency overlaps the
     // key/query copies and the Gram product; stored slice-major ([E][64]) after it
-    float gv[4], kv[4], qv[4], bv = 0.f;
+    // (raw register copies, nothing computed from them until the product has been issued, so
+    // no instruction waits for the loads here)
+    float gv[4], bv = 1.f;
+    unsigned short kv[4], qv[4];
 #pragma unroll
     for (int u = 0; u < 4; ++u) {   // 64 E <= 1024 values: at most four per thread
         const int i = tid + u * kThreads;
-        gv[u] = kv[u] = qv[u] = 0.f;
+        gv[u] = 0.f;
+        kv[u] = qv[u] = 0;   // bf16 zero
         if (i < 64 * E) {
             const int r = i / E, e = i - (i / E) * E;
             const int rr = r < n ? r : n - 1;
             gv[u] = p.G[tok_idx(b, t0 + rr, h, e, T, H, E)];
             if (r < n) {
-                kv[u] = __bfloat162float(p.k2[tok_idx(b, t0 + r, h, e, T, H, E)]);
-                qv[u] = __bfloat162float(p.q2[tok_idx(b, t0 + r, h, e, T, H, E)]);
+                kv[u] = __bfloat16_as_ushort(p.k2[tok_idx(b, t0 + r, h, e, T, H, E)]);
+                qv[u] = __bfloat16_as_ushort(p.q2[tok_idx(b, t0 + r, h, e, T, H, E)]);
             }
         }
     }
-    if (tid < 64) bv = tid < n ? (p.beta ? p.beta[(size_t(b) * T + t0 + tid) * H + h] : 1.f) : 0.f;
+    if (tid < n && p.beta) bv = p.beta[(size_t(b) * T + t0 + tid) * H + h];
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -175,11 +179,11 @@ chunk_prep_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         if (i < 64 * E) {
             const int r = i / E, e = i - (i / E) * E;
             Gs[e * 64 + r] = gv[u];
-            k2s[e * 64 + r] = kv[u];
-            q2s[e * 64 + r] = qv[u];
+            k2s[e * 64 + r] = __bfloat162float(__ushort_as_bfloat16(kv[u]));
+            q2s[e * 64 + r] = __bfloat162float(__ushort_as_bfloat16(qv[u]));
         }
     }
-    if (tid < 64) bs[tid] = bv;
+    if (tid < 64) bs[tid] = tid < n ? bv : 0.f;   // beta, 1 without one, 0 past the chunk's rows
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -252,14 +256,18 @@ chunk_prep_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     // substitution (warps 0-3, lane = column), then the off-diagonal blocks by distance
     if (p.use_delta) {
         if (warp < 4 && lane < 16) {
+            // column s2 of the block's inverse: x_r = delta_{r,s2} - sum_{j<r} L_rj x_j, each
+            // x_r applied to the later rows as soon as it is final (the same terms in the same
+            // order as row-by-row substitution, but a dependent chain of 16 steps, not 120)
             const int o = 16 * warp, s2 = lane;
-            float x[16];
+            float x[16], acc[16];
+#pragma unroll
+            for (int k = 0; k < 16; ++k) acc[k] = (k == s2) ? 1.f : 0.f;
 #pragma unroll
             for (int r = 0; r < 16; ++r) {
-                float acc = (r == s2) ? 1.f : 0.f;
+                x[r] = acc[r];
 #pragma unroll
-                for (int j = 0; j < r; ++j) acc = fmaf(-LT[(o + j) * MP + o + r], x[j], acc);
-                x[r] = acc;
+                for (int k = r + 1; k < 16; ++k) acc[k] = fmaf(-LT[(o + r) * MP + o + k], x[r], acc[k]);
             }
 #pragma unroll
             for (int r = 0; r < 16; ++r) {
