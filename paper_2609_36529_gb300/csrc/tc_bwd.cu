@@ -10,7 +10,9 @@
 // One CTA of 8 warps per (b, h, block of TV value columns) keeps dS for its
 // value columns in TMEM.  Per chunk:
 //   MMA-A'  P' = K dS'_all              (M=64, N=NE, K=dk; dS' MN-major hi/lo, the two halves
-//                                        side by side, N = 2 NE, when that fits one instruction)
+//                                        side by side, N = 2 NE, when that fits one instruction;
+//                                        at E = 16 in two halves of the slices, one after the
+//                                        other, so that P', Y and the slab fit 512 columns)
 //   MMA-0   Y  = A^T dO                 (M=64, N=TV, K=64; A^T hi/lo, dO exact bf16,
 //                                        MN-major as the TMA loads it)
 //   epi     dU = Y + sum_e w_e (.) P'_e  -> dU hi/lo operand, dU to the workspace
@@ -29,6 +31,7 @@
 // Precision, TMA prefetch, bounded waits, the slice-block layout of the state
 // operand and the TMA-stored checkpoints as in the forward kernel.
 #include <cstring>
+#include <type_traits>
 
 #include "common.cuh"
 #include "internal.h"
@@ -90,14 +93,15 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     uint8_t* sKQ = sm;                       // 2 blocks x [K rows | Q rows] x 128 B
     uint8_t* sBT = sKQ + 4 * kBoxBytes;      // A^T hi, A^T lo, T^T hi, T^T lo (64 x 64 each)
     uint8_t* sReg = sBT + 4 * kBoxBytes;     // NE * 512 bytes, reused:
-    uint8_t* sDh = sReg;                     //   dS' hi / lo: E blocks [dk][TV] (MMA-A')
-    uint8_t* sDl = sReg + NE * 256;
-    uint8_t* sUh = sReg;                     //   dU [64][TV] hi / lo, MN-major (MMA-B')
-    uint8_t* sUl = sReg + TV * 128;
+    uint8_t* sDh = sReg;                     //   dS' hi / lo: E blocks [dk][TV] (MMA-A',
+    uint8_t* sDl = sReg + NE * 256;          //   checkpoint source)
     uint8_t* sBh = sReg;                     //   [-a dRes ; b dO] [128][NE] hi / lo (MMA-C')
     uint8_t* sBl = sReg + NE * 256;
     uint8_t* sdO = sReg + NE * 512;          // dO [64][TV] bf16, MN-major operand (TMA, swizzled)
     uint8_t* sDvo = sdO + 64 * TV * 2;       // dv tile [64][TV] (TMA store)
+    uint8_t* sUh = sDvo;                     // dU [64][TV] hi / lo, MN-major (MMA-B'), in the dv
+    uint8_t* sUl = sDvo + TV * 128;          // tile's space: the checkpoint copy of dS' proceeds
+                                             // under the dU epilogue and MMA-B' 
     float* sCoef = reinterpret_cast<float*>(sDvo + 64 * TV * 4);   // 2 x CB
 
     __shared__ __align__(8) uint64_t bar_kq, bar_av, bar_mma;
@@ -112,7 +116,13 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     // hi and lo halves of dS' side by side in one N = 2 NE product K dS' (half the UMMAs on
     // the chain) when N fits one instruction; dRes takes 2 TV columns (hi*hi + lo*hi, hi*lo)
     constexpr bool kSide = 2 * NE <= 256;
-    constexpr int kPc = kSide ? 2 * NE : NE;   // TMEM columns of P'
+    // P' by halves of the slices (the second product issued once the first is consumed) when
+    // all of it, Y and the slab do not fit the 512 TMEM columns together
+    constexpr bool kSplitP = !kSide && 2 * NE + 2 * TV > 512;
+    constexpr int EP = kSplitP ? E / 2 : E;    // slices per P' product
+    static_assert(!kSplitP || (E % 2 == 0 && (E / 2) % GRP == 0), "P' halves: whole batches");
+    constexpr int kPc = kSide ? 2 * NE : EP * TV;   // TMEM columns of P'
+    static_assert(kPc + 2 * TV + NE <= 512, "TMEM map");
     constexpr uint32_t tcols = (kPc + 2 * TV + NE <= 256) ? 256u : 512u;
     constexpr uint64_t kSwz = swizzle_code(2 * TV);
     // token batch, first token, tokens, chunks and first chunk (in the workspaces) of this state
@@ -246,6 +256,25 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         bulk_commit();
     };
 
+    // MMA-A' for slices [half * EP, half * EP + EP) into P' (thread 0)
+    auto issue_pa = [&](int half) {
+        // dS' lo blocks follow the hi blocks: one descriptor spans both when side by side
+        const uint32_t ida = idesc_bf16_f32(64, kSide ? 2 * NE : EP * TV, 0, 1);
+        // descriptors built once; each K step advances their start addresses
+        const uint32_t hb = uint32_t(half) * EP * blk_bytes<TV>();
+        const uint64_t a0 = smem_desc(smem_u32(sKQ), 16, 1024);
+        const uint64_t dh0 = smem_desc(smem_u32(sDh) + hb, blk_bytes<TV>(), 16 * TV, kSwz);
+        const uint64_t dl0 = smem_desc(smem_u32(sDl) + hb, blk_bytes<TV>(), 16 * TV, kSwz);
+#pragma unroll
+        for (int ks = 0; ks < kDk / 16; ++ks) {
+            const int blk = ks >> 2, kk = (ks & 3) * 16;
+            const uint64_t ad = desc_add(a0, blk * 2 * kBoxBytes + kk * 2);
+            const uint32_t ko = ks * 32 * TV;   // 16 rows of the slice blocks per K step
+            umma_bf16(tP, ad, desc_add(dh0, ko), ida, ks > 0 ? 1u : 0u);
+            if (!kSide) umma_bf16(tP, ad, desc_add(dl0, ko), ida, 1u);
+        }
+    };
+
     bool failed = false;
     uint32_t mma_phase = 0;
     int pending_mma = 0;
@@ -286,20 +315,7 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
 
         // ---- MMA-A' (P' = K dS') and MMA-0 (Y = A^T dO)
         if (tid == 0) {
-            // dS' lo blocks follow the hi blocks: one descriptor spans both when side by side
-            const uint32_t ida = idesc_bf16_f32(64, kSide ? 2 * NE : NE, 0, 1);
-            // descriptors built once; each K step advances their start addresses
-            const uint64_t a0 = smem_desc(smem_u32(sKQ), 16, 1024);
-            const uint64_t dh0 = smem_desc(smem_u32(sDh), blk_bytes<TV>(), 16 * TV, kSwz);
-            const uint64_t dl0 = smem_desc(smem_u32(sDl), blk_bytes<TV>(), 16 * TV, kSwz);
-#pragma unroll
-            for (int ks = 0; ks < kDk / 16; ++ks) {
-                const int blk = ks >> 2, kk = (ks & 3) * 16;
-                const uint64_t ad = desc_add(a0, blk * 2 * kBoxBytes + kk * 2);
-                const uint32_t ko = ks * 32 * TV;   // 16 rows of the slice blocks per K step
-                umma_bf16(tP, ad, desc_add(dh0, ko), ida, ks > 0 ? 1u : 0u);
-                if (!kSide) umma_bf16(tP, ad, desc_add(dl0, ko), ida, 1u);
-            }
+            issue_pa(0);
             const uint32_t id0 = idesc_bf16_f32(64, TV, 0, 1);
             const uint64_t o0 = smem_desc(smem_u32(sdO), blk_bytes<TV>(), 16 * TV, kSwz);
             const uint64_t t0d = smem_desc(smem_u32(sBT), 16, 1024);
@@ -333,7 +349,12 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         }
         ok = mbar_wait(&bar_mma, mma_phase);
         mma_phase ^= 1;
-        if (tid == 0) bulk_wait_read_all();   // the dS' blocks are rewritten next
+        // dU is written next into the dv tile's space, so the previous chunk's dv copy must
+        // have read it (the checkpoint copy, the most recent group, may still be reading dS')
+        if (tid == 0) {
+            if (p.ck_tiles) bulk_wait_read_but_last();
+            else bulk_wait_read_all();   // no checkpoint copies: the dv copy is the last group
+        }
         if (__syncthreads_or(!ok)) { failed = true; break; }
         pending_mma = 0;
         tc_fence_after();
@@ -344,26 +365,47 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
 #pragma unroll
             for (int e = 0; e < E; ++e) wr[e] = row_thread ? we[e * 64 + r64] : 0.f;
             tmem_ld<TVH>(tmem_lane_addr(tY, warp, cofs), du);
+            // adds w_e (.) P'_e for the EP slices from EB on (P' columns from 0)
+            auto add_p = [&](auto eb) {
+                constexpr int EB = decltype(eb)::value;
 #pragma unroll
-            for (int e0 = 0; e0 < E; e0 += GRP) {
-                float pv[GRP * TVH];
+                for (int e0 = 0; e0 < EP; e0 += GRP) {
+                    float pv[GRP * TVH];
 #pragma unroll
-                for (int g = 0; g < GRP; ++g) tmem_ld<TVH>(tmem_lane_addr(tP, warp, (e0 + g) * TV + cofs), pv + g * TVH);
-                if constexpr (kSide) {   // the lo part of K dS'
-                    float pl[GRP * TVH];
+                    for (int g = 0; g < GRP; ++g) tmem_ld<TVH>(tmem_lane_addr(tP, warp, (e0 + g) * TV + cofs), pv + g * TVH);
+                    if constexpr (kSide) {   // the lo part of K dS'
+                        float pl[GRP * TVH];
+#pragma unroll
+                        for (int g = 0; g < GRP; ++g)
+                            tmem_ld<TVH>(tmem_lane_addr(tP, warp, NE + (e0 + g) * TV + cofs), pl + g * TVH);
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int i = 0; i < GRP * TVH; ++i) pv[i] += pl[i];
+                    } else {
+                        tmem_wait_ld();
+                    }
 #pragma unroll
                     for (int g = 0; g < GRP; ++g)
-                        tmem_ld<TVH>(tmem_lane_addr(tP, warp, NE + (e0 + g) * TV + cofs), pl + g * TVH);
-                    tmem_wait_ld();
 #pragma unroll
-                    for (int i = 0; i < GRP * TVH; ++i) pv[i] += pl[i];
-                } else {
-                    tmem_wait_ld();
+                        for (int i = 0; i < TVH; ++i) du[i] = fmaf(wr[EB + e0 + g], pv[g * TVH + i], du[i]);
                 }
-#pragma unroll
-                for (int g = 0; g < GRP; ++g)
-#pragma unroll
-                    for (int i = 0; i < TVH; ++i) du[i] = fmaf(wr[e0 + g], pv[g * TVH + i], du[i]);
+            };
+            add_p(std::integral_constant<int, 0>{});
+            if constexpr (kSplitP) {   // the second half of the slices into the same columns
+                tc_fence_before();
+                __syncthreads();
+                tc_fence_after();
+                if (tid == 0) {
+                    issue_pa(1);
+                    umma_commit(&bar_mma);
+                }
+                pending_mma = 1;
+                ok = mbar_wait(&bar_mma, mma_phase);
+                mma_phase ^= 1;
+                if (__syncthreads_or(!ok)) { failed = true; break; }
+                pending_mma = 0;
+                tc_fence_after();
+                add_p(std::integral_constant<int, EP>{});
             }
             if (row_thread) {
 #pragma unroll
@@ -398,6 +440,7 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         pending_mma = 1;
         ok = mbar_wait(&bar_mma, mma_phase);
         mma_phase ^= 1;
+        if (tid == 0) bulk_wait_read_all();   // the MMA-C' operand rows overwrite dS' next
         if (__syncthreads_or(!ok)) { failed = true; break; }
         pending_mma = 0;
         tc_fence_after();
@@ -569,7 +612,8 @@ cudaError_t launch_tv(const tla_problem& p, const FwdPlan& fp, const char* fws, 
 int tc_bwd_ok(const tla_problem& p, int tv) {
     if (tv == 0) return 0;
     const int ne = p.E * tv;
-    const int pc = 2 * ne <= 256 ? 2 * ne : ne;   // TMEM columns of K dS' (side by side or not)
+    int pc = 2 * ne <= 256 ? 2 * ne : ne;   // TMEM columns of K dS' (side by side or not)
+    if (pc == ne && pc + 2 * tv + ne > 512 && p.E % 2 == 0) pc = ne / 2;   // by halves of the slices
     if (pc + 2 * tv + ne > 512) return 0;
     const size_t smem = tv == 16 ? tc_bwd_smem_c<16>(p.E)
                                  : tv == 32 ? tc_bwd_smem_c<32>(p.E) : tc_bwd_smem_c<64>(p.E);
@@ -589,6 +633,7 @@ cudaError_t launch_bwd_recurrence_tc(const tla_problem& p, const FwdPlan& fp, co
         case 6: return launch_tv<32, 6>(p, fp, fws, bp, bws, dO, dht, dv, dh0, err, s);
         case 8: return launch_tv<16, 8>(p, fp, fws, bp, bws, dO, dht, dv, dh0, err, s);
         case 12: return launch_tv<16, 12>(p, fp, fws, bp, bws, dO, dht, dv, dh0, err, s);
+        case 16: return launch_tv<16, 16>(p, fp, fws, bp, bws, dO, dht, dv, dh0, err, s);
         default: return cudaErrorInvalidValue;
     }
 }

@@ -104,14 +104,15 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     uint8_t* sKQ = sm;                         // 2 blocks x [K rows 0-63 | Q rows 64-127] x 128 B
     uint8_t* sA2 = sKQ + 4 * kBoxBytes;        // [T; A T] 128 x 64 bf16: hi tile, lo tile
     uint8_t* sReg = sA2 + 4 * kBoxBytes;       // shared region, NE * 512 bytes:
-    uint8_t* sSh = sReg;                       //   S_all hi: E blocks [dk][TV] (MMA-A operand)
-    uint8_t* sSl = sReg + NE * 256;            //   S_all lo
-    uint8_t* sRh = sReg;                       //   Res [64][TV] hi, lo, MN-major (after MMA-A)
-    uint8_t* sRl = sReg + TV * 128;
-    uint8_t* sUh = sReg + TV * 256;            //   Ut [64][NE] hi, lo, MN-major (after MMA-B)
+    uint8_t* sSh = sReg;                       //   S_all hi: E blocks [dk][TV] (MMA-A operand,
+    uint8_t* sSl = sReg + NE * 256;            //   S_all lo                     checkpoint source)
+    uint8_t* sUh = sReg;                       //   Ut [64][NE] hi, lo, MN-major (after MMA-B)
     uint8_t* sUl = sUh + NE * 128;
     __nv_bfloat16* sV = reinterpret_cast<__nv_bfloat16*>(sReg + NE * 512);  // [64][TV]
     uint8_t* sOo = sReg + NE * 512 + 64 * TV * 2;                             // o tile [64][TV] (TMA store)
+    uint8_t* sRh = sOo;                        // Res [64][TV] hi, lo, MN-major (epi-A to MMA-B),
+    uint8_t* sRl = sOo + TV * 128;             // in the o tile's space: the checkpoint copy of
+                                               // the state operand proceeds under epi-A and MMA-B
     float* sCoef = reinterpret_cast<float*>(sOo + 64 * TV * 4);               // 2 x CB
 
     __shared__ __align__(8) uint64_t bar_kq, bar_av, bar_mma;
@@ -338,11 +339,15 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                 tma_prefetch_l2_4d(&map_k, 64 * j, h, tbeg + (c + 1) * 64, b);
                 tma_prefetch_l2_4d(&map_q, 64 * j, h, tbeg + (c + 1) * 64, b);
             }
-        // ---- wait for MMA-A(c) (issued at the end of the previous step); the operand
-        // region is rewritten next, so the checkpoint copies must have read it
+        // ---- wait for MMA-A(c) (issued at the end of the previous step); Res is written
+        // next into the o tile's space, so the previous chunk's o copy must have read it (the
+        // checkpoint copy, the most recent group, may still be reading the state operand)
         bool ok = mbar_wait(&bar_mma, mma_phase);
         mma_phase ^= 1;
-        if (tid == 0) bulk_wait_read_all();
+        if (tid == 0) {
+            if (p.save && p.ck_tiles) bulk_wait_read_but_last();
+            else bulk_wait_read_all();   // no checkpoint copies: the o copy is the last group
+        }
         tc_fence_before();
         if (__syncthreads_or(!ok)) { failed = true; break; }
         pending_mma = 0;
@@ -428,6 +433,7 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         }
         ok = mbar_wait(&bar_mma, mma_phase);
         mma_phase ^= 1;
+        if (tid == 0) bulk_wait_read_all();   // Ut overwrites the state operand next
         if (__syncthreads_or(!ok)) { failed = true; break; }
         pending_mma = 0;
         tc_fence_after();

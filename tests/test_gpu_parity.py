@@ -215,9 +215,11 @@ def test_bwd_small(dtype, use_delta, T):
 
 @pytest.mark.parametrize("use_delta", [True, False])
 @pytest.mark.parametrize("T,E,dv", [(1, 4, 64), (64, 2, 64), (65, 4, 128), (200, 8, 64),
-                                    (130, 1, 64)])
+                                    (130, 1, 64), (90, 3, 64), (140, 6, 128), (150, 12, 128),
+                                    (193, 16, 128)])
 def test_bwd_tensor_core_path(use_delta, T, E, dv):
-    """bf16, dk = 128: tcgen05 forward and backward recurrences (+ chunk gradients)."""
+    """bf16, dk = 128: tcgen05 forward and backward recurrences (+ chunk gradients); every
+    slice count the tensor-core path takes, E = 16 with its K dS' product in two halves."""
     x = inputs.chunk_inputs(2, T, 2, 128, dv, E, dtype="bf16", with_beta=True, h0_std=0.1,
                             backward=True, device="cuda", seed=1000 + T * 7 + E)
     dht = 0.5 * torch.randn(2, 2, E, 128, dv, device="cuda",
