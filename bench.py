@@ -715,12 +715,17 @@ def _time_steps(step, k, warm, stream, barrier, max_over_ranks):
 def run_variants(args, tla, inputs, w, dev, stream, barrier, max_over_ranks, ws_n, rank,
                  headline):
     """Forward + backward tokens/s of the shape/gate variants: one log gate per head on the
-    headline workload (tensor-core path), the headline with o and the input gradients in
-    bf16 (the input dtype), and E = 32 slices with d_k = 64 (Table 4's iso-state variant;
-    CUDA-core path) on one 8192-token sequence."""
+    headline workload, the headline with o and the input gradients in bf16 (the input dtype),
+    and on one 8192-token sequence the d_k vs E shapes of Table 4 at d_k E = 1024 (E = 8 with
+    d_k = 128, E = 16 with d_k = 64) and E = 32 with d_k = 64.  Each case lists the kernels
+    that ran (tensor-core `*_tc` or CUDA-core) and its state-update rate (tokens/s x E d_k d_v)
+    against the headline's."""
     out = {}
+    lib = tla.lib()
     cases = [("gate_per_head", w.B, w.T, w.H, w.dk, w.dv, w.E, True),
              ("bf16_outputs", w.B, w.T, w.H, w.dk, w.dv, w.E, False),
+             ("E8_dk128", 1, w.T, w.H, 128, w.dv, 8, False),
+             ("E16_dk64", 1, w.T, w.H, 64, w.dv, 16, False),
              ("E32_dk64", 1, w.T, w.H, 64, w.dv, 32, False)]
     for name, B, T, H, dk, dv, E, per_head in cases:
         out_dtype = torch.bfloat16 if name == "bf16_outputs" else OUT_DTYPE
@@ -744,11 +749,17 @@ def run_variants(args, tla, inputs, w, dev, stream, barrier, max_over_ranks, ws_
 
         ms = _time_steps(step, 3, 3, stream, barrier, max_over_ranks)
         val = ws_n * B * T / (ms / 1e3)
+        lib.tla_profile_begin()   # one more step, untimed: which kernels ran
+        step()
+        torch.cuda.synchronize()
+        kernels = sorted(profile_read(lib, stream.cuda_stream))
         out[name] = {"config": {"B": B, "T": T, "H": H, "dk": dk, "dv": dv, "E": E,
                                 "gate": "per head [B,T,H]" if per_head else "per slice",
                                 "outputs": "fp32" if out_dtype == torch.float32 else "bf16"},
                      "value": round(val, 1), "unit": "tokens/s", "ms_per_step": round(ms, 4),
-                     "path": "tensor cores" if dk == 128 else "CUDA cores (fp32 SIMT)"}
+                     "kernels": kernels,
+                     "state_rate_vs_headline": round(val * E * dk * dv /
+                                                     (headline * w.E * w.dk * w.dv), 4)}
         if B == w.B and T == w.T:
             out[name]["vs_headline"] = round(val / headline, 4)
         del x, fws, bws, grads, o

@@ -34,7 +34,8 @@ struct FwdPlan {
                          //    and read by TMA (tma_host.h: make_ckpt_map); U, Res
                          //    and the backward's dU, -dRes are then token tiles: per
                          //    (b,h,chunk) 64 rows x dv bf16 hi then lo, SW128 K-major 64-row
-                         //    blocks, rows past T zero
+                         //    blocks, rows past T zero; with d_k = 64 a checkpoint keeps 128
+                         //    rows, the last 64 zero
     int tc_tv;           // value columns per CTA of the tensor-core recurrence (0: SIMT)
     int need_A;          // 1: the fp32 A matrices are read (a CUDA-core recurrence follows)
     size_t bytes;        // total
@@ -46,6 +47,7 @@ struct BwdPlan {
     size_t dRes;         // fp32 [B,T,H,dv] dRes, or token tiles of -dRes (delta rule)
     size_t dS;           // fp32 [B,H,NT,E,dk,dv] gradient of the state at each chunk's end
     size_t dgE;          // per-head gate: fp32 [B,T,H,E] per-slice gate gradient before the sum
+    size_t gscr;         // tensor-core chunk gradients with E > 8: fp32 [B,H,NT,3,64,E] partials
     size_t bytes;
 };
 
@@ -78,7 +80,7 @@ cudaError_t launch_chunk_prep_tc(const tla_problem& p, const FwdPlan& fp, char* 
 int tc_grads_ok(const tla_problem& p, const FwdPlan& fp);
 int tc_grads_shape_ok(const tla_problem& p);
 cudaError_t launch_bwd_chunk_grads_tc(const tla_problem& p, const FwdPlan& fp, const char* fws,
-                                      const BwdPlan& bp, const char* bws, const void* dO,
+                                      const BwdPlan& bp, char* bws, const void* dO,
                                       void* dq, void* dk, void* dq2, void* dk2, float* dbeta,
                                       float* dg, int* err, cudaStream_t s);
 // Tensor-core backward recurrence (requires the tensor-core forward layout).

@@ -59,6 +59,7 @@ struct TcBwdArgs {
     int* err;
     const int4* dtab;    // packed documents: (first token, chunks, first chunk, tokens); else NULL
     int T, H, dv, E, NT, use_delta, out_f32, ck_tiles;
+    int dk;              // key dimension: 128, or 64 padded to 128 by zero rows (TMA fill)
 };
 
 template <int TV>
@@ -132,10 +133,10 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         b = 0; tbeg = dd.x; nct = dd.y; cb = dd.z; tlen = dd.w;
     }
     if (nct == 0) {   // empty document: the gradient of the initial state is that of the final one
-        if (p.dh0)
+        if (p.dh0 && r < p.dk)
             for (int e = 0; e < E; ++e)
                 for (int n = cofs; n < cofs + TVH; ++n) {
-                    const size_t o = ((size_t(sb * H + h) * E + e) * kDk + r) * dv + n0 + n;
+                    const size_t o = ((size_t(sb * H + h) * E + e) * p.dk + r) * dv + n0 + n;
                     p.dh0[o] = p.dht ? p.dht[o] : 0.f;
                 }
         return;
@@ -186,8 +187,8 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
 #pragma unroll
         for (int n = 0; n < TVH; n += 8)
             st8_split(sDh, sDl, e * blk_bytes<TV>() + blk_offset<TV>(r, cofs + n), v + n);
-        if (!p.ck_tiles) {
-            const size_t slab = (((size_t(b) * H + h) * NT + cb + c) * E + e) * kDk * dv;
+        if (!p.ck_tiles && r < p.dk) {
+            const size_t slab = (((size_t(b) * H + h) * NT + cb + c) * E + e) * p.dk * dv;
             store_f32_row(p.dSck + slab + size_t(r) * dv + n0 + cofs, v, TVH);
         }
     };
@@ -227,9 +228,9 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         #pragma unroll
         for (int e = 0; e < E; ++e) {
             float v[TVH];
-            if (p.dht) {
+            if (p.dht && r < p.dk) {
                 const float4* src = reinterpret_cast<const float4*>(
-                    p.dht + ((size_t(sb * H + h) * E + e) * kDk + r) * dv + n0 + cofs);
+                    p.dht + ((size_t(sb * H + h) * E + e) * p.dk + r) * dv + n0 + cofs);
 #pragma unroll
                 for (int i = 0; i < TVH / 4; ++i) {
                     const float4 x = src[i];
@@ -267,6 +268,7 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         const uint64_t dl0 = smem_desc(smem_u32(sDl) + hb, blk_bytes<TV>(), 16 * TV, kSwz);
 #pragma unroll
         for (int ks = 0; ks < kDk / 16; ++ks) {
+            if (ks * 16 >= p.dk) break;   // the padded key rows are zero
             const int blk = ks >> 2, kk = (ks & 3) * 16;
             const uint64_t ad = desc_add(a0, blk * 2 * kBoxBytes + kk * 2);
             const uint32_t ko = ks * 32 * TV;   // 16 rows of the slice blocks per K step
@@ -542,8 +544,9 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                 tmem_wait_ld();
 #pragma unroll
                 for (int g = 0; g < GRP; ++g)
-                    store_f32_row(p.dh0 + ((size_t(sb * H + h) * E + e0 + g) * kDk + r) * dv + n0 + cofs,
-                                  v + g * TVH, TVH);
+                    if (r < p.dk)
+                        store_f32_row(p.dh0 + ((size_t(sb * H + h) * E + e0 + g) * p.dk + r) * dv + n0 + cofs,
+                                      v + g * TVH, TVH);
             }
         }
         fence_proxy_async_smem();
@@ -570,8 +573,8 @@ cudaError_t launch_tv(const tla_problem& p, const FwdPlan& fp, const char* fws, 
     if (p.E != E || fp.tc_tv != TV) return cudaErrorInvalidValue;
     CUtensorMap mk, mq, mo, mb, mc, mdv;
     const int NT = fp.NT;
-    if (!make_token_map(&mk, p.k, p.B, p.T, p.H, kDk, 64, 64, true) ||
-        !make_token_map(&mq, p.q, p.B, p.T, p.H, kDk, 64, 64, true) ||
+    if (!make_token_map(&mk, p.k, p.B, p.T, p.H, p.dk, 64, 64, true) ||
+        !make_token_map(&mq, p.q, p.B, p.T, p.H, p.dk, 64, 64, true) ||
         !make_token_map_sw(&mo, dO, p.B, p.T, p.H, p.dv, TV, 64) ||
         !make_matrix_map(&mb, fws + fp.BT, (long long)p.B * p.H * NT * 256, 64, 64, 64) ||
         !make_token_map(&mdv, dv, p.B, p.T, p.H, p.dv, TV, 64, false,
@@ -593,6 +596,7 @@ cudaError_t launch_tv(const tla_problem& p, const FwdPlan& fp, const char* fws, 
     a.T = p.T; a.H = p.H; a.dv = p.dv; a.E = p.E; a.NT = NT;
     a.use_delta = p.use_delta; a.out_f32 = p.out_dtype == TLA_FP32;
     a.ck_tiles = fp.ck_tiles;
+    a.dk = p.dk;
     a.dtab = p.cu_seqlens ? (const int4*)(fws + fp.dtab) : nullptr;
     const size_t smem = tc_bwd_smem_c<TV>(E);
     auto kern = bwd_recurrence_tc_kernel<TV, E>;

@@ -70,6 +70,7 @@ struct TcFwdArgs {
     int* err;
     const int4* dtab;    // packed documents: (first token, chunks, first chunk, tokens); else NULL
     int T, H, dv, E, NT, use_delta, save, out_f32, ck_tiles;
+    int dk;              // key dimension: 128, or 64 padded to 128 by zero rows (TMA fill)
 };
 
 template <int TV>
@@ -137,10 +138,10 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         b = 0; tbeg = dd.x; nct = dd.y; cb = dd.z; tlen = dd.w;
     }
     if (nct == 0) {   // empty document: the final state is the initial one
-        if (p.ht)
+        if (p.ht && r < p.dk)
             for (int e = 0; e < E; ++e)
                 for (int n = cofs; n < cofs + TVH; ++n) {
-                    const size_t o = ((size_t(sb * H + h) * E + e) * kDk + r) * dv + n0 + n;
+                    const size_t o = ((size_t(sb * H + h) * E + e) * p.dk + r) * dv + n0 + n;
                     p.ht[o] = p.h0 ? p.h0[o] : 0.f;
                 }
         return;
@@ -191,8 +192,8 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
 #pragma unroll
         for (int n = 0; n < TVH; n += 8)
             st8_split(sSh, sSl, e * blk_bytes<TV>() + blk_offset<TV>(r, cofs + n), v + n);
-        if (p.save && !p.ck_tiles) {
-            const size_t slab = (((size_t(b) * H + h) * NT + cb + c) * E + e) * kDk * dv;
+        if (p.save && !p.ck_tiles && r < p.dk) {
+            const size_t slab = (((size_t(b) * H + h) * NT + cb + c) * E + e) * p.dk * dv;
             store_f32_row(p.Sck + slab + size_t(r) * dv + n0 + cofs, v, TVH);
         }
     };
@@ -233,9 +234,9 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
 #pragma unroll
         for (int e = 0; e < E; ++e) {
             float v[TVH];
-            if (p.h0) {
+            if (p.h0 && r < p.dk) {
                 const float4* src = reinterpret_cast<const float4*>(
-                    p.h0 + ((size_t(sb * H + h) * E + e) * kDk + r) * dv + n0 + cofs);
+                    p.h0 + ((size_t(sb * H + h) * E + e) * p.dk + r) * dv + n0 + cofs);
 #pragma unroll
                 for (int i = 0; i < TVH / 4; ++i) {
                     const float4 x = src[i];
@@ -271,6 +272,7 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         const uint32_t idesc = idesc_bf16_f32(128, kSide ? 2 * NE : NE, 0, 1);
 #pragma unroll
         for (int ks = 0; ks < kDk / 16; ++ks) {
+            if (ks * 16 >= p.dk) break;   // the padded key rows are zero
             const int blk = ks >> 2, kk = (ks & 3) * 16;
             const uint64_t ad = desc_add(a0, blk * 2 * kBoxBytes + kk * 2);
             const uint32_t ko = ks * 32 * TV;
@@ -538,8 +540,9 @@ fwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                 tmem_wait_ld();
 #pragma unroll
                 for (int g = 0; g < GRP; ++g)
-                    store_f32_row(p.ht + ((size_t(sb * H + h) * E + e0 + g) * kDk + r) * dv + n0 + cofs,
-                                  v + g * TVH, TVH);
+                    if (r < p.dk)
+                        store_f32_row(p.ht + ((size_t(sb * H + h) * E + e0 + g) * p.dk + r) * dv + n0 + cofs,
+                                      v + g * TVH, TVH);
             }
         }
     }
@@ -565,8 +568,8 @@ cudaError_t launch_tv(const tla_problem& p, const FwdPlan& fp, char* ws, int sav
     if (p.E != E || fp.tc_tv != TV) return cudaErrorInvalidValue;
     CUtensorMap mk, mq, mv, ma, mc, mo;
     const int NT = fp.NT;
-    if (!make_token_map(&mk, p.k, p.B, p.T, p.H, kDk, 64, 64, true) ||
-        !make_token_map(&mq, p.q, p.B, p.T, p.H, kDk, 64, 64, true) ||
+    if (!make_token_map(&mk, p.k, p.B, p.T, p.H, p.dk, 64, 64, true) ||
+        !make_token_map(&mq, p.q, p.B, p.T, p.H, p.dk, 64, 64, true) ||
         !make_token_map(&mv, p.v, p.B, p.T, p.H, p.dv, TV, 64, false) ||
         !make_matrix_map(&ma, ws + fp.A2, (long long)p.B * p.H * NT * 256, 64, 64, 128) ||
         !make_token_map(&mo, p.o, p.B, p.T, p.H, p.dv, TV, 64, false, p.out_dtype == TLA_FP32 ? 4 : 2))
@@ -587,6 +590,7 @@ cudaError_t launch_tv(const tla_problem& p, const FwdPlan& fp, char* ws, int sav
     a.T = p.T; a.H = p.H; a.dv = p.dv; a.E = p.E; a.NT = NT;
     a.use_delta = p.use_delta; a.save = save; a.out_f32 = p.out_dtype == TLA_FP32;
     a.ck_tiles = fp.ck_tiles;
+    a.dk = p.dk;
     a.dtab = p.cu_seqlens ? (const int4*)(ws + fp.dtab) : nullptr;
     const size_t smem = tc_fwd_smem_c<TV>(E);
     auto kern = fwd_recurrence_tc_kernel<TV, E>;
@@ -604,7 +608,9 @@ cudaError_t launch_tv(const tla_problem& p, const FwdPlan& fp, char* ws, int sav
 // state and Ut operands are MN-major with 64-column swizzle atoms, so E * TV must
 // be a multiple of 64 (and at most 256, the widest UMMA and half of TMEM).
 int tc_fwd_tv(const tla_problem& p) {
-    if (p.dtype != TLA_BF16 || p.dk != kDk) return 0;
+    // d_k = 64 runs as d_k = 128 with zero key rows: the key/query boxes past d_k are filled
+    // with zeros by the copy engine, so the state's padded rows stay zero
+    if (p.dtype != TLA_BF16 || (p.dk != kDk && p.dk != 64)) return 0;
     const int cand[3] = {16, 32, 64};
     for (int tv : cand) {
         const int ne = p.E * tv;

@@ -63,7 +63,10 @@ struct TcGradArgs {
     float* dg;
     int* err;
     const int2* ctab;    // packed documents: (first token, rows) of each chunk; else NULL
+    float* scratch;      // E > 8: per chunk [3][64][E] fp32 partials (dk', dq', dG) in global
+                         // memory, leaving the shared memory to the operands
     int T, H, dv, E, NT, use_delta, out_f32;
+    int kdim;            // key dimension: 128, or 64 padded to 128 by zero rows (TMA fill)
 };
 
 // 4 x 4 block (rows R0.., columns S0..) of a shared row-major matrix.
@@ -152,7 +155,10 @@ __device__ __forceinline__ float unpack_bf16(const uint32_t* pk, int j) {
     return __uint_as_float((j & 1) ? (w & 0xffff0000u) : (w << 16));
 }
 
-template <int OUT_F32, bool PACKED>
+// BIG: more than 8 slices, whose per-token partial sums of dk', dq' and dG live in a per-chunk
+// global scratch (read and written a few times per element, L2-resident) instead of shared
+// memory.
+template <int OUT_F32, bool PACKED, bool BIG>
 __global__ void __launch_bounds__(kThreads, 1)
 bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                           const __grid_constant__ CUtensorMap map_q,
@@ -188,16 +194,17 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     float* Gs = reinterpret_cast<float*>(W + kWorkBytes);
     __nv_bfloat16* k2s = reinterpret_cast<__nv_bfloat16*>(Gs + GP * E);
     __nv_bfloat16* q2s = k2s + GP * E;
-    float* dk2a = reinterpret_cast<float*>(q2s + GP * E);
-    float* dq2a = dk2a + 64 * E;
-    float* dGa = dq2a + 64 * E;
-    float* dwk = dGa + 64 * E;
+    float* dwk = reinterpret_cast<float*>(q2s + GP * E);   // [64][E]
     float* bs = dwk + 64 * E;                  // [64]
     float* dba = bs + 64;                      // [64]
     float* dgc = dba + 64;                     // [16]
     float* scl = dgc + 16;                     // [2][3][64]: b_e, a_e, w_e (slice parity)
     float* red = scl + 384;                    // [3][4][64] row-dot partials per lane quarter
     float* frw = red + 768;                    // [2][8] Frobenius partials per warp (slice parity)
+    // [64][E] partial sums of dk', dq', dG: shared memory, or this chunk's global scratch
+    float* dk2a = BIG ? p.scratch + ((size_t(b) * H + h) * NT + c) * (3 * 64 * E) : frw + 16;
+    float* dq2a = dk2a + 64 * E;
+    float* dGa = dq2a + 64 * E;
 
     __shared__ __align__(8) uint64_t bar_ld, bar_mma, bar_q[4], bar_mh[2], bar_fh[2];
     __shared__ uint32_t tmem_slot;
@@ -296,6 +303,7 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     if (tid == 0) {
         const uint32_t id_kq = idesc_bf16_f32(128, 64, 0, 0);
         for (int ks = 0; ks < kDk / 16; ++ks) {
+            if (ks * 16 >= p.kdim) break;   // zero key columns past d_k
             const uint64_t a = smem_desc(smem_u32(sKQ) + (ks >> 2) * 2 * kBoxBytes + (ks & 3) * 32, 16, 1024);
             umma_bf16(tmem + 128, a, a, id_kq, ks > 0 ? 1u : 0u);   // B = the key rows of the same tile
         }
@@ -820,9 +828,9 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         for (int i = tid; i < 2 * 64 * (kDk / 4); i += kThreads) {
             const int m = i >= 64 * (kDk / 4), j = i - m * 64 * (kDk / 4);
             const int t = j / (kDk / 4), c4 = (j % (kDk / 4)) * 4;
-            if (t >= n) continue;
+            if (t >= n || c4 >= p.kdim) continue;   // padded key columns are not outputs
             const float4 x = *reinterpret_cast<const float4*>((m ? dks : dqs) + t * kDk + c4);
-            const size_t off = tok_idx(b, t0 + t, h, c4, T, H, kDk);
+            const size_t off = tok_idx(b, t0 + t, h, c4, T, H, p.kdim);
             void* dst = m ? p.dk : p.dq;
             if (OUT_F32) {
                 *reinterpret_cast<float4*>(static_cast<float*>(dst) + off) = x;
@@ -834,8 +842,8 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         }
     }
     __syncthreads();
-    if (warp < E) {   // one warp per slice: dgamma^C, then the reverse cumulative sum of dG
-        const int e = warp;
+    for (int e = warp; e < E; e += kThreads / 32) {   // a warp per slice: dgamma^C, then the
+                                                      // reverse cumulative sum of dG
         const float gl = Gs[e * GP + n - 1];
         float dGC = 0.f;
         for (int r = lane; r < n; r += 32)
@@ -874,28 +882,29 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
 
 size_t grads_tc_smem(int E, int dv) {
     const size_t T64 = size_t(64) * dv * 2;
-    const size_t small = size_t(GP) * E * (4 + 2 + 2) + size_t(64) * E * 4 * 4 +
+    // Gs, k2s, q2s, dwk, bs, dba, dgc, scl, red, frw, and dk2a, dq2a, dGa unless E > 8
+    const size_t small = size_t(GP) * E * (4 + 2 + 2) + size_t(64) * E * 4 * (E > 8 ? 1 : 4) +
                          (64 + 64 + 16 + 384 + 768 + 16) * 4;
-    return 1024 + 5 * T64 + kWorkBytes + small;   // small: Gs, k2s, q2s, dk2a, dq2a, dGa, dwk, bs, dba, dgc, scl, red, frw
+    return 1024 + 5 * T64 + kWorkBytes + small;
 }
 
 }  // namespace
 
 int tc_grads_shape_ok(const tla_problem& p) {
-    return p.dk == kDk && p.dv % 64 == 0 && p.dv <= 128 && p.E <= 8 &&
+    return (p.dk == kDk || p.dk == 64) && p.dv % 64 == 0 && p.dv <= 128 && p.E <= 16 &&
            grads_tc_smem(p.E, p.dv) <= 227 * 1024;
 }
 
 int tc_grads_ok(const tla_problem& p, const FwdPlan& fp) { return fp.ck_tiles && tc_grads_shape_ok(p); }
 
 cudaError_t launch_bwd_chunk_grads_tc(const tla_problem& p, const FwdPlan& fp, const char* fws,
-                                      const BwdPlan& bp, const char* bws, const void* dO,
+                                      const BwdPlan& bp, char* bws, const void* dO,
                                       void* dq, void* dk, void* dq2, void* dk2, float* dbeta,
                                       float* dg, int* err, cudaStream_t s) {
     CUtensorMap mk, mq, mo, ms, md;
     const long long nslab = (long long)p.B * p.H * fp.NT * p.E;
-    if (!make_token_map(&mk, p.k, p.B, p.T, p.H, kDk, 64, 64, true) ||
-        !make_token_map(&mq, p.q, p.B, p.T, p.H, kDk, 64, 64, true) ||
+    if (!make_token_map(&mk, p.k, p.B, p.T, p.H, p.dk, 64, 64, true) ||
+        !make_token_map(&mq, p.q, p.B, p.T, p.H, p.dk, 64, 64, true) ||
         !make_token_map(&mo, dO, p.B, p.T, p.H, p.dv, 64, 64, true) ||
         !make_ckpt_map(&ms, fws + fp.S, nslab, p.dv, 64, 1, 128) ||
         !make_ckpt_map(&md, bws + bp.dS, nslab, p.dv, 64, 1, 128))
@@ -915,11 +924,19 @@ cudaError_t launch_bwd_chunk_grads_tc(const tla_problem& p, const FwdPlan& fp, c
     a.dq = dq; a.dk = dk; a.dq2 = dq2; a.dk2 = dk2; a.dbeta = dbeta; a.dg = dg;
     a.err = err;
     a.ctab = p.cu_seqlens ? (const int2*)(fws + fp.ctab) : nullptr;
+    const bool big = p.E > 8;
+    a.scratch = big ? (float*)(bws + bp.gscr) : nullptr;
     a.T = p.T; a.H = p.H; a.dv = p.dv; a.E = p.E; a.NT = fp.NT;
-    a.use_delta = p.use_delta; a.out_f32 = p.out_dtype == TLA_FP32;
+    a.use_delta = p.use_delta; a.out_f32 = p.out_dtype == TLA_FP32; a.kdim = p.dk;
     const size_t smem = grads_tc_smem(p.E, p.dv);
-    auto kern = a.ctab ? (a.out_f32 ? bwd_chunk_grads_tc_kernel<1, true> : bwd_chunk_grads_tc_kernel<0, true>)
-                       : (a.out_f32 ? bwd_chunk_grads_tc_kernel<1, false> : bwd_chunk_grads_tc_kernel<0, false>);
+    auto kern = big ? (a.ctab ? (a.out_f32 ? bwd_chunk_grads_tc_kernel<1, true, true>
+                                           : bwd_chunk_grads_tc_kernel<0, true, true>)
+                              : (a.out_f32 ? bwd_chunk_grads_tc_kernel<1, false, true>
+                                           : bwd_chunk_grads_tc_kernel<0, false, true>))
+                    : (a.ctab ? (a.out_f32 ? bwd_chunk_grads_tc_kernel<1, true, false>
+                                           : bwd_chunk_grads_tc_kernel<0, true, false>)
+                              : (a.out_f32 ? bwd_chunk_grads_tc_kernel<1, false, false>
+                                           : bwd_chunk_grads_tc_kernel<0, false, false>));
     cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     dim3 grid(fp.NT, p.H, p.B);
     prof_before("bwd_chunk_grads_tc", s);

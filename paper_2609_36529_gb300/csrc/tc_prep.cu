@@ -40,6 +40,7 @@ struct TcPrepArgs {
     int* err;
     const int2* ctab;    // packed documents: (first token, rows) of each chunk; else NULL
     int T, H, E, NT, use_delta;
+    int dk;              // key dimension: 128, or 64 (the key/query boxes past it are zero)
 };
 
 __device__ __forceinline__ void ld4(const float* src, float* v) {
@@ -146,6 +147,7 @@ chunk_prep_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     if (tid == 0) {
         const uint32_t id = idesc_bf16_f32(128, 64, 0, 0);
         for (int ks = 0; ks < kDk / 16; ++ks) {
+            if (ks * 16 >= p.dk) break;   // zero key columns past d_k
             const uint64_t a = smem_desc(smem_u32(sKQ) + (ks >> 2) * 2 * kBoxBytes + (ks & 3) * 32, 16, 1024);
             umma_bf16(tmem, a, a, id, ks > 0 ? 1u : 0u);
         }
@@ -413,8 +415,8 @@ size_t prep_tc_smem(int E) { return 1024 + size_t(5) * kSlot * 4 + (3 * 64 * E +
 cudaError_t launch_chunk_prep_tc(const tla_problem& p, const FwdPlan& fp, char* ws, int* err,
                                  cudaStream_t s) {
     CUtensorMap mk, mq;
-    if (!make_token_map(&mk, p.k, p.B, p.T, p.H, kDk, 64, 64, true) ||
-        !make_token_map(&mq, p.q, p.B, p.T, p.H, kDk, 64, 64, true))
+    if (!make_token_map(&mk, p.k, p.B, p.T, p.H, p.dk, 64, 64, true) ||
+        !make_token_map(&mq, p.q, p.B, p.T, p.H, p.dk, 64, 64, true))
         return cudaErrorInvalidValue;
     TcPrepArgs a;
     a.q2 = (const __nv_bfloat16*)p.q2;
@@ -428,7 +430,7 @@ cudaError_t launch_chunk_prep_tc(const tla_problem& p, const FwdPlan& fp, char* 
     a.coef = (float*)(ws + fp.coef);
     a.err = err;
     a.ctab = p.cu_seqlens ? (const int2*)(ws + fp.ctab) : nullptr;
-    a.T = p.T; a.H = p.H; a.E = p.E; a.NT = fp.NT; a.use_delta = p.use_delta;
+    a.T = p.T; a.H = p.H; a.E = p.E; a.NT = fp.NT; a.use_delta = p.use_delta; a.dk = p.dk;
     const size_t smem = prep_tc_smem(p.E);
     cudaFuncSetAttribute(chunk_prep_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     dim3 grid(fp.NT, p.H, p.B);

@@ -102,7 +102,6 @@ FwdPlan plan_fwd(const tla_problem& p, int save) {
     f.tc_tv = tc_fwd_tv(p);   // layout depends on shapes only
     const size_t tokE = (size_t)p.B * p.T * p.H * p.E * 4;
     const size_t mats = (size_t)p.B * p.H * f.NT * kChunk * kChunk * 4;
-    const size_t states = (size_t)p.B * p.H * f.NT * p.E * p.dk * p.dv * 4;
     const size_t tokV = (size_t)p.B * f.NT * kChunk * p.H * p.dv * 4;   // whole chunks (token tiles)
     size_t off = 0;
     f.G = off; off = align256(off + tokE);
@@ -119,7 +118,8 @@ FwdPlan plan_fwd(const tla_problem& p, int save) {
     // A feeds the CUDA-core recurrences only: the forward without tensor cores, or the
     // backward recurrence when it cannot run on tensor cores
     f.need_A = (!f.tc_tv || (save && !f.tcb)) ? 1 : 0;
-    if (save) {
+    if (save) {   // tile checkpoints keep 128 key rows (zero past d_k = 64)
+        const size_t states = (size_t)p.B * p.H * f.NT * p.E * (f.ck_tiles ? 128 : p.dk) * p.dv * 4;
         f.S = off; off = align256(off + states);
         f.U = off; off = align256(off + tokV);
         if (p.use_delta || f.ck_tiles) { f.Res = off; off = align256(off + tokV); }
@@ -138,12 +138,18 @@ BwdPlan plan_bwd(const tla_problem& p) {
     const int NT = chunk_count(p);
     b.tv = simt_tv(p);
     const size_t tokV = (size_t)p.B * NT * kChunk * p.H * p.dv * 4;   // whole chunks (token tiles)
-    const size_t states = (size_t)p.B * p.H * NT * p.E * p.dk * p.dv * 4;
+    // tile checkpoints (the forward plan's choice) keep 128 key rows (zero past d_k = 64)
+    const int ck_rows = plan_fwd(p, 1).ck_tiles ? 128 : p.dk;
+    const size_t states = (size_t)p.B * p.H * NT * p.E * ck_rows * p.dv * 4;
     size_t off = 0;
     b.dU = off; off = align256(off + tokV);
     b.dRes = off; off = align256(off + tokV);
     b.dS = off; off = align256(off + states);
     if (p.gate_per_head) { b.dgE = off; off = align256(off + (size_t)p.B * p.T * p.H * p.E * 4); }
+    if (p.E > 8 && tc_grads_ok(p, plan_fwd(p, 1))) {
+        b.gscr = off;
+        off = align256(off + (size_t)p.B * p.H * NT * 3 * kChunk * p.E * 4);
+    }
     b.bytes = off;
     return b;
 }

@@ -145,8 +145,11 @@ def test_packed_documents_validation(tla):
     p = packed([0, 100])
     p.n_docs = 0
     assert L.tla_chunk_fwd(ctypes.byref(p), None, 0, 0, None) == -1
-    # packed documents run on the tensor-core path only (here d_k = 64): refused before a launch
-    assert L.tla_chunk_fwd(ctypes.byref(ok), ctypes.c_void_p(0x100000), need, 1, None) == -2
+    # packed documents run on the tensor-core path only (d_k = 64 or 128; here d_k = 32):
+    # refused before a launch
+    small = packed([0, 10, 10, 100], dk=32)
+    need32 = L.tla_fwd_workspace_bytes(ctypes.byref(small), 1)
+    assert L.tla_chunk_fwd(ctypes.byref(small), ctypes.c_void_p(0x100000), need32, 1, None) == -2
 
 
 def test_layer_io_validation(tla):

@@ -233,6 +233,27 @@ def test_bwd_tensor_core_path(use_delta, T, E, dv):
         close(n, grads[n], ref[n], TOL["bf16"], rel_l2=0.01)
 
 
+@pytest.mark.parametrize("use_delta", [True, False])
+@pytest.mark.parametrize("T,E,dv", [(130, 4, 128), (200, 8, 64), (150, 16, 128), (64, 2, 64)])
+def test_tensor_core_dk64(use_delta, T, E, dv):
+    """d_k = 64 on the tensor-core kernels (key rows past 64 zero-filled by the copy engine):
+    forward with h0 and final state, backward with dht and dh0, every output."""
+    x = inputs.chunk_inputs(2, T, 2, 64, dv, E, dtype="bf16", with_beta=True, h0_std=0.1,
+                            backward=True, device="cuda", seed=2000 + T + E)
+    dht = 0.5 * torch.randn(2, 2, E, 64, dv, device="cuda",
+                            generator=torch.Generator("cuda").manual_seed(T * E))
+    o, ht, grads = run_bwd(x, use_delta, dht)
+    torch.cuda.synchronize()
+    assert tla.tla_last_device_status() == 0
+    ro, rht = oracle_fwd(x, use_delta)
+    close("o", o, ro, TOL["bf16"], rel_l2=0.01)
+    close("ht", ht, rht, TOL["bf16"], rel_l2=0.01)
+    ref = oracle_bwd(x, use_delta, dht)
+    assert set(ref) == set(grads)
+    for n in ref:
+        close(n, grads[n], ref[n], TOL["bf16"], rel_l2=0.01)
+
+
 def test_bwd_sgla_no_beta_no_h0():
     x = inputs.chunk_inputs(1, 150, 2, 32, 32, 4, dtype="fp32", with_beta=False, backward=True,
                             device="cuda", seed=11)

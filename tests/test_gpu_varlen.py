@@ -43,8 +43,8 @@ def close(name, got, ref, rel_l2=None):
         assert rl < rel_l2, f"{name}: rel L2 {rl:.3e}"
 
 
-def packed(lens, H, dv, E, seed, backward=False):
-    x, cu = inputs.packed_inputs(lens, H, 128, dv, E, dtype="bf16", h0_std=0.1,
+def packed(lens, H, dv, E, seed, backward=False, dk=128):
+    x, cu = inputs.packed_inputs(lens, H, dk, dv, E, dtype="bf16", h0_std=0.1,
                                  backward=backward, device="cuda", seed=seed)
     return x, cu
 
@@ -116,6 +116,27 @@ def test_packed_backward(use_delta, lens):
     assert tla.tla_last_device_status() == 0
     _, _, ref = oracle_docs(x, cu, use_delta, dht=_np(dht))
     assert set(ref) == set(grads)
+    for n in ref:
+        close(n, grads[n], ref[n], rel_l2=0.01)
+
+
+@pytest.mark.parametrize("dk,dv,E", [(64, 128, 4), (128, 64, 12), (64, 64, 16)])
+def test_packed_backward_shapes(dk, dv, E):
+    """Packed documents with d_k = 64 (zero-padded key rows) and more than eight slices."""
+    lens = [70, 0, 129, 64, 3]
+    x, cu = packed(lens, 2, dv, E, seed=dk + E, backward=True, dk=dk)
+    gen = torch.Generator("cuda")
+    gen.manual_seed(dk * E)
+    dht = 0.5 * torch.randn(len(lens), 2, E, dk, dv, device="cuda", generator=gen)
+    o, ht, ws = tla.tla_chunk_fwd(x["q"], x["k"], x["v"], x["q2"], x["k2"], x["g"], x["beta"],
+                                  x["h0"], save_for_bwd=True, cu_seqlens=cu)
+    grads, _ = tla.tla_chunk_bwd(x["q"], x["k"], x["v"], x["q2"], x["k2"], x["g"], x["dO"], ws,
+                                 beta=x["beta"], h0=x["h0"], dht=dht, cu_seqlens=cu)
+    torch.cuda.synchronize()
+    assert tla.tla_last_device_status() == 0
+    ro, rht, ref = oracle_docs(x, cu, True, dht=_np(dht))
+    close("o", o, ro, rel_l2=0.01)
+    close("ht", ht, rht, rel_l2=0.01)
     for n in ref:
         close(n, grads[n], ref[n], rel_l2=0.01)
 
