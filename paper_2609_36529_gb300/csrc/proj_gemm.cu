@@ -67,12 +67,18 @@ __device__ __forceinline__ float silu(float x) { return x * sigm(x); }
 // when n is a multiple of 8).
 __device__ __forceinline__ void put_row(__nv_bfloat16* dst, const float* src, int n, bool norm, float eps) {
     float r = 1.f;
-    if (norm) {
-        float ss = 0.f;
-        for (int i = 0; i < n; ++i) ss = fmaf(src[i], src[i], ss);
-        r = rsqrtf(ss + eps);
+    if (norm) {   // four partial sums: four loads and FMA chains in flight
+        float s4[4] = {0.f, 0.f, 0.f, 0.f};
+        int i = 0;
+#pragma unroll 4
+        for (; i + 4 <= n; i += 4)
+#pragma unroll
+            for (int u = 0; u < 4; ++u) s4[u] = fmaf(src[i + u], src[i + u], s4[u]);
+        for (; i < n; ++i) s4[0] = fmaf(src[i], src[i], s4[0]);
+        r = rsqrtf((s4[0] + s4[1]) + (s4[2] + s4[3]) + eps);
     }
     if (n % 8 == 0) {
+#pragma unroll 4
         for (int i = 0; i < n; i += 8) {
             uint32_t w4[4];
 #pragma unroll
@@ -183,35 +189,55 @@ proj_gemm_kernel(const __grid_constant__ CUtensorMap map_u, const __grid_constan
                 const int nc = grp == 0 ? dk : dv + 2 * E;         // channels of the pass
                 const int c0 = (grp == 0 ? 0 : 2 * dk) + tc0;     // their first channel in the head
                 const int ld = nc + 1;                             // odd stride: no bank conflicts
-                // TMEM -> shared memory (and the raw projection, when requested)
-                for (int j = 0; j < nc; j += 16) {
-                    float v[16];
+                // TMEM -> shared memory (and the raw projection, when requested), 32 columns
+                // per wait (the accumulator's 256 columns cover the second load)
+                for (int j = 0; j < nc; j += 32) {
+                    float v[32];
                     tmem_ld16(tmem_lane_addr(tmem, warp, tc0 + j), v);
+                    tmem_ld16(tmem_lane_addr(tmem, warp, tc0 + j + 16), v + 16);
                     tmem_wait_ld();
-                    const int cnt = nc - j < 16 ? nc - j : 16;
+                    const int cnt = nc - j < 32 ? nc - j : 32;
 #pragma unroll
-                    for (int u = 0; u < 16; ++u)
+                    for (int u = 0; u < 32; ++u)
                         if (u < cnt) S[row * ld + j + u] = v[u];
                     if (p.P && out_row)
-                        for (int u = 0; u < cnt; ++u) p.P[tok * C + c0 + j + u] = __float2bfloat16_rn(v[u]);
+#pragma unroll
+                        for (int u = 0; u < 32; ++u)
+                            if (u < cnt) p.P[tok * C + c0 + j + u] = __float2bfloat16_rn(v[u]);
                 }
                 epi_sync();
                 // causal depthwise convolution and activation, one thread per channel down the rows
                 for (int c = et; c < nc; c += 128) {
                     const int cg = c0 + c;                 // channel within the head
                     const bool soft = cg >= 2 * dk + dv;   // q', k': softplus; q, k, v: SiLU
-                    float w[4] = {0.f, 0.f, 0.f, 0.f};
-                    for (int j = 0; j < K; ++j) w[4 - K + j] = p.conv_w[(size_t(h) * C + cg) * K + j];
-                    float x0 = 0.f, x1 = 0.f, x2 = 0.f;    // raw values of the three previous rows
-                    for (int r = 0; r < 128; ++r) {
-                        const int t = t0 - kHalo + r;
-                        const float x3 = t >= 0 ? S[r * ld + c] : 0.f;
-                        if (r >= kHalo) {
-                            const float a = fmaf(w[0], x0, fmaf(w[1], x1, fmaf(w[2], x2, w[3] * x3)));
-                            S[r * ld + c] = soft ? softplus(a) : silu(a);
+                    float w[4];   // taps padded on the left to four
+#pragma unroll
+                    for (int j = 0; j < 4; ++j)
+                        w[j] = j >= 4 - K ? p.conv_w[(size_t(h) * C + cg) * K + j - (4 - K)] : 0.f;
+                    float* col = S + c;
+                    // eight rows at a time: their raw values are read before any of them is
+                    // overwritten, so the eight loads are in flight together; the activation is
+                    // chosen once per channel, outside the loop, so that the eight rows'
+                    // activations interleave
+                    auto conv_rows = [&](auto act) {
+                        float x0 = 0.f, x1 = 0.f, x2 = 0.f;   // raw values of the three previous rows
+                        for (int r0 = 0; r0 < 128; r0 += 8) {
+                            float xr[8], y[8];
+#pragma unroll
+                            for (int i = 0; i < 8; ++i) xr[i] = t0 - kHalo + r0 + i >= 0 ? col[(r0 + i) * ld] : 0.f;
+#pragma unroll
+                            for (int i = 0; i < 8; ++i) {
+                                const float a = fmaf(w[0], x0, fmaf(w[1], x1, fmaf(w[2], x2, w[3] * xr[i])));
+                                y[i] = act(a);
+                                x0 = x1; x1 = x2; x2 = xr[i];
+                            }
+#pragma unroll
+                            for (int i = 0; i < 8; ++i)
+                                if (r0 + i >= kHalo) col[(r0 + i) * ld] = y[i];
                         }
-                        x0 = x1; x1 = x2; x2 = x3;
-                    }
+                    };
+                    if (soft) conv_rows([](float a) { return softplus(a); });
+                    else conv_rows([](float a) { return silu(a); });
                 }
                 epi_sync();
                 // normalisation and stores, one thread per token row
