@@ -413,20 +413,22 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             load_bf16x4(k2s + e * GP + R0, krv);
             load_bf16x4(q2s + e * GP + R0, qrv);
         }
+        // the block's 16 exponentials first (independent), then the sums
+        float ks2[4][4];
 #pragma unroll
-        for (int a = 0; a < 4; ++a) {
-            const float gr = grv[a];
-            const float kr = krv[a];
-            const float qr = qrv[a];
+        for (int a = 0; a < 4; ++a)
+#pragma unroll
+            for (int c2 = 0; c2 < 4; ++c2)   // exp of a non-positive difference
+                ks2[a][c2] = __expf(fminf(grv[a] - gs[c2], 0.f));
+#pragma unroll
+        for (int a = 0; a < 4; ++a)
 #pragma unroll
             for (int c2 = 0; c2 < 4; ++c2) {
-                // exp of a non-positive difference (entries above the diagonal are discarded)
-                const float gam = __expf(fminf(gr - gs[c2], 0.f));
-                const float ks2 = (R0 + a >= S0 + c2) ? ksv[c2] * gam : 0.f;
-                Rv[a][c2] = fmaf(kr, ks2, Rv[a][c2]);
-                Rq[a][c2] = fmaf(qr, ks2, Rq[a][c2]);
+                // entries above the diagonal are discarded
+                const float kg = (R0 + a >= S0 + c2) ? ksv[c2] * ks2[a][c2] : 0.f;
+                Rv[a][c2] = fmaf(krv[a], kg, Rv[a][c2]);
+                Rq[a][c2] = fmaf(qrv[a], kg, Rq[a][c2]);
             }
-        }
     }
     __syncthreads();
     float dKK[4][4], rp[4];
