@@ -283,48 +283,42 @@ chunk_prep_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         }
         __syncthreads();
         for (int dist = 1; dist < 4; ++dist) {
-            const int tasks = (4 - dist) * 16;   // 4 x 4 blocks of the blocks (i, i - dist)
-            const int bi = dist + (tid >> 4), bj = bi - dist;
-            const int r0 = 16 * bi + 4 * ((tid >> 2) & 3), s0 = 16 * bj + 4 * (tid & 3);
+            // 2 x 2 blocks of the 16 x 16 blocks (i, i - dist): 64 threads per block, so that
+            // 192 / 128 / 64 threads share the work of the three distances
+            const int tasks = (4 - dist) * 64;
+            const int bi = dist + (tid >> 6), bj = bi - dist;
+            const int r0 = 16 * bi + 2 * ((tid >> 3) & 7), s0 = 16 * bj + 2 * (tid & 7);
             if (tid < tasks) {   // W_ij = sum_{k=j}^{i-1} L_ik X_kj
-                float w[4][4];
-#pragma unroll
-                for (int a = 0; a < 4; ++a)
-#pragma unroll
-                    for (int c2 = 0; c2 < 4; ++c2) w[a][c2] = 0.f;
+                float w[2][2] = {{0.f, 0.f}, {0.f, 0.f}};
 #pragma unroll 4
                 for (int x = 16 * bj; x < 16 * bi; ++x) {
-                    float l[4], xv[4];
-                    ld4(LT + x * MP + r0, l);
-                    ld4(MX + x * MP + s0, xv);
-#pragma unroll
-                    for (int a = 0; a < 4; ++a)
-#pragma unroll
-                        for (int c2 = 0; c2 < 4; ++c2) w[a][c2] = fmaf(l[a], xv[c2], w[a][c2]);
+                    const float2 l = *reinterpret_cast<const float2*>(LT + x * MP + r0);
+                    const float2 xv = *reinterpret_cast<const float2*>(MX + x * MP + s0);
+                    w[0][0] = fmaf(l.x, xv.x, w[0][0]);
+                    w[0][1] = fmaf(l.x, xv.y, w[0][1]);
+                    w[1][0] = fmaf(l.y, xv.x, w[1][0]);
+                    w[1][1] = fmaf(l.y, xv.y, w[1][1]);
                 }
 #pragma unroll
-                for (int a = 0; a < 4; ++a) st4(MW + (r0 + a) * MP + s0, w[a][0], w[a][1], w[a][2], w[a][3]);
+                for (int a = 0; a < 2; ++a)
+                    *reinterpret_cast<float2*>(MW + (r0 + a) * MP + s0) = make_float2(w[a][0], w[a][1]);
             }
             __syncthreads();
             if (tid < tasks) {   // X_ij = -X_ii W_ij
-                float xo[4][4];
-#pragma unroll
-                for (int a = 0; a < 4; ++a)
-#pragma unroll
-                    for (int c2 = 0; c2 < 4; ++c2) xo[a][c2] = 0.f;
+                float xo[2][2] = {{0.f, 0.f}, {0.f, 0.f}};
                 const float* xt = XT + bi * 16 * XS;
 #pragma unroll 4
                 for (int x = 0; x < 16; ++x) {
-                    float xi[4], wv[4];
-                    ld4(xt + x * XS + (r0 - 16 * bi), xi);
-                    ld4(MW + (16 * bi + x) * MP + s0, wv);
-#pragma unroll
-                    for (int a = 0; a < 4; ++a)
-#pragma unroll
-                        for (int c2 = 0; c2 < 4; ++c2) xo[a][c2] = fmaf(xi[a], wv[c2], xo[a][c2]);
+                    const float2 xi = *reinterpret_cast<const float2*>(xt + x * XS + (r0 - 16 * bi));
+                    const float2 wv = *reinterpret_cast<const float2*>(MW + (16 * bi + x) * MP + s0);
+                    xo[0][0] = fmaf(xi.x, wv.x, xo[0][0]);
+                    xo[0][1] = fmaf(xi.x, wv.y, xo[0][1]);
+                    xo[1][0] = fmaf(xi.y, wv.x, xo[1][0]);
+                    xo[1][1] = fmaf(xi.y, wv.y, xo[1][1]);
                 }
 #pragma unroll
-                for (int a = 0; a < 4; ++a) st4(MX + (r0 + a) * MP + s0, -xo[a][0], -xo[a][1], -xo[a][2], -xo[a][3]);
+                for (int a = 0; a < 2; ++a)
+                    *reinterpret_cast<float2*>(MX + (r0 + a) * MP + s0) = make_float2(-xo[a][0], -xo[a][1]);
             }
             __syncthreads();
         }
