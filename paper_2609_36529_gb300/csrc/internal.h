@@ -26,7 +26,7 @@ struct FwdPlan {
                          // tiles, where sGLA stores V): fp32 [B,T,H,dv], or token tiles
     size_t A2;           // bf16 [B,H,NT,2,128,64] [T; A T] hi and lo tiles (tensor-core path)
     size_t coef;         // fp32 [B,H,NT,3*64*E+16] per-row coefficients (tensor-core path)
-    size_t BT;           // bf16 [B,H,NT,4,64,64] A^T, T^T hi/lo (tensor-core backward)
+    size_t BT;           // bf16 [B,H,NT,4,64,64] A, T hi/lo row-major (tensor-core backward)
     int tcb;             // 1: the backward recurrence runs on tensor cores
     int ck_tiles;        // 1: state checkpoints (forward S, backward dS) are stored as bf16
                          //    hi/lo pairs: per (b,h,chunk,e) a row-major [dk][dv] hi matrix
@@ -73,7 +73,7 @@ cudaError_t launch_gate_cumsum(const tla_problem& p, const FwdPlan& fp, const ch
                                cudaStream_t s);
 cudaError_t launch_chunk_prep(const tla_problem& p, const float* G, float* A, float* N,
                               __nv_bfloat16* A2, float* coef, __nv_bfloat16* BT, cudaStream_t s);
-// Per-chunk preparation of the tensor-core path (A, N, [T; A T], [A^T; T^T], coefficients).
+// Per-chunk preparation of the tensor-core path (A, N, [T; A T], [A; T], coefficients).
 cudaError_t launch_chunk_prep_tc(const tla_problem& p, const FwdPlan& fp, char* ws, int* err,
                                  cudaStream_t s);
 // Tensor-core chunk-parallel gradients (requires the tensor-core backward recurrence).

@@ -194,15 +194,15 @@ chunk_prep_kernel(const Tin* __restrict__ q, const Tin* __restrict__ k, const Ti
         }
     }
     if (BTout) {
-        // Operands of the tensor-core backward recurrence as bf16 pairs, 64 x 64 each:
-        // [A^T hi | A^T lo | T^T hi | T^T lo], A^T[r][s] = A[s][r], T^T[r][s] = T[s][r].
+        // Operands of the tensor-core backward recurrence as bf16 pairs, 64 x 64 each,
+        // row-major: [A hi | A lo | T hi | T lo] (read there as the MN-major A^T and T^T).
         const size_t m4 = ((size_t(b) * H + h) * NT + c) * (4 * kChunk * kChunk);
         for (int i = tid; i < kChunk * kChunk; i += blockDim.x) {
-            const int r = i >> 6, s = i & 63;   // element (r, s) of the transposes
+            const int r = i >> 6, s = i & 63;   // element (r, s) of A and T
             float at = 0.f, tt = 0.f;
-            if (s >= r) {
-                at = As[s * 65 + r];
-                tt = (use_delta ? Xs[s * 65 + r] : (s == r ? 1.f : 0.f)) * bs[r];
+            if (r >= s) {
+                at = As[r * 65 + s];
+                tt = (use_delta ? Xs[r * 65 + s] : (r == s ? 1.f : 0.f)) * bs[s];
             }
             const __nv_bfloat16 ah = __float2bfloat16_rn(at), th = __float2bfloat16_rn(tt);
             BTout[m4 + i] = ah;

@@ -13,8 +13,9 @@
 //                                        side by side, N = 2 NE, when that fits one instruction;
 //                                        at E = 16 in two halves of the slices, one after the
 //                                        other, so that P', Y and the slab fit 512 columns)
-//   MMA-0   Y  = A^T dO                 (M=64, N=TV, K=64; A^T hi/lo, dO exact bf16,
-//                                        MN-major as the TMA loads it)
+//   MMA-0   Y  = A^T dO                 (M=64, N=TV, K=64; A^T hi/lo read MN-major from the
+//                                        row-major A tiles, dO exact bf16, MN-major as the
+//                                        TMA loads it)
 //   epi     dU = Y + sum_e w_e (.) P'_e  -> dU hi/lo operand, dU to the workspace
 //   MMA-B'  dRes = T^T dU               (M=64, K=64; both hi/lo, the hi*hi and hi*lo terms in
 //                                        one N = 2 TV product)
@@ -92,7 +93,8 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     constexpr int NE = E * TV;
     constexpr int CB = 3 * 64 * E + 16;
     uint8_t* sKQ = sm;                       // 2 blocks x [K rows | Q rows] x 128 B
-    uint8_t* sBT = sKQ + 4 * kBoxBytes;      // A^T hi, A^T lo, T^T hi, T^T lo (64 x 64 each)
+    uint8_t* sBT = sKQ + 4 * kBoxBytes;      // A hi, A lo, T hi, T lo (64 x 64 each, row-major:
+                                             // the MN-major A operands A^T and T^T)
     uint8_t* sReg = sBT + 4 * kBoxBytes;     // NE * 512 bytes, reused:
     uint8_t* sDh = sReg;                     //   dS' hi / lo: E blocks [dk][TV] (MMA-A',
     uint8_t* sDl = sReg + NE * 256;          //   checkpoint source)
@@ -318,14 +320,15 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         // ---- MMA-A' (P' = K dS') and MMA-0 (Y = A^T dO)
         if (tid == 0) {
             issue_pa(0);
-            const uint32_t id0 = idesc_bf16_f32(64, TV, 0, 1);
+            const uint32_t id0 = idesc_bf16_f32(64, TV, 1, 1);
             const uint64_t o0 = smem_desc(smem_u32(sdO), blk_bytes<TV>(), 16 * TV, kSwz);
-            const uint64_t t0d = smem_desc(smem_u32(sBT), 16, 1024);
+            // A^T MN-major: K = the rows of A (16 per step, 2048 bytes), M = its 64 columns
+            const uint64_t t0d = smem_desc(smem_u32(sBT), 2 * kBoxBytes, 1024);
 #pragma unroll
             for (int ks = 0; ks < 4; ++ks) {
                 const uint64_t bd = desc_add(o0, ks * 32 * TV);
-                umma_bf16(tY, desc_add(t0d, ks * 32), bd, id0, ks > 0 ? 1u : 0u);
-                umma_bf16(tY, desc_add(t0d, kBoxBytes + ks * 32), bd, id0, 1u);
+                umma_bf16(tY, desc_add(t0d, ks * 2048), bd, id0, ks > 0 ? 1u : 0u);
+                umma_bf16(tY, desc_add(t0d, kBoxBytes + ks * 2048), bd, id0, 1u);
             }
             umma_commit(&bar_mma);
             issue_ckpt(c);   // the dS' blocks were completed before the last barrier
@@ -425,14 +428,14 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         if (tid == 0) {
             // T^T_hi [dU_hi | dU_lo] (N = 2 TV: the lo block is the next swizzle atom, TV * 128
             // bytes on) into tY columns [0, 2 TV), and T^T_lo dU_hi into [0, TV)
-            const uint32_t idb2 = idesc_bf16_f32(64, 2 * TV, 0, 1);
-            const uint32_t idb = idesc_bf16_f32(64, TV, 0, 1);
-            const uint64_t t0d = smem_desc(smem_u32(sBT), 16, 1024);
+            const uint32_t idb2 = idesc_bf16_f32(64, 2 * TV, 1, 1);
+            const uint32_t idb = idesc_bf16_f32(64, TV, 1, 1);
+            const uint64_t t0d = smem_desc(smem_u32(sBT), 2 * kBoxBytes, 1024);   // T^T MN-major
             const uint64_t u0 = smem_desc(smem_u32(sUh), TV * 128, 16 * TV, kSwz);
 #pragma unroll
             for (int ks = 0; ks < 4; ++ks) {
-                const uint64_t th = desc_add(t0d, 2 * kBoxBytes + ks * 32);
-                const uint64_t tl = desc_add(t0d, 3 * kBoxBytes + ks * 32);
+                const uint64_t th = desc_add(t0d, 2 * kBoxBytes + ks * 2048);
+                const uint64_t tl = desc_add(t0d, 3 * kBoxBytes + ks * 2048);
                 const uint64_t uh = desc_add(u0, ks * 32 * TV);
                 umma_bf16(tY, th, uh, idb2, ks > 0 ? 1u : 0u);
                 umma_bf16(tY, tl, uh, idb, 1u);

@@ -8,7 +8,8 @@
 //                                    off-diagonal blocks by distance (Eq. joint-solve)
 //   T = N diag(beta) (sGLA: diag(beta)), A T
 // and writes A and N (fp32), the bf16 hi/lo tiles [T; A T] (forward recurrence) and
-// [A^T; T^T] (backward recurrence), and the per-row coefficient block
+// [A; T] (backward recurrence, which reads them as the MN-major operands A^T and T^T), and
+// the per-row coefficient block
 // [k'_e gamma_e | q'_e gamma_e | k'_e gamma^C_e / gamma_e | gamma^C_e] (slice-major).
 #include "common.cuh"
 #include "internal.h"
@@ -362,8 +363,9 @@ chunk_prep_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     }
     __syncthreads();   // every matrix slot is free from here
     // images of the two tile blocks in their global layout (bf16 row-major 64-wide rows):
-    // [T; A T] hi (128 x 64) then lo, and [A^T hi, A^T lo, T^T hi, T^T lo] (64 x 64 each),
-    // built in slots 0-3 and written by two bulk copies
+    // [T; A T] hi (128 x 64) then lo, and [A hi, A lo, T hi, T lo] (64 x 64 each), built in
+    // slots 0-3 (each thread writes its rows: no transposed stores) and written by two bulk
+    // copies
     __nv_bfloat16* stA2 = reinterpret_cast<__nv_bfloat16*>(sm);
     __nv_bfloat16* stBT = stA2 + 4 * 64 * 64;
 #pragma unroll
@@ -374,10 +376,10 @@ chunk_prep_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     }
     if (p.BTout) {
 #pragma unroll
-        for (int c2 = 0; c2 < 4; ++c2) {
-            const int o = (S0 + c2) * 64 + R0;
-            put4(stBT + o, stBT + 4096 + o, Av[0][c2], Av[1][c2], Av[2][c2], Av[3][c2]);
-            put4(stBT + 8192 + o, stBT + 12288 + o, Tv[0][c2], Tv[1][c2], Tv[2][c2], Tv[3][c2]);
+        for (int a = 0; a < 4; ++a) {
+            const int o = (R0 + a) * 64 + S0;
+            put4(stBT + o, stBT + 4096 + o, Av[a][0], Av[a][1], Av[a][2], Av[a][3]);
+            put4(stBT + 8192 + o, stBT + 12288 + o, Tv[a][0], Tv[a][1], Tv[a][2], Tv[a][3]);
         }
     }
     fence_proxy_async_smem();
