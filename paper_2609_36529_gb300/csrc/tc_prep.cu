@@ -1,11 +1,14 @@
-// Per-chunk preparation for the tensor-core path (bf16 inputs, dk = 128).
+// Per-chunk preparation for the tensor-core path (bf16 inputs, d_k = 128, or 64 with the
+// key/query boxes zero-filled past it).
 // One CTA of 8 warps per (b, h, chunk) computes, Appendix A:
 //   K K^T and Q K^T                  one UMMA [K; Q] K^T on the TMA key/query tile
 //   R, R' element by element         exp of non-positive log-decay differences (Eq. joint-gram)
 //   A = Q K^T (.) R' (lower incl. diagonal), L = tril(diag(beta)(K K^T (.) R), -1)
 //   N = (I + L)^{-1}                 blocked: the four 16 x 16 diagonal blocks by forward
 //                                    substitution (one warp each, registers only), then the
-//                                    off-diagonal blocks by distance (Eq. joint-solve)
+//                                    off-diagonal blocks in two levels (Eq. joint-solve):
+//                                    blocks (1,0) and (3,2), then the lower-left 32 x 32
+//                                    block from the two 32 x 32 diagonal blocks
 //   T = N diag(beta) (sGLA: diag(beta)), A T
 // and writes A and N (fp32), the bf16 hi/lo tiles [T; A T] (forward recurrence) and
 // [A; T] (backward recurrence, which reads them as the MN-major operands A^T and T^T), and
@@ -256,7 +259,7 @@ chunk_prep_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     __syncthreads();
 
     // ---- N = (I + L)^{-1} (Eq. joint-solve): the four 16 x 16 diagonal blocks by forward
-    // substitution (warps 0-3, lane = column), then the off-diagonal blocks by distance
+    // substitution (warps 0-3, lane = column), then the off-diagonal blocks in two levels
     if (p.use_delta) {
         if (warp < 4 && lane < 16) {
             // column s2 of the block's inverse: x_r = delta_{r,s2} - sum_{j<r} L_rj x_j, each
@@ -283,13 +286,15 @@ chunk_prep_tc_kernel(const __grid_constant__ CUtensorMap map_k,
             if ((s2 >> 4) > (r >> 4)) MX[r * MP + s2] = 0.f;
         }
         __syncthreads();
-        for (int dist = 1; dist < 4; ++dist) {
-            // 2 x 2 blocks of the 16 x 16 blocks (i, i - dist): 64 threads per block, so that
-            // 192 / 128 / 64 threads share the work of the three distances
-            const int tasks = (4 - dist) * 64;
-            const int bi = dist + (tid >> 6), bj = bi - dist;
+        // Off-diagonal blocks in two levels (2 x 2 register blocks, each entry's sum in order):
+        // level 1 the 16 x 16 blocks (1,0) and (3,2), X_ij = -X_ii (L_ij X_jj) (128 threads);
+        // level 2 the lower-left 32 x 32 block, N21 = -N22 (L21 N11), N11 and N22 the 32 x 32
+        // diagonal blocks, complete after level 1 (256 threads) -- a dependent depth of 96
+        // multiply-adds instead of 144 by distance.
+        {
+            const int bi = 1 + 2 * (tid >> 6), bj = bi - 1;
             const int r0 = 16 * bi + 2 * ((tid >> 3) & 7), s0 = 16 * bj + 2 * (tid & 7);
-            if (tid < tasks) {   // W_ij = sum_{k=j}^{i-1} L_ik X_kj
+            if (tid < 128) {   // W = L_ij X_jj
                 float w[2][2] = {{0.f, 0.f}, {0.f, 0.f}};
 #pragma unroll 4
                 for (int x = 16 * bj; x < 16 * bi; ++x) {
@@ -305,7 +310,7 @@ chunk_prep_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                     *reinterpret_cast<float2*>(MW + (r0 + a) * MP + s0) = make_float2(w[a][0], w[a][1]);
             }
             __syncthreads();
-            if (tid < tasks) {   // X_ij = -X_ii W_ij
+            if (tid < 128) {   // X_ij = -X_ii W
                 float xo[2][2] = {{0.f, 0.f}, {0.f, 0.f}};
                 const float* xt = XT + bi * 16 * XS;
 #pragma unroll 4
@@ -321,6 +326,37 @@ chunk_prep_tc_kernel(const __grid_constant__ CUtensorMap map_k,
                 for (int a = 0; a < 2; ++a)
                     *reinterpret_cast<float2*>(MX + (r0 + a) * MP + s0) = make_float2(-xo[a][0], -xo[a][1]);
             }
+            __syncthreads();
+        }
+        {
+            const int i0 = 2 * (tid >> 4), j0 = 2 * (tid & 15);   // rows 32 + i0.., columns j0..
+            float w[2][2] = {{0.f, 0.f}, {0.f, 0.f}};
+#pragma unroll 4
+            for (int k = j0; k < 32; ++k) {   // W = L21 N11 (N11 lower triangular)
+                const float2 l = *reinterpret_cast<const float2*>(LT + k * MP + 32 + i0);
+                const float2 nv = *reinterpret_cast<const float2*>(MX + k * MP + j0);
+                w[0][0] = fmaf(l.x, nv.x, w[0][0]);
+                w[0][1] = fmaf(l.x, nv.y, w[0][1]);
+                w[1][0] = fmaf(l.y, nv.x, w[1][0]);
+                w[1][1] = fmaf(l.y, nv.y, w[1][1]);
+            }
+#pragma unroll
+            for (int a = 0; a < 2; ++a)
+                *reinterpret_cast<float2*>(MW + (32 + i0 + a) * MP + j0) = make_float2(w[a][0], w[a][1]);
+            __syncthreads();
+            float xo[2][2] = {{0.f, 0.f}, {0.f, 0.f}};
+#pragma unroll 4
+            for (int k = 0; k <= i0 + 1; ++k) {   // N21 = -N22 W (N22 lower triangular)
+                const float n0 = MX[(32 + i0) * MP + 32 + k], n1 = MX[(33 + i0) * MP + 32 + k];
+                const float2 wv = *reinterpret_cast<const float2*>(MW + (32 + k) * MP + j0);
+                xo[0][0] = fmaf(n0, wv.x, xo[0][0]);
+                xo[0][1] = fmaf(n0, wv.y, xo[0][1]);
+                xo[1][0] = fmaf(n1, wv.x, xo[1][0]);
+                xo[1][1] = fmaf(n1, wv.y, xo[1][1]);
+            }
+#pragma unroll
+            for (int a = 0; a < 2; ++a)
+                *reinterpret_cast<float2*>(MX + (32 + i0 + a) * MP + j0) = make_float2(-xo[a][0], -xo[a][1]);
             __syncthreads();
         }
         for (int i = tid; i < 64 * 16; i += kThreads) {
