@@ -279,9 +279,24 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         }
     };
 
+    // MMA-0 of the chunk whose A^T/T^T and dO tiles are in shared memory (thread 0): Y = A^T dO
+    auto issue_y = [&]() {
+        const uint32_t id0 = idesc_bf16_f32(64, TV, 1, 1);
+        const uint64_t o0 = smem_desc(smem_u32(sdO), blk_bytes<TV>(), 16 * TV, kSwz);
+        // A^T MN-major: K = the rows of A (16 per step, 2048 bytes), M = its 64 columns
+        const uint64_t t0d = smem_desc(smem_u32(sBT), 2 * kBoxBytes, 1024);
+#pragma unroll
+        for (int ks = 0; ks < 4; ++ks) {
+            const uint64_t bd = desc_add(o0, ks * 32 * TV);
+            umma_bf16(tY, desc_add(t0d, ks * 2048), bd, id0, ks > 0 ? 1u : 0u);
+            umma_bf16(tY, desc_add(t0d, kBoxBytes + ks * 2048), bd, id0, 1u);
+        }
+    };
+
     bool failed = false;
     uint32_t mma_phase = 0;
     int pending_mma = 0;
+    bool y_early = false;   // thread 0: the next chunk's MMA-0 issued, not yet committed
     bool scaled = true;   // the slab already holds gamma^C-scaled values for the current chunk
     if (tid == 0) {
         issue_kq(nct - 1);
@@ -317,20 +332,13 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         if (__syncthreads_or(!ok)) { failed = true; break; }
         tc_fence_after();
 
-        // ---- MMA-A' (P' = K dS') and MMA-0 (Y = A^T dO)
+        // ---- MMA-A' (P' = K dS') and MMA-0 (Y = A^T dO; issued at the end of the previous
+        // chunk, off the chain, except for the first); one commit covers both
         if (tid == 0) {
+            if (!y_early) issue_y();
             issue_pa(0);
-            const uint32_t id0 = idesc_bf16_f32(64, TV, 1, 1);
-            const uint64_t o0 = smem_desc(smem_u32(sdO), blk_bytes<TV>(), 16 * TV, kSwz);
-            // A^T MN-major: K = the rows of A (16 per step, 2048 bytes), M = its 64 columns
-            const uint64_t t0d = smem_desc(smem_u32(sBT), 2 * kBoxBytes, 1024);
-#pragma unroll
-            for (int ks = 0; ks < 4; ++ks) {
-                const uint64_t bd = desc_add(o0, ks * 32 * TV);
-                umma_bf16(tY, desc_add(t0d, ks * 2048), bd, id0, ks > 0 ? 1u : 0u);
-                umma_bf16(tY, desc_add(t0d, kBoxBytes + ks * 2048), bd, id0, 1u);
-            }
             umma_commit(&bar_mma);
+            y_early = false;
             issue_ckpt(c);   // the dS' blocks were completed before the last barrier
         }
         pending_mma = 1;
@@ -534,7 +542,13 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         if (__syncthreads_or(!ok)) { failed = true; break; }
         pending_mma = 0;
         tc_fence_after();
-        if (tid == 0 && c > 0) issue_kq(c - 1);
+        if (tid == 0 && c > 0) {
+            issue_kq(c - 1);
+            // chunk c-1's MMA-0: its tiles have arrived (bar_av above), and Y is free (this
+            // chunk's dRes was read before MMA-C'); it runs under the operand staging below
+            issue_y();
+            y_early = true;
+        }
 
         if (c > 0) {
             stage_operand(c - 1);   // its gamma^C scaling follows the next MMA-A' issue
@@ -561,6 +575,10 @@ bwd_recurrence_tc_kernel(const __grid_constant__ CUtensorMap map_k,
     if (failed && tid == 0) {
         record_device_error(p.err, TLA_ERR_TIMEOUT);
         if (pending_mma) mbar_wait(&bar_mma, mma_phase ^ 1);
+        if (y_early) {   // an MMA-0 issued ahead and not yet committed
+            umma_commit(&bar_mma);
+            mbar_wait(&bar_mma, mma_phase);
+        }
     }
     if (tid == 0) bulk_wait_all();
     tc_fence_before();
