@@ -634,7 +634,7 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         for (int which = 0; which < 2; ++which) {
             uint64_t* bar = &bar_q[2 * j + which];
             mbar_arrive_expect_tx(bar, 32768);   // [hi | lo][128][64 columns]
-            tma_load_4d(quarter(which, j), which ? &map_ds : &map_s, bar, 64 * j, 0, int(sbase + e), 0);
+            tma_load_4d_once(quarter(which, j), which ? &map_ds : &map_s, bar, 64 * j, 0, int(sbase + e), 0);
             pend |= 1u << (2 * j + which);
         }
         pend_slice = e;
