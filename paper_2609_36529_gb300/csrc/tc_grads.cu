@@ -233,17 +233,17 @@ bwd_chunk_grads_tc_kernel(const __grid_constant__ CUtensorMap map_k,
         // tensor loads and the token-tile copies is announced here, before any copy starts
         mbar_arrive_expect_tx(&bar_ld, 4 * kBoxBytes + nb * kBoxBytes + 3 * tt + (p.use_delta ? tt : 0));
         for (int j = 0; j < 2; ++j) {
-            tma_load_4d(sKQ + j * 2 * kBoxBytes, &map_k, &bar_ld, 64 * j, h, t0, b);
-            tma_load_4d(sKQ + j * 2 * kBoxBytes + kBoxBytes, &map_q, &bar_ld, 64 * j, h, t0, b);
+            tma_load_4d_once(sKQ + j * 2 * kBoxBytes, &map_k, &bar_ld, 64 * j, h, t0, b);
+            tma_load_4d_once(sKQ + j * 2 * kBoxBytes + kBoxBytes, &map_q, &bar_ld, 64 * j, h, t0, b);
         }
-        for (int j = 0; j < nb; ++j) tma_load_4d(sB + j * 2 * kBoxBytes, &map_do, &bar_ld, 64 * j, h, t0, b);
-        bulk_load(sUh, reinterpret_cast<const uint8_t*>(p.Ubuf) + ci * tt, tt, &bar_ld);
-        bulk_load(scr, reinterpret_cast<const uint8_t*>(p.dUbuf) + ci * tt, tt, &bar_ld);
-        bulk_load(scr + tt, reinterpret_cast<const uint8_t*>(p.Rbuf) + ci * tt, tt, &bar_ld);
+        for (int j = 0; j < nb; ++j) tma_load_4d_once(sB + j * 2 * kBoxBytes, &map_do, &bar_ld, 64 * j, h, t0, b);
+        bulk_load_once(sUh, reinterpret_cast<const uint8_t*>(p.Ubuf) + ci * tt, tt, &bar_ld);
+        bulk_load_once(scr, reinterpret_cast<const uint8_t*>(p.dUbuf) + ci * tt, tt, &bar_ld);
+        bulk_load_once(scr + tt, reinterpret_cast<const uint8_t*>(p.Rbuf) + ci * tt, tt, &bar_ld);
         if (p.use_delta) {
             const uint8_t* g = reinterpret_cast<const uint8_t*>(p.dRbuf) + ci * tt;
-            for (int j = 0; j < nb; ++j) bulk_load(sB + j * 16384 + 8192, g + j * 8192, 8192, &bar_ld);
-            bulk_load(sRlo, g + T64, T64, &bar_ld);
+            for (int j = 0; j < nb; ++j) bulk_load_once(sB + j * 16384 + 8192, g + j * 8192, 8192, &bar_ld);
+            bulk_load_once(sRlo, g + T64, T64, &bar_ld);
         }
         bulk_prefetch_l2(gS + sbase * slab_bytes, slab_bytes);
         if (p.use_delta) bulk_prefetch_l2(p.Nmat + ((size_t(b) * H + h) * NT + c) * (64 * 64), kNBytes);
