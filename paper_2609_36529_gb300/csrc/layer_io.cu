@@ -26,6 +26,7 @@ namespace {
 constexpr int kThreads = 256;
 constexpr int kFwdRun = 128;   // tokens per CTA of the prologue forward
 constexpr int kSeg = 256;      // tokens per CTA of the prologue backward
+constexpr int kBwdGroup = 2;   // tokens whose row sums the prologue backward reduces together
 constexpr int kGateTile = 64;  // (token, head) rows per CTA of the output gate
 
 
@@ -103,6 +104,14 @@ __device__ __forceinline__ float warp_sum(float x) {
 #pragma unroll
     for (int o = 16; o >= 1; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
     return x;
+}
+// warp_sum of N values at once, their shuffles interleaved (each value summed in warp_sum's order).
+template <int N>
+__device__ __forceinline__ void warp_sum_n(float (&v)[N]) {
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1)
+#pragma unroll
+        for (int i = 0; i < N; ++i) v[i] += __shfl_xor_sync(0xffffffffu, v[i], o);
 }
 
 // Layout of the prologue kernels: a CTA of four warps takes one run of tokens of one
@@ -335,73 +344,101 @@ __device__ __forceinline__ void prologue_bwd_qkv(const tla_prologue_args& a, con
         dxw[i][0] = dxw[i][1] = dxw[i][2] = dxw[i][3] = 0.f;
     }
     const int tl = t1 + 3, tv = min(tl, T), te = min(t1, T);
+    const bool nrm = g != 2;   // q and k are L2-normalised, v is not
     for (int tb = t0; tb < tl; tb += 4) {
-        float xb[4][4], gb[4][4];
+        // rows t-3 .. t+3 of the batch's four tokens t = tb .. tb+3: win[i .. i+3] are token
+        // i's convolution taps
+        float win[7][4], gb[4][4];
+#pragma unroll
+        for (int i = 0; i < 3; ++i)
+#pragma unroll
+            for (int u = 0; u < 4; ++u) win[i][u] = pw[i][u];
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
             if (m.act && tb + i < tv) {
-                ld4<VEC>(pP + (tb + i) * sP, xb[i]);
+                ld4<VEC>(pP + (tb + i) * sP, win[3 + i]);
                 ld4<VEC>(pG + (tb + i) * sG, gb[i]);
             } else {
 #pragma unroll
-                for (int u = 0; u < 4; ++u) xb[i][u] = gb[i][u] = 0.f;
+                for (int u = 0; u < 4; ++u) win[3 + i][u] = gb[i][u] = 0.f;
+            }
+        }
+        // The tokens are independent up to the weight sums: a group's activations first, then
+        // its row sums together (interleaved shuffles), then its gradients; no branch per
+        // token, so that their latencies overlap.  Tokens at or past tv give dx = 0.
+        float dwin[7][4];   // pre-activation gradients of t-3 .. t+3
+#pragma unroll
+        for (int i = 0; i < 3; ++i)
+#pragma unroll
+            for (int u = 0; u < 4; ++u) dwin[i][u] = dxw[i][u];
+#pragma unroll
+        for (int i0 = 0; i0 < 4; i0 += kBwdGroup) {
+            float fd[kBwdGroup][4], y[kBwdGroup][4], rs[2 * kBwdGroup];   // fd = d silu(x) / dx
+#pragma unroll
+            for (int j = 0; j < kBwdGroup; ++j) {
+                const int i = i0 + j;
+                float ss = 0.f, yd = 0.f;
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    float v = w[0][u] * win[i][u];
+                    v = fmaf(w[1][u], win[i + 1][u], v);
+                    v = fmaf(w[2][u], win[i + 2][u], v);
+                    v = fmaf(w[3][u], win[i + 3][u], v);
+                    const float sgv = sigm(v);
+                    y[j][u] = v * sgv;
+                    fd[j][u] = sgv * (1.f + v * (1.f - sgv));
+                    ss = fmaf(y[j][u], y[j][u], ss);
+                    yd = fmaf(y[j][u], gb[i][u], yd);
+                }
+                rs[j] = ss;
+                rs[kBwdGroup + j] = yd;
+            }
+            if (nrm) warp_sum_n(rs);
+#pragma unroll
+            for (int j = 0; j < kBwdGroup; ++j) {
+                const int i = i0 + j, t = tb + i;
+                float dy[4] = {gb[i][0], gb[i][1], gb[i][2], gb[i][3]};
+                if (nrm) {   // through u = y / n:  (dy - u (u . dy)) / n
+                    const float r = rsqrtf(rs[j] + a.eps), kk = r * r * rs[kBwdGroup + j];
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) dy[u] = (dy[u] - y[j][u] * kk) * r;
+                }
+                const bool live = t < tv, own = t < t1;
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const float dx = dy[u] * fd[j][u];
+                    dwin[3 + i][u] = live ? dx : 0.f;
+                    const float dxo = own ? dx : 0.f;   // the conv-weight sums take the run's own tokens
+                    dw[0][u] = fmaf(dxo, win[i][u], dw[0][u]);
+                    dw[1][u] = fmaf(dxo, win[i + 1][u], dw[1][u]);
+                    dw[2][u] = fmaf(dxo, win[i + 2][u], dw[2][u]);
+                    dw[3][u] = fmaf(dxo, win[i + 3][u], dw[3][u]);
+                }
             }
         }
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
-            const int t = tb + i;
-            float dx[4] = {0.f, 0.f, 0.f, 0.f};
-            if (t < tv) {
-                float x[4], sg[4], y[4], ss = 0.f, yd = 0.f;
-#pragma unroll
-                for (int u = 0; u < 4; ++u) {
-                    float v = w[0][u] * pw[0][u];
-                    v = fmaf(w[1][u], pw[1][u], v);
-                    v = fmaf(w[2][u], pw[2][u], v);
-                    v = fmaf(w[3][u], xb[i][u], v);
-                    x[u] = v;
-                    sg[u] = sigm(v);
-                    y[u] = v * sg[u];
-                    ss = fmaf(y[u], y[u], ss);
-                    yd = fmaf(y[u], gb[i][u], yd);
-                }
-                float dy[4] = {gb[i][0], gb[i][1], gb[i][2], gb[i][3]};
-                if (g != 2) {   // through u = y / n:  (dy - u (u . dy)) / n
-                    const float r = rsqrtf(warp_sum(ss) + a.eps), kk = r * r * warp_sum(yd);
-#pragma unroll
-                    for (int u = 0; u < 4; ++u) dy[u] = (dy[u] - y[u] * kk) * r;
-                }
-#pragma unroll
-                for (int u = 0; u < 4; ++u) dx[u] = dy[u] * sg[u] * (1.f + x[u] * (1.f - sg[u]));
-                if (t < t1) {
-#pragma unroll
-                    for (int u = 0; u < 4; ++u) {
-                        dw[0][u] = fmaf(dx[u], pw[0][u], dw[0][u]);
-                        dw[1][u] = fmaf(dx[u], pw[1][u], dw[1][u]);
-                        dw[2][u] = fmaf(dx[u], pw[2][u], dw[2][u]);
-                        dw[3][u] = fmaf(dx[u], xb[i][u], dw[3][u]);
-                    }
-                }
-            }
-            const int tp = t - 3;   // dP of token t - 3 reads dx of t - 3 .. t
+            const int tp = tb + i - 3;   // dP of token t - 3 reads dx of t - 3 .. t
             if (m.act && tp >= t0 && tp < te) {
                 float d[4];
 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
-                    float v = w[0][u] * dx[u];
-                    v = fmaf(w[1][u], dxw[2][u], v);
-                    v = fmaf(w[2][u], dxw[1][u], v);
-                    v = fmaf(w[3][u], dxw[0][u], v);
+                    float v = w[0][u] * dwin[i + 3][u];
+                    v = fmaf(w[1][u], dwin[i + 2][u], v);
+                    v = fmaf(w[2][u], dwin[i + 1][u], v);
+                    v = fmaf(w[3][u], dwin[i][u], v);
                     d[u] = v;
                 }
                 st4<VEC>(pdP + tp * sP, d);
             }
+        }
+#pragma unroll
+        for (int i = 0; i < 3; ++i)
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
-                pw[0][u] = pw[1][u]; pw[1][u] = pw[2][u]; pw[2][u] = xb[i][u];
-                dxw[0][u] = dxw[1][u]; dxw[1][u] = dxw[2][u]; dxw[2][u] = dx[u];
+                pw[i][u] = win[4 + i][u];
+                dxw[i][u] = dwin[4 + i][u];
             }
-        }
     }
     if (m.act)
 #pragma unroll
@@ -450,66 +487,87 @@ __device__ __forceinline__ void prologue_bwd_small(const tla_prologue_args& a, c
         }
     const int tl = t1 + 3, tv = min(tl, T), te = min(t1, T);
     for (int tb = t0; tb < tl; tb += 4) {
-        float xb[4][2], gb[4][2];
+        // as in prologue_bwd_qkv: rows t-3 .. t+3 in win, the four tokens' activations, then
+        // their row sums together, then their gradients, with no branch per token
+        float win[7][2], gb[4][2];
+#pragma unroll
+        for (int i = 0; i < 3; ++i)
+#pragma unroll
+            for (int s = 0; s < 2; ++s) win[i][s] = pw[i][s];
 #pragma unroll
         for (int i = 0; i < 4; ++i)
 #pragma unroll
             for (int s = 0; s < 2; ++s) {
                 const bool ok = act[s] && tb + i < tv;
                 const size_t o = rowE + (tb + i) * sE + col[s];
-                xb[i][s] = ok ? to_f(pP[(tb + i) * sP + 32 * s]) : 0.f;
+                win[3 + i][s] = ok ? to_f(pP[(tb + i) * sP + 32 * s]) : 0.f;
                 gb[i][s] = ok ? to_f(isq[s] ? gq[o] : gk[o]) : 0.f;
             }
+        float sx[4][2], y[4][2], rs[16];   // sx = sigmoid(x); rs: sq, sk, dq, dk of the four tokens
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            float sq = 0.f, sk = 0.f, dq = 0.f, dkk = 0.f;
+#pragma unroll
+            for (int s = 0; s < 2; ++s) {
+                float v = w[0][s] * win[i][s];
+                v = fmaf(w[1][s], win[i + 1][s], v);
+                v = fmaf(w[2][s], win[i + 2][s], v);
+                v = fmaf(w[3][s], win[i + 3][s], v);
+                sx[i][s] = sigm(v);
+                y[i][s] = act[s] ? softplus(v) : 0.f;
+                if (isq[s]) { sq = fmaf(y[i][s], y[i][s], sq); dq = fmaf(y[i][s], gb[i][s], dq); }
+                else { sk = fmaf(y[i][s], y[i][s], sk); dkk = fmaf(y[i][s], gb[i][s], dkk); }
+            }
+            rs[i] = sq;
+            rs[4 + i] = sk;
+            rs[8 + i] = dq;
+            rs[12 + i] = dkk;
+        }
+        warp_sum_n(rs);
+        float dwin[7][2];
+#pragma unroll
+        for (int i = 0; i < 3; ++i)
+#pragma unroll
+            for (int s = 0; s < 2; ++s) dwin[i][s] = dxw[i][s];
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
             const int t = tb + i;
-            float dx[2] = {0.f, 0.f};
-            if (t < tv) {
-                float x[2], y[2], sq = 0.f, sk = 0.f, dq = 0.f, dkk = 0.f;
+            const float rq = rsqrtf(rs[i] + a.eps), rk = rsqrtf(rs[4 + i] + a.eps);
+            const float kq = rq * rq * rs[8 + i], kk = rk * rk * rs[12 + i];
+            const bool live = t < tv, own = t < t1;
 #pragma unroll
-                for (int s = 0; s < 2; ++s) {
-                    float v = w[0][s] * pw[0][s];
-                    v = fmaf(w[1][s], pw[1][s], v);
-                    v = fmaf(w[2][s], pw[2][s], v);
-                    v = fmaf(w[3][s], xb[i][s], v);
-                    x[s] = v;
-                    y[s] = act[s] ? softplus(v) : 0.f;
-                    if (isq[s]) { sq = fmaf(y[s], y[s], sq); dq = fmaf(y[s], gb[i][s], dq); }
-                    else { sk = fmaf(y[s], y[s], sk); dkk = fmaf(y[s], gb[i][s], dkk); }
-                }
-                const float rq = rsqrtf(warp_sum(sq) + a.eps), rk = rsqrtf(warp_sum(sk) + a.eps);
-                const float kq = rq * rq * warp_sum(dq), kk = rk * rk * warp_sum(dkk);
-#pragma unroll
-                for (int s = 0; s < 2; ++s) {
-                    const float r = isq[s] ? rq : rk, k2 = isq[s] ? kq : kk;
-                    dx[s] = act[s] ? (gb[i][s] - y[s] * k2) * r * sigm(x[s]) : 0.f;
-                }
-                if (t < t1)
-#pragma unroll
-                    for (int s = 0; s < 2; ++s) {
-                        dw[0][s] = fmaf(dx[s], pw[0][s], dw[0][s]);
-                        dw[1][s] = fmaf(dx[s], pw[1][s], dw[1][s]);
-                        dw[2][s] = fmaf(dx[s], pw[2][s], dw[2][s]);
-                        dw[3][s] = fmaf(dx[s], xb[i][s], dw[3][s]);
-                    }
+            for (int s = 0; s < 2; ++s) {
+                const float r = isq[s] ? rq : rk, k2 = isq[s] ? kq : kk;
+                const float dx = act[s] ? (gb[i][s] - y[i][s] * k2) * r * sx[i][s] : 0.f;
+                dwin[3 + i][s] = live ? dx : 0.f;
+                const float dxo = own ? dx : 0.f;
+                dw[0][s] = fmaf(dxo, win[i][s], dw[0][s]);
+                dw[1][s] = fmaf(dxo, win[i + 1][s], dw[1][s]);
+                dw[2][s] = fmaf(dxo, win[i + 2][s], dw[2][s]);
+                dw[3][s] = fmaf(dxo, win[i + 3][s], dw[3][s]);
             }
-            const int tp = t - 3;
+        }
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int tp = tb + i - 3;
             if (tp >= t0 && tp < te)
 #pragma unroll
                 for (int s = 0; s < 2; ++s)
                     if (act[s]) {
-                        float v = w[0][s] * dx[s];
-                        v = fmaf(w[1][s], dxw[2][s], v);
-                        v = fmaf(w[2][s], dxw[1][s], v);
-                        v = fmaf(w[3][s], dxw[0][s], v);
+                        float v = w[0][s] * dwin[i + 3][s];
+                        v = fmaf(w[1][s], dwin[i + 2][s], v);
+                        v = fmaf(w[2][s], dwin[i + 1][s], v);
+                        v = fmaf(w[3][s], dwin[i][s], v);
                         pdP[tp * sP + 32 * s] = from_f<Tin>(v);
                     }
+        }
+#pragma unroll
+        for (int i = 0; i < 3; ++i)
 #pragma unroll
             for (int s = 0; s < 2; ++s) {
-                pw[0][s] = pw[1][s]; pw[1][s] = pw[2][s]; pw[2][s] = xb[i][s];
-                dxw[0][s] = dxw[1][s]; dxw[1][s] = dxw[2][s]; dxw[2][s] = dx[s];
+                pw[i][s] = win[4 + i][s];
+                dxw[i][s] = dwin[4 + i][s];
             }
-        }
     }
 #pragma unroll
     for (int s = 0; s < 2; ++s)
