@@ -168,26 +168,36 @@ __device__ __forceinline__ void prologue_fwd_qkv(const tla_prologue_args& a, int
             if (m.act && tb + i < t1) ld4<VEC>(pP + (tb + i) * sP, xb[i]);
             else xb[i][0] = xb[i][1] = xb[i][2] = xb[i][3] = 0.f;
         }
+        // the four tokens' activations, then their row sums together (interleaved shuffles),
+        // then the scaled rows: no branch per token, so that their latencies overlap
+        float y[4][4], rs[4];
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
-            float y[4], ss = 0.f;
+            float ss = 0.f;
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
                 float x = w[0][u] * pw[0][u];
                 x = fmaf(w[1][u], pw[1][u], x);
                 x = fmaf(w[2][u], pw[2][u], x);
                 x = fmaf(w[3][u], xb[i][u], x);
-                y[u] = x * sigm(x);
-                ss = fmaf(y[u], y[u], ss);
+                y[i][u] = x * sigm(x);
+                ss = fmaf(y[i][u], y[i][u], ss);
                 pw[0][u] = pw[1][u]; pw[1][u] = pw[2][u]; pw[2][u] = xb[i][u];
             }
-            if (g != 2) {
-                const float r = rsqrtf(warp_sum(ss) + a.eps);
-#pragma unroll
-                for (int u = 0; u < 4; ++u) y[u] *= r;
-            }
-            if (m.act && tb + i < t1) st4<VEC>(pD + (tb + i) * sD, y);
+            rs[i] = ss;
         }
+        if (g != 2) {   // q and k are L2-normalised, v is not
+            warp_sum_n(rs);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const float r = rsqrtf(rs[i] + a.eps);
+#pragma unroll
+                for (int u = 0; u < 4; ++u) y[i][u] *= r;
+            }
+        }
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+            if (m.act && tb + i < t1) st4<VEC>(pD + (tb + i) * sD, y[i]);
     }
 }
 
@@ -228,28 +238,35 @@ __device__ __forceinline__ void prologue_fwd_small(const tla_prologue_args& a, i
 #pragma unroll
             for (int s = 0; s < 2; ++s)
                 xb[i][s] = (act[s] && tb + i < t1) ? to_f(pP[(tb + i) * sP + 32 * s]) : 0.f;
+        float y[4][2], rs[8];   // rs: sq, sk of the four tokens, reduced together
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
-            float y[2], sq = 0.f, sk = 0.f;
+            float sq = 0.f, sk = 0.f;
 #pragma unroll
             for (int s = 0; s < 2; ++s) {
                 float x = w[0][s] * pw[0][s];
                 x = fmaf(w[1][s], pw[1][s], x);
                 x = fmaf(w[2][s], pw[2][s], x);
                 x = fmaf(w[3][s], xb[i][s], x);
-                y[s] = act[s] ? softplus(x) : 0.f;
-                if (lane + 32 * s < E) sq = fmaf(y[s], y[s], sq);
-                else sk = fmaf(y[s], y[s], sk);
+                y[i][s] = act[s] ? softplus(x) : 0.f;
+                if (lane + 32 * s < E) sq = fmaf(y[i][s], y[i][s], sq);
+                else sk = fmaf(y[i][s], y[i][s], sk);
                 pw[0][s] = pw[1][s]; pw[1][s] = pw[2][s]; pw[2][s] = xb[i][s];
             }
-            const float rq = rsqrtf(warp_sum(sq) + a.eps), rk = rsqrtf(warp_sum(sk) + a.eps);
+            rs[i] = sq;
+            rs[4 + i] = sk;
+        }
+        warp_sum_n(rs);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float rq = rsqrtf(rs[i] + a.eps), rk = rsqrtf(rs[4 + i] + a.eps);
             if (tb + i < t1) {
                 const size_t o = rowE + (tb + i) * sE;
 #pragma unroll
                 for (int s = 0; s < 2; ++s)
                     if (act[s]) {
                         const bool isq = lane + 32 * s < E;
-                        st<Tin>(isq ? a.q2 : a.k2, o + col[s], y[s] * (isq ? rq : rk));
+                        st<Tin>(isq ? a.q2 : a.k2, o + col[s], y[i][s] * (isq ? rq : rk));
                     }
             }
         }
