@@ -111,19 +111,6 @@ __device__ __forceinline__ void tma_load_4d(void* dst, const CUtensorMap* map, u
         : "memory");
 }
 
-// TMA tensor load as tma_load_4d, with the L2 lines marked evict-first: for data read once, so
-// that streaming it does not push out what is still to be read.
-__device__ __forceinline__ void tma_load_4d_once(void* dst, const CUtensorMap* map, uint64_t* bar,
-                                                 int x, int y, int z, int w) {
-    uint64_t pol;
-    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
-    asm volatile(
-        "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
-        " [%0], [%1, {%2, %3, %4, %5}], [%6], %7;" ::"r"(smem_u32(dst)),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(w), "r"(smem_u32(bar)), "l"(pol)
-        : "memory");
-}
-
 // Hint: bring the box at the given coordinates of a 4-d tensor map into L2 (no
 // shared memory, no barrier); a later TMA load of the same box then hits L2.
 __device__ __forceinline__ void tma_prefetch_l2_4d(const CUtensorMap* map, int x, int y, int z, int w) {
@@ -174,17 +161,6 @@ __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wa
 // shared-memory source.
 __device__ __forceinline__ void bulk_wait_read_but_last() {
     asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
-}
-
-// As bulk_load, with the L2 lines marked evict-first (data read once).
-__device__ __forceinline__ void bulk_load_once(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
-    uint64_t pol;
-    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
-    asm volatile(
-        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;" ::"r"(
-            smem_u32(dst)),
-        "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(smem_u32(bar)), "l"(pol)
-        : "memory");
 }
 
 // Hint: bring `bytes` of global memory into L2 (16-byte aligned, size multiple of 16).

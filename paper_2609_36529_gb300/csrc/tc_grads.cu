@@ -69,6 +69,29 @@ struct TcGradArgs {
     int kdim;            // key dimension: 128, or 64 padded to 128 by zero rows (TMA fill)
 };
 
+// Copies of data this kernel reads once (the state and state-gradient slabs, the token
+// tiles), with their L2 lines marked evict-first: streaming them then does not push out the
+// next slice's slabs, which are prefetched into L2 one slice ahead.
+__device__ __forceinline__ void tma_load_4d_once(void* dst, const CUtensorMap* map, uint64_t* bar,
+                                                 int x, int y, int z, int w) {
+    uint64_t pol;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+    asm volatile(
+        "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+        " [%0], [%1, {%2, %3, %4, %5}], [%6], %7;" ::"r"(smem_u32(dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(w), "r"(smem_u32(bar)), "l"(pol)
+        : "memory");
+}
+__device__ __forceinline__ void bulk_load_once(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+    uint64_t pol;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+        " [%0], [%1], %2, [%3], %4;" ::"r"(smem_u32(dst)),
+        "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(smem_u32(bar)), "l"(pol)
+        : "memory");
+}
+
 // 4 x 4 block (rows R0.., columns S0..) of a shared row-major matrix.
 __device__ __forceinline__ void ld4x4(const float* M, int R0, int S0, float (&v)[4][4]) {
 #pragma unroll
