@@ -769,7 +769,7 @@ def run_variants(args, tla, inputs, w, dev, stream, barrier, max_over_ranks, ws_
 
 
 def run_layer_io(args, tla, inputs, w, dev, stream, barrier, max_over_ranks, rank, peaks):
-    """The layer's input path and output gate (Algorithm 4) on the headline's token-heads
+    """The layer's input path and output gate (Algorithm 2) on the headline's token-heads
     (bf16 projection output, K = 4 convolution, fp32 operator output and gradients): device
     time per call and algorithmic bytes (each tensor read or written once) per second."""
     B, T, H, dk, dv, E, K = w.B, w.T, w.H, w.dk, w.dv, w.E, 4

@@ -189,7 +189,7 @@ tla_status tla_decode_step(int B, int H, int dk, int dv, int E, int use_delta, i
 const char *tla_status_string(int status);
 
 /*
- * Layer input path of Algorithm 4 (Appendix A, Input projections): from the
+ * Layer input path of Algorithm 2 (Appendix A, Input projections): from the
  * output P of the one projection GEMM to the operator's inputs.  The GEMMs
  * themselves (W u for P, W_alpha u, W_beta u) are plain GEMMs of the caller.
  * Per (b, t, h), with C = 2 dk + dv + 2 E channels per head ordered
@@ -239,7 +239,7 @@ tla_status tla_layer_prologue_bwd(const tla_prologue_args *a, int grad_dtype, co
                                   size_t workspace_bytes, void *stream);
 
 /*
- * Input projection of Algorithm 4 fused with the input path above (Appendix A, Input
+ * Input projection of Algorithm 2 fused with the input path above (Appendix A, Input
  * projections: one GEMM produces q, k, v, k', q' of every head, then one causal depthwise
  * convolution processes them).  From the normalised layer input u:
  *   P[b,t,h,c] = sum_i u[b,t,i] W[h*C + c, i]      (C = 2 dk + dv + 2 E, [q | k | v | q' | k'])
@@ -271,7 +271,7 @@ typedef struct {
 tla_status tla_layer_projection(const tla_projection_args *a, void *stream);
 
 /*
- * Output gate of Algorithm 4: per (b, t, h) over dv channels
+ * Output gate of Algorithm 2: per (b, t, h) over dv channels
  *   y = o / sqrt(mean(o^2) + eps) * w_norm * sigmoid(z).
  */
 typedef struct {

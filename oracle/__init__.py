@@ -127,7 +127,7 @@ def decode_step(state, q, k, v, q2, k2, g, beta=None, use_delta=True):
 
 
 def projection(u, W, H):
-    """Input projection of Algorithm 4 / Appendix A (Input projections): one GEMM of the
+    """Input projection of Algorithm 2 / Appendix A (Input projections): one GEMM of the
     layer input u [B,T,Dm] with the weight W [H*C, Dm] (rows: head h's channels
     [q|k|v|q'|k'] at h*C..h*C+C-1), P[b,t,h,c] = sum_i u[b,t,i] W[h*C+c, i], in float64
     (the matrix product is the library primitive).  Returns P [B,T,H,C]."""
@@ -138,7 +138,7 @@ def projection(u, W, H):
 
 
 def prologue(P, conv_w, gate_in, gate_bias, A_log, beta_in, dk, dv, E, eps=1e-6):
-    """Layer input path of Algorithm 4: causal depthwise convolution of the projection
+    """Layer input path of Algorithm 2: causal depthwise convolution of the projection
     output P [B,T,H,2dk+dv+2E] (per head [q|k|v|q'|k']) with conv_w [H,C,K], SiLU on
     q,k,v, softplus on q',k', L2 normalisation of q,k,q',k'; log gates
     -exp(A_log) softplus(gate_in + gate_bias) and beta = sigmoid(beta_in).
@@ -180,7 +180,7 @@ def prologue_backward(P, conv_w, gate_in, gate_bias, A_log, beta_in, grads, dk, 
 
 
 def gate_norm(o, z, w_norm, eps=1e-6):
-    """Output gate of Algorithm 4: RMSNorm(o) (weight w_norm [dv]) times sigmoid(z)."""
+    """Output gate of Algorithm 2: RMSNorm(o) (weight w_norm [dv]) times sigmoid(z)."""
     o, z, w_norm = map(_f64, (o, z, w_norm))
     B, T, H, dv = o.shape
     y = np.zeros_like(o)

@@ -503,7 +503,7 @@ void tla_oracle_chunk_forward(int B, int T, int H, int dk, int dv, int E, int us
 }
 
 /* ------------------------------------------------------------------------
- * Layer input path and output gate of Algorithm 4 (and the input-projection
+ * Layer input path and output gate of Algorithm 2 (and the input-projection
  * paragraph of Appendix A): what surrounds the operator in a triadic layer.
  *
  * Input prologue, per (b, t, h), with C = 2 dk + dv + 2 E channels per head in

@@ -1,4 +1,4 @@
-// Activation functions of the layer's input path (Algorithm 4), shared by the
+// Activation functions of the layer's input path (Algorithm 2), shared by the
 // elementwise prologue kernels and the fused projection GEMM epilogue.
 #pragma once
 

@@ -1,4 +1,4 @@
-// Layer input path and output gate of Algorithm 4 (Appendix A, Input projections):
+// Layer input path and output gate of Algorithm 2 (Appendix A, Input projections):
 // the memory-bound steps around the operator, each one kernel per direction.
 //
 // Prologue (per (b, t, h), C = 2 dk + dv + 2 E channels ordered [q | k | v | q' | k']):

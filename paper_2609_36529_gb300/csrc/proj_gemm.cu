@@ -1,4 +1,4 @@
-// Input projection of the layer (Appendix A, Input projections; Algorithm 4): one GEMM
+// Input projection of the layer (Appendix A, Input projections; Algorithm 2): one GEMM
 // produces the q, k, v, q', k' channels of every head,
 //   P[t, h, c] = sum_i u[t, i] W[h C + c, i]      (C = 2 dk + dv + 2 E, channels [q|k|v|q'|k'])
 // on tcgen05 tensor cores, and its epilogue runs the rest of the input path on the

@@ -141,7 +141,7 @@ def packed_lengths(total, mean_len, seed=0, min_len=1):
 
 
 def layer_inputs(B, T, H, dk, dv, E, K=4, dtype="bf16", device="cpu", seed=0):
-    """Inputs of the layer input path and output gate (Algorithm 4), one generator:
+    """Inputs of the layer input path and output gate (Algorithm 2), one generator:
     P ~ N(0,1) [B,T,H,2dk+dv+2E] (dtype), conv_w ~ N(0,1/K) [H,C,K], gate_in ~ N(0,1)
     [B,T,H,E], gate_bias ~ N(1,1) [H,E], A_log ~ N(-1,0.5^2) [H,E], beta_in ~ N(0,1) [B,T,H],
     o ~ N(0,1) [B,T,H,dv] fp32, z ~ N(0,1) [B,T,H,dv] (dtype), w_norm ~ 1 + 0.1 N(0,1) [dv];
@@ -163,7 +163,7 @@ def layer_inputs(B, T, H, dk, dv, E, K=4, dtype="bf16", device="cpu", seed=0):
 
 
 def projection_inputs(B, T, H, dk, dv, E, Dm, K=4, device="cpu", seed=0):
-    """Inputs of the fused input projection (Algorithm 4): the normalised layer input
+    """Inputs of the fused input projection (Algorithm 2): the normalised layer input
     u ~ N(0,1) [B,T,Dm] and the projection weight W ~ N(0, 1/Dm) [H*(2dk+dv+2E), Dm], both
     bf16, then the parameters of layer_inputs (conv_w, gate_in, gate_bias, A_log, beta_in;
     fp32) from the same generator."""

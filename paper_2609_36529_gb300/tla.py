@@ -298,7 +298,7 @@ def tla_version() -> str:
     return lib().tla_version().decode()
 
 
-# --- layer input path and output gate (Algorithm 4)
+# --- layer input path and output gate (Algorithm 2)
 
 def _prologue_args(P, conv_w, gate_in, gate_bias, A_log, beta_in, dk, dv, E, eps, out):
     B, T, H, C = P.shape
@@ -315,7 +315,7 @@ def _prologue_args(P, conv_w, gate_in, gate_bias, A_log, beta_in, dk, dv, E, eps
 
 
 def layer_prologue(P, conv_w, gate_in, gate_bias, A_log, beta_in, dk, dv, E, eps=1e-6):
-    """Input path of Algorithm 4 from the projection output P [B,T,H,2dk+dv+2E] (per head
+    """Input path of Algorithm 2 from the projection output P [B,T,H,2dk+dv+2E] (per head
     [q|k|v|q'|k']): returns q, k, v, q2, k2 (P's dtype), g and beta (fp32)."""
     B, T, H, _ = P.shape
     dev, dt = P.device, P.dtype
@@ -369,7 +369,7 @@ def _gate_args(o, z, w_norm, eps, y):
 
 
 def output_gate(o, z, w_norm, eps=1e-6):
-    """Output gate of Algorithm 4: RMSNorm(o) * w_norm * sigmoid(z), in z's dtype."""
+    """Output gate of Algorithm 2: RMSNorm(o) * w_norm * sigmoid(z), in z's dtype."""
     y = torch.empty(o.shape, dtype=z.dtype, device=o.device)
     a = _gate_args(o, z, w_norm, eps, y)
     _check("tla_output_gate", lib().tla_output_gate(ctypes.byref(a), _stream()))
@@ -390,7 +390,7 @@ def output_gate_bwd(o, z, w_norm, dy, eps=1e-6):
     return out
 
 
-# --- input projection GEMM fused with the input path (Algorithm 4)
+# --- input projection GEMM fused with the input path (Algorithm 2)
 
 def layer_projection(u, W, conv_w, gate_in, gate_bias, A_log, beta_in, dk, dv, E, eps=1e-6,
                      want_P=False):

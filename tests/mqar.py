@@ -1,7 +1,7 @@
 """MQAR capacity smoke study (Section 2.3, Appendix C) with the CUDA kernels under autograd.
 
 A reduced version of the paper's setup: two blocks of vanilla triadic linear attention
-(Algorithm 3: no forgetting, no delta rule, RMSNorm per head on the read-out) and SwiGLU
+(Algorithm 1: no forgetting, no delta rule, RMSNorm per head on the read-out) and SwiGLU
 MLPs, d_model 128, 4 heads of D = 16, E slices.  A sequence holds N key-value pairs, one
 token each (key and value embeddings concatenated), then the N keys in random order as
 read-only queries (key embedding and zeros; their second key is zeroed so they do not

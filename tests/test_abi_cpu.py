@@ -153,7 +153,7 @@ def test_packed_documents_validation(tla):
 
 
 def test_layer_io_validation(tla):
-    """Input prologue and output gate (Algorithm 4): argument checks before any launch."""
+    """Input prologue and output gate (Algorithm 2): argument checks before any launch."""
     L = tla.lib()
     f = ctypes.c_void_p(0x1000)
 
@@ -203,7 +203,7 @@ def test_selftest_limit_checked_on_host(tla):
 
 
 def test_projection_validation(tla):
-    """Fused input projection (Algorithm 4): argument checks before any launch."""
+    """Fused input projection (Algorithm 2): argument checks before any launch."""
     L = tla.lib()
     f = ctypes.c_void_p(0x1000)
 

@@ -1,4 +1,4 @@
-"""Layer input path and output gate (Algorithm 4) through the C ABI against the float64
+"""Layer input path and output gate (Algorithm 2) through the C ABI against the float64
 oracle, and a whole layer forward (prologue -> chunkwise operator -> output gate).
 
 Tolerances: fp32 results max|err| <= 1e-4 * RMS(oracle); results stored in bf16 add

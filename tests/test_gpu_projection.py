@@ -1,4 +1,4 @@
-"""GPU parity of the fused input projection (Algorithm 4; Appendix A, Input projections):
+"""GPU parity of the fused input projection (Algorithm 2; Appendix A, Input projections):
 one tcgen05 GEMM P = u W^T whose epilogue runs the causal convolution, activations, L2
 normalisations, log gates and beta.  Reference: the oracle's float64 projection of the same
 bf16 u and W, then the oracle's input path on P.

@@ -307,7 +307,7 @@ def test_backward_vs_autograd_flat(delta):
                                    err_msg=x)
 
 
-# --- layer input path and output gate (Algorithm 4; Appendix A, Input projections)
+# --- layer input path and output gate (Algorithm 2; Appendix A, Input projections)
 
 def _layer_inputs(seed, B=2, T=37, H=2, dk=8, dv=16, E=3, K=4):
     rng = np.random.default_rng(seed)
@@ -394,7 +394,7 @@ def test_output_gate_matches_library_form_and_autograd():
 
 
 def test_projection_is_the_per_channel_sum():
-    """Input projection of Algorithm 4 (Appendix A, Input projections): every entry of
+    """Input projection of Algorithm 2 (Appendix A, Input projections): every entry of
     P[b,t,h,c] is the explicit sum over the model width of u[b,t,i] W[h C + c, i], head h's
     rows of W in the order [q|k|v|q'|k'] (brute force on a tiny case)."""
     rng = np.random.default_rng(3)
