@@ -72,7 +72,7 @@ BwdPlan plan_bwd(const tla_problem& p);
 cudaError_t launch_gate_cumsum(const tla_problem& p, const FwdPlan& fp, const char* ws, float* G,
                                cudaStream_t s);
 cudaError_t launch_chunk_prep(const tla_problem& p, const float* G, float* A, float* N,
-                              __nv_bfloat16* A2, float* coef, __nv_bfloat16* BT, cudaStream_t s);
+                              cudaStream_t s);
 // Per-chunk preparation of the tensor-core path (A, N, [T; A T], [A; T], coefficients).
 cudaError_t launch_chunk_prep_tc(const tla_problem& p, const FwdPlan& fp, char* ws, int* err,
                                  cudaStream_t s);

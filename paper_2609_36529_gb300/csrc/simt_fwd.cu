@@ -68,9 +68,7 @@ __global__ void __launch_bounds__(256)
 chunk_prep_kernel(const Tin* __restrict__ q, const Tin* __restrict__ k, const Tin* __restrict__ q2,
                   const Tin* __restrict__ k2, const float* __restrict__ G,
                   const float* __restrict__ beta, float* __restrict__ Aout,
-                  float* __restrict__ Nout, __nv_bfloat16* __restrict__ A2out,
-                  float* __restrict__ coef_out, __nv_bfloat16* __restrict__ BTout, int T, int H,
-                  int dk, int E, int use_delta) {
+                  float* __restrict__ Nout, int T, int H, int dk, int E, int use_delta) {
     const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
     const int NT = gridDim.x;
     const int tid = threadIdx.x;
@@ -153,64 +151,6 @@ chunk_prep_kernel(const Tin* __restrict__ q, const Tin* __restrict__ k, const Ti
         }
         for (int i = tid; i < kChunk * kChunk; i += blockDim.x) Nout[mat + i] = Xs[(i >> 6) * 65 + (i & 63)];
     }
-    if (coef_out) {
-        // Per-row coefficients of the tensor-core recurrence, one block per chunk:
-        // [k'_e gamma_e | q'_e gamma_e | k'_e gamma^C_e / gamma_e] as [E][64] each (slice-major),
-        // then gamma^C_e (padded to 16).  Decays are exponentials of non-positive log differences.
-        float* cf = coef_out + ((size_t(b) * H + h) * NT + c) * (3 * kChunk * E + 16);
-        for (int i = tid; i < kChunk * E; i += blockDim.x) {
-            const int e = i / kChunk, r = i % kChunk, ir = r * E + e;
-            const float Gr = Gs[ir], GC = Gs[(n - 1) * E + e];
-            const float gam = expf(Gr);
-            cf[i] = k2s[ir] * gam;
-            cf[kChunk * E + i] = q2s[ir] * gam;
-            cf[2 * kChunk * E + i] = k2s[ir] * expf(GC - Gr);
-        }
-        if (tid < 16) cf[3 * kChunk * E + tid] = tid < E ? expf(Gs[(n - 1) * E + tid]) : 0.f;
-    }
-    if (A2out) {
-        // Operand [T; A T] (128 x 64) of the tensor-core recurrence as a bf16 pair
-        // (hi tile, then lo tile = bf16 of the remainder): T = N diag(beta)
-        // (sGLA: diag(beta)), A T = (Q K^T (.) R') T.
-        const size_t m2 = ((size_t(b) * H + h) * NT + c) * (4 * kChunk * kChunk);
-        for (int i = tid; i < kChunk * kChunk; i += blockDim.x) {
-            const int r = i >> 6, s = i & 63;
-            float t = 0.f, at = 0.f;
-            if (r >= s) {
-                const float bsv = bs[s];
-                t = (use_delta ? Xs[r * 65 + s] : (r == s ? 1.f : 0.f)) * bsv;
-                if (use_delta) {
-                    for (int j = s; j <= r; ++j) at = fmaf(As[r * 65 + j], Xs[j * 65 + s], at);
-                    at *= bsv;
-                } else {
-                    at = As[r * 65 + s] * bsv;
-                }
-            }
-            const __nv_bfloat16 th = __float2bfloat16_rn(t), ath = __float2bfloat16_rn(at);
-            A2out[m2 + i] = th;
-            A2out[m2 + kChunk * kChunk + i] = ath;
-            A2out[m2 + 2 * kChunk * kChunk + i] = __float2bfloat16_rn(t - __bfloat162float(th));
-            A2out[m2 + 3 * kChunk * kChunk + i] = __float2bfloat16_rn(at - __bfloat162float(ath));
-        }
-    }
-    if (BTout) {
-        // Operands of the tensor-core backward recurrence as bf16 pairs, 64 x 64 each,
-        // row-major: [A hi | A lo | T hi | T lo] (read there as the MN-major A^T and T^T).
-        const size_t m4 = ((size_t(b) * H + h) * NT + c) * (4 * kChunk * kChunk);
-        for (int i = tid; i < kChunk * kChunk; i += blockDim.x) {
-            const int r = i >> 6, s = i & 63;   // element (r, s) of A and T
-            float at = 0.f, tt = 0.f;
-            if (r >= s) {
-                at = As[r * 65 + s];
-                tt = (use_delta ? Xs[r * 65 + s] : (r == s ? 1.f : 0.f)) * bs[s];
-            }
-            const __nv_bfloat16 ah = __float2bfloat16_rn(at), th = __float2bfloat16_rn(tt);
-            BTout[m4 + i] = ah;
-            BTout[m4 + kChunk * kChunk + i] = __float2bfloat16_rn(at - __bfloat162float(ah));
-            BTout[m4 + 2 * kChunk * kChunk + i] = th;
-            BTout[m4 + 3 * kChunk * kChunk + i] = __float2bfloat16_rn(tt - __bfloat162float(th));
-        }
-    }
 }
 
 static size_t prep_smem(const tla_problem& p) {
@@ -218,7 +158,7 @@ static size_t prep_smem(const tla_problem& p) {
 }
 
 cudaError_t launch_chunk_prep(const tla_problem& p, const float* G, float* A, float* N,
-                              __nv_bfloat16* A2, float* coef, __nv_bfloat16* BT, cudaStream_t s) {
+                              cudaStream_t s) {
     int NT = (p.T + kChunk - 1) / kChunk;
     dim3 grid(NT, p.H, p.B);
     size_t smem = prep_smem(p);
@@ -228,13 +168,13 @@ cudaError_t launch_chunk_prep(const tla_problem& p, const float* G, float* A, fl
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         kern<<<grid, 256, smem, s>>>((const __nv_bfloat16*)p.q, (const __nv_bfloat16*)p.k,
                                      (const __nv_bfloat16*)p.q2, (const __nv_bfloat16*)p.k2, G,
-                                     p.beta, A, N, A2, coef, BT, p.T, p.H, p.dk, p.E, p.use_delta);
+                                     p.beta, A, N, p.T, p.H, p.dk, p.E, p.use_delta);
     } else {
         auto kern = chunk_prep_kernel<float>;
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         kern<<<grid, 256, smem, s>>>((const float*)p.q, (const float*)p.k, (const float*)p.q2,
-                                     (const float*)p.k2, G, p.beta, A, N, nullptr, nullptr, nullptr,
-                                     p.T, p.H, p.dk, p.E, p.use_delta);
+                                     (const float*)p.k2, G, p.beta, A, N, p.T, p.H, p.dk, p.E,
+                                     p.use_delta);
     }
     prof_after(s);
     return cudaGetLastError();

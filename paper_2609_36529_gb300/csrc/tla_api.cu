@@ -244,8 +244,7 @@ tla_status tla_chunk_fwd(const tla_problem* p, void* workspace, size_t workspace
             e = launch_chunk_prep_tc(*p, fp, ws, err, s);
         else
             e = launch_chunk_prep(*p, (const float*)(ws + fp.G), (float*)(ws + fp.A),
-                                  p->use_delta ? (float*)(ws + fp.N) : nullptr, nullptr, nullptr,
-                                  nullptr, s);
+                                  p->use_delta ? (float*)(ws + fp.N) : nullptr, s);
     }
     if (e == cudaSuccess) {
         if (fp.tc_tv)
